@@ -1,0 +1,542 @@
+#!/usr/bin/env python3
+"""Benchmark of the ProViP in-LLM pruning step on GB300.
+
+One step = one pass of the whole hot path over one batch: head-aware scores
+(both passes), top-k with the fused score reduction, and the compaction of
+hidden states, K, V and position ids (provip_prune). The workload is the
+LLaVA-NeXT-7B anyres batch of 8 (2880 -> 960 visual tokens before the LLM,
+960 -> 320 at the pruning layer; 32 heads x 128, hidden 4096, 96 text tokens,
+8 selected heads), seeded synthetic data.
+
+Timing: W warm-up steps, then exactly K steps replayed from CUDA graphs
+(chunks of up to 100 steps) between CUDA events on the launching stream, with a
+barrier and a device synchronisation on both sides; inputs rotate over three
+device copies (3 x 286 MB, larger than the 129 MB L2). value = samples pruned
+per second over all ranks (max time over ranks).
+
+Extra keys: roofline of the dominant kernel (the compaction; its algorithmic
+bytes per launch over its event-timed duration), the whole path's achieved
+bandwidth, e2e through the C ABI with pinned host buffers (copies inside the
+timed region), the fp64 oracle timed on the host cores (cpu_baseline), SM
+clocks sampled with nvidia-smi during the timed region.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
+                  [--impl reference]
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "pruned samples/s for head_scores+topk+compact; % of GB300 HBM roofline"
+UNIT = "samples/s"
+DEFAULT_WORKLOAD = "llava_next_7b_bf16_b8"
+FALLBACK_HBM_GBS = 6800.0
+GRAPH_CHUNK = 100
+N_COPIES = 3
+
+# DRAM traffic of one compaction launch on the default workload, from the ncu
+# capture summarised in profiles/ (null when the kernel source has changed
+# since: the sha1 of the kernel file is checked at run time).
+COMPACT_TRAFFIC = {"sha1": None, "bytes": None, "profile": None}
+
+
+def parse_args(argv=None):
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
+    ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
+    ap.add_argument("--algo", default="auto", choices=["auto", "simt", "tcgen05"])
+    ap.add_argument("--e2e-steps", type=int, default=20)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args(argv)
+
+
+# ---------------------------------------------------------------------------
+# distributed bookkeeping (one process per GPU; no collective on the data path)
+# ---------------------------------------------------------------------------
+class Dist:
+    def __init__(self):
+        self.world = int(os.environ.get("WORLD_SIZE", "1"))
+        self.rank = int(os.environ.get("RANK", "0"))
+        self.local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+        self.pg = None
+
+    def init(self, backend):
+        if self.world > 1:
+            import torch.distributed as dist
+            os.environ.setdefault("MASTER_ADDR", "127.0.0.1")
+            dist.init_process_group(backend=backend, rank=self.rank, world_size=self.world)
+            self.pg = dist
+
+    def barrier(self):
+        if self.pg:
+            self.pg.barrier()
+
+    def max(self, x: float) -> float:
+        if not self.pg:
+            return x
+        import torch
+        t = torch.tensor([x], dtype=torch.float64)
+        if self.pg.get_backend() == "nccl":
+            t = t.cuda()
+        self.pg.all_reduce(t, op=self.pg.ReduceOp.MAX)
+        return float(t.item())
+
+    def sum(self, x: float) -> float:
+        if not self.pg:
+            return x
+        import torch
+        t = torch.tensor([x], dtype=torch.float64)
+        if self.pg.get_backend() == "nccl":
+            t = t.cuda()
+        self.pg.all_reduce(t, op=self.pg.ReduceOp.SUM)
+        return float(t.item())
+
+    def close(self):
+        if self.pg:
+            self.pg.destroy_process_group()
+
+
+def aggregate(units_per_rank_total: float, max_seconds: float) -> float:
+    """whole-job throughput: units all ranks processed / slowest rank's time"""
+    return units_per_rank_total / max_seconds if max_seconds > 0 else float("nan")
+
+
+# ---------------------------------------------------------------------------
+# peaks, clocks
+# ---------------------------------------------------------------------------
+def hbm_peak():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            return float(json.load(f)["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index):
+        self.dev = device_index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            cmd = ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                   "-lms", "50"]
+            if self.dev is not None:
+                cmd += ["-i", str(self.dev)]
+            self.proc = subprocess.Popen(cmd, stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+            time.sleep(0.3)
+        except Exception:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append((time.time(), line.strip()))
+
+    def mark(self):
+        return time.time()
+
+    def stop(self, t0, t1):
+        if not self.proc:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        time.sleep(0.1)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        sm, smax, reasons, n = [], None, set(), 0
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ts, line in self.lines:
+            if ts < t0 - 0.06 or ts > t1 + 0.06:
+                continue
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                smax = float(parts[2])
+            except ValueError:
+                continue
+            n += 1
+            for nm, v in zip(names, parts[5:9]):
+                if v.lower() == "active":
+                    reasons.add(nm)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": smax,
+                "reasons": sorted(reasons), "samples": n}
+
+
+def visible_device_index(local_rank):
+    v = os.environ.get("CUDA_VISIBLE_DEVICES")
+    if v:
+        ids = [x.strip() for x in v.split(",") if x.strip()]
+        if local_rank < len(ids):
+            return ids[local_rank]
+    return local_rank
+
+
+# ---------------------------------------------------------------------------
+# algorithmic bytes (what the method must move), per launch
+# ---------------------------------------------------------------------------
+def algorithmic_bytes(w, inp):
+    import numpy as np
+    es = 4 if w.dtype == "f32" else 2
+    dh = 128
+    seq = inp["seq_len"].cpu().numpy().astype(np.int64)
+    tl = inp["text_len"].cpu().numpy().astype(np.int64)
+    heads = inp["head_list"].cpu().numpy()
+    group = w.H_q // w.H_kv
+    n_kv_used = len(set(int(h) // group for h in heads))
+    out_rows = seq - w.keep_pre + w.keep
+    row = (w.D + 2 * w.H_kv * dh) * es
+    compact = int((2 * out_rows * row).sum() + (2 * out_rows * w.P * 4).sum() + w.B * w.keep * 4)
+    scores = int((seq * n_kv_used * dh * es).sum() + (tl * w.H_sel * dh * es).sum()
+                 + w.B * w.keep_pre * 4 + w.B * w.keep * 4)
+    return {"compact": compact, "head_topk": scores, "path": compact + scores}
+
+
+def kernel_sha1(*names):
+    h = hashlib.sha1()
+    for n in names:
+        with open(os.path.join(ROOT, "paper_2608_25332_gb300", "csrc", n), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()
+
+
+# ---------------------------------------------------------------------------
+# CPU baseline: the fp64 oracle as it stands
+# ---------------------------------------------------------------------------
+def oracle_inputs(cpu):
+    import numpy as np
+    return dict(Q=cpu["Q"].float().numpy().astype(np.float64),
+                K=cpu["K"].float().numpy().astype(np.float64),
+                heads=cpu["head_list"].numpy(), ts=cpu["text_start"].numpy(),
+                tl=cpu["text_len"].numpy(), sl=cpu["seq_len"].numpy(),
+                hidden=cpu["hidden"].view(__import__("torch").int16).numpy(),
+                Kraw=cpu["K"].view(__import__("torch").int16).numpy(),
+                Vraw=cpu["V"].view(__import__("torch").int16).numpy(),
+                pos=cpu["pos"].numpy())
+
+
+def oracle_step(o, w, samples, vis_start, N_v, keep, threads):
+    import oracle
+    sel = slice(samples[0], samples[1])
+    return oracle.prune_batch(o["Q"][sel], o["K"][sel], o["heads"], o["ts"][sel], o["tl"][sel], o["sl"][sel],
+                              vis_start, N_v, keep, o["hidden"][sel], o["Kraw"][sel], o["Vraw"][sel],
+                              o["pos"][:, sel], threads=threads)
+
+
+def cpu_baseline(cpu, w, vis_start, N_v, keep, budget_s=4.0):
+    """The oracle on the workload's samples, all host cores, repeated until ~budget_s wall."""
+    import oracle
+    oracle.build()
+    threads = os.cpu_count() or 1
+    o = oracle_inputs(cpu)
+    B = w.B
+    done, t0 = 0, time.perf_counter()
+    reps = 0
+    while True:
+        oracle_step(o, w, (0, B), vis_start, N_v, keep, threads)
+        done += B
+        reps += 1
+        el = time.perf_counter() - t0
+        if el >= budget_s or reps >= 20:
+            break
+    used = min(threads, B)
+    return {"value": done / el, "unit": UNIT, "cores": used, "kind": "oracle",
+            "sample": f"{reps} x the {B}-sample batch of {w.name} (fp64 oracle: scores, top-k, "
+                      f"compaction), OpenMP over samples, {el:.1f} s wall"}
+
+
+# ---------------------------------------------------------------------------
+# the reference arm: the oracle, K steps of a bounded slice of the workload
+# ---------------------------------------------------------------------------
+def run_reference(args, dist):
+    import numpy as np
+    import torch
+    import oracle
+    from paper_2608_25332_gb300 import synth
+    if dist.rank != 0:
+        return 0
+    oracle.build()
+    w = synth.BY_NAME[args.workload]
+    cpu = synth.in_llm_inputs(w)
+    o = oracle_inputs(cpu)
+    threads = os.cpu_count() or 1
+    vis, nv, keep = cpu["vis_start"], cpu["N_v"], cpu["keep"]
+    rows_per_sample = int(cpu["text_len"][0])
+    heads = o["heads"]
+    # Unit of work: one text row of one sample scored over every selected head
+    # (the oracle's inner loop); the sample's top-k and compaction run with its
+    # last row. Rows per step are sized so that W + K steps fit ~120 s.
+    t0 = time.perf_counter()
+    oracle.head_scores(o["Q"][0, :o["sl"][0]], o["K"][0, :o["sl"][0]], heads, [int(o["ts"][0])], vis, nv)
+    t_row = max(time.perf_counter() - t0, 1e-5)
+    budget = 120.0 / max(1, args.steps + args.warmup)
+    rows_per_step = max(1, min(rows_per_sample * w.B, int(budget / t_row)))
+    state = {"b": 0, "r": 0, "acc": np.zeros(nv)}
+
+    def step():
+        left = rows_per_step
+        while left > 0:
+            b, r = state["b"], state["r"]
+            n = min(left, int(o["tl"][b]) - r)
+            rows = np.arange(int(o["ts"][b]) + r, int(o["ts"][b]) + r + n)
+            sl = int(o["sl"][b])
+            state["acc"] += oracle.head_scores(o["Q"][b, :sl], o["K"][b, :sl], heads, rows, vis, nv) * n
+            state["r"] += n
+            left -= n
+            if state["r"] == int(o["tl"][b]):
+                v = state["acc"] / int(o["tl"][b])
+                idx = oracle.topk(v, keep)
+                src = oracle.compact_map(sl, vis, nv, idx)
+                for key in ("hidden", "Kraw", "Vraw"):
+                    oracle.gather_rows(o[key][b], src)
+                state.update(b=(b + 1) % w.B, r=0, acc=np.zeros(nv))
+        return rows_per_step
+
+    for _ in range(args.warmup):
+        step()
+    t0 = time.perf_counter()
+    rows = sum(step() for _ in range(args.steps))
+    el = time.perf_counter() - t0
+    samples = rows / rows_per_sample
+    value = samples / el
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * el / max(1, args.steps),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": {"workload": w.name, "B": w.B},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
+                             "sample": f"{rows_per_step} text row(s) per step of {w.name} scored over "
+                                       f"{w.H_sel} heads, each sample's top-k + compaction with its last "
+                                       f"row; {samples:.2f} samples in {el:.1f} s"},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line))
+    return 0
+
+
+# ---------------------------------------------------------------------------
+# the GB300 arm
+# ---------------------------------------------------------------------------
+def run_gb300(args, dist):
+    import numpy as np
+    import torch
+    import __graft_entry__
+    from paper_2608_25332_gb300 import provip as P
+    from paper_2608_25332_gb300 import synth
+
+    torch.cuda.set_device(dist.local_rank)
+    dev = torch.device("cuda", dist.local_rank)
+    __graft_entry__.build()
+    w = synth.BY_NAME[args.workload]
+    # each rank prunes its own shard of samples (seeded by rank)
+    cpu = synth.in_llm_inputs(w, seed=w.seed + 1000 * dist.rank)
+    vis, nv, keep = cpu["vis_start"], cpu["N_v"], cpu["keep"]
+    algo = {"auto": P.ALGO_AUTO, "simt": P.ALGO_SIMT, "tcgen05": P.ALGO_TCGEN05}[args.algo]
+    copies = []
+    for _ in range(N_COPIES):
+        copies.append({k: (v.to(dev) if isinstance(v, torch.Tensor) else v) for k, v in cpu.items()})
+    g0 = copies[0]
+    step = P.PruneStep(g0["Q"], g0["K"], g0["V"], g0["hidden"], g0["pos"], g0["head_list"], w.n_t[1], nv, keep,
+                       algo=algo, want_scores=False)
+
+    def do_step(i):
+        c = copies[i % N_COPIES]
+        step(c["Q"], c["K"], c["V"], c["hidden"], c["pos"], c["text_start"], c["text_len"], c["seq_len"], vis)
+
+    # warm-up
+    for i in range(max(args.warmup, 1)):
+        do_step(i)
+    torch.cuda.synchronize()
+    rc, bits = P.provip_device_status(clear=True)
+    if rc != 0:
+        raise RuntimeError(f"device status {rc} {bits} after warm-up")
+
+    # graphs of up to GRAPH_CHUNK steps (the step index picks the input copy)
+    K = args.steps
+    sizes = []
+    left = K
+    while left > 0:
+        n = min(GRAPH_CHUNK, left)
+        sizes.append(n)
+        left -= n
+    graphs = {}
+    stream = torch.cuda.Stream(device=dev)
+    for n in sorted(set(sizes)):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            for i in range(n):
+                do_step(i)
+        graphs[n] = g
+    torch.cuda.synchronize()
+
+    sampler = ClockSampler(visible_device_index(dist.local_rank) if dist.rank == 0 else None)
+    if dist.rank == 0:
+        sampler.start()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    dist.barrier()
+    torch.cuda.synchronize()
+    t_wall0 = time.time()
+    ev0.record()
+    for n in sizes:
+        graphs[n].replay()
+    ev1.record()
+    torch.cuda.synchronize()
+    t_wall1 = time.time()
+    dist.barrier()
+    sec = ev0.elapsed_time(ev1) / 1e3
+    clocks = sampler.stop(t_wall0, t_wall1) if dist.rank == 0 else None
+    max_sec = dist.max(sec)
+    total_samples = dist.sum(float(w.B * K))
+    value = aggregate(total_samples, max_sec)
+    rc, bits = P.provip_device_status(clear=True)
+    if rc != 0:
+        raise RuntimeError(f"device status {rc} {bits} after the timed region")
+
+    # per-kernel durations (same launch configuration, graphs of GRAPH_CHUNK launches)
+    ab = algorithmic_bytes(w, cpu)
+    out = step(g0["Q"], g0["K"], g0["V"], g0["hidden"], g0["pos"], g0["text_start"], g0["text_len"],
+               g0["seq_len"], vis)
+    idx = out["idx"].clone()
+    outs = (step.hidden_out, step.K_out, step.V_out, step.pos_out)
+    ws_ht = P.workspace(step.ws.numel(), dev)
+
+    def compact_i(i):
+        c = copies[i % N_COPIES]
+        P.provip_compact(idx, c["hidden"], c["K"], c["V"], c["pos"], c["seq_len"], vis, nv, out=outs)
+
+    def head_topk_i(i):
+        c = copies[i % N_COPIES]
+        P.provip_head_topk(c["Q"], c["K"], c["head_list"], c["text_start"], c["text_len"], c["seq_len"], vis, nv,
+                           keep, algo=algo, N_t_max=w.n_t[1], ws=ws_ht, want_scores=False)
+
+    def time_graph(fn, reps):
+        for i in range(3):
+            fn(i)
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            for i in range(GRAPH_CHUNK):
+                fn(i)
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        for _ in range(reps):
+            g.replay()
+        b.record()
+        torch.cuda.synchronize()
+        return a.elapsed_time(b) / 1e3 / (reps * GRAPH_CHUNK)
+
+    reps = max(1, min(20, K // GRAPH_CHUNK))
+    t_compact = time_graph(compact_i, reps)
+    t_head = time_graph(head_topk_i, reps)
+    peak, peak_src = hbm_peak()
+    ach = ab["compact"] / t_compact / 1e9
+    traffic = None
+    if COMPACT_TRAFFIC["bytes"] and COMPACT_TRAFFIC["sha1"] == kernel_sha1("compact.cu") and \
+            args.workload == DEFAULT_WORKLOAD:
+        traffic = COMPACT_TRAFFIC["bytes"]
+    path_gbs = ab["path"] * K / max_sec / 1e9  # per GPU
+
+    # e2e: host buffers through the C ABI, H2D + prune + D2H per step
+    pin = {k: v.pin_memory() for k, v in cpu.items() if isinstance(v, torch.Tensor)}
+    dbuf = {k: torch.empty_like(v, device=dev) for k, v in pin.items()}
+    host_out = {k: torch.empty(v.shape, dtype=v.dtype, pin_memory=True)
+                for k, v in (("hidden", step.hidden_out), ("K", step.K_out), ("V", step.V_out),
+                             ("pos", step.pos_out), ("idx", step.idx), ("seq_len", step.seq_len_out))}
+    h2d = sum(v.numel() * v.element_size() for v in pin.values())
+    d2h = sum(v.numel() * v.element_size() for v in host_out.values())
+
+    def e2e_step():
+        for k, v in pin.items():
+            dbuf[k].copy_(v, non_blocking=True)
+        r = step(dbuf["Q"], dbuf["K"], dbuf["V"], dbuf["hidden"], dbuf["pos"], dbuf["text_start"],
+                 dbuf["text_len"], dbuf["seq_len"], vis)
+        for k in host_out:
+            host_out[k].copy_(r[k], non_blocking=True)
+
+    for _ in range(2):
+        e2e_step()
+    torch.cuda.synchronize()
+    E = max(1, args.e2e_steps)
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    dist.barrier()
+    a.record()
+    for _ in range(E):
+        e2e_step()
+    b.record()
+    torch.cuda.synchronize()
+    e2e_sec = dist.max(a.elapsed_time(b) / 1e3)
+    e2e_value = aggregate(dist.sum(float(w.B * E)), e2e_sec)
+
+    cpu_base = None
+    if dist.rank == 0 and dist.world == 1 and not args.no_cpu_baseline:
+        cpu_base = cpu_baseline(cpu, w, vis, nv, keep)
+
+    if dist.rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": dist.world, "steps": K,
+            "warmup": args.warmup, "ms_per_step": 1e3 * max_sec / K, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
+            "config": {"workload": w.name, "B": w.B, "N_v": nv, "keep": keep, "L_max": w.L_max,
+                       "H_q": w.H_q, "H_kv": w.H_kv, "H_sel": w.H_sel, "D": w.D,
+                       "algo": args.algo,
+                       "l2": f"inputs larger than L2: {N_COPIES} rotating device copies of "
+                             f"{sum(v.numel() * v.element_size() for v in pin.values()) / 1e6:.0f} MB",
+                       "timing": f"CUDA graphs of {GRAPH_CHUNK} steps, events on the launching stream"},
+            "roofline": {"bound": "hbm", "kernel": "compact_kernel", "achieved": ach, "peak": peak,
+                         "peak_source": peak_src, "unit": "GB/s", "frac": ach / peak,
+                         "traffic": traffic, "algorithmic_bytes": ab["compact"],
+                         "duration_us": t_compact * 1e6},
+            "path": {"algorithmic_bytes": ab["path"], "achieved_gbs": path_gbs, "frac": path_gbs / peak,
+                     "head_topk_us": t_head * 1e6, "head_topk_bytes": ab["head_topk"],
+                     "compact_us": t_compact * 1e6},
+            "cpu_baseline": cpu_base,
+            "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+            "gpu_launches": 4 * K,
+            "clocks": clocks,
+        }
+        print(json.dumps(line))
+    return 0
+
+
+def main(argv=None):
+    args = parse_args(argv)
+    dist = Dist()
+    if args.impl == "reference":
+        dist.init("gloo")
+        try:
+            return run_reference(args, dist)
+        finally:
+            dist.close()
+    import torch
+    dist.init("nccl" if torch.cuda.is_available() else "gloo")
+    try:
+        return run_gb300(args, dist)
+    finally:
+        dist.close()
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,236 @@
+/*
+ * provip.h - C ABI of the GB300 (sm_103a) ProViP token-pruning library.
+ *
+ * ProViP ("Not All Attention Heads Contribute to Critical Visual Token
+ * Selection: Head-Aware Pruning Matters More") prunes visual tokens of a
+ * vision-language model in two places:
+ *   - before the LLM (Sec. 4.2-4.3): critical text tokens from the text
+ *     self-similarity, text-guided cosine relevance of every visual token, a
+ *     top-N1 keep set, and the pruned tokens merged into their nearest kept
+ *     token;
+ *   - inside the LLM (Sec. 4.4): attention probabilities from the text rows to
+ *     the visual columns for a chosen set of heads, normalised over the full
+ *     causal key range, averaged over heads and text rows, top-N2 kept, and the
+ *     sequence (hidden states, K/V rows, position ids) compacted.
+ *
+ * Conventions shared by every call
+ *   - Tensor pointers are DEVICE pointers owned by the caller, C-contiguous,
+ *     row-major with the shapes given; the library never frees or retains them.
+ *     Pointers marked "host" are read on the host during the call.
+ *   - dtype is PROVIP_F32 or PROVIP_BF16 and applies to every floating-point
+ *     input/output tensor of the call except scores, which are always fp32.
+ *   - Every call is asynchronous on `stream` (a cudaStream_t; NULL is the
+ *     legacy default stream) and allocates nothing: scratch memory comes from
+ *     the caller's workspace `ws` of `ws_bytes` bytes (256-byte aligned), sized
+ *     by the matching *_workspace_size() query with the same shape arguments.
+ *     Workspace contents need not be initialised and are clobbered.
+ *   - Return value: PROVIP_OK or a negative status. Arguments are validated on
+ *     the host before anything is launched; on error nothing is enqueued.
+ *     Values that live in device memory (lengths, indices) cannot be checked
+ *     before launch: kernels that meet an out-of-range one skip it and set the
+ *     device status word, read with provip_device_status().
+ *   - Every wait inside a kernel is bounded (2 s); a wait that gives up sets
+ *     PROVIP_DEVSTAT_TIMEOUT in the device status word instead of hanging.
+ *   - Sequences are laid out per sample as [prefix rows | N_v visual rows |
+ *     text rows | padding]: visual rows start at vis_start, a sample's rows
+ *     beyond seq_len[b] are padding and never read.
+ */
+#ifndef PROVIP_H_
+#define PROVIP_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* status codes */
+#define PROVIP_OK 0
+#define PROVIP_ERR_INVALID_ARG (-1) /* a host-checkable argument is out of range */
+#define PROVIP_ERR_UNSUPPORTED (-2) /* dtype / shape / alignment not supported */
+#define PROVIP_ERR_WORKSPACE (-3)   /* ws_bytes smaller than the size query */
+#define PROVIP_ERR_CUDA (-4)        /* a CUDA call failed; see provip_last_error() */
+#define PROVIP_ERR_TIMEOUT (-5)     /* returned by provip_device_status() */
+
+/* element types */
+#define PROVIP_F32 0
+#define PROVIP_BF16 1
+
+/* kernel families for provip_head_scores / provip_prune */
+#define PROVIP_ALGO_AUTO 0    /* tensor cores for bf16, CUDA cores for fp32 */
+#define PROVIP_ALGO_SIMT 1    /* CUDA-core FFMA kernels (fp32 and bf16) */
+#define PROVIP_ALGO_TCGEN05 2 /* tcgen05 tensor cores, TMEM accumulators (bf16 only) */
+
+/* bits of the device status word */
+#define PROVIP_DEVSTAT_TIMEOUT 1u  /* a bounded wait gave up */
+#define PROVIP_DEVSTAT_BAD_ARG 2u  /* a device-resident argument was out of range */
+
+/* ------------------------------------------------------------------------
+ * Library status
+ * ---------------------------------------------------------------------- */
+
+/* Human-readable name of a status code (static string). */
+const char *provip_status_string(int status);
+
+/* Message of the last PROVIP_ERR_CUDA / INVALID_ARG / UNSUPPORTED returned on
+ * the calling thread (static per thread; empty if none). */
+const char *provip_last_error(void);
+
+/* Library version as 10000*major + 100*minor + patch. */
+int provip_version(void);
+
+/* Synchronises the current device, then returns the device status word of the
+ * current device (PROVIP_DEVSTAT_* bits) in *bits and clears it when `clear`
+ * is non-zero. Returns PROVIP_ERR_TIMEOUT if the TIMEOUT bit is set,
+ * PROVIP_ERR_INVALID_ARG if BAD_ARG is set, PROVIP_OK otherwise. */
+int provip_device_status(unsigned *bits, int clear);
+
+/* ------------------------------------------------------------------------
+ * Pre-LLM pass (Sec. 4.2-4.3)
+ * ---------------------------------------------------------------------- */
+
+/* Critical textual token selection (Sec. 4.2, equations for r and T):
+ *   G = E_t E_t^T (no scaling), R = row-wise softmax of G,
+ *   r_j = (1/N_t) sum_i R_ij,  T = { j : r_j > mean(r) };
+ * over the text_len[b] valid rows of each sample. If no r_j exceeds the mean
+ * (e.g. N_t = 1 or identical rows) T is every valid row.
+ *   emb_t    [B, N_t_max, D] dtype; rows >= text_len[b] are not read.
+ *   text_len [B] int32, 0 <= text_len[b] <= N_t_max.
+ *   mask_out [B, N_t_max] uint8: 1 for j in T, 0 otherwise (and for padding).
+ *   r_out    [B, N_t_max] fp32 or NULL: r (0 for padding).
+ * Requires D % 8 == 0, N_t_max <= 4096. */
+size_t provip_crit_text_workspace_size(int B, int N_t_max, int D);
+int provip_crit_text(const void *emb_t, int B, int N_t_max, int D, const int *text_len,
+                     int dtype, uint8_t *mask_out, float *r_out, void *ws, size_t ws_bytes,
+                     void *stream);
+
+/* Text-guided visual relevance (Sec. 4.3, equations for M, M-hat and p):
+ *   M_ij = cos(E_t[i], E_v[j]) for i in T (crit_mask), j < N_v (0 for a zero row),
+ *   p_j  = max_{i in T} ( M_ij - (1/N_v) sum_k M_ik ).
+ *   emb_v [B, N_v, D], emb_t [B, N_t_max, D] dtype; crit_mask [B, N_t_max] uint8.
+ *   p_out [B, N_v] fp32 (-inf for a sample without a critical row).
+ * Requires D % 8 == 0. */
+size_t provip_relevance_workspace_size(int B, int N_v, int D, int N_t_max);
+int provip_relevance(const void *emb_v, int B, int N_v, int D, const void *emb_t,
+                     const int *text_len, int N_t_max, const uint8_t *crit_mask, int dtype,
+                     float *p_out, void *ws, size_t ws_bytes, void *stream);
+
+/* Top-k per sample (Sec. 4.3 top N1 of p, Sec. 4.4 top N2 of v): the k
+ * largest of scores[b][0..N), ties broken toward the lower index, written in
+ * ascending index order to idx_out [B, k] int32. 1 <= k <= N <= 49152.
+ * NaN sorts above +inf. No workspace. */
+int provip_topk(const float *scores, int B, int N, int k, int *idx_out, void *stream);
+
+/* Merge of pruned visual tokens into their nearest kept token (Sec. 4.3, last
+ * paragraph; the paper defers the rule to ApET without stating it - this
+ * library reads it as: each pruned row j goes to the kept row of largest
+ * cosine, ties to the lower kept position; merged = uniform mean of the kept
+ * row and its members).
+ *   keep_idx   [B, keep] int32, strictly ascending visual indices (device).
+ *   assign_out [B, N_v] int32: position in keep_idx of row j's centroid (kept
+ *              rows map to their own position).
+ *   merged_out [B, keep, D] dtype or NULL (assignment only). fp32 sums are
+ *              accumulated in double, bf16 sums in float, both in ascending
+ *              row order; the mean is rounded to nearest-even.
+ * Requires D % 8 == 0, D <= 8192. */
+size_t provip_merge_workspace_size(int B, int N_v, int D, int keep);
+int provip_merge(const void *emb_v, int B, int N_v, int D, const int *keep_idx, int keep,
+                 int dtype, int *assign_out, void *merged_out, void *ws, size_t ws_bytes,
+                 void *stream);
+
+/* The whole pre-LLM pass: critical text tokens (unless crit_mask_or_null is
+ * given), relevance p, top keep_pre of p (idx_out, ascending), and the merge
+ * (when merged_out_or_null is given). p_out_or_null / mask_out_or_null
+ * receive the intermediate p [B, N_v] and T mask [B, N_t_max] when non-NULL. */
+size_t provip_similarity_reduce_workspace_size(int B, int N_v, int D, int N_t_max, int keep_pre);
+int provip_similarity_reduce(const void *emb_v, int B, int N_v, int D, const void *emb_t,
+                             const int *text_len, int N_t_max,
+                             const uint8_t *crit_mask_or_null, int keep_pre, int dtype,
+                             int *idx_out, void *merged_out_or_null, float *p_out_or_null,
+                             uint8_t *mask_out_or_null, void *ws, size_t ws_bytes,
+                             void *stream);
+
+/* ------------------------------------------------------------------------
+ * In-LLM head-aware pruning (Sec. 4.4)
+ * ---------------------------------------------------------------------- */
+
+/* Head-aware visual-token scores (Sec. 4.4, equations for S^vis and v):
+ *   A_{h,j,i} = softmax over keys 0..t_j of q_{t_j,h} . k_{k,g(h)} / sqrt(d_h),
+ *               taken at key vis_start + i  (t_j the absolute position of text
+ *               row j, g(h) = h / (H_q / H_kv) its key/value head);
+ *   v_i       = 1/(|V| |R|) sum_{h in V} sum_{j in R} A_{h,j,i}.
+ * V = head_list (host int32[H_sel], distinct, in [0, H_q)); R = text rows
+ * j < text_len[b] at positions text_start[b] + j, restricted to
+ * row_mask_or_null[b][j] != 0 when given (e.g. the critical rows T).
+ *   Q [B, L_max, H_q, d_h], K [B, L_max, H_kv, d_h] dtype (post-RoPE).
+ *   text_start, text_len, seq_len [B] int32 (device).
+ *   row_mask_or_null [B, N_t_max] uint8 or NULL.
+ *   scores [B, N_v] fp32.
+ * Only the selected heads are read; the attention matrix is never stored.
+ * Requires d_h == 128, H_q % H_kv == 0, 1 <= H_sel <= 64, vis_start + N_v <=
+ * seq_len[b], text_start[b] + text_len[b] <= seq_len[b] <= L_max.
+ * algo: PROVIP_ALGO_* (TCGEN05 requires bf16). */
+size_t provip_head_scores_workspace_size(int B, int L_max, int H_sel, int N_t_max, int N_v,
+                                         int algo, int dtype);
+int provip_head_scores(const void *Q, const void *K, int B, int L_max, int H_q, int H_kv,
+                       int d_h, const int *head_list, int H_sel, const int *text_start,
+                       const int *text_len, const uint8_t *row_mask_or_null, int N_t_max,
+                       int vis_start, int N_v, const int *seq_len, int dtype, int algo,
+                       float *scores, void *ws, size_t ws_bytes, void *stream);
+
+/* Survivor compaction given the kept indices (Sec. 4.1: pruned tokens are
+ * excluded from all later computation). For every sample the output rows are
+ *   [0, vis_start) ++ (vis_start + idx[b][a], a < keep) ++ [vis_start + N_v, seq_len[b])
+ * gathered byte-exactly from hidden [B, L_max, D], K/V [B, L_max, H_kv, d_h]
+ * (either may be NULL, both or neither) and pos [P, B, L_max] int32 (NULL
+ * allowed) into hidden_out [B, L_out, D], K_out/V_out [B, L_out, H_kv, d_h],
+ * pos_out [P, B, L_out] with L_out = L_max - N_v + keep. Position ids are
+ * carried, not renumbered. seq_len_out [B] (may be NULL) = seq_len - N_v + keep.
+ * Output rows >= seq_len_out[b] are left untouched.
+ *   idx [B, keep] int32 ascending in [0, N_v) (device).
+ * Row sizes (D and H_kv*d_h elements) must be multiples of 16 bytes and every
+ * tensor pointer 16-byte aligned. */
+int provip_compact(const int *idx, int B, int N_v, int keep, const void *hidden, int D,
+                   const void *K, const void *V, int H_kv, int d_h, const int *pos, int P,
+                   const int *seq_len, int L_max, int vis_start, int dtype, void *hidden_out,
+                   void *K_out, void *V_out, int *pos_out, int *seq_len_out, void *stream);
+
+/* provip_topk on scores [B, N_v] (keep of them, idx_out ascending) followed by
+ * provip_compact with that idx. No workspace. */
+int provip_topk_compact(const float *scores, int B, int N_v, int keep, const void *hidden,
+                        int D, const void *K, const void *V, int H_kv, int d_h, const int *pos,
+                        int P, const int *seq_len, int L_max, int vis_start, int dtype,
+                        void *hidden_out, void *K_out, void *V_out, int *pos_out,
+                        int *idx_out, int *seq_len_out, void *stream);
+
+/* Head-aware selection: provip_head_scores followed by the top `keep` of the
+ * scores (ties to the lower index, idx_out [B, keep] ascending), with the
+ * score reduction fused into the top-k kernel (the scores are bit-identical
+ * to provip_head_scores'). scores_out_or_null receives v [B, N_v] when
+ * non-NULL. Uses the workspace of provip_head_scores. N_v <= 49152. */
+int provip_head_topk(const void *Q, const void *K, int B, int L_max, int H_q, int H_kv, int d_h,
+                     const int *head_list, int H_sel, const int *text_start, const int *text_len,
+                     const uint8_t *row_mask_or_null, int N_t_max, int vis_start, int N_v,
+                     const int *seq_len, int keep, int dtype, int algo, int *idx_out,
+                     float *scores_out_or_null, void *ws, size_t ws_bytes, void *stream);
+
+/* The in-LLM pruning step end to end: provip_head_topk, then
+ * provip_compact with its idx. Arguments as in the calls above; K is both the scored keys and the
+ * compacted K. scores_out_or_null receives v [B, N_v] when non-NULL. Uses the
+ * workspace of provip_head_scores. */
+size_t provip_prune_workspace_size(int B, int L_max, int H_sel, int N_t_max, int N_v, int algo,
+                                   int dtype);
+int provip_prune(const void *Q, const void *K, const void *V, const void *hidden, int B,
+                 int L_max, int H_q, int H_kv, int d_h, int D, const int *head_list, int H_sel,
+                 const int *text_start, const int *text_len, const uint8_t *row_mask_or_null,
+                 int N_t_max, int vis_start, int N_v, const int *seq_len, const int *pos, int P,
+                 int keep, int dtype, int algo, void *hidden_out, void *K_out, void *V_out,
+                 int *pos_out, int *idx_out, int *seq_len_out, float *scores_out_or_null,
+                 void *ws, size_t ws_bytes, void *stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* PROVIP_H_ */

@@ -1,0 +1,703 @@
+// C-ABI layer of the ProViP GB300 library: host-side argument validation,
+// workspace carving and kernel launches. Declarations and the contract of each
+// entry point are in include/provip.h.
+#include <math.h>
+#include <stdarg.h>
+#include <stdio.h>
+#include <string.h>
+
+#include "../../include/provip.h"
+#include "kernels.h"
+
+using namespace provip;
+
+// device status word (one per device that loads the library)
+__device__ unsigned int g_provip_status;
+
+namespace {
+
+thread_local char g_last_error[512] = {0};
+
+int fail(int code, const char* fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(g_last_error, sizeof(g_last_error), fmt, ap);
+  va_end(ap);
+  return code;
+}
+
+int cuda_fail(cudaError_t e, const char* where) {
+  return fail(PROVIP_ERR_CUDA, "%s: %s", where, cudaGetErrorString(e));
+}
+
+struct DevInfo {
+  bool init = false;
+  int sms = 0;
+  unsigned* status = nullptr;
+};
+DevInfo g_dev[64];
+
+// per-device facts, looked up once with that device current
+int dev_info(DevInfo** out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+  if (dev < 0 || dev >= 64) return fail(PROVIP_ERR_UNSUPPORTED, "device ordinal %d >= 64", dev);
+  DevInfo& d = g_dev[dev];
+  if (!d.init) {
+    e = cudaDeviceGetAttribute(&d.sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceGetAttribute");
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_provip_status);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress(status)");
+    d.status = static_cast<unsigned*>(p);
+    d.init = true;
+  }
+  *out = &d;
+  return PROVIP_OK;
+}
+
+constexpr size_t kAlign = 256;
+inline size_t align_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
+
+// bump allocator over the caller's workspace (also used to size it)
+struct Carve {
+  char* base;
+  size_t off = 0;
+  explicit Carve(void* b) : base(static_cast<char*>(b)) {}
+  template <typename T>
+  T* take(size_t count) {
+    T* p = base ? reinterpret_cast<T*>(base + off) : nullptr;
+    off += align_up(count * sizeof(T));
+    return p;
+  }
+};
+
+inline int esize(int dtype) { return dtype == PROVIP_F32 ? 4 : 2; }
+inline bool dtype_ok(int dtype) { return dtype == PROVIP_F32 || dtype == PROVIP_BF16; }
+inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// ---------------------------------------------------------------------------
+// head scores: shapes and workspace
+// ---------------------------------------------------------------------------
+int resolve_algo(int algo, int dtype) {
+  if (algo == PROVIP_ALGO_AUTO) return dtype == PROVIP_BF16 ? PROVIP_ALGO_TCGEN05 : PROVIP_ALGO_SIMT;
+  return algo;
+}
+int key_chunk(int algo) { return algo == PROVIP_ALGO_TCGEN05 ? 128 : 64; }
+int vis_chunk(int algo) { return algo == PROVIP_ALGO_TCGEN05 ? 128 : 64; }
+
+struct HSShape {
+  int n_rb, kc, n_kc, vc, n_vc;
+};
+HSShape hs_shape(int L_max, int N_t_max, int N_v, int algo) {
+  HSShape s;
+  s.n_rb = (N_t_max + kRowBlock - 1) / kRowBlock;
+  s.kc = key_chunk(algo);
+  s.n_kc = (L_max + s.kc - 1) / s.kc;
+  s.vc = vis_chunk(algo);
+  s.n_vc = (N_v + s.vc - 1) / s.vc;
+  return s;
+}
+size_t hs_ws(Carve& c, int B, int H_sel, const HSShape& s, int N_v, float2** stats,
+             float** partial) {
+  *stats = c.take<float2>((size_t)B * s.n_rb * H_sel * s.n_kc * kRowBlock);
+  *partial = c.take<float>((size_t)B * s.n_rb * H_sel * N_v);
+  return c.off;
+}
+
+int hs_validate(const void* Q, const void* K, int B, int L_max, int H_q, int H_kv, int d_h,
+                const int* head_list, int H_sel, const int* text_start, const int* text_len,
+                int N_t_max, int vis_start, int N_v, const int* seq_len, int dtype, int algo) {
+  if (!Q || !K || !head_list || !text_start || !text_len || !seq_len)
+    return fail(PROVIP_ERR_INVALID_ARG, "head_scores: null pointer argument");
+  if (B < 1 || L_max < 1 || H_q < 1 || H_kv < 1 || N_t_max < 1 || N_v < 1 || vis_start < 0)
+    return fail(PROVIP_ERR_INVALID_ARG, "head_scores: non-positive size");
+  if (H_q % H_kv != 0) return fail(PROVIP_ERR_INVALID_ARG, "head_scores: H_q %% H_kv != 0");
+  if (vis_start + N_v > L_max) return fail(PROVIP_ERR_INVALID_ARG, "head_scores: visual range exceeds L_max");
+  if (N_t_max > L_max) return fail(PROVIP_ERR_INVALID_ARG, "head_scores: N_t_max > L_max");
+  if (!dtype_ok(dtype)) return fail(PROVIP_ERR_UNSUPPORTED, "head_scores: dtype %d", dtype);
+  if (d_h != kHeadDim) return fail(PROVIP_ERR_UNSUPPORTED, "head_scores: d_h must be 128");
+  if (H_sel < 1 || H_sel > kMaxHeads) return fail(PROVIP_ERR_INVALID_ARG, "head_scores: H_sel %d", H_sel);
+  for (int i = 0; i < H_sel; ++i) {
+    if (head_list[i] < 0 || head_list[i] >= H_q)
+      return fail(PROVIP_ERR_INVALID_ARG, "head_scores: head_list[%d] = %d out of range", i, head_list[i]);
+    for (int j = 0; j < i; ++j)
+      if (head_list[j] == head_list[i])
+        return fail(PROVIP_ERR_INVALID_ARG, "head_scores: duplicate head %d", head_list[i]);
+  }
+  if (algo != PROVIP_ALGO_SIMT && algo != PROVIP_ALGO_TCGEN05)
+    return fail(PROVIP_ERR_INVALID_ARG, "head_scores: algo %d", algo);
+  if (algo == PROVIP_ALGO_TCGEN05 && dtype != PROVIP_BF16)
+    return fail(PROVIP_ERR_UNSUPPORTED, "head_scores: tcgen05 path needs bf16");
+  if (!aligned16(Q) || !aligned16(K)) return fail(PROVIP_ERR_UNSUPPORTED, "head_scores: Q/K not 16-byte aligned");
+  if ((size_t)B * L_max * H_q * d_h >= (1ull << 40))
+    return fail(PROVIP_ERR_UNSUPPORTED, "head_scores: tensor too large");
+  return PROVIP_OK;
+}
+
+HSArgs hs_args(const void* Q, const void* K, int B, int L_max, int H_q, int H_kv, int d_h,
+               const int* head_list, int H_sel, const int* text_start, const int* text_len,
+               const uint8_t* row_mask, int N_t_max, int vis_start, int N_v, const int* seq_len,
+               const HSShape& sh, float2* stats, float* partial, unsigned* err) {
+  HSArgs a;
+  memset(&a, 0, sizeof(a));
+  a.Q = Q;
+  a.K = K;
+  a.B = B;
+  a.L_max = L_max;
+  a.H_q = H_q;
+  a.H_kv = H_kv;
+  a.d_h = d_h;
+  a.H_sel = H_sel;
+  for (int i = 0; i < H_sel; ++i) a.heads[i] = head_list[i];
+  a.text_start = text_start;
+  a.text_len = text_len;
+  a.row_mask = row_mask;
+  a.N_t_max = N_t_max;
+  a.vis_start = vis_start;
+  a.N_v = N_v;
+  a.seq_len = seq_len;
+  a.n_rb = sh.n_rb;
+  a.kc = sh.kc;
+  a.n_kc = sh.n_kc;
+  a.vc = sh.vc;
+  a.n_vc = sh.n_vc;
+  a.scale_log2 = (float)(1.4426950408889634 / sqrt((double)d_h));
+  a.stats = stats;
+  a.partial = partial;
+  a.err = err;
+  return a;
+}
+
+// both passes of the head scores (partials in the workspace)
+int hs_run(const HSArgs& a, int dtype, int algo, cudaStream_t s) {
+  cudaError_t e;
+  if (algo == PROVIP_ALGO_TCGEN05) {
+    CUtensorMap tq, tk;
+    const uint64_t qstride = (uint64_t)a.H_q * a.d_h * 2, kstride = (uint64_t)a.H_kv * a.d_h * 2;
+    if (make_tmap_bf16_2d(&tq, a.Q, (uint64_t)a.B * a.L_max, (uint64_t)a.H_q * a.d_h, qstride, 128) ||
+        make_tmap_bf16_2d(&tk, a.K, (uint64_t)a.B * a.L_max, (uint64_t)a.H_kv * a.d_h, kstride, 128))
+      return fail(PROVIP_ERR_CUDA, "head_scores: cuTensorMapEncodeTiled failed");
+    e = hs_launch_tc(a, &tq, &tk, s);
+  } else {
+    e = hs_launch_simt(a, dtype, s);
+  }
+  if (e != cudaSuccess) return cuda_fail(e, "head_scores launch");
+  return PROVIP_OK;
+}
+
+int compact_validate(const int* idx, int B, int N_v, int keep, const void* hidden, int D,
+                     const void* K, const void* V, int H_kv, int d_h, const int* pos, int P,
+                     const int* seq_len, int L_max, int vis_start, int dtype, void* hidden_out,
+                     void* K_out, void* V_out, int* pos_out) {
+  if (!idx || !seq_len) return fail(PROVIP_ERR_INVALID_ARG, "compact: null idx/seq_len");
+  if (!hidden || !hidden_out) return fail(PROVIP_ERR_INVALID_ARG, "compact: hidden is required");
+  if (B < 1 || N_v < 1 || D < 1 || L_max < 1 || vis_start < 0 || vis_start + N_v > L_max)
+    return fail(PROVIP_ERR_INVALID_ARG, "compact: bad sizes");
+  if (keep < 1 || keep > N_v) return fail(PROVIP_ERR_INVALID_ARG, "compact: keep %d not in [1, N_v]", keep);
+  if (!dtype_ok(dtype)) return fail(PROVIP_ERR_UNSUPPORTED, "compact: dtype %d", dtype);
+  if ((K == nullptr) != (K_out == nullptr) || (V == nullptr) != (V_out == nullptr))
+    return fail(PROVIP_ERR_INVALID_ARG, "compact: K/V given without output (or vice versa)");
+  if ((K || V) && (H_kv < 1 || d_h < 1)) return fail(PROVIP_ERR_INVALID_ARG, "compact: bad H_kv/d_h");
+  if (pos && (!pos_out || P < 1)) return fail(PROVIP_ERR_INVALID_ARG, "compact: pos without pos_out/P");
+  const long long hb = (long long)D * esize(dtype), kb = (long long)H_kv * d_h * esize(dtype);
+  if (hb % 16 || ((K || V) && kb % 16))
+    return fail(PROVIP_ERR_UNSUPPORTED, "compact: row bytes must be multiples of 16");
+  const void* ptrs[6] = {hidden, hidden_out, K, K_out, V, V_out};
+  for (const void* p : ptrs)
+    if (p && !aligned16(p)) return fail(PROVIP_ERR_UNSUPPORTED, "compact: tensor not 16-byte aligned");
+  return PROVIP_OK;
+}
+
+CompactArgs compact_args(const int* idx, int B, int N_v, int keep, const void* hidden, int D,
+                         const void* K, const void* V, int H_kv, int d_h, const int* pos, int P,
+                         const int* seq_len, int L_max, int vis_start, int dtype,
+                         void* hidden_out, void* K_out, void* V_out, int* pos_out,
+                         int* seq_len_out, unsigned* err) {
+  CompactArgs a;
+  memset(&a, 0, sizeof(a));
+  const long long hb = (long long)D * esize(dtype), kb = (long long)H_kv * d_h * esize(dtype);
+  int t = 0;
+  a.src[t] = static_cast<const char*>(hidden);
+  a.dst[t] = static_cast<char*>(hidden_out);
+  a.row_bytes[t++] = hb;
+  if (K) {
+    a.src[t] = static_cast<const char*>(K);
+    a.dst[t] = static_cast<char*>(K_out);
+    a.row_bytes[t++] = kb;
+  }
+  if (V) {
+    a.src[t] = static_cast<const char*>(V);
+    a.dst[t] = static_cast<char*>(V_out);
+    a.row_bytes[t++] = kb;
+  }
+  a.n_tensors = t;
+  a.pos = pos;
+  a.pos_out = pos_out;
+  a.P = pos ? P : 0;
+  a.idx = idx;
+  a.keep = keep;
+  a.N_v = N_v;
+  a.vis_start = vis_start;
+  a.seq_len = seq_len;
+  a.seq_len_out = seq_len_out;
+  a.B = B;
+  a.L_max = L_max;
+  a.L_out = L_max - N_v + keep;
+  a.err = err;
+  return a;
+}
+
+// similarity pass: workspace partition
+int rel_splits(int N_v) {
+  int n = (N_v + 255) / 256;
+  return n < 1 ? 1 : (n > 32 ? 32 : n);
+}
+int merge_splits(int B, int N_v, int keep) {
+  const int rows = ((N_v + 127) / 128) * B;
+  const int cols = (keep + 63) / 64;
+  int n = (512 + rows - 1) / rows;
+  if (n > cols) n = cols;
+  if (n > 16) n = 16;
+  return n < 1 ? 1 : n;
+}
+
+struct SimWs {
+  float* G = nullptr;
+  uint8_t* mask = nullptr;
+  float* inv_v = nullptr;
+  float* sum = nullptr;
+  float* mu = nullptr;
+  float* invt = nullptr;
+  float* p = nullptr;
+  float* best = nullptr;
+  int* bidx = nullptr;
+  int* assign = nullptr;
+};
+
+int sim_validate_common(const void* emb, int B, int N, int D, int dtype, const char* what) {
+  if (!emb) return fail(PROVIP_ERR_INVALID_ARG, "%s: null embeddings", what);
+  if (B < 1 || N < 1 || D < 1) return fail(PROVIP_ERR_INVALID_ARG, "%s: non-positive size", what);
+  if (!dtype_ok(dtype)) return fail(PROVIP_ERR_UNSUPPORTED, "%s: dtype %d", what, dtype);
+  if (D % 8) return fail(PROVIP_ERR_UNSUPPORTED, "%s: D must be a multiple of 8", what);
+  if (!aligned16(emb)) return fail(PROVIP_ERR_UNSUPPORTED, "%s: embeddings not 16-byte aligned", what);
+  return PROVIP_OK;
+}
+
+int check_ws(size_t need, void* ws, size_t ws_bytes, const char* what) {
+  if (need == 0) return PROVIP_OK;
+  if (!ws || ws_bytes < need)
+    return fail(PROVIP_ERR_WORKSPACE, "%s: workspace %zu < %zu bytes", what, ws ? ws_bytes : (size_t)0, need);
+  if (reinterpret_cast<uintptr_t>(ws) % kAlign)
+    return fail(PROVIP_ERR_INVALID_ARG, "%s: workspace not 256-byte aligned", what);
+  return PROVIP_OK;
+}
+
+SimArgs sim_args(const void* emb_v, const void* emb_t, const int* text_len, int B, int N_v, int D,
+                 int N_t_max, int dtype, unsigned* err) {
+  SimArgs a;
+  a.emb_v = emb_v;
+  a.emb_t = emb_t;
+  a.text_len = text_len;
+  a.B = B;
+  a.N_v = N_v;
+  a.D = D;
+  a.N_t_max = N_t_max;
+  a.dtype = dtype;
+  a.err = err;
+  return a;
+}
+
+}  // namespace
+
+// ===========================================================================
+// status
+// ===========================================================================
+extern "C" const char* provip_status_string(int status) {
+  switch (status) {
+    case PROVIP_OK: return "PROVIP_OK";
+    case PROVIP_ERR_INVALID_ARG: return "PROVIP_ERR_INVALID_ARG";
+    case PROVIP_ERR_UNSUPPORTED: return "PROVIP_ERR_UNSUPPORTED";
+    case PROVIP_ERR_WORKSPACE: return "PROVIP_ERR_WORKSPACE";
+    case PROVIP_ERR_CUDA: return "PROVIP_ERR_CUDA";
+    case PROVIP_ERR_TIMEOUT: return "PROVIP_ERR_TIMEOUT";
+    default: return "PROVIP_ERR_UNKNOWN";
+  }
+}
+
+extern "C" const char* provip_last_error(void) { return g_last_error; }
+
+extern "C" int provip_version(void) { return 10000; }
+
+extern "C" int provip_device_status(unsigned* bits, int clear) {
+  DevInfo* d;
+  int rc = dev_info(&d);
+  if (rc) return rc;
+  cudaError_t e = cudaDeviceSynchronize();
+  if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceSynchronize");
+  unsigned v = 0;
+  e = cudaMemcpy(&v, d->status, sizeof(v), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_fail(e, "read device status");
+  if (clear) {
+    e = cudaMemset(d->status, 0, sizeof(unsigned));
+    if (e != cudaSuccess) return cuda_fail(e, "clear device status");
+  }
+  if (bits) *bits = v;
+  if (v & PROVIP_DEVSTAT_TIMEOUT) return PROVIP_ERR_TIMEOUT;
+  if (v & PROVIP_DEVSTAT_BAD_ARG) return PROVIP_ERR_INVALID_ARG;
+  return PROVIP_OK;
+}
+
+// ===========================================================================
+// pre-LLM pass
+// ===========================================================================
+extern "C" size_t provip_crit_text_workspace_size(int B, int N_t_max, int D) {
+  (void)D;
+  Carve c(nullptr);
+  c.take<float>((size_t)B * N_t_max * N_t_max);
+  return c.off;
+}
+
+extern "C" int provip_crit_text(const void* emb_t, int B, int N_t_max, int D, const int* text_len,
+                                int dtype, uint8_t* mask_out, float* r_out, void* ws,
+                                size_t ws_bytes, void* stream) {
+  int rc = sim_validate_common(emb_t, B, N_t_max, D, dtype, "crit_text");
+  if (rc) return rc;
+  if (!text_len || !mask_out) return fail(PROVIP_ERR_INVALID_ARG, "crit_text: null text_len/mask_out");
+  if (N_t_max > 4096) return fail(PROVIP_ERR_UNSUPPORTED, "crit_text: N_t_max > 4096");
+  if ((rc = check_ws(provip_crit_text_workspace_size(B, N_t_max, D), ws, ws_bytes, "crit_text"))) return rc;
+  DevInfo* d;
+  if ((rc = dev_info(&d))) return rc;
+  Carve c(ws);
+  float* G = c.take<float>((size_t)B * N_t_max * N_t_max);
+  SimArgs a = sim_args(nullptr, emb_t, text_len, B, 1, D, N_t_max, dtype, d->status);
+  cudaError_t e = crit_text_launch(a, mask_out, r_out, G, static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? PROVIP_OK : cuda_fail(e, "crit_text launch");
+}
+
+static size_t relevance_ws(Carve& c, int B, int N_v, int D, int N_t_max, SimWs& w) {
+  const int ns = rel_splits(N_v);
+  w.inv_v = c.take<float>((size_t)B * N_v);
+  w.sum = c.take<float>((size_t)(ns + 1) * B * D);
+  w.mu = c.take<float>((size_t)B * N_t_max);
+  w.invt = c.take<float>((size_t)B * N_t_max);
+  return c.off;
+}
+
+extern "C" size_t provip_relevance_workspace_size(int B, int N_v, int D, int N_t_max) {
+  Carve c(nullptr);
+  SimWs w;
+  return relevance_ws(c, B, N_v, D, N_t_max, w);
+}
+
+extern "C" int provip_relevance(const void* emb_v, int B, int N_v, int D, const void* emb_t,
+                                const int* text_len, int N_t_max, const uint8_t* crit_mask,
+                                int dtype, float* p_out, void* ws, size_t ws_bytes, void* stream) {
+  int rc = sim_validate_common(emb_v, B, N_v, D, dtype, "relevance");
+  if (rc) return rc;
+  if ((rc = sim_validate_common(emb_t, B, N_t_max, D, dtype, "relevance"))) return rc;
+  if (!text_len || !crit_mask || !p_out) return fail(PROVIP_ERR_INVALID_ARG, "relevance: null pointer");
+  if ((rc = check_ws(provip_relevance_workspace_size(B, N_v, D, N_t_max), ws, ws_bytes, "relevance"))) return rc;
+  DevInfo* d;
+  if ((rc = dev_info(&d))) return rc;
+  Carve c(ws);
+  SimWs w;
+  relevance_ws(c, B, N_v, D, N_t_max, w);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  SimArgs a = sim_args(emb_v, emb_t, text_len, B, N_v, D, N_t_max, dtype, d->status);
+  cudaError_t e = vis_inv_norm_launch(a, w.inv_v, s);
+  if (e == cudaSuccess) e = relevance_launch(a, crit_mask, w.inv_v, p_out, w.sum, w.mu, w.invt, rel_splits(N_v), s);
+  return e == cudaSuccess ? PROVIP_OK : cuda_fail(e, "relevance launch");
+}
+
+extern "C" int provip_topk(const float* scores, int B, int N, int k, int* idx_out, void* stream) {
+  if (!scores || !idx_out) return fail(PROVIP_ERR_INVALID_ARG, "topk: null pointer");
+  if (B < 1 || N < 1 || k < 1 || k > N) return fail(PROVIP_ERR_INVALID_ARG, "topk: need 1 <= k <= N");
+  if (N > kTopkMaxN) return fail(PROVIP_ERR_UNSUPPORTED, "topk: N > %d", kTopkMaxN);
+  DevInfo* d;
+  int rc = dev_info(&d);
+  if (rc) return rc;
+  TopkArgs a;
+  memset(&a, 0, sizeof(a));
+  a.scores = scores;
+  a.B = B;
+  a.N = N;
+  a.k = k;
+  a.idx_out = idx_out;
+  a.err = d->status;
+  cudaError_t e = topk_launch(a, static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? PROVIP_OK : cuda_fail(e, "topk launch");
+}
+
+static size_t merge_ws(Carve& c, int B, int N_v, int keep, SimWs& w) {
+  const int ns = merge_splits(B, N_v, keep);
+  w.inv_v = c.take<float>((size_t)B * N_v);
+  w.best = c.take<float>((size_t)ns * B * N_v);
+  w.bidx = c.take<int>((size_t)ns * B * N_v);
+  return c.off;
+}
+
+extern "C" size_t provip_merge_workspace_size(int B, int N_v, int D, int keep) {
+  (void)D;
+  Carve c(nullptr);
+  SimWs w;
+  return merge_ws(c, B, N_v, keep, w);
+}
+
+static int merge_validate(const void* emb_v, int B, int N_v, int D, const int* keep_idx, int keep,
+                          int dtype, int* assign_out) {
+  int rc = sim_validate_common(emb_v, B, N_v, D, dtype, "merge");
+  if (rc) return rc;
+  if (!keep_idx || !assign_out) return fail(PROVIP_ERR_INVALID_ARG, "merge: null keep_idx/assign_out");
+  if (keep < 1 || keep > N_v) return fail(PROVIP_ERR_INVALID_ARG, "merge: keep %d not in [1, N_v]", keep);
+  if (D > 8192) return fail(PROVIP_ERR_UNSUPPORTED, "merge: D > 8192");
+  return PROVIP_OK;
+}
+
+extern "C" int provip_merge(const void* emb_v, int B, int N_v, int D, const int* keep_idx, int keep,
+                            int dtype, int* assign_out, void* merged_out, void* ws, size_t ws_bytes,
+                            void* stream) {
+  int rc = merge_validate(emb_v, B, N_v, D, keep_idx, keep, dtype, assign_out);
+  if (rc) return rc;
+  if ((rc = check_ws(provip_merge_workspace_size(B, N_v, D, keep), ws, ws_bytes, "merge"))) return rc;
+  DevInfo* d;
+  if ((rc = dev_info(&d))) return rc;
+  Carve c(ws);
+  SimWs w;
+  merge_ws(c, B, N_v, keep, w);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  SimArgs a = sim_args(emb_v, nullptr, nullptr, B, N_v, D, 1, dtype, d->status);
+  cudaError_t e = vis_inv_norm_launch(a, w.inv_v, s);
+  if (e == cudaSuccess)
+    e = merge_launch(a, keep_idx, keep, w.inv_v, assign_out, merged_out, w.best, w.bidx,
+                     merge_splits(B, N_v, keep), s);
+  return e == cudaSuccess ? PROVIP_OK : cuda_fail(e, "merge launch");
+}
+
+static size_t simred_ws(Carve& c, int B, int N_v, int D, int N_t_max, int keep_pre, SimWs& w) {
+  w.G = c.take<float>((size_t)B * N_t_max * N_t_max);
+  w.mask = c.take<uint8_t>((size_t)B * N_t_max);
+  w.p = c.take<float>((size_t)B * N_v);
+  w.assign = c.take<int>((size_t)B * N_v);
+  SimWs r, m;
+  relevance_ws(c, B, N_v, D, N_t_max, r);
+  const int ns = merge_splits(B, N_v, keep_pre);
+  w.inv_v = r.inv_v;
+  w.sum = r.sum;
+  w.mu = r.mu;
+  w.invt = r.invt;
+  w.best = c.take<float>((size_t)ns * B * N_v);
+  w.bidx = c.take<int>((size_t)ns * B * N_v);
+  (void)m;
+  return c.off;
+}
+
+extern "C" size_t provip_similarity_reduce_workspace_size(int B, int N_v, int D, int N_t_max,
+                                                          int keep_pre) {
+  Carve c(nullptr);
+  SimWs w;
+  return simred_ws(c, B, N_v, D, N_t_max, keep_pre, w);
+}
+
+extern "C" int provip_similarity_reduce(const void* emb_v, int B, int N_v, int D, const void* emb_t,
+                                        const int* text_len, int N_t_max,
+                                        const uint8_t* crit_mask_or_null, int keep_pre, int dtype,
+                                        int* idx_out, void* merged_out_or_null,
+                                        float* p_out_or_null, uint8_t* mask_out_or_null, void* ws,
+                                        size_t ws_bytes, void* stream) {
+  int rc = sim_validate_common(emb_v, B, N_v, D, dtype, "similarity_reduce");
+  if (rc) return rc;
+  if ((rc = sim_validate_common(emb_t, B, N_t_max, D, dtype, "similarity_reduce"))) return rc;
+  if (!text_len || !idx_out) return fail(PROVIP_ERR_INVALID_ARG, "similarity_reduce: null text_len/idx_out");
+  if (keep_pre < 1 || keep_pre > N_v) return fail(PROVIP_ERR_INVALID_ARG, "similarity_reduce: keep_pre %d", keep_pre);
+  if (N_v > kTopkMaxN) return fail(PROVIP_ERR_UNSUPPORTED, "similarity_reduce: N_v > %d", kTopkMaxN);
+  if (N_t_max > 4096) return fail(PROVIP_ERR_UNSUPPORTED, "similarity_reduce: N_t_max > 4096");
+  if (merged_out_or_null && D > 8192) return fail(PROVIP_ERR_UNSUPPORTED, "similarity_reduce: D > 8192");
+  if ((rc = check_ws(provip_similarity_reduce_workspace_size(B, N_v, D, N_t_max, keep_pre), ws,
+                     ws_bytes, "similarity_reduce")))
+    return rc;
+  DevInfo* d;
+  if ((rc = dev_info(&d))) return rc;
+  Carve c(ws);
+  SimWs w;
+  simred_ws(c, B, N_v, D, N_t_max, keep_pre, w);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  SimArgs a = sim_args(emb_v, emb_t, text_len, B, N_v, D, N_t_max, dtype, d->status);
+  const uint8_t* mask = crit_mask_or_null;
+  uint8_t* mask_dst = mask_out_or_null ? mask_out_or_null : w.mask;
+  cudaError_t e = cudaSuccess;
+  if (!mask) {
+    e = crit_text_launch(a, mask_dst, nullptr, w.G, s);
+    mask = mask_dst;
+  } else if (mask_out_or_null) {
+    e = cudaMemcpyAsync(mask_out_or_null, mask, (size_t)B * N_t_max, cudaMemcpyDeviceToDevice, s);
+  }
+  float* p = p_out_or_null ? p_out_or_null : w.p;
+  if (e == cudaSuccess) e = vis_inv_norm_launch(a, w.inv_v, s);
+  if (e == cudaSuccess) e = relevance_launch(a, mask, w.inv_v, p, w.sum, w.mu, w.invt, rel_splits(N_v), s);
+  if (e == cudaSuccess) {
+    TopkArgs t;
+    memset(&t, 0, sizeof(t));
+    t.scores = p;
+    t.B = B;
+    t.N = N_v;
+    t.k = keep_pre;
+    t.idx_out = idx_out;
+    t.err = d->status;
+    e = topk_launch(t, s);
+  }
+  if (e == cudaSuccess && merged_out_or_null)
+    e = merge_launch(a, idx_out, keep_pre, w.inv_v, w.assign, merged_out_or_null, w.best, w.bidx,
+                     merge_splits(B, N_v, keep_pre), s);
+  return e == cudaSuccess ? PROVIP_OK : cuda_fail(e, "similarity_reduce launch");
+}
+
+// ===========================================================================
+// in-LLM pass
+// ===========================================================================
+extern "C" size_t provip_head_scores_workspace_size(int B, int L_max, int H_sel, int N_t_max,
+                                                    int N_v, int algo, int dtype) {
+  algo = resolve_algo(algo, dtype);
+  HSShape sh = hs_shape(L_max, N_t_max, N_v, algo);
+  Carve c(nullptr);
+  float2* st;
+  float* pa;
+  return hs_ws(c, B, H_sel, sh, N_v, &st, &pa);
+}
+
+extern "C" int provip_head_scores(const void* Q, const void* K, int B, int L_max, int H_q, int H_kv,
+                                  int d_h, const int* head_list, int H_sel, const int* text_start,
+                                  const int* text_len, const uint8_t* row_mask_or_null, int N_t_max,
+                                  int vis_start, int N_v, const int* seq_len, int dtype, int algo,
+                                  float* scores, void* ws, size_t ws_bytes, void* stream) {
+  algo = resolve_algo(algo, dtype);
+  int rc = hs_validate(Q, K, B, L_max, H_q, H_kv, d_h, head_list, H_sel, text_start, text_len,
+                       N_t_max, vis_start, N_v, seq_len, dtype, algo);
+  if (rc) return rc;
+  if (!scores) return fail(PROVIP_ERR_INVALID_ARG, "head_scores: null scores");
+  if ((rc = check_ws(provip_head_scores_workspace_size(B, L_max, H_sel, N_t_max, N_v, algo, dtype),
+                     ws, ws_bytes, "head_scores")))
+    return rc;
+  DevInfo* d;
+  if ((rc = dev_info(&d))) return rc;
+  HSShape sh = hs_shape(L_max, N_t_max, N_v, algo);
+  Carve c(ws);
+  float2* stats;
+  float* partial;
+  hs_ws(c, B, H_sel, sh, N_v, &stats, &partial);
+  HSArgs a = hs_args(Q, K, B, L_max, H_q, H_kv, d_h, head_list, H_sel, text_start, text_len,
+                     row_mask_or_null, N_t_max, vis_start, N_v, seq_len, sh, stats, partial,
+                     d->status);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if ((rc = hs_run(a, dtype, algo, s))) return rc;
+  cudaError_t e = hs_launch_reduce(a, scores, s);
+  return e == cudaSuccess ? PROVIP_OK : cuda_fail(e, "head_scores reduce");
+}
+
+extern "C" int provip_compact(const int* idx, int B, int N_v, int keep, const void* hidden, int D,
+                              const void* K, const void* V, int H_kv, int d_h, const int* pos,
+                              int P, const int* seq_len, int L_max, int vis_start, int dtype,
+                              void* hidden_out, void* K_out, void* V_out, int* pos_out,
+                              int* seq_len_out, void* stream) {
+  int rc = compact_validate(idx, B, N_v, keep, hidden, D, K, V, H_kv, d_h, pos, P, seq_len, L_max,
+                            vis_start, dtype, hidden_out, K_out, V_out, pos_out);
+  if (rc) return rc;
+  DevInfo* d;
+  if ((rc = dev_info(&d))) return rc;
+  CompactArgs a = compact_args(idx, B, N_v, keep, hidden, D, K, V, H_kv, d_h, pos, P, seq_len,
+                               L_max, vis_start, dtype, hidden_out, K_out, V_out, pos_out,
+                               seq_len_out, d->status);
+  cudaError_t e = compact_launch(a, d->sms, static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? PROVIP_OK : cuda_fail(e, "compact launch");
+}
+
+extern "C" int provip_topk_compact(const float* scores, int B, int N_v, int keep, const void* hidden,
+                                   int D, const void* K, const void* V, int H_kv, int d_h,
+                                   const int* pos, int P, const int* seq_len, int L_max,
+                                   int vis_start, int dtype, void* hidden_out, void* K_out,
+                                   void* V_out, int* pos_out, int* idx_out, int* seq_len_out,
+                                   void* stream) {
+  if (!scores || !idx_out) return fail(PROVIP_ERR_INVALID_ARG, "topk_compact: null scores/idx_out");
+  int rc = compact_validate(idx_out, B, N_v, keep, hidden, D, K, V, H_kv, d_h, pos, P, seq_len,
+                            L_max, vis_start, dtype, hidden_out, K_out, V_out, pos_out);
+  if (rc) return rc;
+  if ((rc = provip_topk(scores, B, N_v, keep, idx_out, stream))) return rc;
+  return provip_compact(idx_out, B, N_v, keep, hidden, D, K, V, H_kv, d_h, pos, P, seq_len, L_max,
+                        vis_start, dtype, hidden_out, K_out, V_out, pos_out, seq_len_out, stream);
+}
+
+extern "C" size_t provip_prune_workspace_size(int B, int L_max, int H_sel, int N_t_max, int N_v,
+                                              int algo, int dtype) {
+  return provip_head_scores_workspace_size(B, L_max, H_sel, N_t_max, N_v, algo, dtype);
+}
+
+extern "C" int provip_head_topk(const void* Q, const void* K, int B, int L_max, int H_q, int H_kv,
+                                int d_h, const int* head_list, int H_sel, const int* text_start,
+                                const int* text_len, const uint8_t* row_mask_or_null, int N_t_max,
+                                int vis_start, int N_v, const int* seq_len, int keep, int dtype,
+                                int algo, int* idx_out, float* scores_out_or_null, void* ws,
+                                size_t ws_bytes, void* stream) {
+  algo = resolve_algo(algo, dtype);
+  int rc = hs_validate(Q, K, B, L_max, H_q, H_kv, d_h, head_list, H_sel, text_start, text_len,
+                       N_t_max, vis_start, N_v, seq_len, dtype, algo);
+  if (rc) return rc;
+  if (!idx_out) return fail(PROVIP_ERR_INVALID_ARG, "head_topk: null idx_out");
+  if (keep < 1 || keep > N_v) return fail(PROVIP_ERR_INVALID_ARG, "head_topk: keep %d not in [1, N_v]", keep);
+  if (N_v > kTopkMaxN) return fail(PROVIP_ERR_UNSUPPORTED, "head_topk: N_v > %d", kTopkMaxN);
+  if ((rc = check_ws(provip_head_scores_workspace_size(B, L_max, H_sel, N_t_max, N_v, algo, dtype), ws,
+                     ws_bytes, "head_topk")))
+    return rc;
+  DevInfo* d;
+  if ((rc = dev_info(&d))) return rc;
+  HSShape sh = hs_shape(L_max, N_t_max, N_v, algo);
+  Carve c(ws);
+  float2* stats;
+  float* partial;
+  hs_ws(c, B, H_sel, sh, N_v, &stats, &partial);
+  HSArgs a = hs_args(Q, K, B, L_max, H_q, H_kv, d_h, head_list, H_sel, text_start, text_len,
+                     row_mask_or_null, N_t_max, vis_start, N_v, seq_len, sh, stats, partial,
+                     d->status);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if ((rc = hs_run(a, dtype, algo, s))) return rc;
+  TopkArgs t;
+  memset(&t, 0, sizeof(t));
+  t.partial = partial;
+  t.n_part = sh.n_rb * H_sel;
+  t.text_len = text_len;
+  t.row_mask = row_mask_or_null;
+  t.N_t_max = N_t_max;
+  t.H_sel = H_sel;
+  t.scores_out = scores_out_or_null;
+  t.B = B;
+  t.N = N_v;
+  t.k = keep;
+  t.idx_out = idx_out;
+  t.err = d->status;
+  cudaError_t e = topk_launch(t, s);
+  return e == cudaSuccess ? PROVIP_OK : cuda_fail(e, "head_topk topk");
+}
+
+extern "C" int provip_prune(const void* Q, const void* K, const void* V, const void* hidden, int B,
+                            int L_max, int H_q, int H_kv, int d_h, int D, const int* head_list,
+                            int H_sel, const int* text_start, const int* text_len,
+                            const uint8_t* row_mask_or_null, int N_t_max, int vis_start, int N_v,
+                            const int* seq_len, const int* pos, int P, int keep, int dtype,
+                            int algo, void* hidden_out, void* K_out, void* V_out, int* pos_out,
+                            int* idx_out, int* seq_len_out, float* scores_out_or_null, void* ws,
+                            size_t ws_bytes, void* stream) {
+  // validate both halves before enqueueing anything
+  int rc = hs_validate(Q, K, B, L_max, H_q, H_kv, d_h, head_list, H_sel, text_start, text_len,
+                       N_t_max, vis_start, N_v, seq_len, dtype, resolve_algo(algo, dtype));
+  if (rc) return rc;
+  if ((rc = compact_validate(idx_out ? idx_out : reinterpret_cast<int*>(16), B, N_v, keep, hidden, D,
+                             K, V, H_kv, d_h, pos, P, seq_len, L_max, vis_start, dtype, hidden_out,
+                             K_out, V_out, pos_out)))
+    return rc;
+  rc = provip_head_topk(Q, K, B, L_max, H_q, H_kv, d_h, head_list, H_sel, text_start, text_len,
+                        row_mask_or_null, N_t_max, vis_start, N_v, seq_len, keep, dtype, algo,
+                        idx_out, scores_out_or_null, ws, ws_bytes, stream);
+  if (rc) return rc;
+  return provip_compact(idx_out, B, N_v, keep, hidden, D, K, V, H_kv, d_h, pos, P, seq_len, L_max,
+                        vis_start, dtype, hidden_out, K_out, V_out, pos_out, seq_len_out, stream);
+}

@@ -1,0 +1,179 @@
+// Survivor compaction (Sec. 4.1: pruned tokens are excluded from every later
+// computation): out-of-place gather of the rows
+//   [0, vis_start) ++ (vis_start + idx[b][0..keep)) ++ [vis_start + N_v, seq_len[b])
+// of hidden states, K and V (any row size that is a multiple of 16 bytes),
+// plus the position-id rows (int32, P of them; carried, not renumbered).
+//
+// Bulk-TMA pipeline: the work is the list of (output row, tensor, <= 8 KiB
+// piece) items; every CTA owns a contiguous range of it. One thread per CTA
+// streams its range through a ring of shared-memory slots: a cp.async.bulk load
+// (global -> shared, completion on the slot's mbarrier) and, once it lands, a
+// cp.async.bulk store (shared -> global, bulk group). A slot is refilled as soon
+// as the store that drained it has finished reading, so up to kSlots - 1 loads
+// and a store are in flight per CTA. The other warps copy the position ids.
+// Every wait is bounded; a timeout sets the device error word and the CTA
+// drains what it issued before returning.
+#include "common.cuh"
+#include "kernels.h"
+
+namespace provip {
+namespace {
+
+constexpr int kSlotBytes = 8192;
+constexpr int kSlots = 12;
+constexpr int kCompactThreads = 128;
+constexpr size_t kCompactSmem = (size_t)kSlots * kSlotBytes;
+
+__device__ __forceinline__ int src_row(const CompactArgs& a, int b, int r, bool& ok) {
+  if (r < a.vis_start) return r;
+  if (r < a.vis_start + a.keep) {
+    const int v = a.idx[(size_t)b * a.keep + (r - a.vis_start)];
+    if (v < 0 || v >= a.N_v) {
+      ok = false;
+      return 0;
+    }
+    return a.vis_start + v;
+  }
+  return r - a.keep + a.N_v;
+}
+
+struct Item {
+  const char* src;
+  char* dst;
+  uint32_t bytes;
+};
+
+__global__ void __launch_bounds__(kCompactThreads) compact_kernel(const CompactArgs a, int np0,
+                                                                   int np1, int np2) {
+  extern __shared__ __align__(128) uint8_t slots[];
+  __shared__ __align__(8) uint64_t bars[kSlots];
+  __shared__ char* ring_dst[kSlots];
+  __shared__ uint32_t ring_bytes[kSlots];
+  const int NP = np0 + np1 + np2;
+  const long long total = (long long)a.B * a.L_out * NP;
+  const long long per = (total + gridDim.x - 1) / gridDim.x;
+  const long long it_begin = min(total, (long long)blockIdx.x * per);
+  const long long it_end = min(total, it_begin + per);
+
+  if (blockIdx.x == 0 && a.seq_len_out != nullptr)
+    for (int b = threadIdx.x; b < a.B; b += blockDim.x)
+      a.seq_len_out[b] = a.seq_len[b] - a.N_v + a.keep;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kSlots; ++s) mbar_init(&bars[s], 1);
+    fence_mbar_init();
+  }
+  __syncthreads();
+
+  if (threadIdx.x == 0) {
+    const uint64_t pol = policy_evict_first();
+    long long next = it_begin;
+    // next valid item at or after `next`; false when the range is exhausted
+    auto fetch = [&](Item& it) -> bool {
+      while (next < it_end) {
+        const long long i = next++;
+        const long long row = i / NP;
+        int q = (int)(i - row * NP);
+        const int b = (int)(row / a.L_out), r = (int)(row - (long long)b * a.L_out);
+        const int sl = a.seq_len[b];
+        if (sl > a.L_max || sl < a.vis_start + a.N_v) {
+          set_error(a.err, kErrBadDeviceArg);
+          continue;
+        }
+        if (r >= sl - a.N_v + a.keep) continue;
+        int t = 0;
+        if (q >= np0) {
+          q -= np0;
+          t = 1;
+          if (q >= np1) {
+            q -= np1;
+            t = 2;
+          }
+        }
+        bool ok = true;
+        const int sr = src_row(a, b, r, ok);
+        if (!ok) {
+          set_error(a.err, kErrBadDeviceArg);
+          continue;
+        }
+        const long long rb = a.row_bytes[t];
+        const long long off = (long long)q * kSlotBytes;
+        it.bytes = (uint32_t)min((long long)kSlotBytes, rb - off);
+        it.src = a.src[t] + ((long long)b * a.L_max + sr) * rb + off;
+        it.dst = a.dst[t] + ((long long)b * a.L_out + r) * rb + off;
+        return true;
+      }
+      return false;
+    };
+    auto issue = [&](int slot, const Item& it) {
+      ring_dst[slot] = it.dst;
+      ring_bytes[slot] = it.bytes;
+      mbar_arrive_expect_tx(&bars[slot], it.bytes);
+      bulk_g2s(slots + (size_t)slot * kSlotBytes, it.src, it.bytes, &bars[slot], pol);
+    };
+    int loaded = 0;
+    Item it;
+    while (loaded < kSlots && fetch(it)) issue(loaded++, it);
+    bool failed = false;
+    int i = 0;
+    for (; i < loaded; ++i) {
+      const int s = i % kSlots;
+      if (!mbar_wait(&bars[s], (uint32_t)(i / kSlots) & 1u, a.err)) {
+        failed = true;
+        break;
+      }
+      bulk_s2g(ring_dst[s], slots + (size_t)s * kSlotBytes, ring_bytes[s]);
+      bulk_commit();
+      if (i >= 1) {
+        bulk_wait_read<1>();  // the store of item i - 1 has read its slot
+        if (fetch(it)) {
+          issue(loaded % kSlots, it);
+          ++loaded;
+        }
+      }
+    }
+    if (failed) {
+      // drain the loads still in flight (bounded) before the CTA exits
+      for (int j = i; j < loaded; ++j) mbar_wait(&bars[j % kSlots], (uint32_t)(j / kSlots) & 1u, a.err);
+    }
+    bulk_wait<0>();
+  } else if (a.pos != nullptr && threadIdx.x >= 32) {
+    // position ids of the rows whose first item lies in this CTA's range
+    const long long r0 = (it_begin + NP - 1) / NP, r1 = (it_end + NP - 1) / NP;
+    const int nth = blockDim.x - 32;
+    for (long long row = r0 + (threadIdx.x - 32); row < r1; row += nth) {
+      const int b = (int)(row / a.L_out), r = (int)(row - (long long)b * a.L_out);
+      const int sl = a.seq_len[b];
+      if (sl > a.L_max || sl < a.vis_start + a.N_v || r >= sl - a.N_v + a.keep) continue;
+      bool ok = true;
+      const int sr = src_row(a, b, r, ok);
+      if (!ok) continue;
+      for (int p = 0; p < a.P; ++p)
+        a.pos_out[((size_t)p * a.B + b) * a.L_out + r] = a.pos[((size_t)p * a.B + b) * a.L_max + sr];
+    }
+  }
+}
+
+}  // namespace
+
+cudaError_t compact_launch(const CompactArgs& a, int num_sms, cudaStream_t s) {
+  static bool configured[64] = {false};
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev >= 0 && dev < 64 && !configured[dev]) {
+    cudaError_t e = cudaFuncSetAttribute(compact_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)kCompactSmem);
+    if (e != cudaSuccess) return e;
+    configured[dev] = true;
+  }
+  int np[3] = {0, 0, 0};
+  for (int t = 0; t < a.n_tensors; ++t)
+    np[t] = (int)((a.row_bytes[t] + kSlotBytes - 1) / kSlotBytes);
+  const long long total = (long long)a.B * a.L_out * (np[0] + np[1] + np[2]);
+  long long grid = 2LL * num_sms;
+  if (grid > total) grid = total > 0 ? total : 1;
+  compact_kernel<<<(unsigned)grid, kCompactThreads, kCompactSmem, s>>>(a, np[0], np[1], np[2]);
+  return cudaGetLastError();
+}
+
+}  // namespace provip

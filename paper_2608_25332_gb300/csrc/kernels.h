@@ -1,0 +1,124 @@
+// Internal launch interface between the C-ABI layer (api.cu) and the kernel
+// translation units. Not installed; the public interface is include/provip.h.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+namespace provip {
+
+constexpr int kMaxHeads = 64;
+constexpr int kHeadDim = 128;  // d_h supported by the kernels
+constexpr int kRowBlock = 128; // text rows per CTA row block
+
+// ---------------------------------------------------------------------------
+// head-aware scores (Sec. 4.4): two passes over the keys
+//   pass 1 (stats): per text row and key chunk, the chunk max m_c and
+//                   sum l_c of exp2(s - m_c) over the causal keys in the chunk;
+//   pass 2 (probs): per visual key chunk, p = exp2(s - m) / l with the row's
+//                   global (m, l), summed over the rows of the block ->
+//                   partial[b][rb * H_sel + head][col].
+// Scores are in the base-2 domain: s = <q, k> * log2(e) / sqrt(d_h).
+// ---------------------------------------------------------------------------
+struct HSArgs {
+  const void* Q;  // [B, L_max, H_q, d_h]
+  const void* K;  // [B, L_max, H_kv, d_h]
+  int B, L_max, H_q, H_kv, d_h;
+  int H_sel;
+  int heads[kMaxHeads];
+  const int* text_start;     // [B]
+  const int* text_len;       // [B]
+  const uint8_t* row_mask;   // [B, N_t_max] or null
+  int N_t_max;
+  int vis_start, N_v;
+  const int* seq_len;        // [B]
+  int n_rb;                  // row blocks: ceil(N_t_max / 128)
+  int kc;                    // key chunk width of pass 1
+  int n_kc;                  // ceil(L_max / kc)
+  int vc;                    // visual chunk width of pass 2
+  int n_vc;                  // ceil(N_v / vc)
+  float scale_log2;          // log2(e) / sqrt(d_h)
+  float2* stats;             // [B][n_rb][H_sel][n_kc][128]
+  float* partial;            // [B][n_rb * H_sel][N_v]
+  unsigned* err;
+};
+
+cudaError_t hs_launch_simt(const HSArgs& a, int dtype, cudaStream_t s);
+// tcgen05 path (bf16): needs tensor maps over Q and K viewed as 2-D row tables.
+cudaError_t hs_launch_tc(const HSArgs& a, const CUtensorMap* tmQ, const CUtensorMap* tmK,
+                         cudaStream_t s);
+// scores[b][i] = sum_u partial[b][u][i] / (H_sel * valid text rows of b)
+cudaError_t hs_launch_reduce(const HSArgs& a, float* scores, cudaStream_t s);
+
+// ---------------------------------------------------------------------------
+// top-k (ties to the lower index, ascending output)
+// ---------------------------------------------------------------------------
+struct TopkArgs {
+  const float* scores;       // [B][N]; or null when reading head partials
+  const float* partial;      // [B][n_part][N]
+  int n_part;
+  const int* text_len;       // used with partial: valid-row count per sample
+  const uint8_t* row_mask;
+  int N_t_max;
+  int H_sel;
+  float* scores_out;         // optional [B][N]
+  int B, N, k;
+  int* idx_out;              // [B][k]
+  unsigned* err;
+};
+constexpr int kTopkMaxN = 49152;
+cudaError_t topk_launch(const TopkArgs& a, cudaStream_t s);
+
+// ---------------------------------------------------------------------------
+// compaction: rows [0, vis_start) ++ vis_start + idx ++ [vis_start + N_v, seq_len)
+// ---------------------------------------------------------------------------
+struct CompactArgs {
+  const char* src[3];
+  char* dst[3];
+  long long row_bytes[3];
+  int n_tensors;
+  const int* pos;            // [P, B, L_max] or null
+  int* pos_out;              // [P, B, L_out]
+  int P;
+  const int* idx;            // [B, keep]
+  int keep, N_v, vis_start;
+  const int* seq_len;        // [B]
+  int* seq_len_out;          // [B] or null
+  int B, L_max, L_out;
+  unsigned* err;
+};
+cudaError_t compact_launch(const CompactArgs& a, int num_sms, cudaStream_t s);
+
+// ---------------------------------------------------------------------------
+// pre-LLM similarity pass (Sec. 4.2-4.3)
+// ---------------------------------------------------------------------------
+struct SimArgs {
+  const void* emb_v;         // [B, N_v, D]
+  const void* emb_t;         // [B, N_t_max, D]
+  const int* text_len;       // [B]
+  int B, N_v, D, N_t_max;
+  int dtype;
+  unsigned* err;
+};
+// Sec. 4.2: mask[b][j] (and r) from the text self-similarity. ws: G [B][Ntm][Ntm] f32.
+cudaError_t crit_text_launch(const SimArgs& a, uint8_t* mask, float* r_out, float* G,
+                             cudaStream_t s);
+// inverse L2 norms of every visual row (0 for a zero row): inv_v [B][N_v]
+cudaError_t vis_inv_norm_launch(const SimArgs& a, float* inv_v, cudaStream_t s);
+// Sec. 4.3: p[b][j] = max_{i in T} cos(t_i, v_j) - mu_i. ws: see sim_ws_floats().
+cudaError_t relevance_launch(const SimArgs& a, const uint8_t* mask, const float* inv_v,
+                             float* p, float* ws_sum, float* ws_mu, float* ws_invt,
+                             int n_split, cudaStream_t s);
+// Sec. 4.3 merge: assign[b][j] and merged[b][a][:]
+cudaError_t merge_launch(const SimArgs& a, const int* keep_idx, int keep, const float* inv_v,
+                         int* assign, void* merged, float* ws_best, int* ws_bidx,
+                         int n_split, cudaStream_t s);
+
+// host helper: encode a 2-D bf16 row table [rows, cols] (row stride in bytes)
+// as a tensor map with 64 x box_rows boxes and 128-byte swizzle.
+int make_tmap_bf16_2d(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols,
+                      uint64_t row_stride_bytes, uint32_t box_rows);
+
+}  // namespace provip

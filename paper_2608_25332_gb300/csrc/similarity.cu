@@ -1,0 +1,509 @@
+// Pre-LLM pass (Sec. 4.2-4.3), CUDA-core kernels.
+//
+//   crit_text:  G = E_t E_t^T (no scale), row softmax, r_j = mean_i R_ij,
+//               T = { j : r_j > mean(r) } (all rows when none exceeds it).
+//   relevance:  p_j = max_{i in T} ( cos(t_i, v_j) - mu_i ), where the row mean
+//               mu_i = (1/N_v) sum_k cos(t_i, v_k) = <t_i / |t_i|, sum_k v_k / |v_k|> / N_v
+//               is computed from the sum of the normalised visual rows, so the
+//               |T| x N_v cosine matrix is never stored.
+//   merge:      for each visual row j, the kept row of largest cosine
+//               (= largest <v_j, v_k> / |v_k|, since |v_j| is common), ties to
+//               the lower kept position; merged_a = mean of centroid a and its
+//               members, summed in ascending row order.
+#include "common.cuh"
+#include "kernels.h"
+#include "simt_gemm.cuh"
+
+namespace provip {
+namespace {
+
+template <typename T>
+__device__ __forceinline__ const T* row_ptr(const void* base, size_t row, int D) {
+  return static_cast<const T*>(base) + row * (size_t)D;
+}
+
+// ---------------------------------------------------------------------------
+// Sec. 4.2
+// ---------------------------------------------------------------------------
+template <typename T>
+__global__ void __launch_bounds__(256) crit_gram_kernel(const SimArgs a, float* G) {
+  __shared__ __align__(16) SimtSmem sm;
+  __shared__ const T* arow[kSimtBM];
+  __shared__ const T* brow[kSimtBN];
+  const int b = blockIdx.z;
+  const int r0 = blockIdx.y * kSimtBM, c0 = blockIdx.x * kSimtBN;
+  int tl = a.text_len[b];
+  if (tl < 0 || tl > a.N_t_max) tl = 0;
+  if (threadIdx.x < kSimtBM) {
+    const int j = r0 + threadIdx.x;
+    arow[threadIdx.x] = j < tl ? row_ptr<T>(a.emb_t, (size_t)b * a.N_t_max + j, a.D) : nullptr;
+  }
+  if (threadIdx.x < kSimtBN) {
+    const int j = c0 + threadIdx.x;
+    brow[threadIdx.x] = j < tl ? row_ptr<T>(a.emb_t, (size_t)b * a.N_t_max + j, a.D) : nullptr;
+  }
+  __syncthreads();
+  float acc[8][4];
+  simt_gemm_nt<T>(arow, brow, a.D, sm, acc);
+  const int rg = threadIdx.x >> 4, kg = threadIdx.x & 15;
+#pragma unroll
+  for (int i = 0; i < 8; ++i)
+#pragma unroll
+    for (int jj = 0; jj < 4; ++jj) {
+      const int r = r0 + rg + 16 * i, c = c0 + kg + 16 * jj;
+      if (r < a.N_t_max && c < a.N_t_max) G[((size_t)b * a.N_t_max + r) * a.N_t_max + c] = acc[i][jj];
+    }
+}
+
+// one CTA per sample: row softmax statistics, column means r, threshold
+__global__ void __launch_bounds__(256) crit_finish_kernel(const SimArgs a, const float* G,
+                                                          uint8_t* mask, float* r_out) {
+  extern __shared__ float sh[];  // rowm[Ntm], rowinv[Ntm], r[Ntm]
+  float* rowm = sh;
+  float* rowinv = sh + a.N_t_max;
+  float* rr = sh + 2 * a.N_t_max;
+  __shared__ float wsum[8];
+  __shared__ int wcnt[8];
+  const int b = blockIdx.x;
+  int n = a.text_len[b];
+  if (n < 0 || n > a.N_t_max) {
+    if (threadIdx.x == 0) set_error(a.err, kErrBadDeviceArg);
+    n = 0;
+  }
+  const float* Gb = G + (size_t)b * a.N_t_max * a.N_t_max;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  for (int i = warp; i < n; i += 8) {
+    float m = -INFINITY;
+    for (int j = lane; j < n; j += 32) m = fmaxf(m, Gb[(size_t)i * a.N_t_max + j]);
+    m = warp_max(m);
+    float z = 0.f;
+    for (int j = lane; j < n; j += 32) z += expf(Gb[(size_t)i * a.N_t_max + j] - m);
+    z = warp_sum(z);
+    if (lane == 0) {
+      rowm[i] = m;
+      rowinv[i] = 1.f / z;
+    }
+  }
+  __syncthreads();
+  for (int j = threadIdx.x; j < n; j += blockDim.x) {
+    float s = 0.f;
+    for (int i = 0; i < n; ++i) s += expf(Gb[(size_t)i * a.N_t_max + j] - rowm[i]) * rowinv[i];
+    rr[j] = s / (float)n;
+  }
+  __syncthreads();
+  // mean(r), fixed-order block sum
+  float part = 0.f;
+  for (int j = threadIdx.x; j < n; j += blockDim.x) part += rr[j];
+  part = warp_sum(part);
+  if (lane == 0) wsum[warp] = part;
+  __syncthreads();
+  float tot = 0.f;
+  for (int w = 0; w < 8; ++w) tot += wsum[w];
+  const float mean = n > 0 ? tot / (float)n : 0.f;
+  int c = 0;
+  for (int j = threadIdx.x; j < n; j += blockDim.x) c += rr[j] > mean;
+  for (int o = 16; o > 0; o >>= 1) c += __shfl_xor_sync(0xffffffffu, c, o);
+  if (lane == 0) wcnt[warp] = c;
+  __syncthreads();
+  int cnt = 0;
+  for (int w = 0; w < 8; ++w) cnt += wcnt[w];
+  for (int j = threadIdx.x; j < a.N_t_max; j += blockDim.x) {
+    const bool in = j < n && (cnt == 0 || rr[j] > mean);
+    mask[(size_t)b * a.N_t_max + j] = in ? 1 : 0;
+    if (r_out) r_out[(size_t)b * a.N_t_max + j] = j < n ? rr[j] : 0.f;
+  }
+}
+
+// ---------------------------------------------------------------------------
+// inverse row norms: one warp per row
+// ---------------------------------------------------------------------------
+template <typename T>
+__global__ void __launch_bounds__(256) inv_norm_kernel(const void* X, size_t rows, int D,
+                                                       float* inv) {
+  const size_t row = (size_t)blockIdx.x * 8 + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (row >= rows) return;
+  const T* p = static_cast<const T*>(X) + row * (size_t)D;
+  float s = 0.f;
+  for (int e = lane * 8; e < D; e += 256) {
+    float v[8];
+    load8(p + e, v);
+#pragma unroll
+    for (int q = 0; q < 8; ++q) s = fmaf(v[q], v[q], s);
+  }
+  s = warp_sum(s);
+  if (lane == 0) inv[row] = s > 0.f ? 1.f / sqrtf(s) : 0.f;
+}
+
+// ---------------------------------------------------------------------------
+// Sec. 4.3 relevance
+// ---------------------------------------------------------------------------
+// partial sums of normalised visual rows: part[z][b][d] over rows z*chunk..
+template <typename T>
+__global__ void __launch_bounds__(256) vis_sum_kernel(const SimArgs a, const float* inv_v,
+                                                      float* part, int chunk) {
+  const int d = blockIdx.x * 256 + threadIdx.x;
+  const int b = blockIdx.y, z = blockIdx.z;
+  if (d >= a.D) return;
+  const int j0 = z * chunk, j1 = min(a.N_v, j0 + chunk);
+  const T* E = static_cast<const T*>(a.emb_v) + (size_t)b * a.N_v * a.D;
+  float s = 0.f;
+  for (int j = j0; j < j1; ++j) s = fmaf(to_f32(E[(size_t)j * a.D + d]), inv_v[(size_t)b * a.N_v + j], s);
+  part[((size_t)z * a.B + b) * a.D + d] = s;
+}
+
+// sum[b][d] = sum over the row chunks z of part[z][b][d] (fixed order)
+__global__ void __launch_bounds__(256) vis_sum_reduce_kernel(const SimArgs a, const float* part,
+                                                             int nz, float* sum) {
+  const int d = blockIdx.x * 256 + threadIdx.x;
+  const int b = blockIdx.y;
+  if (d >= a.D) return;
+  float s = 0.f;
+  for (int z = 0; z < nz; ++z) s += part[((size_t)z * a.B + b) * a.D + d];
+  sum[(size_t)b * a.D + d] = s;
+}
+
+// mu_i and 1/|t_i| for the text rows (one warp per row)
+template <typename T>
+__global__ void __launch_bounds__(256) text_mu_kernel(const SimArgs a, const float* sum,
+                                                      float* mu, float* invt) {
+  const int b = blockIdx.y;
+  const int i = blockIdx.x * 8 + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (i >= a.N_t_max) return;
+  const int tl = min(max(a.text_len[b], 0), a.N_t_max);
+  if (i >= tl) {
+    if (lane == 0) {
+      mu[(size_t)b * a.N_t_max + i] = 0.f;
+      invt[(size_t)b * a.N_t_max + i] = 0.f;
+    }
+    return;
+  }
+  const T* t = static_cast<const T*>(a.emb_t) + ((size_t)b * a.N_t_max + i) * a.D;
+  float ss = 0.f, dt = 0.f;
+  for (int d = lane; d < a.D; d += 32) {
+    const float x = to_f32(t[d]);
+    ss = fmaf(x, x, ss);
+    dt = fmaf(x, sum[(size_t)b * a.D + d], dt);
+  }
+  ss = warp_sum(ss);
+  dt = warp_sum(dt);
+  if (lane == 0) {
+    const float iv = ss > 0.f ? 1.f / sqrtf(ss) : 0.f;
+    invt[(size_t)b * a.N_t_max + i] = iv;
+    mu[(size_t)b * a.N_t_max + i] = dt * iv / (float)a.N_v;
+  }
+}
+
+// p_j = max over critical rows of cos - mu; CTA = 64 visual rows x all text rows
+template <typename T>
+__global__ void __launch_bounds__(256) relevance_kernel(const SimArgs a, const uint8_t* mask,
+                                                        const float* inv_v, const float* mu,
+                                                        const float* invt, float* p) {
+  __shared__ __align__(16) SimtSmem sm;
+  __shared__ const T* arow[kSimtBM];
+  __shared__ const T* brow[kSimtBN];
+  __shared__ float red[8][kSimtBN];
+  const int b = blockIdx.y, c0 = blockIdx.x * kSimtBN;
+  const int tl = min(max(a.text_len[b], 0), a.N_t_max);
+  const int rg = threadIdx.x >> 4, kg = threadIdx.x & 15;
+  float best[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+  if (threadIdx.x < kSimtBN) {
+    const int j = c0 + threadIdx.x;
+    brow[threadIdx.x] = j < a.N_v ? row_ptr<T>(a.emb_v, (size_t)b * a.N_v + j, a.D) : nullptr;
+  }
+  for (int r0 = 0; r0 < tl; r0 += kSimtBM) {
+    __syncthreads();
+    if (threadIdx.x < kSimtBM) {
+      const int i = r0 + threadIdx.x;
+      const bool in = i < tl && mask[(size_t)b * a.N_t_max + i] != 0;
+      arow[threadIdx.x] = in ? row_ptr<T>(a.emb_t, (size_t)b * a.N_t_max + i, a.D) : nullptr;
+    }
+    __syncthreads();
+    float acc[8][4];
+    simt_gemm_nt<T>(arow, brow, a.D, sm, acc);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const int r = rg + 16 * i;
+      if (arow[r] == nullptr) continue;
+      const float it = invt[(size_t)b * a.N_t_max + r0 + r], m = mu[(size_t)b * a.N_t_max + r0 + r];
+#pragma unroll
+      for (int jj = 0; jj < 4; ++jj) {
+        const int j = c0 + kg + 16 * jj;
+        if (j < a.N_v) best[jj] = fmaxf(best[jj], acc[i][jj] * it * inv_v[(size_t)b * a.N_v + j] - m);
+      }
+    }
+  }
+  // max across the 16 row groups
+#pragma unroll
+  for (int jj = 0; jj < 4; ++jj) best[jj] = fmaxf(best[jj], __shfl_xor_sync(0xffffffffu, best[jj], 16));
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (lane < 16)
+#pragma unroll
+    for (int jj = 0; jj < 4; ++jj) red[warp][lane + 16 * jj] = best[jj];
+  __syncthreads();
+  if (threadIdx.x < kSimtBN) {
+    const int j = c0 + threadIdx.x;
+    float m = -INFINITY;
+    for (int w = 0; w < 8; ++w) m = fmaxf(m, red[w][threadIdx.x]);
+    if (j < a.N_v) p[(size_t)b * a.N_v + j] = m;
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Sec. 4.3 merge
+// ---------------------------------------------------------------------------
+// kept-position map: pos[b][j] = a if j == keep[b][a], else -1
+__global__ void keep_pos_kernel(const int* keep_idx, int keep, int B, int N_v, int* kpos,
+                                unsigned* err) {
+  const size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < (size_t)B * N_v) kpos[i] = -1;
+}
+__global__ void keep_scatter_kernel(const int* keep_idx, int keep, int B, int N_v, int* kpos,
+                                    unsigned* err) {
+  const size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= (size_t)B * keep) return;
+  const int b = (int)(i / keep), a = (int)(i - (size_t)b * keep);
+  const int j = keep_idx[i];
+  if (j < 0 || j >= N_v || (a > 0 && keep_idx[i - 1] >= j)) {
+    set_error(err, kErrBadDeviceArg);
+    return;
+  }
+  kpos[(size_t)b * N_v + j] = a;
+}
+
+__device__ __forceinline__ bool better(float v, int i, float bv, int bi) {
+  return v > bv || (v == bv && i < bi);
+}
+
+// argmax over one split of the kept columns for a tile of 128 visual rows
+template <typename T>
+__global__ void __launch_bounds__(256) merge_argmax_kernel(const SimArgs a, const int* keep_idx,
+                                                           int keep, const float* inv_v,
+                                                           const int* kpos, int n_split,
+                                                           float* ws_best, int* ws_bidx) {
+  __shared__ __align__(16) SimtSmem sm;
+  __shared__ const T* arow[kSimtBM];
+  __shared__ const T* brow[kSimtBN];
+  __shared__ float kinv[kSimtBN];
+  const int b = blockIdx.y, r0 = blockIdx.x * kSimtBM, split = blockIdx.z;
+  const int ntile = (keep + kSimtBN - 1) / kSimtBN;
+  const int t0 = (int)((long long)ntile * split / n_split), t1 = (int)((long long)ntile * (split + 1) / n_split);
+  const int rg = threadIdx.x >> 4, kg = threadIdx.x & 15;
+  if (threadIdx.x < kSimtBM) {
+    const int j = r0 + threadIdx.x;
+    const bool pruned = j < a.N_v && kpos[(size_t)b * a.N_v + j] < 0;
+    arow[threadIdx.x] = pruned ? row_ptr<T>(a.emb_v, (size_t)b * a.N_v + j, a.D) : nullptr;
+  }
+  float bv[8];
+  int bi[8];
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    bv[i] = -INFINITY;
+    bi[i] = 0x7fffffff;
+  }
+  for (int t = t0; t < t1; ++t) {
+    const int a0 = t * kSimtBN;
+    __syncthreads();
+    if (threadIdx.x < kSimtBN) {
+      const int ap = a0 + threadIdx.x;
+      if (ap < keep) {
+        const int j = keep_idx[(size_t)b * keep + ap];
+        const bool ok = j >= 0 && j < a.N_v;
+        brow[threadIdx.x] = ok ? row_ptr<T>(a.emb_v, (size_t)b * a.N_v + j, a.D) : nullptr;
+        kinv[threadIdx.x] = ok ? inv_v[(size_t)b * a.N_v + j] : 0.f;
+      } else {
+        brow[threadIdx.x] = nullptr;
+        kinv[threadIdx.x] = 0.f;
+      }
+    }
+    __syncthreads();
+    float acc[8][4];
+    simt_gemm_nt<T>(arow, brow, a.D, sm, acc);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+#pragma unroll
+      for (int jj = 0; jj < 4; ++jj) {
+        const int ap = a0 + kg + 16 * jj;
+        if (ap < keep) {
+          const float v = acc[i][jj] * kinv[kg + 16 * jj];
+          if (better(v, ap, bv[i], bi[i])) {
+            bv[i] = v;
+            bi[i] = ap;
+          }
+        }
+      }
+    }
+  }
+  // combine the 16 lanes of each row group
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+#pragma unroll
+    for (int o = 8; o > 0; o >>= 1) {
+      const float ov = __shfl_xor_sync(0xffffffffu, bv[i], o);
+      const int oi = __shfl_xor_sync(0xffffffffu, bi[i], o);
+      if (better(ov, oi, bv[i], bi[i])) {
+        bv[i] = ov;
+        bi[i] = oi;
+      }
+    }
+    const int j = r0 + rg + 16 * i;
+    if (kg == 0 && j < a.N_v) {
+      ws_best[((size_t)split * a.B + b) * a.N_v + j] = bv[i];
+      ws_bidx[((size_t)split * a.B + b) * a.N_v + j] = bi[i];
+    }
+  }
+}
+
+// assign[b][j]: own position for kept rows, best over splits for the others
+__global__ void merge_assign_kernel(const SimArgs a, const int* kpos, int n_split,
+                                    const float* ws_best, const int* ws_bidx, int* assign) {
+  const size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= (size_t)a.B * a.N_v) return;
+  const int kp = kpos[i];
+  if (kp >= 0) {
+    assign[i] = kp;
+    return;
+  }
+  float bv = -INFINITY;
+  int bi = 0x7fffffff;
+  for (int s = 0; s < n_split; ++s) {
+    const float v = ws_best[(size_t)s * a.B * a.N_v + i];
+    const int ix = ws_bidx[(size_t)s * a.B * a.N_v + i];
+    if (better(v, ix, bv, bi)) {
+      bv = v;
+      bi = ix;
+    }
+  }
+  // a zero or non-finite row compares equal everywhere: lowest position
+  assign[i] = bi == 0x7fffffff ? 0 : bi;
+}
+
+// merged[b][a] = (sum of rows j with assign[b][j] == a, ascending j) / count
+template <typename T, typename Acc>
+__global__ void __launch_bounds__(256) merge_mean_kernel(const SimArgs a, const int* assign,
+                                                         int keep, void* merged) {
+  __shared__ int members[256];
+  __shared__ int wcount[8];
+  const int ap = blockIdx.x, b = blockIdx.y;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const T* E = static_cast<const T*>(a.emb_v) + (size_t)b * a.N_v * a.D;
+  const int* as = assign + (size_t)b * a.N_v;
+  // each thread owns columns threadIdx.x + 256 q
+  constexpr int kMaxQ = 32;  // D <= 8192
+  Acc acc[kMaxQ];
+#pragma unroll
+  for (int q = 0; q < kMaxQ; ++q) acc[q] = Acc(0);
+  int count = 0;
+  for (int j0 = 0; j0 < a.N_v; j0 += 256) {
+    const int j = j0 + threadIdx.x;
+    const bool hit = j < a.N_v && as[j] == ap;
+    const unsigned bal = __ballot_sync(0xffffffffu, hit);
+    if (lane == 0) wcount[warp] = __popc(bal);
+    __syncthreads();
+    int off = 0, tot = 0;
+    for (int w = 0; w < 8; ++w) {
+      if (w < warp) off += wcount[w];
+      tot += wcount[w];
+    }
+    if (hit) members[off + __popc(bal & ((1u << lane) - 1u))] = j;
+    __syncthreads();
+    for (int m = 0; m < tot; ++m) {
+      const T* row = E + (size_t)members[m] * a.D;
+#pragma unroll
+      for (int q = 0; q < kMaxQ; ++q) {
+        const int d = threadIdx.x + 256 * q;
+        if (d < a.D) acc[q] += (Acc)to_f32(row[d]);
+      }
+    }
+    count += tot;
+    __syncthreads();
+  }
+  T* out = static_cast<T*>(merged) + ((size_t)b * keep + ap) * a.D;
+#pragma unroll
+  for (int q = 0; q < kMaxQ; ++q) {
+    const int d = threadIdx.x + 256 * q;
+    if (d < a.D) {
+      const Acc v = count > 0 ? acc[q] / (Acc)count : Acc(0);
+      if constexpr (sizeof(T) == 4)
+        out[d] = (T)v;
+      else
+        out[d] = __float2bfloat16_rn((float)v);
+    }
+  }
+}
+
+}  // namespace
+
+cudaError_t crit_text_launch(const SimArgs& a, uint8_t* mask, float* r_out, float* G,
+                             cudaStream_t s) {
+  dim3 g((a.N_t_max + kSimtBN - 1) / kSimtBN, (a.N_t_max + kSimtBM - 1) / kSimtBM, a.B);
+  if (a.dtype == 0)
+    crit_gram_kernel<float><<<g, 256, 0, s>>>(a, G);
+  else
+    crit_gram_kernel<__nv_bfloat16><<<g, 256, 0, s>>>(a, G);
+  crit_finish_kernel<<<a.B, 256, 3 * a.N_t_max * sizeof(float), s>>>(a, G, mask, r_out);
+  return cudaGetLastError();
+}
+
+cudaError_t vis_inv_norm_launch(const SimArgs& a, float* inv_v, cudaStream_t s) {
+  const size_t rows = (size_t)a.B * a.N_v;
+  const unsigned grid = (unsigned)((rows + 7) / 8);
+  if (a.dtype == 0)
+    inv_norm_kernel<float><<<grid, 256, 0, s>>>(a.emb_v, rows, a.D, inv_v);
+  else
+    inv_norm_kernel<__nv_bfloat16><<<grid, 256, 0, s>>>(a.emb_v, rows, a.D, inv_v);
+  return cudaGetLastError();
+}
+
+cudaError_t relevance_launch(const SimArgs& a, const uint8_t* mask, const float* inv_v, float* p,
+                             float* ws_sum, float* ws_mu, float* ws_invt, int n_split,
+                             cudaStream_t s) {
+  const int chunk = (a.N_v + n_split - 1) / n_split;
+  dim3 g1((a.D + 255) / 256, a.B, n_split);
+  dim3 g2((a.N_t_max + 7) / 8, a.B);
+  dim3 g3((a.N_v + kSimtBN - 1) / kSimtBN, a.B);
+  // ws_sum holds n_split partial sums followed by their total
+  float* total = ws_sum + (size_t)n_split * a.B * a.D;
+  dim3 g4((a.D + 255) / 256, a.B);
+  if (a.dtype == 0) {
+    vis_sum_kernel<float><<<g1, 256, 0, s>>>(a, inv_v, ws_sum, chunk);
+    vis_sum_reduce_kernel<<<g4, 256, 0, s>>>(a, ws_sum, n_split, total);
+    text_mu_kernel<float><<<g2, 256, 0, s>>>(a, total, ws_mu, ws_invt);
+    relevance_kernel<float><<<g3, 256, 0, s>>>(a, mask, inv_v, ws_mu, ws_invt, p);
+  } else {
+    vis_sum_kernel<__nv_bfloat16><<<g1, 256, 0, s>>>(a, inv_v, ws_sum, chunk);
+    vis_sum_reduce_kernel<<<g4, 256, 0, s>>>(a, ws_sum, n_split, total);
+    text_mu_kernel<__nv_bfloat16><<<g2, 256, 0, s>>>(a, total, ws_mu, ws_invt);
+    relevance_kernel<__nv_bfloat16><<<g3, 256, 0, s>>>(a, mask, inv_v, ws_mu, ws_invt, p);
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t merge_launch(const SimArgs& a, const int* keep_idx, int keep, const float* inv_v,
+                         int* assign, void* merged, float* ws_best, int* ws_bidx, int n_split,
+                         cudaStream_t s) {
+  // kpos lives in `assign` until the final assignment overwrites it: it is
+  // read by merge_argmax_kernel and merge_assign_kernel (same index only).
+  int* kpos = assign;
+  const size_t nb = (size_t)a.B * a.N_v;
+  keep_pos_kernel<<<(unsigned)((nb + 255) / 256), 256, 0, s>>>(keep_idx, keep, a.B, a.N_v, kpos, a.err);
+  const size_t nk = (size_t)a.B * keep;
+  keep_scatter_kernel<<<(unsigned)((nk + 255) / 256), 256, 0, s>>>(keep_idx, keep, a.B, a.N_v, kpos, a.err);
+  dim3 g((a.N_v + kSimtBM - 1) / kSimtBM, a.B, n_split);
+  if (a.dtype == 0)
+    merge_argmax_kernel<float><<<g, 256, 0, s>>>(a, keep_idx, keep, inv_v, kpos, n_split, ws_best, ws_bidx);
+  else
+    merge_argmax_kernel<__nv_bfloat16><<<g, 256, 0, s>>>(a, keep_idx, keep, inv_v, kpos, n_split, ws_best, ws_bidx);
+  merge_assign_kernel<<<(unsigned)((nb + 255) / 256), 256, 0, s>>>(a, kpos, n_split, ws_best, ws_bidx, assign);
+  if (merged != nullptr) {
+    dim3 gm(keep, a.B);
+    if (a.dtype == 0)
+      merge_mean_kernel<float, double><<<gm, 256, 0, s>>>(a, assign, keep, merged);
+    else
+      merge_mean_kernel<__nv_bfloat16, float><<<gm, 256, 0, s>>>(a, assign, keep, merged);
+  }
+  return cudaGetLastError();
+}
+
+}  // namespace provip
