@@ -49,7 +49,8 @@ N_COPIES = 3
 # DRAM traffic of one compaction launch on the default workload, from the ncu
 # capture summarised in profiles/ (null when the kernel source has changed
 # since: the sha1 of the kernel file is checked at run time).
-COMPACT_TRAFFIC = {"sha1": None, "bytes": None, "profile": None}
+COMPACT_TRAFFIC = {"sha1": "589b2b87d1b4ea8803beb9af644e4f40730ff41b", "bytes": 116439296,
+                   "profile": "profiles/prune_llava_next_b8_kernels.md"}
 
 
 def parse_args(argv=None):
@@ -62,6 +63,7 @@ def parse_args(argv=None):
     ap.add_argument("--algo", default="auto", choices=["auto", "simt", "tcgen05"])
     ap.add_argument("--e2e-steps", type=int, default=20)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--copies", type=int, default=N_COPIES, help="rotating device copies of the inputs")
     return ap.parse_args(argv)
 
 
@@ -356,14 +358,15 @@ def run_gb300(args, dist):
     vis, nv, keep = cpu["vis_start"], cpu["N_v"], cpu["keep"]
     algo = {"auto": P.ALGO_AUTO, "simt": P.ALGO_SIMT, "tcgen05": P.ALGO_TCGEN05}[args.algo]
     copies = []
-    for _ in range(N_COPIES):
+    n_copies = max(1, args.copies)
+    for _ in range(n_copies):
         copies.append({k: (v.to(dev) if isinstance(v, torch.Tensor) else v) for k, v in cpu.items()})
     g0 = copies[0]
     step = P.PruneStep(g0["Q"], g0["K"], g0["V"], g0["hidden"], g0["pos"], g0["head_list"], w.n_t[1], nv, keep,
                        algo=algo, want_scores=False)
 
     def do_step(i):
-        c = copies[i % N_COPIES]
+        c = copies[i % len(copies)]
         step(c["Q"], c["K"], c["V"], c["hidden"], c["pos"], c["text_start"], c["text_len"], c["seq_len"], vis)
 
     # warm-up
@@ -424,12 +427,14 @@ def run_gb300(args, dist):
     ws_ht = P.workspace(step.ws.numel(), dev)
 
     def compact_i(i):
-        c = copies[i % N_COPIES]
+        c = copies[i % len(copies)]
         P.provip_compact(idx, c["hidden"], c["K"], c["V"], c["pos"], c["seq_len"], vis, nv, out=outs)
 
+    heads_host = cpu["head_list"].tolist()
+
     def head_topk_i(i):
-        c = copies[i % N_COPIES]
-        P.provip_head_topk(c["Q"], c["K"], c["head_list"], c["text_start"], c["text_len"], c["seq_len"], vis, nv,
+        c = copies[i % len(copies)]
+        P.provip_head_topk(c["Q"], c["K"], heads_host, c["text_start"], c["text_len"], c["seq_len"], vis, nv,
                            keep, algo=algo, N_t_max=w.n_t[1], ws=ws_ht, want_scores=False)
 
     def time_graph(fn, reps):
@@ -502,7 +507,7 @@ def run_gb300(args, dist):
             "config": {"workload": w.name, "B": w.B, "N_v": nv, "keep": keep, "L_max": w.L_max,
                        "H_q": w.H_q, "H_kv": w.H_kv, "H_sel": w.H_sel, "D": w.D,
                        "algo": args.algo,
-                       "l2": f"inputs larger than L2: {N_COPIES} rotating device copies of "
+                       "l2": f"inputs larger than L2: {len(copies)} rotating device copies of "
                              f"{sum(v.numel() * v.element_size() for v in pin.values()) / 1e6:.0f} MB",
                        "timing": f"CUDA graphs of {GRAPH_CHUNK} steps, events on the launching stream"},
             "roofline": {"bound": "hbm", "kernel": "compact_kernel", "achieved": ach, "peak": peak,

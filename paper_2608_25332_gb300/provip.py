@@ -227,6 +227,7 @@ def provip_similarity_reduce(emb_v, emb_t, text_len, keep_pre, crit_mask=None, w
 # in-LLM pass
 # ---------------------------------------------------------------------------
 def _heads_arg(head_list):
+    """head_list is read on the host (a list, a CPU tensor, or a device tensor copied once)."""
     hl = [int(h) for h in (head_list.tolist() if hasattr(head_list, "tolist") else head_list)]
     arr = (ctypes.c_int * len(hl))(*hl)
     return arr, len(hl)
