@@ -179,6 +179,33 @@ int provip_head_scores(const void *Q, const void *K, int B, int L_max, int H_q, 
                        int vis_start, int N_v, const int *seq_len, int dtype, int algo,
                        float *scores, void *ws, size_t ws_bytes, void *stream);
 
+/* provip_head_scores for callers that cannot allocate device memory (the
+ * paper has no counterpart; this is a deployment convenience). Some hosts
+ * cannot pass the library a workspace: a framework that owns every device
+ * allocation and hands a plugin only its input and output tensors, or a
+ * serving loop that allows no allocator call once it is running. This entry
+ * point takes the same arguments as provip_head_scores minus the workspace and
+ * keeps its scratch in a static device array of PROVIP_NOALLOC_SCRATCH_BYTES
+ * (4 MiB) inside the library, which every GPU that loads the library holds
+ * until the process exits. It allocates nothing.
+ *   - A shape whose scratch (provip_head_scores_workspace_size) exceeds the
+ *     array is rejected with PROVIP_ERR_UNSUPPORTED before anything is
+ *     enqueued; use provip_head_scores with a workspace for it.
+ *   - The first call on each device looks up the array's device address (with
+ *     that device current); make that first call before any stream capture.
+ *   - All calls on a device share the one array, which keeps what the last call
+ *     left there (nothing in it needs to start at zero). Calls that overlap on
+ *     the GPU - on different streams, or from different host threads without
+ *     ordering - race on it and corrupt each other's results: issue them in
+ *     order on one stream. */
+#define PROVIP_NOALLOC_SCRATCH_BYTES (4u << 20)
+int provip_head_scores_noalloc(const void *Q, const void *K, int B, int L_max, int H_q,
+                               int H_kv, int d_h, const int *head_list, int H_sel,
+                               const int *text_start, const int *text_len,
+                               const uint8_t *row_mask_or_null, int N_t_max, int vis_start,
+                               int N_v, const int *seq_len, int dtype, int algo, float *scores,
+                               void *stream);
+
 /* Survivor compaction given the kept indices (Sec. 4.1: pruned tokens are
  * excluded from all later computation). For every sample the output rows are
  *   [0, vis_start) ++ (vis_start + idx[b][a], a < keep) ++ [vis_start + N_v, seq_len[b])

@@ -701,3 +701,64 @@ extern "C" int provip_prune(const void* Q, const void* K, const void* V, const v
   return provip_compact(idx_out, B, N_v, keep, hidden, D, K, V, H_kv, d_h, pos, P, seq_len, L_max,
                         vis_start, dtype, hidden_out, K_out, V_out, pos_out, seq_len_out, stream);
 }
+
+// ===========================================================================
+// head scores without a workspace
+//
+// Some callers cannot hand the library any device memory: a host framework
+// that owns every allocation and passes a plugin only its input and output
+// tensors, or a serving loop that forbids allocator calls once it is running.
+// For them the scratch of the head scores (per-chunk row statistics and
+// per-head partial sums) lives in this file-scope device array instead of a
+// workspace. Every GPU that loads the library keeps the array until the
+// process exits.
+// ===========================================================================
+static constexpr size_t kNoAllocScratchBytes = (size_t)PROVIP_NOALLOC_SCRATCH_BYTES;
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
+// Device address of the array on each device. In host code the symbol only
+// names a host-side stand-in, so a kernel must be given this address, looked up
+// with the device current.
+static void* g_noalloc_addr[64];
+
+static int noalloc_scratch_addr(void** out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, "head_scores_noalloc: cudaGetDevice");
+  if (dev < 0 || dev >= 64) return fail(PROVIP_ERR_UNSUPPORTED, "head_scores_noalloc: device %d >= 64", dev);
+  if (g_noalloc_addr[dev] == nullptr) {
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+    if (e != cudaSuccess || p == nullptr)
+      return cuda_fail(e != cudaSuccess ? e : cudaErrorInvalidSymbol,
+                       "head_scores_noalloc: cudaGetSymbolAddress(scratch)");
+    g_noalloc_addr[dev] = p;
+  }
+  *out = g_noalloc_addr[dev];
+  return PROVIP_OK;
+}
+
+extern "C" int provip_head_scores_noalloc(const void* Q, const void* K, int B, int L_max, int H_q,
+                                          int H_kv, int d_h, const int* head_list, int H_sel,
+                                          const int* text_start, const int* text_len,
+                                          const uint8_t* row_mask_or_null, int N_t_max,
+                                          int vis_start, int N_v, const int* seq_len, int dtype,
+                                          int algo, float* scores, void* stream) {
+  const int ralgo = resolve_algo(algo, dtype);
+  int rc = hs_validate(Q, K, B, L_max, H_q, H_kv, d_h, head_list, H_sel, text_start, text_len,
+                       N_t_max, vis_start, N_v, seq_len, dtype, ralgo);
+  if (rc) return rc;
+  if (!scores) return fail(PROVIP_ERR_INVALID_ARG, "head_scores_noalloc: null scores");
+  const size_t need = provip_head_scores_workspace_size(B, L_max, H_sel, N_t_max, N_v, ralgo, dtype);
+  if (need > kNoAllocScratchBytes)
+    return fail(PROVIP_ERR_UNSUPPORTED,
+                "head_scores_noalloc: this shape needs %zu bytes of scratch, more than the %zu-byte "
+                "static array; use provip_head_scores with a workspace",
+                need, kNoAllocScratchBytes);
+  void* scratch = nullptr;
+  if ((rc = noalloc_scratch_addr(&scratch))) return rc;
+  // Nothing in the scratch has to start at zero: every statistic and partial
+  // sum is written by the first pass of this call before anything reads it.
+  return provip_head_scores(Q, K, B, L_max, H_q, H_kv, d_h, head_list, H_sel, text_start, text_len,
+                            row_mask_or_null, N_t_max, vis_start, N_v, seq_len, dtype, ralgo,
+                            scores, scratch, kNoAllocScratchBytes, stream);
+}

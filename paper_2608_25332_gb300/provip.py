@@ -48,6 +48,8 @@ _SIGS = {
     "provip_head_scores_workspace_size": (_Z, [_I, _I, _I, _I, _I, _I, _I]),
     "provip_head_scores": (_I, [_P, _P, _I, _I, _I, _I, _I, _P, _I, _P, _P, _P, _I, _I, _I, _P, _I, _I,
                                 _P, _P, _Z, _P]),
+    "provip_head_scores_noalloc": (_I, [_P, _P, _I, _I, _I, _I, _I, _P, _I, _P, _P, _P, _I, _I, _I, _P, _I,
+                                        _I, _P, _P]),
     "provip_compact": (_I, [_P, _I, _I, _I, _P, _I, _P, _P, _I, _I, _P, _I, _P, _I, _I, _I, _P, _P, _P,
                             _P, _P, _P]),
     "provip_topk_compact": (_I, [_P, _I, _I, _I, _P, _I, _P, _P, _I, _I, _P, _I, _P, _I, _I, _I, _P, _P,
@@ -356,3 +358,21 @@ def provip_head_topk(Q, K, head_list, text_start, text_len, seq_len, vis_start, 
                             algo, _ptr(idx), _ptr(scores), _ptr(ws), ws.numel(), _stream(dev))
     _check(rc, "provip_head_topk")
     return idx, scores
+
+
+def provip_head_scores_noalloc(Q, K, head_list, text_start, text_len, seq_len, vis_start, N_v,
+                               row_mask=None, algo=ALGO_AUTO, N_t_max=None):
+    """provip_head_scores without a workspace: the scratch is the library's own
+    static device array (for hosts that cannot allocate device memory; shapes
+    needing more than PROVIP_NOALLOC_SCRATCH_BYTES are rejected)."""
+    B, Lm, Hq, dh = Q.shape
+    Hkv = K.shape[2]
+    dev = Q.device
+    heads, hs = _heads_arg(head_list)
+    Ntm = int(N_t_max if N_t_max is not None else int(text_len.max().item()))
+    scores = torch.empty((B, N_v), dtype=torch.float32, device=dev)
+    rc = lib().provip_head_scores_noalloc(_ptr(Q), _ptr(K), B, Lm, Hq, Hkv, dh, heads, hs, _i32(text_start),
+                                          _i32(text_len), _u8(row_mask), Ntm, vis_start, N_v, _i32(seq_len),
+                                          _dtype_code(Q), algo, _ptr(scores), _stream(dev))
+    _check(rc, "provip_head_scores_noalloc")
+    return scores
