@@ -60,7 +60,12 @@ extern "C" {
 /* kernel families for provip_head_scores / provip_prune */
 #define PROVIP_ALGO_AUTO 0    /* tensor cores for bf16, CUDA cores for fp32 */
 #define PROVIP_ALGO_SIMT 1    /* CUDA-core FFMA kernels (fp32 and bf16) */
-#define PROVIP_ALGO_TCGEN05 2 /* tcgen05 tensor cores, TMEM accumulators (bf16 only) */
+#define PROVIP_ALGO_TCGEN05 2 /* tcgen05 tensor cores, one pass over K in a cluster per
+                                 (head, sample), logits kept in TMEM (bf16 only); falls
+                                 back to the two-pass form when L_max > 8192 or no
+                                 cluster shape fits */
+#define PROVIP_ALGO_TCGEN05_TWOPASS 3 /* tcgen05, two kernels: chunk statistics, then
+                                         probabilities (bf16 only) */
 
 /* bits of the device status word */
 #define PROVIP_DEVSTAT_TIMEOUT 1u  /* a bounded wait gave up */

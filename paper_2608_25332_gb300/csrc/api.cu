@@ -84,8 +84,9 @@ int resolve_algo(int algo, int dtype) {
   if (algo == PROVIP_ALGO_AUTO) return dtype == PROVIP_BF16 ? PROVIP_ALGO_TCGEN05 : PROVIP_ALGO_SIMT;
   return algo;
 }
-int key_chunk(int algo) { return algo == PROVIP_ALGO_TCGEN05 ? 128 : 64; }
-int vis_chunk(int algo) { return algo == PROVIP_ALGO_TCGEN05 ? 128 : 64; }
+bool is_tc(int algo) { return algo == PROVIP_ALGO_TCGEN05 || algo == PROVIP_ALGO_TCGEN05_TWOPASS; }
+int key_chunk(int algo) { return is_tc(algo) ? 128 : 64; }
+int vis_chunk(int algo) { return is_tc(algo) ? 128 : 64; }
 
 struct HSShape {
   int n_rb, kc, n_kc, vc, n_vc;
@@ -126,9 +127,9 @@ int hs_validate(const void* Q, const void* K, int B, int L_max, int H_q, int H_k
       if (head_list[j] == head_list[i])
         return fail(PROVIP_ERR_INVALID_ARG, "head_scores: duplicate head %d", head_list[i]);
   }
-  if (algo != PROVIP_ALGO_SIMT && algo != PROVIP_ALGO_TCGEN05)
+  if (algo != PROVIP_ALGO_SIMT && !is_tc(algo))
     return fail(PROVIP_ERR_INVALID_ARG, "head_scores: algo %d", algo);
-  if (algo == PROVIP_ALGO_TCGEN05 && dtype != PROVIP_BF16)
+  if (is_tc(algo) && dtype != PROVIP_BF16)
     return fail(PROVIP_ERR_UNSUPPORTED, "head_scores: tcgen05 path needs bf16");
   if (!aligned16(Q) || !aligned16(K)) return fail(PROVIP_ERR_UNSUPPORTED, "head_scores: Q/K not 16-byte aligned");
   if ((size_t)B * L_max * H_q * d_h >= (1ull << 40))
@@ -173,13 +174,16 @@ HSArgs hs_args(const void* Q, const void* K, int B, int L_max, int H_q, int H_kv
 // both passes of the head scores (partials in the workspace)
 int hs_run(const HSArgs& a, int dtype, int algo, cudaStream_t s) {
   cudaError_t e;
-  if (algo == PROVIP_ALGO_TCGEN05) {
+  if (is_tc(algo)) {
     CUtensorMap tq, tk;
     const uint64_t qstride = (uint64_t)a.H_q * a.d_h * 2, kstride = (uint64_t)a.H_kv * a.d_h * 2;
     if (make_tmap_bf16_2d(&tq, a.Q, (uint64_t)a.B * a.L_max, (uint64_t)a.H_q * a.d_h, qstride, 128) ||
         make_tmap_bf16_2d(&tk, a.K, (uint64_t)a.B * a.L_max, (uint64_t)a.H_kv * a.d_h, kstride, 128))
       return fail(PROVIP_ERR_CUDA, "head_scores: cuTensorMapEncodeTiled failed");
-    e = hs_launch_tc(a, &tq, &tk, s);
+    bool launched = false;
+    e = cudaSuccess;
+    if (algo == PROVIP_ALGO_TCGEN05) e = hs_launch_fused(a, &tq, &tk, s, &launched);
+    if (e == cudaSuccess && !launched) e = hs_launch_tc(a, &tq, &tk, s);
   } else {
     e = hs_launch_simt(a, dtype, s);
   }
@@ -674,7 +678,9 @@ extern "C" int provip_head_topk(const void* Q, const void* K, int B, int L_max, 
   t.k = keep;
   t.idx_out = idx_out;
   t.err = d->status;
-  cudaError_t e = topk_launch(t, s);
+  // a programmatic dependent of the head-score kernel: launched early, waits
+  // for the partials on the device
+  cudaError_t e = topk_launch(t, s, true);
   return e == cudaSuccess ? PROVIP_OK : cuda_fail(e, "head_topk topk");
 }
 
@@ -698,8 +704,15 @@ extern "C" int provip_prune(const void* Q, const void* K, const void* V, const v
                         row_mask_or_null, N_t_max, vis_start, N_v, seq_len, keep, dtype, algo,
                         idx_out, scores_out_or_null, ws, ws_bytes, stream);
   if (rc) return rc;
-  return provip_compact(idx_out, B, N_v, keep, hidden, D, K, V, H_kv, d_h, pos, P, seq_len, L_max,
-                        vis_start, dtype, hidden_out, K_out, V_out, pos_out, seq_len_out, stream);
+  // the compaction is a programmatic dependent of the selection: the rows that
+  // do not depend on idx are copied while the selection finishes
+  DevInfo* d;
+  if ((rc = dev_info(&d))) return rc;
+  CompactArgs ca = compact_args(idx_out, B, N_v, keep, hidden, D, K, V, H_kv, d_h, pos, P, seq_len,
+                                L_max, vis_start, dtype, hidden_out, K_out, V_out, pos_out,
+                                seq_len_out, d->status);
+  cudaError_t e = compact_launch(ca, d->sms, static_cast<cudaStream_t>(stream), true);
+  return e == cudaSuccess ? PROVIP_OK : cuda_fail(e, "prune compact");
 }
 
 // ===========================================================================

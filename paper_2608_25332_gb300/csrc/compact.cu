@@ -5,7 +5,11 @@
 // plus the position-id rows (int32, P of them; carried, not renumbered).
 //
 // Bulk-TMA pipeline: the work is the list of (output row, tensor, <= 8 KiB
-// piece) items; every CTA owns a contiguous range of it. One thread per CTA
+// piece) items, in two phases - first the rows that do not depend on the kept
+// indices (prefix and text rows), then the kept visual rows - and every CTA
+// owns a contiguous range of each phase. Launched as a programmatic dependent
+// of the kernel that writes idx, the first phase overlaps that kernel; the
+// threads that read idx wait for it (griddepcontrol.wait, a no-op otherwise). One thread per CTA
 // streams its range through a ring of shared-memory slots: a cp.async.bulk load
 // (global -> shared, completion on the slot's mbarrier) and, once it lands, a
 // cp.async.bulk store (shared -> global, bulk group). A slot is refilled as soon
@@ -43,6 +47,23 @@ struct Item {
   uint32_t bytes;
 };
 
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
+// Output row of item-space row q: phase 0 enumerates, per sample, the
+// L_out - keep rows outside the kept block; phase 1 the keep kept rows.
+__device__ __forceinline__ void phase_row(const CompactArgs& a, int phase, long long row, int& b,
+                                          int& r) {
+  if (phase == 0) {
+    const int per = a.L_out - a.keep;
+    b = (int)(row / per);
+    const int q = (int)(row - (long long)b * per);
+    r = q < a.vis_start ? q : q + a.keep;
+  } else {
+    b = (int)(row / a.keep);
+    r = a.vis_start + (int)(row - (long long)b * a.keep);
+  }
+}
+
 __global__ void __launch_bounds__(kCompactThreads) compact_kernel(const CompactArgs a, int np0,
                                                                    int np1, int np2) {
   extern __shared__ __align__(128) uint8_t slots[];
@@ -50,10 +71,14 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(const CompactA
   __shared__ char* ring_dst[kSlots];
   __shared__ uint32_t ring_bytes[kSlots];
   const int NP = np0 + np1 + np2;
-  const long long total = (long long)a.B * a.L_out * NP;
-  const long long per = (total + gridDim.x - 1) / gridDim.x;
-  const long long it_begin = min(total, (long long)blockIdx.x * per);
-  const long long it_end = min(total, it_begin + per);
+  long long rows[2] = {(long long)a.B * (a.L_out - a.keep), (long long)a.B * a.keep};
+  long long beg[2], fin[2];
+  for (int ph = 0; ph < 2; ++ph) {
+    const long long total = rows[ph] * NP;
+    const long long per = (total + gridDim.x - 1) / gridDim.x;
+    beg[ph] = min(total, (long long)blockIdx.x * per);
+    fin[ph] = min(total, beg[ph] + per);
+  }
 
   if (blockIdx.x == 0 && a.seq_len_out != nullptr)
     for (int b = threadIdx.x; b < a.B; b += blockDim.x)
@@ -67,14 +92,27 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(const CompactA
 
   if (threadIdx.x == 0) {
     const uint64_t pol = policy_evict_first();
-    long long next = it_begin;
-    // next valid item at or after `next`; false when the range is exhausted
+    int phase = 0;
+    long long next = beg[0];
+    bool waited = false;
+    // next valid item; false when both phases are exhausted
     auto fetch = [&](Item& it) -> bool {
-      while (next < it_end) {
+      for (;;) {
+        if (next >= fin[phase]) {
+          if (phase == 1) return false;
+          phase = 1;
+          next = beg[1];
+          continue;
+        }
+        if (phase == 1 && !waited) {
+          pdl_wait();  // idx is written by the previous kernel
+          waited = true;
+        }
         const long long i = next++;
         const long long row = i / NP;
         int q = (int)(i - row * NP);
-        const int b = (int)(row / a.L_out), r = (int)(row - (long long)b * a.L_out);
+        int b, r;
+        phase_row(a, phase, row, b, r);
         const int sl = a.seq_len[b];
         if (sl > a.L_max || sl < a.vis_start + a.N_v) {
           set_error(a.err, kErrBadDeviceArg);
@@ -103,7 +141,6 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(const CompactA
         it.dst = a.dst[t] + ((long long)b * a.L_out + r) * rb + off;
         return true;
       }
-      return false;
     };
     auto issue = [&](int slot, const Item& it) {
       ring_dst[slot] = it.dst;
@@ -138,25 +175,29 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(const CompactA
     }
     bulk_wait<0>();
   } else if (a.pos != nullptr && threadIdx.x >= 32) {
-    // position ids of the rows whose first item lies in this CTA's range
-    const long long r0 = (it_begin + NP - 1) / NP, r1 = (it_end + NP - 1) / NP;
+    // position ids of the rows whose first item lies in this CTA's ranges
     const int nth = blockDim.x - 32;
-    for (long long row = r0 + (threadIdx.x - 32); row < r1; row += nth) {
-      const int b = (int)(row / a.L_out), r = (int)(row - (long long)b * a.L_out);
-      const int sl = a.seq_len[b];
-      if (sl > a.L_max || sl < a.vis_start + a.N_v || r >= sl - a.N_v + a.keep) continue;
-      bool ok = true;
-      const int sr = src_row(a, b, r, ok);
-      if (!ok) continue;
-      for (int p = 0; p < a.P; ++p)
-        a.pos_out[((size_t)p * a.B + b) * a.L_out + r] = a.pos[((size_t)p * a.B + b) * a.L_max + sr];
+    for (int ph = 0; ph < 2; ++ph) {
+      if (ph == 1) pdl_wait();
+      const long long r0 = (beg[ph] + NP - 1) / NP, r1 = (fin[ph] + NP - 1) / NP;
+      for (long long row = r0 + (threadIdx.x - 32); row < r1; row += nth) {
+        int b, r;
+        phase_row(a, ph, row, b, r);
+        const int sl = a.seq_len[b];
+        if (sl > a.L_max || sl < a.vis_start + a.N_v || r >= sl - a.N_v + a.keep) continue;
+        bool ok = true;
+        const int sr = src_row(a, b, r, ok);
+        if (!ok) continue;
+        for (int p = 0; p < a.P; ++p)
+          a.pos_out[((size_t)p * a.B + b) * a.L_out + r] = a.pos[((size_t)p * a.B + b) * a.L_max + sr];
+      }
     }
   }
 }
 
 }  // namespace
 
-cudaError_t compact_launch(const CompactArgs& a, int num_sms, cudaStream_t s) {
+cudaError_t compact_launch(const CompactArgs& a, int num_sms, cudaStream_t s, bool pdl) {
   static bool configured[64] = {false};
   int dev = 0;
   cudaGetDevice(&dev);
@@ -172,8 +213,17 @@ cudaError_t compact_launch(const CompactArgs& a, int num_sms, cudaStream_t s) {
   const long long total = (long long)a.B * a.L_out * (np[0] + np[1] + np[2]);
   long long grid = 2LL * num_sms;
   if (grid > total) grid = total > 0 ? total : 1;
-  compact_kernel<<<(unsigned)grid, kCompactThreads, kCompactSmem, s>>>(a, np[0], np[1], np[2]);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  cfg.gridDim = dim3((unsigned)grid);
+  cfg.blockDim = dim3(kCompactThreads);
+  cfg.dynamicSmemBytes = kCompactSmem;
+  cfg.stream = s;
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, compact_kernel, a, np[0], np[1], np[2]);
 }
 
 }  // namespace provip

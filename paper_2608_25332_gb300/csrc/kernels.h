@@ -49,6 +49,10 @@ cudaError_t hs_launch_simt(const HSArgs& a, int dtype, cudaStream_t s);
 // tcgen05 path (bf16): needs tensor maps over Q and K viewed as 2-D row tables.
 cudaError_t hs_launch_tc(const HSArgs& a, const CUtensorMap* tmQ, const CUtensorMap* tmK,
                          cudaStream_t s);
+// one-pass tcgen05 path (clusters, TMEM-resident logits): writes the partials
+// directly; *launched is false when no cluster shape fits this problem.
+cudaError_t hs_launch_fused(const HSArgs& a, const CUtensorMap* tmQ, const CUtensorMap* tmK,
+                            cudaStream_t s, bool* launched);
 // scores[b][i] = sum_u partial[b][u][i] / (H_sel * valid text rows of b)
 cudaError_t hs_launch_reduce(const HSArgs& a, float* scores, cudaStream_t s);
 
@@ -69,7 +73,9 @@ struct TopkArgs {
   unsigned* err;
 };
 constexpr int kTopkMaxN = 49152;
-cudaError_t topk_launch(const TopkArgs& a, cudaStream_t s);
+// pdl: launched as a programmatic dependent of the previous kernel on the
+// stream (the kernel waits for it before reading its inputs)
+cudaError_t topk_launch(const TopkArgs& a, cudaStream_t s, bool pdl = false);
 
 // ---------------------------------------------------------------------------
 // compaction: rows [0, vis_start) ++ vis_start + idx ++ [vis_start + N_v, seq_len)
@@ -89,7 +95,9 @@ struct CompactArgs {
   int B, L_max, L_out;
   unsigned* err;
 };
-cudaError_t compact_launch(const CompactArgs& a, int num_sms, cudaStream_t s);
+// pdl: launched as a programmatic dependent of the previous kernel on the
+// stream; rows that do not depend on idx are copied before waiting for it.
+cudaError_t compact_launch(const CompactArgs& a, int num_sms, cudaStream_t s, bool pdl = false);
 
 // ---------------------------------------------------------------------------
 // pre-LLM similarity pass (Sec. 4.2-4.3)

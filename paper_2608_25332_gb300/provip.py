@@ -24,7 +24,7 @@ ERR_WORKSPACE = -3
 ERR_CUDA = -4
 ERR_TIMEOUT = -5
 F32, BF16 = 0, 1
-ALGO_AUTO, ALGO_SIMT, ALGO_TCGEN05 = 0, 1, 2
+ALGO_AUTO, ALGO_SIMT, ALGO_TCGEN05, ALGO_TCGEN05_TWOPASS = 0, 1, 2, 3
 
 _P = ctypes.c_void_p
 _I = ctypes.c_int

@@ -65,7 +65,8 @@ def ref_scores(name):
 
 
 CASES = [(w.name, a) for w in synth.WORKLOADS
-         for a in ([P.ALGO_SIMT] if w.dtype == "f32" else [P.ALGO_SIMT, P.ALGO_TCGEN05])]
+         for a in ([P.ALGO_SIMT] if w.dtype == "f32" else
+                   [P.ALGO_SIMT, P.ALGO_TCGEN05, P.ALGO_TCGEN05_TWOPASS])]
 
 
 @pytest.mark.parametrize("name,algo", CASES)
@@ -140,7 +141,7 @@ def _small_case(seed, B=3, Hq=6, Hkv=2, nsys=5, nv=37, tls=(1, 9, 130), dtype=to
     return dict(Q=Qt, K=Kt, tl=tl, sl=sl, ts=np.full(B, nsys + nv, np.int32), nsys=nsys, nv=nv, Ntm=Ntm)
 
 
-@pytest.mark.parametrize("algo", [P.ALGO_SIMT, P.ALGO_TCGEN05])
+@pytest.mark.parametrize("algo", [P.ALGO_SIMT, P.ALGO_TCGEN05, P.ALGO_TCGEN05_TWOPASS])
 def test_head_scores_ragged_and_masked_rows(algo):
     c = _small_case(7)
     heads = [1, 2, 5]
@@ -158,6 +159,23 @@ def test_head_scores_ragged_and_masked_rows(algo):
             rows = [c["ts"][b] + j for j in range(c["tl"][b]) if rm is None or rm[b, j]]
             ref = oracle.head_scores(Qn[b, :c["sl"][b]], Kn[b, :c["sl"][b]], heads, rows, c["nsys"], c["nv"])
             assert_close_rel(s[b].cpu().numpy(), ref, 2e-3, f"small case b={b} mask={rm is not None}")
+
+
+@pytest.mark.parametrize("nv,tl", [(4000, 200), (8000, 316)])
+def test_head_scores_long_sequences(nv, tl):
+    # 4205 keys: 33 chunks -> clusters of 9 CTAs with 4 chunks each; 8321 keys: more
+    # than 64 chunks -> the two-pass kernels take over
+    c = _small_case(9, B=1, Hq=4, Hkv=2, nsys=5, nv=nv, tls=(tl,))
+    heads = [0, 3]
+    Qd, Kd = c["Q"].to(DEV), c["K"].to(DEV)
+    ts, tlt, sl = (torch.from_numpy(x).to(DEV) for x in (c["ts"], c["tl"], c["sl"]))
+    Qn, Kn = c["Q"].float().numpy(), c["K"].float().numpy()
+    ref = oracle.head_scores(Qn[0, :c["sl"][0]], Kn[0, :c["sl"][0]], heads,
+                             np.arange(c["ts"][0], c["ts"][0] + c["tl"][0]), c["nsys"], c["nv"])
+    for algo in (P.ALGO_TCGEN05, P.ALGO_TCGEN05_TWOPASS, P.ALGO_SIMT):
+        s = P.provip_head_scores(Qd, Kd, heads, ts, tlt, sl, c["nsys"], c["nv"], algo=algo, N_t_max=c["Ntm"])
+        torch.cuda.synchronize()
+        assert_close_rel(s[0].cpu().numpy(), ref, 2e-3, f"long L={c['sl'][0]} algo={algo}")
 
 
 def test_topk_matches_oracle_with_ties():
