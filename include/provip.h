@@ -247,10 +247,24 @@ int provip_head_topk(const void *Q, const void *K, int B, int L_max, int H_q, in
                      const int *seq_len, int keep, int dtype, int algo, int *idx_out,
                      float *scores_out_or_null, void *ws, size_t ws_bytes, void *stream);
 
-/* The in-LLM pruning step end to end: provip_head_topk, then
- * provip_compact with its idx. Arguments as in the calls above; K is both the scored keys and the
- * compacted K. scores_out_or_null receives v [B, N_v] when non-NULL. Uses the
- * workspace of provip_head_scores. */
+/* The in-LLM pruning step end to end: provip_head_topk, then provip_compact
+ * with its idx. Arguments as in the calls above; K is both the scored keys and
+ * the compacted K. scores_out_or_null receives v [B, N_v] when non-NULL. Uses
+ * the workspace of provip_head_scores.
+ *
+ * Kernels: the head scores, the top-k and the compaction run back to back on
+ * the stream; the top-k and the compaction are launched as programmatic
+ * dependents (the compaction copies the rows that do not depend on the kept
+ * indices while the selection finishes).
+ *
+ * flags: 0, or PROVIP_PRUNE_OVERLAP_PREVIOUS - the call's head-score kernel may
+ * start while the kernel before it on the stream (typically the previous
+ * call's compaction) is still running; it only waits for that kernel before
+ * writing its workspace. Pass it only when this call's Q and K were not written
+ * by the kernel launched just before it on the stream (for instance when
+ * pruning a stream of independent batches); other kernels in between (e.g. the
+ * LLM layers that produce Q/K) make the flag harmless. */
+#define PROVIP_PRUNE_OVERLAP_PREVIOUS 1u
 size_t provip_prune_workspace_size(int B, int L_max, int H_sel, int N_t_max, int N_v, int algo,
                                    int dtype);
 int provip_prune(const void *Q, const void *K, const void *V, const void *hidden, int B,
@@ -259,7 +273,7 @@ int provip_prune(const void *Q, const void *K, const void *V, const void *hidden
                  int N_t_max, int vis_start, int N_v, const int *seq_len, const int *pos, int P,
                  int keep, int dtype, int algo, void *hidden_out, void *K_out, void *V_out,
                  int *pos_out, int *idx_out, int *seq_len_out, float *scores_out_or_null,
-                 void *ws, size_t ws_bytes, void *stream);
+                 void *ws, size_t ws_bytes, unsigned flags, void *stream);
 
 #ifdef __cplusplus
 }

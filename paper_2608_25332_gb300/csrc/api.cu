@@ -171,8 +171,9 @@ HSArgs hs_args(const void* Q, const void* K, int B, int L_max, int H_q, int H_kv
   return a;
 }
 
-// both passes of the head scores (partials in the workspace)
-int hs_run(const HSArgs& a, int dtype, int algo, cudaStream_t s) {
+// both passes of the head scores (partials in the workspace); overlap: the
+// one-pass kernel may start before the previous kernel on the stream finishes
+int hs_run(const HSArgs& a, int dtype, int algo, cudaStream_t s, bool overlap = false) {
   cudaError_t e;
   if (is_tc(algo)) {
     CUtensorMap tq, tk;
@@ -182,7 +183,7 @@ int hs_run(const HSArgs& a, int dtype, int algo, cudaStream_t s) {
       return fail(PROVIP_ERR_CUDA, "head_scores: cuTensorMapEncodeTiled failed");
     bool launched = false;
     e = cudaSuccess;
-    if (algo == PROVIP_ALGO_TCGEN05) e = hs_launch_fused(a, &tq, &tk, s, &launched);
+    if (algo == PROVIP_ALGO_TCGEN05) e = hs_launch_fused(a, &tq, &tk, s, &launched, overlap);
     if (e == cudaSuccess && !launched) e = hs_launch_tc(a, &tq, &tk, s);
   } else {
     e = hs_launch_simt(a, dtype, s);
@@ -636,12 +637,12 @@ extern "C" size_t provip_prune_workspace_size(int B, int L_max, int H_sel, int N
   return provip_head_scores_workspace_size(B, L_max, H_sel, N_t_max, N_v, algo, dtype);
 }
 
-extern "C" int provip_head_topk(const void* Q, const void* K, int B, int L_max, int H_q, int H_kv,
+static int head_topk_impl(const void* Q, const void* K, int B, int L_max, int H_q, int H_kv,
                                 int d_h, const int* head_list, int H_sel, const int* text_start,
                                 const int* text_len, const uint8_t* row_mask_or_null, int N_t_max,
                                 int vis_start, int N_v, const int* seq_len, int keep, int dtype,
                                 int algo, int* idx_out, float* scores_out_or_null, void* ws,
-                                size_t ws_bytes, void* stream) {
+                                size_t ws_bytes, void* stream, bool overlap) {
   algo = resolve_algo(algo, dtype);
   int rc = hs_validate(Q, K, B, L_max, H_q, H_kv, d_h, head_list, H_sel, text_start, text_len,
                        N_t_max, vis_start, N_v, seq_len, dtype, algo);
@@ -663,7 +664,7 @@ extern "C" int provip_head_topk(const void* Q, const void* K, int B, int L_max, 
                      row_mask_or_null, N_t_max, vis_start, N_v, seq_len, sh, stats, partial,
                      d->status);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  if ((rc = hs_run(a, dtype, algo, s))) return rc;
+  if ((rc = hs_run(a, dtype, algo, s, overlap))) return rc;
   TopkArgs t;
   memset(&t, 0, sizeof(t));
   t.partial = partial;
@@ -684,6 +685,17 @@ extern "C" int provip_head_topk(const void* Q, const void* K, int B, int L_max, 
   return e == cudaSuccess ? PROVIP_OK : cuda_fail(e, "head_topk topk");
 }
 
+extern "C" int provip_head_topk(const void* Q, const void* K, int B, int L_max, int H_q, int H_kv,
+                                int d_h, const int* head_list, int H_sel, const int* text_start,
+                                const int* text_len, const uint8_t* row_mask_or_null, int N_t_max,
+                                int vis_start, int N_v, const int* seq_len, int keep, int dtype,
+                                int algo, int* idx_out, float* scores_out_or_null, void* ws,
+                                size_t ws_bytes, void* stream) {
+  return head_topk_impl(Q, K, B, L_max, H_q, H_kv, d_h, head_list, H_sel, text_start, text_len,
+                        row_mask_or_null, N_t_max, vis_start, N_v, seq_len, keep, dtype, algo,
+                        idx_out, scores_out_or_null, ws, ws_bytes, stream, false);
+}
+
 extern "C" int provip_prune(const void* Q, const void* K, const void* V, const void* hidden, int B,
                             int L_max, int H_q, int H_kv, int d_h, int D, const int* head_list,
                             int H_sel, const int* text_start, const int* text_len,
@@ -691,8 +703,9 @@ extern "C" int provip_prune(const void* Q, const void* K, const void* V, const v
                             const int* seq_len, const int* pos, int P, int keep, int dtype,
                             int algo, void* hidden_out, void* K_out, void* V_out, int* pos_out,
                             int* idx_out, int* seq_len_out, float* scores_out_or_null, void* ws,
-                            size_t ws_bytes, void* stream) {
+                            size_t ws_bytes, unsigned flags, void* stream) {
   // validate both halves before enqueueing anything
+  if (flags & ~(unsigned)PROVIP_PRUNE_OVERLAP_PREVIOUS) return fail(PROVIP_ERR_INVALID_ARG, "prune: unknown flags 0x%x", flags);
   int rc = hs_validate(Q, K, B, L_max, H_q, H_kv, d_h, head_list, H_sel, text_start, text_len,
                        N_t_max, vis_start, N_v, seq_len, dtype, resolve_algo(algo, dtype));
   if (rc) return rc;
@@ -700,9 +713,10 @@ extern "C" int provip_prune(const void* Q, const void* K, const void* V, const v
                              K, V, H_kv, d_h, pos, P, seq_len, L_max, vis_start, dtype, hidden_out,
                              K_out, V_out, pos_out)))
     return rc;
-  rc = provip_head_topk(Q, K, B, L_max, H_q, H_kv, d_h, head_list, H_sel, text_start, text_len,
-                        row_mask_or_null, N_t_max, vis_start, N_v, seq_len, keep, dtype, algo,
-                        idx_out, scores_out_or_null, ws, ws_bytes, stream);
+  rc = head_topk_impl(Q, K, B, L_max, H_q, H_kv, d_h, head_list, H_sel, text_start, text_len,
+                      row_mask_or_null, N_t_max, vis_start, N_v, seq_len, keep, dtype, algo,
+                      idx_out, scores_out_or_null, ws, ws_bytes, stream,
+                      (flags & PROVIP_PRUNE_OVERLAP_PREVIOUS) != 0);
   if (rc) return rc;
   // the compaction is a programmatic dependent of the selection: the rows that
   // do not depend on idx are copied while the selection finishes

@@ -23,8 +23,15 @@
 namespace provip {
 namespace {
 
+#ifndef PROVIP_COMPACT_SLOTS
+#define PROVIP_COMPACT_SLOTS 6
+#endif
+#ifndef PROVIP_COMPACT_CTAS_PER_SM
+#define PROVIP_COMPACT_CTAS_PER_SM 3
+#endif
 constexpr int kSlotBytes = 8192;
-constexpr int kSlots = 12;
+constexpr int kSlots = PROVIP_COMPACT_SLOTS;          // ring of shared-memory slots per CTA
+constexpr int kCtasPerSm = PROVIP_COMPACT_CTAS_PER_SM;
 constexpr int kCompactThreads = 128;
 constexpr size_t kCompactSmem = (size_t)kSlots * kSlotBytes;
 
@@ -80,6 +87,9 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(const CompactA
     fin[ph] = min(total, beg[ph] + per);
   }
 
+  // a kernel launched as this grid's programmatic dependent may start now (it
+  // waits for this grid's completion before touching anything written here)
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   if (blockIdx.x == 0 && a.seq_len_out != nullptr)
     for (int b = threadIdx.x; b < a.B; b += blockDim.x)
       a.seq_len_out[b] = a.seq_len[b] - a.N_v + a.keep;
@@ -211,7 +221,7 @@ cudaError_t compact_launch(const CompactArgs& a, int num_sms, cudaStream_t s, bo
   for (int t = 0; t < a.n_tensors; ++t)
     np[t] = (int)((a.row_bytes[t] + kSlotBytes - 1) / kSlotBytes);
   const long long total = (long long)a.B * a.L_out * (np[0] + np[1] + np[2]);
-  long long grid = 2LL * num_sms;
+  long long grid = (long long)kCtasPerSm * num_sms;
   if (grid > total) grid = total > 0 ? total : 1;
   cudaLaunchConfig_t cfg = {};
   cudaLaunchAttribute attr[1];

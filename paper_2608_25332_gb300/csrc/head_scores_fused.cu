@@ -293,6 +293,9 @@ __global__ void __launch_bounds__(kThreads, CPC == 1 ? 3 : (CPC == 2 ? 2 : 1))
     red[quad][col0 + cb * 32 + lane] = v[0];
   }
   __syncthreads();
+  // When launched as a programmatic dependent of the previous call's
+  // compaction, wait for it before overwriting the partials (a no-op otherwise).
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   if (good) {
     float* out = a.partial + ((size_t)b * a.n_rb * a.H_sel + (size_t)rb * a.H_sel + hi) * a.N_v;
     for (int c = threadIdx.x; c < (int)kCols; c += kThreads) {
@@ -317,7 +320,7 @@ FusedCfg g_cfg[64][3];
 
 template <int CPC>
 cudaError_t launch_cpc(const HSArgs& a, const CUtensorMap* tmQ, const CUtensorMap* tmK, int C,
-                       cudaStream_t s, bool* launched) {
+                       cudaStream_t s, bool* launched, bool pdl) {
   *launched = false;
   // dynamic shared memory large enough that (CTAs per SM) x (TMEM columns) <= 512
   constexpr int max_ctas = 512 / (CPC * kTile);
@@ -330,7 +333,7 @@ cudaError_t launch_cpc(const HSArgs& a, const CUtensorMap* tmQ, const CUtensorMa
   const int slot = CPC == 1 ? 0 : (CPC == 2 ? 1 : 2);
   FusedCfg& fc = g_cfg[dev < 64 ? dev : 0][slot];
   cudaLaunchConfig_t cfg = {};
-  cudaLaunchAttribute attr[2];
+  cudaLaunchAttribute attr[3];
   cfg.gridDim = dim3((unsigned)C, (unsigned)(a.H_sel * a.n_rb), (unsigned)a.B);
   cfg.blockDim = dim3(kThreads);
   cfg.dynamicSmemBytes = smem;
@@ -343,6 +346,8 @@ cudaError_t launch_cpc(const HSArgs& a, const CUtensorMap* tmQ, const CUtensorMa
   // policy spreads them one per SM, which caps the CTAs in flight at ~1 per SM)
   attr[1].id = cudaLaunchAttributeClusterSchedulingPolicyPreference;
   attr[1].val.clusterSchedulingPolicyPreference = cudaClusterSchedulingPolicyLoadBalancing;
+  attr[2].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[2].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 2;
   if (!fc.checked) {
@@ -371,6 +376,7 @@ cudaError_t launch_cpc(const HSArgs& a, const CUtensorMap* tmQ, const CUtensorMa
     fc.clusters_ok[C] = (q == cudaSuccess && nclusters >= 1) ? 1 : -1;
   }
   if (fc.clusters_ok[C] < 0) return cudaSuccess;
+  if (pdl) cfg.numAttrs = 3;
   cudaError_t e = cudaLaunchKernelEx(&cfg, hs_fused_tc<CPC>, a, *tmQ, *tmK);
   if (e == cudaSuccess) *launched = true;
   return e;
@@ -381,12 +387,12 @@ cudaError_t launch_cpc(const HSArgs& a, const CUtensorMap* tmQ, const CUtensorMa
 // One-pass head scores; *launched is false when no cluster shape fits (the
 // caller then runs the two-kernel path).
 cudaError_t hs_launch_fused(const HSArgs& a, const CUtensorMap* tmQ, const CUtensorMap* tmK,
-                            cudaStream_t s, bool* launched) {
+                            cudaStream_t s, bool* launched, bool pdl) {
   *launched = false;
   const int chunks = (a.L_max + kTile - 1) / kTile;
-  if (chunks <= 16) return launch_cpc<1>(a, tmQ, tmK, chunks, s, launched);
-  if (chunks <= 32) return launch_cpc<2>(a, tmQ, tmK, (chunks + 1) / 2, s, launched);
-  if (chunks <= 64) return launch_cpc<4>(a, tmQ, tmK, (chunks + 3) / 4, s, launched);
+  if (chunks <= 16) return launch_cpc<1>(a, tmQ, tmK, chunks, s, launched, pdl);
+  if (chunks <= 32) return launch_cpc<2>(a, tmQ, tmK, (chunks + 1) / 2, s, launched, pdl);
+  if (chunks <= 64) return launch_cpc<4>(a, tmQ, tmK, (chunks + 3) / 4, s, launched, pdl);
   return cudaSuccess;
 }
 

@@ -50,9 +50,11 @@ cudaError_t hs_launch_simt(const HSArgs& a, int dtype, cudaStream_t s);
 cudaError_t hs_launch_tc(const HSArgs& a, const CUtensorMap* tmQ, const CUtensorMap* tmK,
                          cudaStream_t s);
 // one-pass tcgen05 path (clusters, TMEM-resident logits): writes the partials
-// directly; *launched is false when no cluster shape fits this problem.
+// directly; *launched is false when no cluster shape fits this problem. pdl:
+// launched as a programmatic dependent of the previous kernel on the stream
+// (it reads Q/K at once and waits for that kernel only before writing).
 cudaError_t hs_launch_fused(const HSArgs& a, const CUtensorMap* tmQ, const CUtensorMap* tmK,
-                            cudaStream_t s, bool* launched);
+                            cudaStream_t s, bool* launched, bool pdl = false);
 // scores[b][i] = sum_u partial[b][u][i] / (H_sel * valid text rows of b)
 cudaError_t hs_launch_reduce(const HSArgs& a, float* scores, cudaStream_t s);
 

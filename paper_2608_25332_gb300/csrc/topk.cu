@@ -31,10 +31,12 @@ __device__ __forceinline__ int block_count_rows(const TopkArgs& a, int b) {
 __global__ void __launch_bounds__(kTopkMaxThreads) topk_kernel(const TopkArgs a) {
   extern __shared__ uint32_t keys[];
   __shared__ TopkShared sh;
-  // launched as a programmatic dependent: let the next kernel be scheduled,
-  // then wait until the kernel that writes the scores has completed
-  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  // launched as a programmatic dependent: wait until the kernel that writes the
+  // scores has completed, then let the next kernel (the compaction) start. The
+  // trigger comes after the wait so that a compaction never overlaps the
+  // previous call's compaction.
   asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   const int b = blockIdx.x;
   const int N = a.N;
   float* so = a.scores_out ? a.scores_out + (size_t)b * N : nullptr;

@@ -25,6 +25,7 @@ ERR_CUDA = -4
 ERR_TIMEOUT = -5
 F32, BF16 = 0, 1
 ALGO_AUTO, ALGO_SIMT, ALGO_TCGEN05, ALGO_TCGEN05_TWOPASS = 0, 1, 2, 3
+PRUNE_OVERLAP_PREVIOUS = 1
 
 _P = ctypes.c_void_p
 _I = ctypes.c_int
@@ -58,7 +59,7 @@ _SIGS = {
                               _P, _P, _P, _Z, _P]),
     "provip_prune_workspace_size": (_Z, [_I, _I, _I, _I, _I, _I, _I]),
     "provip_prune": (_I, [_P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _P, _I, _P, _P, _P, _I, _I, _I, _P, _P,
-                          _I, _I, _I, _I, _P, _P, _P, _P, _P, _P, _P, _P, _Z, _P]),
+                          _I, _I, _I, _I, _P, _P, _P, _P, _P, _P, _P, _P, _Z, ctypes.c_uint, _P]),
 }
 
 
@@ -300,11 +301,12 @@ class PruneStep:
     """Pre-allocated outputs + workspace for repeated provip_prune calls (one shape)."""
 
     def __init__(self, Q, K, V, hidden, pos, head_list, N_t_max, N_v, keep, algo=ALGO_AUTO,
-                 want_scores=True):
+                 want_scores=True, flags=0, ws=None):
         B, Lm, Hq, dh = Q.shape
         self.shape = (B, Lm, Hq, K.shape[2], dh, hidden.shape[2])
         self.heads, self.H_sel = _heads_arg(head_list)
         self.N_t_max, self.N_v, self.keep, self.algo = int(N_t_max), int(N_v), int(keep), algo
+        self.flags = int(flags)
         dev = Q.device
         self.dtype = _dtype_code(Q)
         L_out = Lm - N_v + keep
@@ -313,7 +315,7 @@ class PruneStep:
         self.seq_len_out = torch.empty(B, dtype=torch.int32, device=dev)
         self.scores = torch.empty((B, N_v), dtype=torch.float32, device=dev) if want_scores else None
         need = lib().provip_prune_workspace_size(B, Lm, self.H_sel, self.N_t_max, N_v, algo, self.dtype)
-        self.ws = workspace(need, dev)
+        self.ws = ws if ws is not None and ws.numel() >= need else workspace(need, dev)
 
     def __call__(self, Q, K, V, hidden, pos, text_start, text_len, seq_len, vis_start,
                  row_mask=None, stream=None):
@@ -326,7 +328,7 @@ class PruneStep:
                                 _i32(pos), P, self.keep, self.dtype, self.algo, _ptr(self.hidden_out),
                                 _ptr(self.K_out), _ptr(self.V_out), _i32(self.pos_out),
                                 _ptr(self.idx), _i32(self.seq_len_out), _ptr(self.scores),
-                                _ptr(self.ws), self.ws.numel(), st)
+                                _ptr(self.ws), self.ws.numel(), self.flags, st)
         _check(rc, "provip_prune")
         return dict(hidden=self.hidden_out, K=self.K_out, V=self.V_out, pos=self.pos_out,
                     idx=self.idx, seq_len=self.seq_len_out, scores=self.scores)

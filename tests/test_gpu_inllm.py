@@ -123,6 +123,34 @@ def test_fused_and_standalone_scores_are_identical():
     assert torch.equal(idx2, out["idx"])
 
 
+def test_overlapped_calls_match_serial_calls():
+    """PROVIP_PRUNE_OVERLAP_PREVIOUS: back-to-back calls on three different batches
+    sharing one workspace give the same bits as calls separated by a sync."""
+    name = "llava_next_7b_bf16_b8"
+    w, cpu, g0 = inputs(name)
+    batches = [g0] + [{k: (v.to(DEV) if isinstance(v, torch.Tensor) else v)
+                       for k, v in synth.in_llm_inputs(w, seed=w.seed + 77 + i).items()} for i in range(2)]
+    ws = P.workspace(P.lib().provip_prune_workspace_size(w.B, w.L_max, w.H_sel, w.n_t[1], w.keep_pre,
+                                                         P.ALGO_AUTO, P.BF16), DEV)
+    def run(flags, sync):
+        outs = []
+        for c in batches:
+            st = P.PruneStep(c["Q"], c["K"], c["V"], c["hidden"], c["pos"], c["head_list"], w.n_t[1], c["N_v"],
+                             c["keep"], flags=flags, ws=ws)
+            outs.append(st(c["Q"], c["K"], c["V"], c["hidden"], c["pos"], c["text_start"], c["text_len"],
+                           c["seq_len"], c["vis_start"]))
+            if sync:
+                torch.cuda.synchronize()
+        torch.cuda.synchronize()
+        return [{k: v.clone() for k, v in o.items() if v is not None} for o in outs]
+    serial = run(0, True)
+    for rep in range(3):
+        over = run(P.PRUNE_OVERLAP_PREVIOUS, False)
+        for a, b in zip(serial, over):
+            for k in a:
+                assert torch.equal(a[k], b[k]), f"overlapped call differs in {k} (rep {rep})"
+
+
 def _small_case(seed, B=3, Hq=6, Hkv=2, nsys=5, nv=37, tls=(1, 9, 130), dtype=torch.bfloat16):
     """ragged: 37 visual columns, a one-row sample and a 130-row sample (two row blocks)."""
     rng = np.random.default_rng(seed)
