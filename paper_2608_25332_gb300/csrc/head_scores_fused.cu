@@ -293,9 +293,6 @@ __global__ void __launch_bounds__(kThreads, CPC == 1 ? 3 : (CPC == 2 ? 2 : 1))
     red[quad][col0 + cb * 32 + lane] = v[0];
   }
   __syncthreads();
-  // When launched as a programmatic dependent of the previous call's
-  // compaction, wait for it before overwriting the partials (a no-op otherwise).
-  asm volatile("griddepcontrol.wait;" ::: "memory");
   if (good) {
     float* out = a.partial + ((size_t)b * a.n_rb * a.H_sel + (size_t)rb * a.H_sel + hi) * a.N_v;
     for (int c = threadIdx.x; c < (int)kCols; c += kThreads) {
@@ -308,7 +305,14 @@ __global__ void __launch_bounds__(kThreads, CPC == 1 ? 3 : (CPC == 2 ? 2 : 1))
   __syncthreads();
   if (threadIdx.x < 32) tmem_dealloc(ctl.tmem, kCols);
   cluster_wait();  // every peer has read this CTA's rowstat
-
+  // When this grid is a programmatic dependent of the previous call's
+  // compaction (independent batches), one CTA waits for that kernel before
+  // exiting, so that this grid - and therefore the top-k that follows it and
+  // rewrites idx - completes only after the compaction has read idx. The
+  // partials need no such wait: the previous top-k has loaded them before the
+  // compaction could start. A no-op without a programmatic dependency.
+  if (blockIdx.x == 0 && blockIdx.y == 0 && blockIdx.z == 0)
+    asm volatile("griddepcontrol.wait;" ::: "memory");
 }
 
 struct FusedCfg {

@@ -32,11 +32,9 @@ __global__ void __launch_bounds__(kTopkMaxThreads) topk_kernel(const TopkArgs a)
   extern __shared__ uint32_t keys[];
   __shared__ TopkShared sh;
   // launched as a programmatic dependent: wait until the kernel that writes the
-  // scores has completed, then let the next kernel (the compaction) start. The
-  // trigger comes after the wait so that a compaction never overlaps the
-  // previous call's compaction.
+  // scores has completed (which, for overlapped calls, implies the previous
+  // compaction has completed too)
   asm volatile("griddepcontrol.wait;" ::: "memory");
-  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   const int b = blockIdx.x;
   const int N = a.N;
   float* so = a.scores_out ? a.scores_out + (size_t)b * N : nullptr;
@@ -52,6 +50,10 @@ __global__ void __launch_bounds__(kTopkMaxThreads) topk_kernel(const TopkArgs a)
     }
   }
   __syncthreads();
+  // The scores are in shared memory now: the next kernel (the compaction, and
+  // through it the next call's head scores, which rewrite the partials) may
+  // start. idx is only read by the compaction after this grid completes.
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   topk_block_select(keys, N, a.k, a.idx_out + (size_t)b * a.k, sh);
 }
 
