@@ -130,6 +130,53 @@ def hbm_peak():
         return FALLBACK_HBM_GBS, "fallback"
 
 
+def bf16_peak():
+    """burst figure: the pre-LLM kernels are timed alone"""
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            return float(json.load(f)["bf16_tflops"]), "measured"
+    except Exception:
+        return 1900.0, "fallback"
+
+
+def prellm_measure(w, dev, reps=20):
+    """The pre-LLM pass (Sec. 4.2-4.3) on the same workload: the whole
+    provip_similarity_reduce call, and the nearest-centroid assignment alone
+    (provip_merge without the mean), whose pruned x kept Gram is the pass's
+    dominant contraction T_RT = 2 d (N_v - N1) N1."""
+    import torch
+    from paper_2608_25332_gb300 import provip as P
+    from paper_2608_25332_gb300 import synth
+    g = {k: v.to(dev) for k, v in synth.pre_llm_inputs(w).items()}
+    ws = P.workspace(P.lib().provip_similarity_reduce_workspace_size(w.B, w.N_v, w.D, w.n_t[1], w.keep_pre), dev)
+    full = lambda: P.provip_similarity_reduce(g["emb_v"], g["emb_t"], g["text_len"], w.keep_pre, ws=ws)
+    idx = full()["idx"]
+    assign_only = lambda: P.provip_merge(g["emb_v"], idx, want_merged=False)
+
+    def t(f):
+        for _ in range(3):
+            f()
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        for _ in range(reps):
+            f()
+        b.record()
+        torch.cuda.synchronize()
+        return a.elapsed_time(b) / reps * 1e3
+
+    us_full, us_assign = t(full), t(assign_only)
+    flops = 2.0 * w.D * (w.N_v - w.keep_pre) * w.keep_pre * w.B
+    peak, src = bf16_peak()
+    ach = flops / us_assign / 1e6
+    return {"workload": w.name, "us_per_call": us_full, "samples_per_s": w.B / us_full * 1e6,
+            "assign_us": us_assign, "assign_gram_flops": flops,
+            "tensor_roofline": {"bound": "tensor", "kernel": "merge_argmax_tc (timed with its gather, "
+                                "norm and assignment kernels)", "achieved": ach, "peak": peak,
+                                "peak_source": src, "unit": "TFLOP/s", "frac": ach / peak}}
+
+
 class ClockSampler:
     FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
@@ -508,6 +555,8 @@ def run_gb300(args, dist):
     e2e_sec = dist.max(a.elapsed_time(b) / 1e3)
     e2e_value = aggregate(dist.sum(float(w.B * E)), e2e_sec)
 
+    prellm = prellm_measure(w, dev) if dist.rank == 0 else None
+
     cpu_base = None
     if dist.rank == 0 and dist.world == 1 and not args.no_cpu_baseline:
         cpu_base = cpu_baseline(cpu, w, vis, nv, keep)
@@ -536,6 +585,7 @@ def run_gb300(args, dist):
             "cpu_baseline": cpu_base,
             "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
             "gpu_launches": launches_per_step * K,
+            "prellm": prellm,
             "clocks": clocks,
         }
         print(json.dumps(line))

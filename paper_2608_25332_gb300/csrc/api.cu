@@ -267,6 +267,11 @@ int merge_splits(int B, int N_v, int keep) {
   if (n > 16) n = 16;
   return n < 1 ? 1 : n;
 }
+// rows of the per-split argmax workspace: enough for either merge path
+int merge_ws_splits(int B, int N_v, int keep) {
+  const int a = merge_splits(B, N_v, keep);
+  return a > kMergeMaxSplit ? a : kMergeMaxSplit;
+}
 
 struct SimWs {
   float* G = nullptr;
@@ -279,6 +284,8 @@ struct SimWs {
   float* best = nullptr;
   int* bidx = nullptr;
   int* assign = nullptr;
+  int* pruned = nullptr;
+  void* perm = nullptr;
 };
 
 int sim_validate_common(const void* emb, int B, int N, int D, int dtype, const char* what) {
@@ -435,19 +442,20 @@ extern "C" int provip_topk(const float* scores, int B, int N, int k, int* idx_ou
   return e == cudaSuccess ? PROVIP_OK : cuda_fail(e, "topk launch");
 }
 
-static size_t merge_ws(Carve& c, int B, int N_v, int keep, SimWs& w) {
-  const int ns = merge_splits(B, N_v, keep);
+static size_t merge_ws(Carve& c, int B, int N_v, int D, int keep, SimWs& w) {
+  const int ns = merge_ws_splits(B, N_v, keep);
   w.inv_v = c.take<float>((size_t)B * N_v);
   w.best = c.take<float>((size_t)ns * B * N_v);
   w.bidx = c.take<int>((size_t)ns * B * N_v);
+  w.pruned = c.take<int>((size_t)B * N_v);
+  w.perm = c.take<uint16_t>((size_t)B * N_v * D);
   return c.off;
 }
 
 extern "C" size_t provip_merge_workspace_size(int B, int N_v, int D, int keep) {
-  (void)D;
   Carve c(nullptr);
   SimWs w;
-  return merge_ws(c, B, N_v, keep, w);
+  return merge_ws(c, B, N_v, D, keep, w);
 }
 
 static int merge_validate(const void* emb_v, int B, int N_v, int D, const int* keep_idx, int keep,
@@ -470,13 +478,14 @@ extern "C" int provip_merge(const void* emb_v, int B, int N_v, int D, const int*
   if ((rc = dev_info(&d))) return rc;
   Carve c(ws);
   SimWs w;
-  merge_ws(c, B, N_v, keep, w);
+  merge_ws(c, B, N_v, D, keep, w);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   SimArgs a = sim_args(emb_v, nullptr, nullptr, B, N_v, D, 1, dtype, d->status);
   cudaError_t e = vis_inv_norm_launch(a, w.inv_v, s);
   if (e == cudaSuccess)
     e = merge_launch(a, keep_idx, keep, w.inv_v, assign_out, merged_out, w.best, w.bidx,
-                     merge_splits(B, N_v, keep), s);
+                     merge_splits(B, N_v, keep), w.pruned, dtype == PROVIP_BF16 ? w.perm : nullptr,
+                     d->sms, s);
   return e == cudaSuccess ? PROVIP_OK : cuda_fail(e, "merge launch");
 }
 
@@ -487,13 +496,15 @@ static size_t simred_ws(Carve& c, int B, int N_v, int D, int N_t_max, int keep_p
   w.assign = c.take<int>((size_t)B * N_v);
   SimWs r, m;
   relevance_ws(c, B, N_v, D, N_t_max, r);
-  const int ns = merge_splits(B, N_v, keep_pre);
+  const int ns = merge_ws_splits(B, N_v, keep_pre);
   w.inv_v = r.inv_v;
   w.sum = r.sum;
   w.mu = r.mu;
   w.invt = r.invt;
   w.best = c.take<float>((size_t)ns * B * N_v);
   w.bidx = c.take<int>((size_t)ns * B * N_v);
+  w.pruned = c.take<int>((size_t)B * N_v);
+  w.perm = c.take<uint16_t>((size_t)B * N_v * D);
   (void)m;
   return c.off;
 }
@@ -554,7 +565,8 @@ extern "C" int provip_similarity_reduce(const void* emb_v, int B, int N_v, int D
   }
   if (e == cudaSuccess && merged_out_or_null)
     e = merge_launch(a, idx_out, keep_pre, w.inv_v, w.assign, merged_out_or_null, w.best, w.bidx,
-                     merge_splits(B, N_v, keep_pre), s);
+                     merge_splits(B, N_v, keep_pre), w.pruned,
+                     dtype == PROVIP_BF16 ? w.perm : nullptr, d->sms, s);
   return e == cudaSuccess ? PROVIP_OK : cuda_fail(e, "similarity_reduce launch");
 }
 

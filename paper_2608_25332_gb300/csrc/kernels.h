@@ -122,9 +122,26 @@ cudaError_t relevance_launch(const SimArgs& a, const uint8_t* mask, const float*
                              float* p, float* ws_sum, float* ws_mu, float* ws_invt,
                              int n_split, cudaStream_t s);
 // Sec. 4.3 merge: assign[b][j] and merged[b][a][:]
+// n_split: the SIMT split (sized by the caller); ws_pruned: [B][N_v] ints and
+// ws_perm: [B][N_v][D] bf16 for the tcgen05 path (null: CUDA-core path);
+// num_sms for its split choice
 cudaError_t merge_launch(const SimArgs& a, const int* keep_idx, int keep, const float* inv_v,
                          int* assign, void* merged, float* ws_best, int* ws_bidx,
-                         int n_split, cudaStream_t s);
+                         int n_split, int* ws_pruned, void* ws_perm, int num_sms, cudaStream_t s);
+
+// tcgen05 forms of the pre-LLM Grams (bf16), used by the launchers above
+bool crit_gram_tc_supported(const SimArgs& a);
+cudaError_t crit_gram_tc_launch(const SimArgs& a, float* G, cudaStream_t s);
+bool relevance_tc_supported(const SimArgs& a);
+cudaError_t relevance_tc_launch(const SimArgs& a, const uint8_t* mask, const float* inv_v,
+                                const float* mu, const float* invt, float* p, cudaStream_t s);
+bool merge_tc_supported(const SimArgs& a, int keep, int n_split);
+cudaError_t merge_argmax_tc_launch(const SimArgs& a, const int* keep_idx, int keep,
+                                   const float* inv_v, const int* kpos, int* pruned, void* perm,
+                                   int n_split, float* ws_best, int* ws_bidx, cudaStream_t s);
+// N split of the tcgen05 merge Gram (fewest waves x tiles per CTA) and its upper bound
+int merge_tc_split(int B, int N_v, int keep, int num_sms);
+constexpr int kMergeMaxSplit = 16;
 
 // host helper: encode a 2-D bf16 row table [rows, cols] (row stride in bytes)
 // as a tensor map with 64 x box_rows boxes and 128-byte swizzle.

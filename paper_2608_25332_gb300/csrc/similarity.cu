@@ -139,6 +139,7 @@ __global__ void __launch_bounds__(256) inv_norm_kernel(const void* X, size_t row
 // Sec. 4.3 relevance
 // ---------------------------------------------------------------------------
 // partial sums of normalised visual rows: part[z][b][d] over rows z*chunk..
+// (8 rows in flight per step; the adds stay in row order)
 template <typename T>
 __global__ void __launch_bounds__(256) vis_sum_kernel(const SimArgs a, const float* inv_v,
                                                       float* part, int chunk) {
@@ -147,8 +148,20 @@ __global__ void __launch_bounds__(256) vis_sum_kernel(const SimArgs a, const flo
   if (d >= a.D) return;
   const int j0 = z * chunk, j1 = min(a.N_v, j0 + chunk);
   const T* E = static_cast<const T*>(a.emb_v) + (size_t)b * a.N_v * a.D;
+  const float* iv = inv_v + (size_t)b * a.N_v;
   float s = 0.f;
-  for (int j = j0; j < j1; ++j) s = fmaf(to_f32(E[(size_t)j * a.D + d]), inv_v[(size_t)b * a.N_v + j], s);
+  int j = j0;
+  for (; j + 8 <= j1; j += 8) {
+    float x[8], w[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      x[u] = to_f32(E[(size_t)(j + u) * a.D + d]);
+      w[u] = iv[j + u];
+    }
+#pragma unroll
+    for (int u = 0; u < 8; ++u) s = fmaf(x[u], w[u], s);
+  }
+  for (; j < j1; ++j) s = fmaf(to_f32(E[(size_t)j * a.D + d]), iv[j], s);
   part[((size_t)z * a.B + b) * a.D + d] = s;
 }
 
@@ -163,7 +176,7 @@ __global__ void __launch_bounds__(256) vis_sum_reduce_kernel(const SimArgs a, co
   sum[(size_t)b * a.D + d] = s;
 }
 
-// mu_i and 1/|t_i| for the text rows (one warp per row)
+// mu_i and 1/|t_i| for the text rows (one warp per row, 8 elements per lane step)
 template <typename T>
 __global__ void __launch_bounds__(256) text_mu_kernel(const SimArgs a, const float* sum,
                                                       float* mu, float* invt) {
@@ -180,11 +193,19 @@ __global__ void __launch_bounds__(256) text_mu_kernel(const SimArgs a, const flo
     return;
   }
   const T* t = static_cast<const T*>(a.emb_t) + ((size_t)b * a.N_t_max + i) * a.D;
+  const float* sv = sum + (size_t)b * a.D;
   float ss = 0.f, dt = 0.f;
-  for (int d = lane; d < a.D; d += 32) {
-    const float x = to_f32(t[d]);
-    ss = fmaf(x, x, ss);
-    dt = fmaf(x, sum[(size_t)b * a.D + d], dt);
+  for (int d = lane * 8; d < a.D; d += 256) {
+    float x[8];
+    load8(t + d, x);
+    const float4 s0 = *reinterpret_cast<const float4*>(sv + d);
+    const float4 s1 = *reinterpret_cast<const float4*>(sv + d + 4);
+    const float sw[8] = {s0.x, s0.y, s0.z, s0.w, s1.x, s1.y, s1.z, s1.w};
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+      ss = fmaf(x[q], x[q], ss);
+      dt = fmaf(x[q], sw[q], dt);
+    }
   }
   ss = warp_sum(ss);
   dt = warp_sum(dt);
@@ -379,52 +400,163 @@ __global__ void merge_assign_kernel(const SimArgs a, const int* kpos, int n_spli
   assign[i] = bi == 0x7fffffff ? 0 : bi;
 }
 
-// merged[b][a] = (sum of rows j with assign[b][j] == a, ascending j) / count
+// merged[b][a] = (sum of rows j with assign[b][j] == a, ascending j) / count.
+// The member lists come from a counting sort per sample: counts (atomics),
+// exclusive offsets, unordered fill; each kept row's CTA then orders its
+// members by rank (ascending row index, so the sum order is fixed) and sums
+// them with four member rows in flight. A centroid with more members than the
+// sort buffer falls back to scanning assign in windows.
+constexpr int kMeanThreads = 256;
+constexpr int kMeanSort = 1024;
+
+__global__ void merge_count_kernel(const int* assign, int B, int N_v, int keep, int* count) {
+  const size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= (size_t)B * N_v) return;
+  const int b = (int)(i / N_v);
+  const int ap = assign[i];
+  if (ap >= 0 && ap < keep) atomicAdd(&count[(size_t)b * keep + ap], 1);
+}
+
+// exclusive scan of count[b][0..keep) -> offset[b][..], cursor[b][..] = 0
+__global__ void __launch_bounds__(1024) merge_offsets_kernel(const int* count, int keep, int* offset,
+                                                              int* cursor) {
+  __shared__ uint32_t warp_tot[32];
+  __shared__ uint32_t carry;
+  const int b = blockIdx.x;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  if (threadIdx.x == 0) carry = 0;
+  __syncthreads();
+  for (int a0 = 0; a0 < keep; a0 += 1024) {
+    const int ap = a0 + threadIdx.x;
+    const uint32_t v = ap < keep ? (uint32_t)count[(size_t)b * keep + ap] : 0u;
+    uint32_t incl = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const uint32_t y = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += y;
+    }
+    if (lane == 31) warp_tot[warp] = incl;
+    __syncthreads();
+    if (warp == 0) {
+      const uint32_t t = warp_tot[lane];
+      uint32_t ti = t;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t y = __shfl_up_sync(0xffffffffu, ti, o);
+        if (lane >= o) ti += y;
+      }
+      warp_tot[lane] = ti - t;
+    }
+    __syncthreads();
+    if (ap < keep) {
+      offset[(size_t)b * keep + ap] = (int)(carry + warp_tot[warp] + incl - v);
+      cursor[(size_t)b * keep + ap] = 0;
+    }
+    __syncthreads();
+    if (threadIdx.x == 1023) carry += warp_tot[31] + incl;
+    __syncthreads();
+  }
+}
+
+__global__ void merge_fill_kernel(const int* assign, int B, int N_v, int keep, const int* offset,
+                                  int* cursor, int* members) {
+  const size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= (size_t)B * N_v) return;
+  const int b = (int)(i / N_v), j = (int)(i - (size_t)b * N_v);
+  const int ap = assign[i];
+  if (ap < 0 || ap >= keep) return;
+  const size_t k = (size_t)b * keep + ap;
+  members[(size_t)b * N_v + offset[k] + atomicAdd(&cursor[k], 1)] = j;
+}
+
 template <typename T, typename Acc>
-__global__ void __launch_bounds__(256) merge_mean_kernel(const SimArgs a, const int* assign,
-                                                         int keep, void* merged) {
-  __shared__ int members[256];
-  __shared__ int wcount[8];
+__global__ void __launch_bounds__(kMeanThreads) merge_mean_kernel(const SimArgs a, const int* assign,
+                                                                  const int* count, const int* offset,
+                                                                  const int* members_all, int keep,
+                                                                  void* merged) {
+  __shared__ int members[kMeanSort];
+  __shared__ int unsorted[kMeanSort];
   const int ap = blockIdx.x, b = blockIdx.y;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const T* E = static_cast<const T*>(a.emb_v) + (size_t)b * a.N_v * a.D;
-  const int* as = assign + (size_t)b * a.N_v;
-  // each thread owns columns threadIdx.x + 256 q
+  T* out = static_cast<T*>(merged) + ((size_t)b * keep + ap) * a.D;
   constexpr int kMaxQ = 32;  // D <= 8192
   Acc acc[kMaxQ];
 #pragma unroll
   for (int q = 0; q < kMaxQ; ++q) acc[q] = Acc(0);
-  int count = 0;
-  for (int j0 = 0; j0 < a.N_v; j0 += 256) {
-    const int j = j0 + threadIdx.x;
-    const bool hit = j < a.N_v && as[j] == ap;
-    const unsigned bal = __ballot_sync(0xffffffffu, hit);
-    if (lane == 0) wcount[warp] = __popc(bal);
-    __syncthreads();
-    int off = 0, tot = 0;
-    for (int w = 0; w < 8; ++w) {
-      if (w < warp) off += wcount[w];
-      tot += wcount[w];
-    }
-    if (hit) members[off + __popc(bal & ((1u << lane) - 1u))] = j;
-    __syncthreads();
-    for (int m = 0; m < tot; ++m) {
-      const T* row = E + (size_t)members[m] * a.D;
+  const int n_all = count[(size_t)b * keep + ap];
+  auto add_rows = [&](int n) {
+    int m = 0;
+    for (; m + 4 <= n; m += 4) {
+      const T* r0 = E + (size_t)members[m] * a.D;
+      const T* r1 = E + (size_t)members[m + 1] * a.D;
+      const T* r2 = E + (size_t)members[m + 2] * a.D;
+      const T* r3 = E + (size_t)members[m + 3] * a.D;
 #pragma unroll
       for (int q = 0; q < kMaxQ; ++q) {
-        const int d = threadIdx.x + 256 * q;
-        if (d < a.D) acc[q] += (Acc)to_f32(row[d]);
+        const int d = threadIdx.x + kMeanThreads * q;
+        if (d < a.D) {
+          const float x0 = to_f32(r0[d]), x1 = to_f32(r1[d]), x2 = to_f32(r2[d]), x3 = to_f32(r3[d]);
+          acc[q] += (Acc)x0;
+          acc[q] += (Acc)x1;
+          acc[q] += (Acc)x2;
+          acc[q] += (Acc)x3;
+        }
       }
     }
-    count += tot;
+    for (; m < n; ++m) {
+      const T* r0 = E + (size_t)members[m] * a.D;
+#pragma unroll
+      for (int q = 0; q < kMaxQ; ++q) {
+        const int d = threadIdx.x + kMeanThreads * q;
+        if (d < a.D) acc[q] += (Acc)to_f32(r0[d]);
+      }
+    }
+  };
+  if (n_all <= kMeanSort) {
+    const int* src = members_all + (size_t)b * a.N_v + offset[(size_t)b * keep + ap];
+    for (int m = threadIdx.x; m < n_all; m += kMeanThreads) unsorted[m] = src[m];
     __syncthreads();
+    // rank = number of smaller row indices (they are distinct)
+    for (int m = threadIdx.x; m < n_all; m += kMeanThreads) {
+      const int v = unsorted[m];
+      int rank = 0;
+      for (int q = 0; q < n_all; ++q) rank += unsorted[q] < v;
+      members[rank] = v;
+    }
+    __syncthreads();
+    add_rows(n_all);
+  } else {
+    // many members: scan assign in windows, members in ascending order
+    const int* as = assign + (size_t)b * a.N_v;
+    __shared__ int wcount[kMeanThreads / 32];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    int base = 0;
+    for (int j0 = 0; j0 < a.N_v; j0 += kMeanThreads) {
+      const int j = j0 + threadIdx.x;
+      const bool hit = j < a.N_v && as[j] == ap;
+      const unsigned bal = __ballot_sync(0xffffffffu, hit);
+      if (lane == 0) wcount[warp] = __popc(bal);
+      __syncthreads();
+      int off = 0, tot = 0;
+      for (int w = 0; w < kMeanThreads / 32; ++w) {
+        off += w < warp ? wcount[w] : 0;
+        tot += wcount[w];
+      }
+      if (hit) members[base + off + __popc(bal & ((1u << lane) - 1u))] = j;
+      __syncthreads();
+      base += tot;
+      if (base > kMeanSort - kMeanThreads || j0 + kMeanThreads >= a.N_v) {
+        add_rows(base);
+        __syncthreads();
+        base = 0;
+      }
+    }
   }
-  T* out = static_cast<T*>(merged) + ((size_t)b * keep + ap) * a.D;
 #pragma unroll
   for (int q = 0; q < kMaxQ; ++q) {
-    const int d = threadIdx.x + 256 * q;
+    const int d = threadIdx.x + kMeanThreads * q;
     if (d < a.D) {
-      const Acc v = count > 0 ? acc[q] / (Acc)count : Acc(0);
+      const Acc v = n_all > 0 ? acc[q] / (Acc)n_all : Acc(0);
       if constexpr (sizeof(T) == 4)
         out[d] = (T)v;
       else
@@ -438,10 +570,14 @@ __global__ void __launch_bounds__(256) merge_mean_kernel(const SimArgs a, const 
 cudaError_t crit_text_launch(const SimArgs& a, uint8_t* mask, float* r_out, float* G,
                              cudaStream_t s) {
   dim3 g((a.N_t_max + kSimtBN - 1) / kSimtBN, (a.N_t_max + kSimtBM - 1) / kSimtBM, a.B);
-  if (a.dtype == 0)
+  if (a.dtype == 0) {
     crit_gram_kernel<float><<<g, 256, 0, s>>>(a, G);
-  else
+  } else if (crit_gram_tc_supported(a)) {
+    cudaError_t e = crit_gram_tc_launch(a, G, s);
+    if (e != cudaSuccess) return e;
+  } else {
     crit_gram_kernel<__nv_bfloat16><<<g, 256, 0, s>>>(a, G);
+  }
   crit_finish_kernel<<<a.B, 256, 3 * a.N_t_max * sizeof(float), s>>>(a, G, mask, r_out);
   return cudaGetLastError();
 }
@@ -475,6 +611,11 @@ cudaError_t relevance_launch(const SimArgs& a, const uint8_t* mask, const float*
     vis_sum_kernel<__nv_bfloat16><<<g1, 256, 0, s>>>(a, inv_v, ws_sum, chunk);
     vis_sum_reduce_kernel<<<g4, 256, 0, s>>>(a, ws_sum, n_split, total);
     text_mu_kernel<__nv_bfloat16><<<g2, 256, 0, s>>>(a, total, ws_mu, ws_invt);
+    if (relevance_tc_supported(a)) {
+      cudaError_t e = cudaGetLastError();
+      if (e != cudaSuccess) return e;
+      return relevance_tc_launch(a, mask, inv_v, ws_mu, ws_invt, p, s);
+    }
     relevance_kernel<__nv_bfloat16><<<g3, 256, 0, s>>>(a, mask, inv_v, ws_mu, ws_invt, p);
   }
   return cudaGetLastError();
@@ -482,7 +623,7 @@ cudaError_t relevance_launch(const SimArgs& a, const uint8_t* mask, const float*
 
 cudaError_t merge_launch(const SimArgs& a, const int* keep_idx, int keep, const float* inv_v,
                          int* assign, void* merged, float* ws_best, int* ws_bidx, int n_split,
-                         cudaStream_t s) {
+                         int* ws_pruned, void* ws_perm, int num_sms, cudaStream_t s) {
   // kpos lives in `assign` until the final assignment overwrites it: it is
   // read by merge_argmax_kernel and merge_assign_kernel (same index only).
   int* kpos = assign;
@@ -490,18 +631,38 @@ cudaError_t merge_launch(const SimArgs& a, const int* keep_idx, int keep, const 
   keep_pos_kernel<<<(unsigned)((nb + 255) / 256), 256, 0, s>>>(keep_idx, keep, a.B, a.N_v, kpos, a.err);
   const size_t nk = (size_t)a.B * keep;
   keep_scatter_kernel<<<(unsigned)((nk + 255) / 256), 256, 0, s>>>(keep_idx, keep, a.B, a.N_v, kpos, a.err);
-  dim3 g((a.N_v + kSimtBM - 1) / kSimtBM, a.B, n_split);
-  if (a.dtype == 0)
-    merge_argmax_kernel<float><<<g, 256, 0, s>>>(a, keep_idx, keep, inv_v, kpos, n_split, ws_best, ws_bidx);
-  else
-    merge_argmax_kernel<__nv_bfloat16><<<g, 256, 0, s>>>(a, keep_idx, keep, inv_v, kpos, n_split, ws_best, ws_bidx);
+  const int tc_split = merge_tc_split(a.B, a.N_v, keep, num_sms);
+  if (ws_pruned != nullptr && ws_perm != nullptr && merge_tc_supported(a, keep, tc_split)) {
+    cudaError_t e = merge_argmax_tc_launch(a, keep_idx, keep, inv_v, kpos, ws_pruned, ws_perm, tc_split,
+                                           ws_best, ws_bidx, s);
+    if (e != cudaSuccess) return e;
+    n_split = tc_split;
+  } else {
+    dim3 g((a.N_v + kSimtBM - 1) / kSimtBM, a.B, n_split);
+    if (a.dtype == 0)
+      merge_argmax_kernel<float><<<g, 256, 0, s>>>(a, keep_idx, keep, inv_v, kpos, n_split, ws_best, ws_bidx);
+    else
+      merge_argmax_kernel<__nv_bfloat16><<<g, 256, 0, s>>>(a, keep_idx, keep, inv_v, kpos, n_split, ws_best,
+                                                           ws_bidx);
+  }
   merge_assign_kernel<<<(unsigned)((nb + 255) / 256), 256, 0, s>>>(a, kpos, n_split, ws_best, ws_bidx, assign);
   if (merged != nullptr) {
+    // counting sort of the rows by centroid; the scratch reuses ws_best/ws_bidx
+    // (the argmax partials are consumed by merge_assign_kernel above)
+    int* cnt = ws_bidx;
+    int* off = cnt + (size_t)a.B * keep;
+    int* cur = off + (size_t)a.B * keep;
+    int* mem = reinterpret_cast<int*>(ws_best);
+    cudaMemsetAsync(cnt, 0, (size_t)a.B * keep * sizeof(int), s);
+    merge_count_kernel<<<(unsigned)((nb + 255) / 256), 256, 0, s>>>(assign, a.B, a.N_v, keep, cnt);
+    merge_offsets_kernel<<<a.B, 1024, 0, s>>>(cnt, keep, off, cur);
+    merge_fill_kernel<<<(unsigned)((nb + 255) / 256), 256, 0, s>>>(assign, a.B, a.N_v, keep, off, cur, mem);
     dim3 gm(keep, a.B);
     if (a.dtype == 0)
-      merge_mean_kernel<float, double><<<gm, 256, 0, s>>>(a, assign, keep, merged);
+      merge_mean_kernel<float, double><<<gm, kMeanThreads, 0, s>>>(a, assign, cnt, off, mem, keep, merged);
     else
-      merge_mean_kernel<__nv_bfloat16, float><<<gm, 256, 0, s>>>(a, assign, keep, merged);
+      merge_mean_kernel<__nv_bfloat16, float><<<gm, kMeanThreads, 0, s>>>(a, assign, cnt, off, mem, keep,
+                                                                          merged);
   }
   return cudaGetLastError();
 }

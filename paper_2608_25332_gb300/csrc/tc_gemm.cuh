@@ -1,0 +1,159 @@
+// Warp-specialised tcgen05 "NT" Gram core for the pre-LLM pass (Sec. 4.3):
+//   D[M x N] = A[M x K] * B[N x K]^T, bf16 operands, fp32 accumulation in TMEM,
+// with A and B rows fetched by 2-D TMA (128-byte swizzle), either as a block of
+// consecutive rows or gathered by row index with tile::gather4 (boxes one row
+// high, four rows per instruction).
+//
+// One CTA owns one 128-row M tile and sweeps a range of BN-column N tiles
+// (BN = 128 or 256):
+//   warp 0 (one lane)  TMA producer: K slices of 64 elements, kStages-deep ring
+//                      of shared-memory stages (A 16 KiB + B BN x 128 B each);
+//   warp 1 (one lane)  MMA issuer: 4 x tcgen05.mma (M=128, N=BN, K=16) per
+//                      stage, tcgen05.commit frees the stage, and a commit per
+//                      N tile hands the accumulator to the epilogue;
+//   warps 2-5          epilogue: thread = TMEM lane = row of the M tile; two
+//                      BN-column accumulators alternate so that the epilogue
+//                      of tile n overlaps the main loop of tile n + 1.
+// Every mbarrier wait is bounded (mbar_wait); a timeout marks the CTA failed,
+// and the roles drain and exit.
+#pragma once
+
+#include "common.cuh"
+
+namespace provip {
+namespace tcg {
+
+constexpr int kBM = 128;
+constexpr int kBK = 64;                      // bf16 elements per stage row (128 B)
+constexpr int kStages = 4;
+constexpr int kABytes = kBM * kBK * 2;       // 16 KiB
+constexpr int kThreads = 192;                // 6 warps
+
+// per N-tile width (128 or 256)
+template <int BN>
+struct Cfg {
+  static constexpr int kBBytes = BN * kBK * 2;
+  static constexpr int kStageBytes = kABytes + kBBytes;
+  static constexpr uint32_t kIdesc = idesc_bf16_f32(kBM, BN);
+  static constexpr size_t kStagesBytes = (size_t)kStages * kStageBytes;
+  static constexpr uint32_t kTmemCols = 2 * BN;  // two accumulators
+};
+
+__device__ __forceinline__ void tma_gather4(void* smem_dst, const CUtensorMap* map, int x, int r0,
+                                            int r1, int r2, int r3, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile::gather4.mbarrier::complete_tx::bytes "
+      "[%0], [%1, {%2, %3, %4, %5, %6}], [%7];" ::"r"(smem_u32(smem_dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(r0), "r"(r1), "r"(r2), "r"(r3),
+      "r"(smem_u32(bar))
+      : "memory");
+}
+
+struct Pipe {
+  uint64_t full[kStages];
+  uint64_t empty[kStages];
+  uint64_t acc_full[2];
+  uint64_t acc_empty[2];
+  uint32_t tmem;
+  volatile int fail;
+};
+
+// Row source of an operand: either rows base + r (contiguous) or rows idx[r].
+struct RowSrc {
+  const int* idx;  // in shared memory, or null for contiguous rows
+  int base;        // first row (contiguous) or offset added to idx[r]
+  int count;       // valid rows; rows >= count load row `base` (masked later)
+  __device__ __forceinline__ int row(int r) const {
+    const int rr = r < count ? r : 0;
+    return idx ? base + idx[rr] : base + rr;
+  }
+};
+
+// Loads rows [r0, r0 + nrows) of an operand for K slice x into a 128-B-row tile.
+__device__ __forceinline__ void load_rows(uint8_t* dst, const CUtensorMap* map, const RowSrc& src,
+                                          int r0, int nrows, int x, uint64_t* bar, bool gather) {
+  if (gather) {
+    for (int r = 0; r < nrows; r += 4)
+      tma_gather4(dst + r * 128, map, x, src.row(r0 + r), src.row(r0 + r + 1), src.row(r0 + r + 2),
+                  src.row(r0 + r + 3), bar);
+  } else {
+    // contiguous: boxes of 128 rows (the tensor map's box height)
+    for (int r = 0; r < nrows; r += 128) tma_load_2d(dst + r * 128, map, x, src.base + r0 + r, bar);
+  }
+}
+
+// Producer: for each N tile t in [0, n_tiles), all K slices.
+template <int BN>
+__device__ __forceinline__ void producer(Pipe& p, uint8_t* stages, const CUtensorMap* mapA,
+                                         const CUtensorMap* mapB, const RowSrc& a, bool gatherA,
+                                         const RowSrc& b, bool gatherB, int n_tiles, int n_k,
+                                         unsigned* err) {
+  int it = 0;
+  for (int t = 0; t < n_tiles && !p.fail; ++t) {
+    for (int kb = 0; kb < n_k; ++kb, ++it) {
+      const int s = it % kStages;
+      const uint32_t ph = (uint32_t)(it / kStages) & 1u;
+      if (!mbar_wait(&p.empty[s], ph ^ 1u, err)) {
+        p.fail = 1;
+        return;
+      }
+      uint8_t* sa = stages + (size_t)s * Cfg<BN>::kStageBytes;
+      uint8_t* sb = sa + kABytes;
+      mbar_arrive_expect_tx(&p.full[s], Cfg<BN>::kStageBytes);
+      load_rows(sa, mapA, a, 0, kBM, kb * kBK, &p.full[s], gatherA);
+      load_rows(sb, mapB, b, t * BN, BN, kb * kBK, &p.full[s], gatherB);
+    }
+  }
+}
+
+// MMA issuer.
+template <int BN>
+__device__ __forceinline__ void mma_issuer(Pipe& p, uint8_t* stages, int n_tiles, int n_k,
+                                           unsigned* err) {
+  int it = 0;
+  for (int t = 0; t < n_tiles; ++t) {
+    const int buf = t & 1;
+    const uint32_t acc_addr = p.tmem + (uint32_t)(buf * BN);
+    if (!mbar_wait(&p.acc_empty[buf], ((uint32_t)(t >> 1) & 1u) ^ 1u, err)) {
+      p.fail = 1;
+    }
+    for (int kb = 0; kb < n_k; ++kb, ++it) {
+      const int s = it % kStages;
+      const uint32_t ph = (uint32_t)(it / kStages) & 1u;
+      if (p.fail || !mbar_wait(&p.full[s], ph, err)) {
+        p.fail = 1;
+        break;
+      }
+      tc_fence_after();
+      const uint32_t sa = smem_u32(stages + (size_t)s * Cfg<BN>::kStageBytes);
+      const uint32_t sb = sa + kABytes;
+#pragma unroll
+      for (int k = 0; k < kBK / 16; ++k)
+        tc_mma_bf16(acc_addr, smem_desc_sw128(sa + k * 32), smem_desc_sw128(sb + k * 32),
+                    Cfg<BN>::kIdesc, (kb > 0 || k > 0) ? 1u : 0u);
+      tc_commit(&p.empty[s]);
+    }
+    tc_commit(&p.acc_full[buf]);  // arrives when every MMA above has completed
+    if (p.fail) {
+      // let the epilogue drain: the commit above still arrives
+      for (int t2 = t + 1; t2 < n_tiles; ++t2) tc_commit(&p.acc_full[t2 & 1]);
+      return;
+    }
+  }
+}
+
+__device__ __forceinline__ void pipe_init(Pipe& p) {
+  for (int s = 0; s < kStages; ++s) {
+    mbar_init(&p.full[s], 1);
+    mbar_init(&p.empty[s], 1);
+  }
+  for (int b = 0; b < 2; ++b) {
+    mbar_init(&p.acc_full[b], 1);
+    mbar_init(&p.acc_empty[b], 4);  // one arrival per epilogue warp
+  }
+  p.fail = 0;
+  fence_mbar_init();
+}
+
+}  // namespace tcg
+}  // namespace provip
