@@ -49,7 +49,7 @@ N_COPIES = 3
 # DRAM traffic of one compaction launch on the default workload, from the ncu
 # capture summarised in profiles/ (null when the kernel source has changed
 # since: the sha1 of the kernel file is checked at run time).
-COMPACT_TRAFFIC = {"sha1": "589b2b87d1b4ea8803beb9af644e4f40730ff41b", "bytes": 116439296,
+COMPACT_TRAFFIC = {"sha1": "22df982433f5f05c15fdb4033ceeaa5eb47a29fd", "bytes": 119081728,
                    "profile": "profiles/prune_llava_next_b8_kernels.md"}
 
 
@@ -64,6 +64,9 @@ def parse_args(argv=None):
     ap.add_argument("--e2e-steps", type=int, default=20)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--copies", type=int, default=N_COPIES, help="rotating device copies of the inputs")
+    ap.add_argument("--prellm-only", action="store_true",
+                    help="time only the pre-LLM pass (provip_similarity_reduce) and print its JSON")
+    ap.add_argument("--prellm-reps", type=int, default=20)
     return ap.parse_args(argv)
 
 
@@ -592,8 +595,20 @@ def run_gb300(args, dist):
     return 0
 
 
+def run_prellm_only(args):
+    import torch
+    import __graft_entry__
+    from paper_2608_25332_gb300 import synth
+    __graft_entry__.build()
+    dev = torch.device("cuda", 0)
+    print(json.dumps({"prellm": prellm_measure(synth.BY_NAME[args.workload], dev, reps=args.prellm_reps)}))
+    return 0
+
+
 def main(argv=None):
     args = parse_args(argv)
+    if args.prellm_only:
+        return run_prellm_only(args)
     dist = Dist()
     if args.impl == "reference":
         dist.init("gloo")
