@@ -252,6 +252,17 @@ def visible_device_index(local_rank):
 # ---------------------------------------------------------------------------
 # algorithmic bytes (what the method must move), per launch
 # ---------------------------------------------------------------------------
+def workload_config(w, algo="auto", copies=N_COPIES, input_mb=None):
+    """the config object both arms print for the workload"""
+    return {"workload": w.name, "B": w.B, "N_v": w.keep_pre, "keep": w.keep, "L_max": w.L_max,
+            "H_q": w.H_q, "H_kv": w.H_kv, "H_sel": w.H_sel, "D": w.D, "algo": algo,
+            "l2": f"inputs larger than L2: {copies} rotating device copies of "
+                  f"{input_mb if input_mb is not None else 286:.0f} MB",
+            "timing": f"CUDA graphs of {GRAPH_CHUNK} steps, events on the launching stream",
+            "overlap": "independent batches: each step's head scores may start under the previous "
+                       "step's compaction (PROVIP_PRUNE_OVERLAP_PREVIOUS)"}
+
+
 def algorithmic_bytes(w, inp):
     import numpy as np
     es = 4 if w.dtype == "f32" else 2
@@ -379,7 +390,7 @@ def run_reference(args, dist):
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * el / max(1, args.steps),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-            "data": "synthetic", "config": {"workload": w.name, "B": w.B},
+            "data": "synthetic", "config": workload_config(w),
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
                              "sample": f"{rows_per_step} text row(s) per step of {w.name} scored over "
                                        f"{w.H_sel} heads, each sample's top-k + compaction with its last "
@@ -569,14 +580,8 @@ def run_gb300(args, dist):
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": dist.world, "steps": K,
             "warmup": args.warmup, "ms_per_step": 1e3 * max_sec / K, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
-            "config": {"workload": w.name, "B": w.B, "N_v": nv, "keep": keep, "L_max": w.L_max,
-                       "H_q": w.H_q, "H_kv": w.H_kv, "H_sel": w.H_sel, "D": w.D,
-                       "algo": args.algo,
-                       "l2": f"inputs larger than L2: {len(copies)} rotating device copies of "
-                             f"{sum(v.numel() * v.element_size() for v in pin.values()) / 1e6:.0f} MB",
-                       "timing": f"CUDA graphs of {GRAPH_CHUNK} steps, events on the launching stream",
-                       "overlap": "independent batches: each step's head scores may start under the previous "
-                                  "step's compaction (PROVIP_PRUNE_OVERLAP_PREVIOUS)"},
+            "config": workload_config(w, args.algo, len(copies),
+                                      sum(v.numel() * v.element_size() for v in pin.values()) / 1e6),
             "roofline": {"bound": "hbm", "kernel": "compact_kernel", "achieved": ach, "peak": peak,
                          "peak_source": peak_src, "unit": "GB/s", "frac": ach / peak,
                          "traffic": traffic, "algorithmic_bytes": ab["compact"],
