@@ -165,7 +165,9 @@ int provip_similarity_reduce(const void *emb_v, int B, int N_v, int D, const voi
  *               taken at key vis_start + i  (t_j the absolute position of text
  *               row j, g(h) = h / (H_q / H_kv) its key/value head);
  *   v_i       = 1/(|V| |R|) sum_{h in V} sum_{j in R} A_{h,j,i}.
- * V = head_list (host int32[H_sel], distinct, in [0, H_q)); R = text rows
+ * V = head_list (host int32[H_sel], distinct, in [0, H_q)), or every head
+ * when head_list is NULL and H_sel == H_q (the paper's "all attention heads"
+ * variant used at the middle pruning layer, Sec. 4.4); R = text rows
  * j < text_len[b] at positions text_start[b] + j, restricted to
  * row_mask_or_null[b][j] != 0 when given (e.g. the critical rows T).
  *   Q [B, L_max, H_q, d_h], K [B, L_max, H_kv, d_h] dtype (post-RoPE).
@@ -259,8 +261,9 @@ int provip_head_topk(const void *Q, const void *K, int B, int L_max, int H_q, in
  *
  * flags: 0, or PROVIP_PRUNE_OVERLAP_PREVIOUS - the call's head-score kernel may
  * start while the kernel before it on the stream (typically the previous
- * call's compaction) is still running; it only waits for that kernel before
- * writing its workspace. Pass it only when this call's Q and K were not written
+ * call's compaction) is still running; it waits for that kernel only before
+ * it completes (its workspace writes do not conflict with the previous
+ * call's kernels, which have consumed the workspace by then). Pass it only when this call's Q and K were not written
  * by the kernel launched just before it on the stream (for instance when
  * pruning a stream of independent batches); other kernels in between (e.g. the
  * LLM layers that produce Q/K) make the flag harmless. */
@@ -274,6 +277,59 @@ int provip_prune(const void *Q, const void *K, const void *V, const void *hidden
                  int keep, int dtype, int algo, void *hidden_out, void *K_out, void *V_out,
                  int *pos_out, int *idx_out, int *seq_len_out, float *scores_out_or_null,
                  void *ws, size_t ws_bytes, unsigned flags, void *stream);
+
+/* ------------------------------------------------------------------------
+ * Visual-head identification (Sec. 4.4, the head confidence C^h and the set
+ * V_l of the N_vis most confident heads) and pruning with those heads
+ * ---------------------------------------------------------------------- */
+
+/* Head confidence over every query head h of the pruning layer:
+ *   C[b][h] = sum over critical text rows j of Var_i(A_{h,j,i}),
+ * A_{h,j,i} the cross-modal attention of provip_head_scores (softmax over the
+ * full causal key range, taken at the N_v visual keys) and Var the population
+ * variance over the N_v visual columns (1/N_v; the ranking is the same with
+ * 1/(N_v - 1)). The critical rows are the text rows j < text_len[b] with
+ * crit_mask_or_null[b][j] != 0 (the set T of Sec. 4.2, e.g. from
+ * provip_crit_text); NULL takes every text row. Then, per sample, the N_vis
+ * heads of largest C (ties to the lower head index) are the visual heads:
+ *   vis_heads_out [B, N_vis] int32, ascending head indices (device);
+ *   conf_out_or_null [B, H_q] fp32 receives C when non-NULL.
+ * The selection is per sample (T and the attention maps are per input). An
+ * empty critical set gives C = 0 for every head, hence heads 0..N_vis-1.
+ * Every head is read once (all H_q heads' queries on the text rows, every
+ * key/value head's keys). Requires H_q <= 64, 1 <= N_vis <= H_q and the shape
+ * rules of provip_head_scores. Variances are accumulated per row in fp32 with
+ * a pairwise (mean, M2) merge over column chunks.
+ * Workspace: provip_visual_heads_workspace_size. */
+size_t provip_visual_heads_workspace_size(int B, int L_max, int H_q, int N_t_max, int N_v,
+                                          int N_vis, int algo, int dtype);
+int provip_head_confidence(const void *Q, const void *K, int B, int L_max, int H_q, int H_kv,
+                           int d_h, const int *text_start, const int *text_len,
+                           const uint8_t *crit_mask_or_null, int N_t_max, int vis_start,
+                           int N_v, const int *seq_len, int N_vis, int dtype, int algo,
+                           float *conf_out_or_null, int *vis_heads_out, void *ws,
+                           size_t ws_bytes, void *stream);
+
+/* Shallow-layer pruning with visual heads only (Sec. 4.4): the confidence and
+ * visual heads of provip_head_confidence, then v from the visual heads of each
+ * sample over all its text rows (S^vis and v of Sec. 4.4), the top `keep` of v
+ * (idx_out [B, keep] ascending, ties to the lower index) and the compaction of
+ * provip_compact. One pass over the keys computes the attention statistics of
+ * every head; the scores of a sample's visual heads are bit-identical to
+ * provip_prune called on that sample alone with head_list = its visual heads.
+ * scores_out_or_null [B, N_v], vis_heads_out_or_null [B, N_vis] and
+ * conf_out_or_null [B, H_q] receive v, the visual heads and C when non-NULL.
+ * flags as in provip_prune. Workspace: provip_visual_heads_workspace_size. */
+int provip_prune_visual_heads(const void *Q, const void *K, const void *V, const void *hidden,
+                              int B, int L_max, int H_q, int H_kv, int d_h, int D,
+                              const int *text_start, const int *text_len,
+                              const uint8_t *crit_mask_or_null, int N_t_max, int vis_start,
+                              int N_v, const int *seq_len, const int *pos, int P, int N_vis,
+                              int keep, int dtype, int algo, void *hidden_out, void *K_out,
+                              void *V_out, int *pos_out, int *idx_out, int *seq_len_out,
+                              float *scores_out_or_null, int *vis_heads_out_or_null,
+                              float *conf_out_or_null, void *ws, size_t ws_bytes,
+                              unsigned flags, void *stream);
 
 #ifdef __cplusplus
 }

@@ -107,10 +107,26 @@ size_t hs_ws(Carve& c, int B, int H_sel, const HSShape& s, int N_v, float2** sta
   return c.off;
 }
 
+// head confidence: chunk capacity per row (every chunk layout the resolved
+// path may take) and the workspace it needs
+int conf_stride(const HSShape& sh, int algo) {
+  return algo == PROVIP_ALGO_TCGEN05 ? (sh.n_vc > kFusedMaxChunks ? sh.n_vc : kFusedMaxChunks) : sh.n_vc;
+}
+struct ConfWs {
+  float2* part = nullptr;
+  int* sel = nullptr;
+};
+size_t conf_ws(Carve& c, int B, int H_sel, int N_t_max, const HSShape& sh, int algo, int n_vis,
+               ConfWs& w) {
+  w.part = c.take<float2>((size_t)B * H_sel * N_t_max * conf_stride(sh, algo));
+  w.sel = c.take<int>((size_t)B * (n_vis > 0 ? n_vis : 1));
+  return c.off;
+}
+
 int hs_validate(const void* Q, const void* K, int B, int L_max, int H_q, int H_kv, int d_h,
                 const int* head_list, int H_sel, const int* text_start, const int* text_len,
                 int N_t_max, int vis_start, int N_v, const int* seq_len, int dtype, int algo) {
-  if (!Q || !K || !head_list || !text_start || !text_len || !seq_len)
+  if (!Q || !K || !text_start || !text_len || !seq_len)
     return fail(PROVIP_ERR_INVALID_ARG, "head_scores: null pointer argument");
   if (B < 1 || L_max < 1 || H_q < 1 || H_kv < 1 || N_t_max < 1 || N_v < 1 || vis_start < 0)
     return fail(PROVIP_ERR_INVALID_ARG, "head_scores: non-positive size");
@@ -120,7 +136,9 @@ int hs_validate(const void* Q, const void* K, int B, int L_max, int H_q, int H_k
   if (!dtype_ok(dtype)) return fail(PROVIP_ERR_UNSUPPORTED, "head_scores: dtype %d", dtype);
   if (d_h != kHeadDim) return fail(PROVIP_ERR_UNSUPPORTED, "head_scores: d_h must be 128");
   if (H_sel < 1 || H_sel > kMaxHeads) return fail(PROVIP_ERR_INVALID_ARG, "head_scores: H_sel %d", H_sel);
-  for (int i = 0; i < H_sel; ++i) {
+  if (!head_list && H_sel != H_q)
+    return fail(PROVIP_ERR_INVALID_ARG, "head_scores: a null head_list (all heads) needs H_sel == H_q");
+  for (int i = 0; head_list && i < H_sel; ++i) {
     if (head_list[i] < 0 || head_list[i] >= H_q)
       return fail(PROVIP_ERR_INVALID_ARG, "head_scores: head_list[%d] = %d out of range", i, head_list[i]);
     for (int j = 0; j < i; ++j)
@@ -151,7 +169,7 @@ HSArgs hs_args(const void* Q, const void* K, int B, int L_max, int H_q, int H_kv
   a.H_kv = H_kv;
   a.d_h = d_h;
   a.H_sel = H_sel;
-  for (int i = 0; i < H_sel; ++i) a.heads[i] = head_list[i];
+  for (int i = 0; i < H_sel; ++i) a.heads[i] = head_list ? head_list[i] : i;
   a.text_start = text_start;
   a.text_len = text_len;
   a.row_mask = row_mask;
@@ -172,8 +190,10 @@ HSArgs hs_args(const void* Q, const void* K, int B, int L_max, int H_q, int H_kv
 }
 
 // both passes of the head scores (partials in the workspace); overlap: the
-// one-pass kernel may start before the previous kernel on the stream finishes
-int hs_run(const HSArgs& a, int dtype, int algo, cudaStream_t s, bool overlap = false) {
+// one-pass kernel may start before the previous kernel on the stream finishes;
+// geom: the chunks of the confidence statistics, when a.conf_part is set
+int hs_run(const HSArgs& a, int dtype, int algo, cudaStream_t s, bool overlap = false,
+           ConfGeom* geom = nullptr) {
   cudaError_t e;
   if (is_tc(algo)) {
     CUtensorMap tq, tk;
@@ -183,10 +203,10 @@ int hs_run(const HSArgs& a, int dtype, int algo, cudaStream_t s, bool overlap = 
       return fail(PROVIP_ERR_CUDA, "head_scores: cuTensorMapEncodeTiled failed");
     bool launched = false;
     e = cudaSuccess;
-    if (algo == PROVIP_ALGO_TCGEN05) e = hs_launch_fused(a, &tq, &tk, s, &launched, overlap);
-    if (e == cudaSuccess && !launched) e = hs_launch_tc(a, &tq, &tk, s);
+    if (algo == PROVIP_ALGO_TCGEN05) e = hs_launch_fused(a, &tq, &tk, s, &launched, overlap, geom);
+    if (e == cudaSuccess && !launched) e = hs_launch_tc(a, &tq, &tk, s, geom);
   } else {
-    e = hs_launch_simt(a, dtype, s);
+    e = hs_launch_simt(a, dtype, s, geom);
   }
   if (e != cudaSuccess) return cuda_fail(e, "head_scores launch");
   return PROVIP_OK;
@@ -662,6 +682,8 @@ static int head_topk_impl(const void* Q, const void* K, int B, int L_max, int H_
   if (!idx_out) return fail(PROVIP_ERR_INVALID_ARG, "head_topk: null idx_out");
   if (keep < 1 || keep > N_v) return fail(PROVIP_ERR_INVALID_ARG, "head_topk: keep %d not in [1, N_v]", keep);
   if (N_v > kTopkMaxN) return fail(PROVIP_ERR_UNSUPPORTED, "head_topk: N_v > %d", kTopkMaxN);
+  if ((long long)((N_t_max + kRowBlock - 1) / kRowBlock) * H_sel * N_v >= (1ll << 31))
+    return fail(PROVIP_ERR_UNSUPPORTED, "head_topk: too many head partials");
   if ((rc = check_ws(provip_head_scores_workspace_size(B, L_max, H_sel, N_t_max, N_v, algo, dtype), ws,
                      ws_bytes, "head_topk")))
     return rc;
@@ -739,6 +761,135 @@ extern "C" int provip_prune(const void* Q, const void* K, const void* V, const v
                                 seq_len_out, d->status);
   cudaError_t e = compact_launch(ca, d->sms, static_cast<cudaStream_t>(stream), true);
   return e == cudaSuccess ? PROVIP_OK : cuda_fail(e, "prune compact");
+}
+
+// ===========================================================================
+// visual-head identification (Sec. 4.4): head confidence over every head on
+// the critical text rows, the N_vis most confident heads per sample, and the
+// token importance from those heads alone
+// ===========================================================================
+extern "C" size_t provip_visual_heads_workspace_size(int B, int L_max, int H_q, int N_t_max,
+                                                     int N_v, int N_vis, int algo, int dtype) {
+  algo = resolve_algo(algo, dtype);
+  HSShape sh = hs_shape(L_max, N_t_max, N_v, algo);
+  Carve c(nullptr);
+  float2* st;
+  float* pa;
+  hs_ws(c, B, H_q, sh, N_v, &st, &pa);
+  ConfWs w;
+  return conf_ws(c, B, H_q, N_t_max, sh, algo, N_vis, w);
+}
+
+// keep == 0: confidence and selection only; keep >= 1: also the top-keep
+// tokens by the selected heads' scores
+static int visual_heads_impl(const void* Q, const void* K, int B, int L_max, int H_q, int H_kv,
+                             int d_h, const int* text_start, const int* text_len,
+                             const uint8_t* crit_mask_or_null, int N_t_max, int vis_start, int N_v,
+                             const int* seq_len, int N_vis, int keep, int dtype, int algo,
+                             float* conf_out_or_null, int* vis_heads_out, int* idx_out,
+                             float* scores_out_or_null, void* ws, size_t ws_bytes, void* stream,
+                             bool overlap, const char* what) {
+  algo = resolve_algo(algo, dtype);
+  if (H_q > kMaxHeads) return fail(PROVIP_ERR_UNSUPPORTED, "%s: H_q %d > %d", what, H_q, kMaxHeads);
+  int rc = hs_validate(Q, K, B, L_max, H_q, H_kv, d_h, nullptr, H_q, text_start, text_len, N_t_max,
+                       vis_start, N_v, seq_len, dtype, algo);
+  if (rc) return rc;
+  if (N_vis < 1 || N_vis > H_q) return fail(PROVIP_ERR_INVALID_ARG, "%s: N_vis %d not in [1, H_q]", what, N_vis);
+  if (keep > 0) {
+    if (!idx_out) return fail(PROVIP_ERR_INVALID_ARG, "%s: null idx_out", what);
+    if (keep > N_v) return fail(PROVIP_ERR_INVALID_ARG, "%s: keep %d not in [1, N_v]", what, keep);
+    if (N_v > kTopkMaxN) return fail(PROVIP_ERR_UNSUPPORTED, "%s: N_v > %d", what, kTopkMaxN);
+  }
+  const HSShape sh = hs_shape(L_max, N_t_max, N_v, algo);
+  if ((long long)sh.n_rb * H_q * N_v >= (1ll << 31))
+    return fail(PROVIP_ERR_UNSUPPORTED, "%s: too many head partials", what);
+  if ((rc = check_ws(provip_visual_heads_workspace_size(B, L_max, H_q, N_t_max, N_v, N_vis, algo, dtype),
+                     ws, ws_bytes, what)))
+    return rc;
+  DevInfo* d;
+  if ((rc = dev_info(&d))) return rc;
+  Carve c(ws);
+  float2* stats;
+  float* partial;
+  hs_ws(c, B, H_q, sh, N_v, &stats, &partial);
+  ConfWs cw;
+  conf_ws(c, B, H_q, N_t_max, sh, algo, N_vis, cw);
+  HSArgs a = hs_args(Q, K, B, L_max, H_q, H_kv, d_h, nullptr, H_q, text_start, text_len, nullptr,
+                     N_t_max, vis_start, N_v, seq_len, sh, stats, partial, d->status);
+  a.conf_mask = crit_mask_or_null;
+  a.conf_part = cw.part;
+  a.conf_stride = conf_stride(sh, algo);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  ConfGeom geom{0, 0, 0};
+  if ((rc = hs_run(a, dtype, algo, s, overlap, &geom))) return rc;
+  ConfArgs ca;
+  ca.n_vis = N_vis;
+  ca.sel_out = cw.sel;
+  ca.vis_heads_out = vis_heads_out;
+  ca.conf_out = conf_out_or_null;
+  cudaError_t e = conf_select_launch(a, geom, ca, s, true);
+  if (e != cudaSuccess) return cuda_fail(e, "visual heads: selection launch");
+  if (keep <= 0) return PROVIP_OK;
+  TopkArgs t;
+  memset(&t, 0, sizeof(t));
+  t.partial = partial;
+  t.n_part = sh.n_rb * H_q;
+  t.text_len = text_len;
+  t.N_t_max = N_t_max;
+  t.H_sel = H_q;
+  t.sel = cw.sel;
+  t.n_sel = N_vis;
+  t.scores_out = scores_out_or_null;
+  t.B = B;
+  t.N = N_v;
+  t.k = keep;
+  t.idx_out = idx_out;
+  t.err = d->status;
+  e = topk_launch(t, s, true);
+  return e == cudaSuccess ? PROVIP_OK : cuda_fail(e, "visual heads: top-k launch");
+}
+
+extern "C" int provip_head_confidence(const void* Q, const void* K, int B, int L_max, int H_q,
+                                      int H_kv, int d_h, const int* text_start, const int* text_len,
+                                      const uint8_t* crit_mask_or_null, int N_t_max, int vis_start,
+                                      int N_v, const int* seq_len, int N_vis, int dtype, int algo,
+                                      float* conf_out_or_null, int* vis_heads_out, void* ws,
+                                      size_t ws_bytes, void* stream) {
+  if (!vis_heads_out) return fail(PROVIP_ERR_INVALID_ARG, "head_confidence: null vis_heads_out");
+  return visual_heads_impl(Q, K, B, L_max, H_q, H_kv, d_h, text_start, text_len, crit_mask_or_null,
+                           N_t_max, vis_start, N_v, seq_len, N_vis, 0, dtype, algo,
+                           conf_out_or_null, vis_heads_out, nullptr, nullptr, ws, ws_bytes, stream,
+                           false, "head_confidence");
+}
+
+extern "C" int provip_prune_visual_heads(
+    const void* Q, const void* K, const void* V, const void* hidden, int B, int L_max, int H_q,
+    int H_kv, int d_h, int D, const int* text_start, const int* text_len,
+    const uint8_t* crit_mask_or_null, int N_t_max, int vis_start, int N_v, const int* seq_len,
+    const int* pos, int P, int N_vis, int keep, int dtype, int algo, void* hidden_out, void* K_out,
+    void* V_out, int* pos_out, int* idx_out, int* seq_len_out, float* scores_out_or_null,
+    int* vis_heads_out_or_null, float* conf_out_or_null, void* ws, size_t ws_bytes,
+    unsigned flags, void* stream) {
+  if (flags & ~(unsigned)PROVIP_PRUNE_OVERLAP_PREVIOUS)
+    return fail(PROVIP_ERR_INVALID_ARG, "prune_visual_heads: unknown flags 0x%x", flags);
+  if (keep < 1) return fail(PROVIP_ERR_INVALID_ARG, "prune_visual_heads: keep %d < 1", keep);
+  int rc = compact_validate(idx_out ? idx_out : reinterpret_cast<int*>(16), B, N_v, keep, hidden, D,
+                            K, V, H_kv, d_h, pos, P, seq_len, L_max, vis_start, dtype, hidden_out,
+                            K_out, V_out, pos_out);
+  if (rc) return rc;
+  rc = visual_heads_impl(Q, K, B, L_max, H_q, H_kv, d_h, text_start, text_len, crit_mask_or_null,
+                         N_t_max, vis_start, N_v, seq_len, N_vis, keep, dtype, algo,
+                         conf_out_or_null, vis_heads_out_or_null, idx_out, scores_out_or_null, ws,
+                         ws_bytes, stream, (flags & PROVIP_PRUNE_OVERLAP_PREVIOUS) != 0,
+                         "prune_visual_heads");
+  if (rc) return rc;
+  DevInfo* d;
+  if ((rc = dev_info(&d))) return rc;
+  CompactArgs ca = compact_args(idx_out, B, N_v, keep, hidden, D, K, V, H_kv, d_h, pos, P, seq_len,
+                                L_max, vis_start, dtype, hidden_out, K_out, V_out, pos_out,
+                                seq_len_out, d->status);
+  cudaError_t e = compact_launch(ca, d->sms, static_cast<cudaStream_t>(stream), true);
+  return e == cudaSuccess ? PROVIP_OK : cuda_fail(e, "prune_visual_heads compact");
 }
 
 // ===========================================================================

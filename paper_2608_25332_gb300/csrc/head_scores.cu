@@ -12,6 +12,8 @@
 //   partial[b][rb * H_sel + head][col]. Deterministic: fixed reduction orders,
 //   no atomics.
 // hs_reduce: scores = sum of partials over (row block, head) / (|V| |R|).
+// conf_select: head confidence from the pass-2 row statistics and the top
+//   n_vis heads per sample.
 #include "common.cuh"
 #include "kernels.h"
 #include "simt_gemm.cuh"
@@ -138,17 +140,36 @@ __global__ void __launch_bounds__(256) hs_probs_simt(const HSArgs a) {
   float acc[8][4];
   simt_gemm_nt<T>(arow, brow, a.d_h, sm, acc);
   const int rg = threadIdx.x >> 4, kg = threadIdx.x & 15;
+  const bool conf = a.conf_part != nullptr;  // block-uniform
+  const int ncol = min(kSimtBN, a.N_v - col0);
   float cs[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
   for (int i = 0; i < 8; ++i) {
     const int r = rg + 16 * i;
-    if (arow[r] == nullptr) continue;
+    const bool rv = arow[r] != nullptr;
     const int t = smp.ts + rb * kSimtBM + r;
     const float m = rowm[r], inv = rowinv[r];
+    float pv[4];
 #pragma unroll
     for (int jj = 0; jj < 4; ++jj) {
       const int col = col0 + kg + 16 * jj;
-      if (col < a.N_v && a.vis_start + col <= t) cs[jj] += exp2f(acc[i][jj] * a.scale_log2 - m) * inv;
+      pv[jj] = (rv && col < a.N_v && a.vis_start + col <= t) ? exp2f(acc[i][jj] * a.scale_log2 - m) * inv : 0.f;
+      cs[jj] += pv[jj];
+    }
+    if (conf) {
+      // head confidence: the row's mean and M2 over the chunk's visual columns
+      // (two-pass over the values in registers; row groups of 16 lanes)
+      const float mean = rowgroup_sum((pv[0] + pv[1]) + (pv[2] + pv[3])) / (float)ncol;
+      float q = 0.f;
+#pragma unroll
+      for (int jj = 0; jj < 4; ++jj) {
+        const float d = (kg + 16 * jj < ncol) ? pv[jj] - mean : 0.f;
+        q += d * d;
+      }
+      q = rowgroup_sum(q);
+      const int j = rb * kSimtBM + r;
+      if (kg == 0 && rv && (a.conf_mask == nullptr || a.conf_mask[(size_t)b * a.N_t_max + j] != 0))
+        a.conf_part[(((size_t)b * a.H_sel + hi) * a.N_t_max + j) * a.conf_stride + vc] = make_float2(mean, q);
     }
   }
   // rows rg and rg + 1 of a warp: fold lanes 16..31 onto 0..15, then across warps
@@ -195,9 +216,89 @@ __global__ void __launch_bounds__(256) hs_reduce_kernel(const HSArgs a, float* s
   scores[(size_t)b * a.N_v + i] = n > 0 ? s / ((float)a.H_sel * (float)n) : 0.f;
 }
 
+// Head confidence and visual-head selection (Sec. 4.4), one CTA per sample.
+// C[i] = sum over the confidence rows of (merged M2) / N_v for head-list
+// position i; each warp takes heads i = warp, warp + 8, ...; each lane a
+// strided set of rows, folded by a fixed butterfly, so C is deterministic.
+// The chunk statistics of a row are merged in chunk order with Chan, Golub and
+// LeVeque's pairwise update; chunk c holds the visual columns of
+// [g.lo0 + c * g.w, g.lo0 + (c + 1) * g.w).
+constexpr int kConfThreads = 256;
+__global__ void __launch_bounds__(kConfThreads) conf_select_kernel(const HSArgs a, const ConfGeom g,
+                                                                  const ConfArgs c) {
+  __shared__ float C[kMaxHeads];
+  __shared__ int chosen[kMaxHeads];
+  // programmatic dependent of the head-score kernel: wait for its statistics
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  const int b = blockIdx.x;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const HSRow smp = hs_sample(a, b);
+  const int vlo = a.vis_start, vhi = a.vis_start + a.N_v;
+  for (int i = warp; i < a.H_sel; i += kConfThreads / 32) {
+    float acc = 0.f;
+    for (int j = lane; j < a.N_t_max; j += 32) {
+      if (!hs_row_valid(a, smp, b, j)) continue;
+      if (a.conf_mask != nullptr && a.conf_mask[(size_t)b * a.N_t_max + j] == 0) continue;
+      const float2* st = a.conf_part + (((size_t)b * a.H_sel + i) * a.N_t_max + j) * a.conf_stride;
+      float n = 0.f, mean = 0.f, m2 = 0.f;
+      for (int q = 0; q < g.n; ++q) {
+        const int lo = max(g.lo0 + q * g.w, vlo), hi = min(g.lo0 + (q + 1) * g.w, vhi);
+        if (hi <= lo) continue;
+        const float nb = (float)(hi - lo);
+        const float2 v = st[q];
+        const float nn = n + nb, dl = v.x - mean;
+        mean += dl * (nb / nn);
+        m2 += v.y + dl * dl * (n * nb / nn);
+        n = nn;
+      }
+      acc += m2 / (float)a.N_v;
+    }
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+    if (lane == 0) C[i] = acc;
+  }
+  __syncthreads();
+  // the next kernel (the top-k) may be scheduled; it waits for this grid
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  const int i = threadIdx.x;
+  if (i < a.H_sel) {
+    const uint32_t ki = float_key(C[i]);
+    int rank = 0;
+    for (int q = 0; q < a.H_sel; ++q) {
+      const uint32_t kq = float_key(C[q]);
+      rank += (kq > ki) || (kq == ki && q < i);
+    }
+    chosen[i] = rank < c.n_vis;
+    if (c.conf_out) c.conf_out[(size_t)b * a.H_q + a.heads[i]] = C[i];
+  }
+  __syncthreads();
+  if (i < a.H_sel && chosen[i]) {
+    int pos = 0;
+    for (int q = 0; q < i; ++q) pos += chosen[q];
+    c.sel_out[(size_t)b * c.n_vis + pos] = i;
+    if (c.vis_heads_out) c.vis_heads_out[(size_t)b * c.n_vis + pos] = a.heads[i];
+  }
+}
+
 }  // namespace
 
-cudaError_t hs_launch_simt(const HSArgs& a, int dtype, cudaStream_t s) {
+cudaError_t conf_select_launch(const HSArgs& a, const ConfGeom& g, const ConfArgs& c,
+                               cudaStream_t s, bool pdl) {
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  cfg.gridDim = dim3((unsigned)a.B);
+  cfg.blockDim = dim3(kConfThreads);
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = s;
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, conf_select_kernel, a, g, c);
+}
+
+cudaError_t hs_launch_simt(const HSArgs& a, int dtype, cudaStream_t s, ConfGeom* geom) {
+  if (geom) *geom = ConfGeom{a.vis_start, kSimtBN, a.n_vc};
   dim3 g1(a.n_kc, a.H_sel * a.n_rb, a.B), g2(a.n_vc, a.H_sel * a.n_rb, a.B);
   if (dtype == 0) {
     hs_stats_simt<float><<<g1, 256, 0, s>>>(a);

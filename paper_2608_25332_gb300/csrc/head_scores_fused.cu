@@ -18,6 +18,8 @@
 //   4. turns its visual columns into probabilities p = e * exp2(mb - M) / L and
 //      sums them over the 128 rows (warp butterfly transpose-reduction, then a
 //      fixed-order sum over the 4 warps) into partial[b][rb * H_sel + h][col];
+//      the CONF variant also keeps, per row, the mean and M2 of its visual
+//      probabilities (head confidence) and writes them per cluster rank;
 //   5. waits on a second cluster barrier (peers may still read its shared
 //      memory) and frees its TMEM.
 // Every key is read from HBM once and every logit is exponentiated once; the
@@ -101,7 +103,8 @@ constexpr size_t smem_bytes() {
   return (size_t)(1 + CPC) * kTileBytes + 1024;
 }
 
-template <int CPC>
+// CONF: also the head-confidence statistics of the visual probabilities
+template <int CPC, bool CONF>
 __global__ void __launch_bounds__(kThreads, CPC == 1 ? 3 : (CPC == 2 ? 2 : 1))
     hs_fused_tc(const HSArgs a,
                                                         const __grid_constant__ CUtensorMap tmQ,
@@ -261,7 +264,11 @@ __global__ void __launch_bounds__(kThreads, CPC == 1 ? 3 : (CPC == 2 ? 2 : 1))
   const float invL = (rv && L > 0.f) ? 1.f / L : 0.f;
   cluster_arrive();  // done reading the peers' rowstat
 
-  // pass 2: probabilities of the visual columns, summed over the rows
+  // pass 2: probabilities of the visual columns, summed over the rows; with
+  // CONF, the row's mean and M2 over this warp's visual columns as well (the
+  // statistics of each 32-column block merged pairwise: Chan, Golub and
+  // LeVeque's update)
+  float cn = 0.f, cmean = 0.f, cm2 = 0.f;
 #pragma unroll
   for (int cb = 0; cb < kBlocks; ++cb) {
     const int k0 = key0 + col0 + cb * 32;
@@ -276,6 +283,24 @@ __global__ void __launch_bounds__(kThreads, CPC == 1 ? 3 : (CPC == 2 ? 2 : 1))
         const int k = k0 + i;
         const bool kv = k >= a.vis_start && k < a.vis_start + a.N_v;
         v[i] = kv ? v[i] * w : 0.f;
+      }
+      if (CONF) {
+        const int lo = max(k0, a.vis_start), hi = min(k0 + 32, a.vis_start + a.N_v);
+        const float nb = (float)(hi - lo);
+        float s4[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int i = 0; i < 32; ++i) s4[i & 3] += v[i];  // zero outside the visual range
+        const float mb = ((s4[0] + s4[1]) + (s4[2] + s4[3])) / nb;
+        float q4[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int i = 0; i < 32; ++i) {
+          const float d = (k0 + i >= lo && k0 + i < hi) ? v[i] - mb : 0.f;
+          q4[i & 3] += d * d;
+        }
+        const float n = cn + nb, dl = mb - cmean;
+        cmean += dl * (nb / n);
+        cm2 += ((q4[0] + q4[1]) + (q4[2] + q4[3])) + dl * dl * (cn * nb / n);
+        cn = n;
       }
 #pragma unroll
       for (int sh = 16; sh >= 1; sh >>= 1) {
@@ -292,7 +317,26 @@ __global__ void __launch_bounds__(kThreads, CPC == 1 ? 3 : (CPC == 2 ? 2 : 1))
     }
     red[quad][col0 + cb * 32 + lane] = v[0];
   }
+  if (CONF) halfstat[half][r] = make_float2(cmean, cm2);  // last read before the cluster barrier
   __syncthreads();
+  if (CONF && half == 0 && rv &&
+      (a.conf_mask == nullptr || a.conf_mask[(size_t)b * a.N_t_max + j] != 0)) {
+    // merge the two column halves of the row; counts from the column ranges
+    const int vlo = a.vis_start, vhi = a.vis_start + a.N_v;
+    const float n0 = (float)max(0, min(key0 + kHalfCols, vhi) - max(key0, vlo));
+    const float n1 = (float)max(0, min(key0 + (int)kCols, vhi) - max(key0 + kHalfCols, vlo));
+    const float2 s0 = halfstat[0][r], s1 = halfstat[1][r];
+    float2 o = s0;
+    if (n1 > 0.f) {
+      if (n0 > 0.f) {
+        const float n = n0 + n1, dl = s1.x - s0.x;
+        o = make_float2(s0.x + dl * (n1 / n), s0.y + s1.y + dl * dl * (n0 * n1 / n));
+      } else {
+        o = s1;
+      }
+    }
+    a.conf_part[(((size_t)b * a.H_sel + hi) * a.N_t_max + j) * a.conf_stride + rank] = o;
+  }
   if (good) {
     float* out = a.partial + ((size_t)b * a.n_rb * a.H_sel + (size_t)rb * a.H_sel + hi) * a.N_v;
     for (int c = threadIdx.x; c < (int)kCols; c += kThreads) {
@@ -320,9 +364,9 @@ struct FusedCfg {
   bool usable = false;
   signed char clusters_ok[17] = {0};  // per cluster size: 0 unknown, 1 placeable, -1 not
 };
-FusedCfg g_cfg[64][3];
+FusedCfg g_cfg[64][3][2];
 
-template <int CPC>
+template <int CPC, bool CONF>
 cudaError_t launch_cpc(const HSArgs& a, const CUtensorMap* tmQ, const CUtensorMap* tmK, int C,
                        cudaStream_t s, bool* launched, bool pdl) {
   *launched = false;
@@ -335,7 +379,7 @@ cudaError_t launch_cpc(const HSArgs& a, const CUtensorMap* tmQ, const CUtensorMa
   int dev = 0;
   cudaGetDevice(&dev);
   const int slot = CPC == 1 ? 0 : (CPC == 2 ? 1 : 2);
-  FusedCfg& fc = g_cfg[dev < 64 ? dev : 0][slot];
+  FusedCfg& fc = g_cfg[dev < 64 ? dev : 0][slot][CONF ? 1 : 0];
   cudaLaunchConfig_t cfg = {};
   cudaLaunchAttribute attr[3];
   cfg.gridDim = dim3((unsigned)C, (unsigned)(a.H_sel * a.n_rb), (unsigned)a.B);
@@ -356,14 +400,14 @@ cudaError_t launch_cpc(const HSArgs& a, const CUtensorMap* tmQ, const CUtensorMa
   cfg.numAttrs = 2;
   if (!fc.checked) {
     fc.checked = true;
-    cudaError_t e = cudaFuncSetAttribute(hs_fused_tc<CPC>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e == cudaSuccess) e = cudaFuncSetAttribute(hs_fused_tc<CPC>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    cudaError_t e = cudaFuncSetAttribute(hs_fused_tc<CPC, CONF>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(hs_fused_tc<CPC, CONF>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
     if (e != cudaSuccess) {
       cudaGetLastError();
       return cudaSuccess;  // not usable: the caller takes the two-kernel path
     }
     int per = 0;
-    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per, hs_fused_tc<CPC>, kThreads, smem);
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per, hs_fused_tc<CPC, CONF>, kThreads, smem);
     if (e != cudaSuccess || per < 1 || per * CPC * kTile > 512) {
       cudaGetLastError();
       return cudaSuccess;
@@ -375,14 +419,24 @@ cudaError_t launch_cpc(const HSArgs& a, const CUtensorMap* tmQ, const CUtensorMa
   if (C < 1 || C > 16) return cudaSuccess;
   if (fc.clusters_ok[C] == 0) {
     int nclusters = 0;
-    cudaError_t q = cudaOccupancyMaxActiveClusters(&nclusters, hs_fused_tc<CPC>, &cfg);
+    cudaError_t q = cudaOccupancyMaxActiveClusters(&nclusters, hs_fused_tc<CPC, CONF>, &cfg);
     if (q != cudaSuccess) cudaGetLastError();
     fc.clusters_ok[C] = (q == cudaSuccess && nclusters >= 1) ? 1 : -1;
   }
   if (fc.clusters_ok[C] < 0) return cudaSuccess;
   if (pdl) cfg.numAttrs = 3;
-  cudaError_t e = cudaLaunchKernelEx(&cfg, hs_fused_tc<CPC>, a, *tmQ, *tmK);
+  cudaError_t e = cudaLaunchKernelEx(&cfg, hs_fused_tc<CPC, CONF>, a, *tmQ, *tmK);
   if (e == cudaSuccess) *launched = true;
+  return e;
+}
+
+template <int CPC>
+cudaError_t launch_conf(const HSArgs& a, const CUtensorMap* tmQ, const CUtensorMap* tmK, int C,
+                        cudaStream_t s, bool* launched, bool pdl, ConfGeom* geom) {
+  if (a.conf_part != nullptr && C > a.conf_stride) return cudaSuccess;  // no room: two-pass path
+  cudaError_t e = a.conf_part != nullptr ? launch_cpc<CPC, true>(a, tmQ, tmK, C, s, launched, pdl)
+                                         : launch_cpc<CPC, false>(a, tmQ, tmK, C, s, launched, pdl);
+  if (*launched && geom) *geom = ConfGeom{0, CPC * kTile, C};
   return e;
 }
 
@@ -391,12 +445,12 @@ cudaError_t launch_cpc(const HSArgs& a, const CUtensorMap* tmQ, const CUtensorMa
 // One-pass head scores; *launched is false when no cluster shape fits (the
 // caller then runs the two-kernel path).
 cudaError_t hs_launch_fused(const HSArgs& a, const CUtensorMap* tmQ, const CUtensorMap* tmK,
-                            cudaStream_t s, bool* launched, bool pdl) {
+                            cudaStream_t s, bool* launched, bool pdl, ConfGeom* geom) {
   *launched = false;
   const int chunks = (a.L_max + kTile - 1) / kTile;
-  if (chunks <= 16) return launch_cpc<1>(a, tmQ, tmK, chunks, s, launched, pdl);
-  if (chunks <= 32) return launch_cpc<2>(a, tmQ, tmK, (chunks + 1) / 2, s, launched, pdl);
-  if (chunks <= 64) return launch_cpc<4>(a, tmQ, tmK, (chunks + 3) / 4, s, launched, pdl);
+  if (chunks <= 16) return launch_conf<1>(a, tmQ, tmK, chunks, s, launched, pdl, geom);
+  if (chunks <= 32) return launch_conf<2>(a, tmQ, tmK, (chunks + 1) / 2, s, launched, pdl, geom);
+  if (chunks <= 64) return launch_conf<4>(a, tmQ, tmK, (chunks + 3) / 4, s, launched, pdl, geom);
   return cudaSuccess;
 }
 

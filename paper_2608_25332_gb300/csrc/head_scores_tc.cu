@@ -13,7 +13,9 @@
 // chunk. Pass 2 turns the visual logits into probabilities with the row's
 // global (max, sum) and sums them over the 128 rows: a butterfly
 // transpose-reduction inside each warp (31 shuffles per 32 columns) and a
-// fixed-order sum over the 4 warps, so the result is deterministic.
+// fixed-order sum over the 4 warps, so the result is deterministic. When asked,
+// pass 2 also writes each row's mean and M2 over the chunk's visual
+// probabilities (head confidence).
 #include "common.cuh"
 #include "kernels.h"
 
@@ -214,6 +216,10 @@ __global__ void __launch_bounds__(kTcThreads) hs_probs_tc(const HSArgs a,
   const bool good = tc_wait_mma(&ctl, a.err);
   rv = rv && good;
   const int col0 = vc * kTile;
+  // head confidence: the row's mean and M2 over this chunk's visual columns
+  // (per 32-column block, merged pairwise: Chan, Golub and LeVeque's update)
+  const bool conf = a.conf_part != nullptr;
+  float cn = 0.f, cmean = 0.f, cm2 = 0.f;
 #pragma unroll 1
   for (int cb = 0; cb < kTile / 32; ++cb) {
     float v[32];
@@ -224,6 +230,24 @@ __global__ void __launch_bounds__(kTcThreads) hs_probs_tc(const HSArgs a,
       const int col = col0 + cb * 32 + i;
       const bool kv = rv && col < a.N_v && (a.vis_start + col) <= t;
       v[i] = kv ? exp2f(v[i] * a.scale_log2 - m) * inv : 0.f;
+    }
+    const int nbi = min(32, a.N_v - (col0 + cb * 32));
+    if (conf && nbi > 0) {
+      const float nb = (float)nbi;
+      float s4[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+      for (int i = 0; i < 32; ++i) s4[i & 3] += v[i];
+      const float mb = ((s4[0] + s4[1]) + (s4[2] + s4[3])) / nb;
+      float q4[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+      for (int i = 0; i < 32; ++i) {
+        const float d = i < nbi ? v[i] - mb : 0.f;
+        q4[i & 3] += d * d;
+      }
+      const float n = cn + nb, dl = mb - cmean;
+      cmean += dl * (nb / n);
+      cm2 += ((q4[0] + q4[1]) + (q4[2] + q4[3])) + dl * dl * (cn * nb / n);
+      cn = n;
     }
     // butterfly transpose-reduction: lane ends with the column sum of column `lane`
 #pragma unroll
@@ -238,6 +262,9 @@ __global__ void __launch_bounds__(kTcThreads) hs_probs_tc(const HSArgs a,
     }
     red[warp][cb * 32 + lane] = v[0];
   }
+  if (conf && rv && (a.conf_mask == nullptr || a.conf_mask[(size_t)b * a.N_t_max + j] != 0))
+    a.conf_part[(((size_t)b * a.H_sel + hi) * a.N_t_max + j) * a.conf_stride + vc] =
+        make_float2(cmean, cm2);
   __syncthreads();
   {
     const int col = col0 + threadIdx.x;
@@ -251,7 +278,8 @@ __global__ void __launch_bounds__(kTcThreads) hs_probs_tc(const HSArgs a,
 }  // namespace
 
 cudaError_t hs_launch_tc(const HSArgs& a, const CUtensorMap* tmQ, const CUtensorMap* tmK,
-                         cudaStream_t s) {
+                         cudaStream_t s, ConfGeom* geom) {
+  if (geom) *geom = ConfGeom{a.vis_start, kTile, a.n_vc};
   static bool configured[64] = {false};
   int dev = 0;
   cudaGetDevice(&dev);

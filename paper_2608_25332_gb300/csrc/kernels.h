@@ -42,21 +42,60 @@ struct HSArgs {
   float scale_log2;          // log2(e) / sqrt(d_h)
   float2* stats;             // [B][n_rb][H_sel][n_kc][128]
   float* partial;            // [B][n_rb * H_sel][N_v]
+  // head confidence (Sec. 4.4), optional: for every valid text row j with
+  // conf_mask[b][j] != 0 (null: every valid row), the mean and the sum of
+  // squared deviations (M2) of the row's visual probabilities over the columns
+  // of each column chunk c the pass-2 kernels own:
+  //   conf_part[((b * H_sel + head) * N_t_max + j) * conf_stride + c] = (mean, M2).
+  // Chunk c covers the keys [conf_lo0 + c * conf_w, conf_lo0 + (c + 1) * conf_w)
+  // intersected with the visual range (ConfGeom below).
+  const uint8_t* conf_mask;
+  float2* conf_part;         // null: no confidence statistics
+  int conf_stride;           // chunk capacity per row
   unsigned* err;
 };
 
-cudaError_t hs_launch_simt(const HSArgs& a, int dtype, cudaStream_t s);
+// column chunks of the confidence statistics written by the path that ran
+struct ConfGeom {
+  int lo0;  // first key of chunk 0
+  int w;    // keys per chunk
+  int n;    // chunks
+};
+
+// geom (optional): the column chunks of the confidence statistics
+cudaError_t hs_launch_simt(const HSArgs& a, int dtype, cudaStream_t s, ConfGeom* geom = nullptr);
 // tcgen05 path (bf16): needs tensor maps over Q and K viewed as 2-D row tables.
 cudaError_t hs_launch_tc(const HSArgs& a, const CUtensorMap* tmQ, const CUtensorMap* tmK,
-                         cudaStream_t s);
+                         cudaStream_t s, ConfGeom* geom = nullptr);
 // one-pass tcgen05 path (clusters, TMEM-resident logits): writes the partials
 // directly; *launched is false when no cluster shape fits this problem. pdl:
 // launched as a programmatic dependent of the previous kernel on the stream
 // (it reads Q/K at once and waits for that kernel only before writing).
+// geom (optional): the confidence chunks of the launched shape.
 cudaError_t hs_launch_fused(const HSArgs& a, const CUtensorMap* tmQ, const CUtensorMap* tmK,
-                            cudaStream_t s, bool* launched, bool pdl = false);
+                            cudaStream_t s, bool* launched, bool pdl = false,
+                            ConfGeom* geom = nullptr);
+// largest number of confidence chunks the one-pass kernel uses (its cluster size)
+constexpr int kFusedMaxChunks = 16;
 // scores[b][i] = sum_u partial[b][u][i] / (H_sel * valid text rows of b)
 cudaError_t hs_launch_reduce(const HSArgs& a, float* scores, cudaStream_t s);
+
+// Head confidence and visual-head selection (Sec. 4.4): per sample,
+//   C[head] = sum over confidence rows j of M2(j) / N_v (population variance of
+//   the row's visual probabilities, its chunk statistics merged in chunk order),
+// then the n_vis heads of largest C (ties to the lower position in the head
+// list), in ascending list position:
+//   sel_out[b][s]       position in the head list (for the partial sums),
+//   vis_heads_out[b][s] head index (optional), conf_out[b][heads[i]] = C (optional).
+// pdl: launched as a programmatic dependent of the head-score kernel.
+struct ConfArgs {
+  int n_vis;
+  int* sel_out;        // [B][n_vis]
+  int* vis_heads_out;  // [B][n_vis] or null
+  float* conf_out;     // [B][H_q] or null
+};
+cudaError_t conf_select_launch(const HSArgs& a, const ConfGeom& g, const ConfArgs& c,
+                               cudaStream_t s, bool pdl = false);
 
 // ---------------------------------------------------------------------------
 // top-k (ties to the lower index, ascending output)
@@ -69,6 +108,10 @@ struct TopkArgs {
   const uint8_t* row_mask;
   int N_t_max;
   int H_sel;
+  // optional per-sample head subset [B][n_sel] (positions in the head list,
+  // ascending): only those heads' partials are summed, divided by n_sel x rows
+  const int* sel;
+  int n_sel;
   float* scores_out;         // optional [B][N]
   int B, N, k;
   int* idx_out;              // [B][k]

@@ -6,6 +6,8 @@
 // When fed head partials (the in-LLM path), the kernel first sums them per
 // column in a fixed order and divides by (heads x valid text rows): the same
 // arithmetic as the stand-alone score reduction, so both give identical bits.
+// With a per-sample head subset (the visual heads picked by their confidence)
+// only the subset's partials are summed, in head-list order.
 #include "common.cuh"
 #include "kernels.h"
 #include "topk_block.cuh"
@@ -39,9 +41,14 @@ __global__ void __launch_bounds__(kTopkMaxThreads) topk_kernel(const TopkArgs a)
   const int N = a.N;
   float* so = a.scores_out ? a.scores_out + (size_t)b * N : nullptr;
   if (a.partial != nullptr) {
-    const int nrows = block_count_rows(a, b);
-    topk_load_partials<false>(a.partial + (size_t)b * a.n_part * N, a.n_part, N,
-                              (float)a.H_sel * (float)nrows, nrows <= 0, so, keys);
+    __shared__ int sel[kMaxHeads];
+    if (a.sel != nullptr)
+      for (int q = threadIdx.x; q < a.n_sel; q += blockDim.x) sel[q] = a.sel[(size_t)b * a.n_sel + q];
+    const int nrows = block_count_rows(a, b);  // synchronises the block
+    const float nh = (float)(a.sel != nullptr ? a.n_sel : a.H_sel);
+    topk_load_partials<false>(a.partial + (size_t)b * a.n_part * N, a.n_part, N, nh * (float)nrows,
+                              nrows <= 0, so, keys, a.sel != nullptr ? sel : nullptr, a.n_sel,
+                              a.H_sel);
   } else {
     for (int i = threadIdx.x; i < N; i += blockDim.x) {
       const float v = a.scores[(size_t)b * N + i];

@@ -1,7 +1,6 @@
 // Block-wide top-k of one sample held in shared memory (Sec. 4.3 top N1, Sec.
 // 4.4 top N2): ties broken toward the lower index, indices in ascending order.
-// Used by the stand-alone top-k kernel and by the tail of the one-pass head-score
-// kernel. Any block size that is a multiple of 32 (<= 1024) works.
+// Used by the top-k kernel. Any block size that is a multiple of 32 (<= 1024) works.
 //
 // keys[0..N) are order-preserving uint32 keys (float_key). An 8-bit MSD radix
 // select (4 passes of a 256-bin shared histogram, one increment per group of
@@ -133,15 +132,27 @@ __device__ __forceinline__ void topk_block_select(const uint32_t* keys, int N, i
   }
 }
 
-// v_i = (sum over u of partial[u][i], in order) / (H_sel x rows): the head-score
-// reduction shared by every path, so all of them give identical bits.
+// v_i = (sum over u of partial[row(u)][i], in order) / div: the head-score
+// reduction shared by every path, so all of them give identical bits. Without
+// a head subset, row(u) = u for u < n_part; with one (sel, n_sel positions in a
+// head list of H_sel, in shared memory), row(u) = (u / n_sel) * H_sel +
+// sel[u % n_sel] for u < (n_part / H_sel) * n_sel: the same rows, in the same
+// order, as a head list made of the subset alone.
 // Loads keys[i] and optionally writes the scores. cg: read through L2 only
 // (the partials were written by other CTAs of a still-running grid).
 template <bool CG>
 __device__ __forceinline__ void topk_load_partials(const float* P0, int n_part, int N, float div,
-                                                   bool zero, float* scores_out, uint32_t* keys) {
+                                                   bool zero, float* scores_out, uint32_t* keys,
+                                                   const int* sel = nullptr, int n_sel = 0,
+                                                   int H_sel = 1) {
   const int tid = threadIdx.x, nth = blockDim.x;
-  if (n_part <= 8) {
+  const int n_sum = sel ? (n_part / H_sel) * n_sel : n_part;
+  auto row = [&](int u) -> int { return sel ? (u / n_sel) * H_sel + sel[u % n_sel] : u; };
+  auto ld = [&](size_t off) -> float { return CG ? __ldcg(P0 + off) : __ldg(P0 + off); };
+  if (n_sum <= 8) {
+    int ro[8];  // row offsets: n_part x N is below 2^31 (N <= 49152, n_part <= 2^15)
+#pragma unroll
+    for (int u = 0; u < 8; ++u) ro[u] = u < n_sum ? row(u) * N : 0;
     for (int i0 = 0; i0 < N; i0 += 4 * nth) {
       float t[4][8];
 #pragma unroll
@@ -149,7 +160,7 @@ __device__ __forceinline__ void topk_load_partials(const float* P0, int n_part, 
         const int i = i0 + c * nth + tid;
 #pragma unroll
         for (int u = 0; u < 8; ++u)
-          if (u < n_part && i < N) t[c][u] = CG ? __ldcg(P0 + (size_t)u * N + i) : __ldg(P0 + (size_t)u * N + i);
+          if (u < n_sum && i < N) t[c][u] = ld((size_t)ro[u] + i);
       }
 #pragma unroll
       for (int c = 0; c < 4; ++c) {
@@ -158,7 +169,7 @@ __device__ __forceinline__ void topk_load_partials(const float* P0, int n_part, 
         float s = 0.f;
 #pragma unroll
         for (int u = 0; u < 8; ++u)
-          if (u < n_part) s += t[c][u];
+          if (u < n_sum) s += t[c][u];
         const float v = zero ? 0.f : s / div;
         if (scores_out) scores_out[i] = v;
         keys[i] = float_key(v);
@@ -167,7 +178,7 @@ __device__ __forceinline__ void topk_load_partials(const float* P0, int n_part, 
   } else {
     for (int i = tid; i < N; i += nth) {
       float s = 0.f;
-      for (int u = 0; u < n_part; ++u) s += CG ? __ldcg(P0 + (size_t)u * N + i) : __ldg(P0 + (size_t)u * N + i);
+      for (int u = 0; u < n_sum; ++u) s += ld((size_t)row(u) * N + i);
       const float v = zero ? 0.f : s / div;
       if (scores_out) scores_out[i] = v;
       keys[i] = float_key(v);

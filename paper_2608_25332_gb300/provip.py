@@ -60,6 +60,12 @@ _SIGS = {
     "provip_prune_workspace_size": (_Z, [_I, _I, _I, _I, _I, _I, _I]),
     "provip_prune": (_I, [_P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _P, _I, _P, _P, _P, _I, _I, _I, _P, _P,
                           _I, _I, _I, _I, _P, _P, _P, _P, _P, _P, _P, _P, _Z, ctypes.c_uint, _P]),
+    "provip_visual_heads_workspace_size": (_Z, [_I, _I, _I, _I, _I, _I, _I, _I]),
+    "provip_head_confidence": (_I, [_P, _P, _I, _I, _I, _I, _I, _P, _P, _P, _I, _I, _I, _P, _I, _I, _I,
+                                    _P, _P, _P, _Z, _P]),
+    "provip_prune_visual_heads": (_I, [_P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _P, _P, _P, _I, _I, _I, _P,
+                                       _P, _I, _I, _I, _I, _I, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _Z,
+                                       ctypes.c_uint, _P]),
 }
 
 
@@ -229,8 +235,11 @@ def provip_similarity_reduce(emb_v, emb_t, text_len, keep_pre, crit_mask=None, w
 # ---------------------------------------------------------------------------
 # in-LLM pass
 # ---------------------------------------------------------------------------
-def _heads_arg(head_list):
-    """head_list is read on the host (a list, a CPU tensor, or a device tensor copied once)."""
+def _heads_arg(head_list, H_q):
+    """head_list is read on the host (a list, a CPU tensor, or a device tensor copied once);
+    None means every head (a NULL list with H_sel = H_q)."""
+    if head_list is None:
+        return None, int(H_q)
     hl = [int(h) for h in (head_list.tolist() if hasattr(head_list, "tolist") else head_list)]
     arr = (ctypes.c_int * len(hl))(*hl)
     return arr, len(hl)
@@ -241,7 +250,7 @@ def provip_head_scores(Q, K, head_list, text_start, text_len, seq_len, vis_start
     B, Lm, Hq, dh = Q.shape
     Hkv = K.shape[2]
     dev = Q.device
-    heads, hs = _heads_arg(head_list)
+    heads, hs = _heads_arg(head_list, Hq)
     Ntm = int(N_t_max if N_t_max is not None else (row_mask.shape[1] if row_mask is not None
                                                    else int(text_len.max().item())))
     scores = torch.empty((B, N_v), dtype=torch.float32, device=dev)
@@ -304,7 +313,7 @@ class PruneStep:
                  want_scores=True, flags=0, ws=None):
         B, Lm, Hq, dh = Q.shape
         self.shape = (B, Lm, Hq, K.shape[2], dh, hidden.shape[2])
-        self.heads, self.H_sel = _heads_arg(head_list)
+        self.heads, self.H_sel = _heads_arg(head_list, Q.shape[2])
         self.N_t_max, self.N_v, self.keep, self.algo = int(N_t_max), int(N_v), int(keep), algo
         self.flags = int(flags)
         dev = Q.device
@@ -346,7 +355,7 @@ def provip_head_topk(Q, K, head_list, text_start, text_len, seq_len, vis_start, 
     B, Lm, Hq, dh = Q.shape
     Hkv = K.shape[2]
     dev = Q.device
-    heads, hs = _heads_arg(head_list)
+    heads, hs = _heads_arg(head_list, Hq)
     Ntm = int(N_t_max if N_t_max is not None else int(text_len.max().item()))
     idx = torch.empty((B, keep), dtype=torch.int32, device=dev)
     scores = torch.empty((B, N_v), dtype=torch.float32, device=dev) if want_scores else None
@@ -370,7 +379,7 @@ def provip_head_scores_noalloc(Q, K, head_list, text_start, text_len, seq_len, v
     B, Lm, Hq, dh = Q.shape
     Hkv = K.shape[2]
     dev = Q.device
-    heads, hs = _heads_arg(head_list)
+    heads, hs = _heads_arg(head_list, Hq)
     Ntm = int(N_t_max if N_t_max is not None else int(text_len.max().item()))
     scores = torch.empty((B, N_v), dtype=torch.float32, device=dev)
     rc = lib().provip_head_scores_noalloc(_ptr(Q), _ptr(K), B, Lm, Hq, Hkv, dh, heads, hs, _i32(text_start),
@@ -378,3 +387,78 @@ def provip_head_scores_noalloc(Q, K, head_list, text_start, text_len, seq_len, v
                                           _dtype_code(Q), algo, _ptr(scores), _stream(dev))
     _check(rc, "provip_head_scores_noalloc")
     return scores
+
+
+# ---------------------------------------------------------------------------
+# visual-head identification (Sec. 4.4)
+# ---------------------------------------------------------------------------
+def provip_head_confidence(Q, K, text_start, text_len, seq_len, vis_start, N_v, N_vis,
+                           crit_mask=None, algo=ALGO_AUTO, N_t_max=None, ws=None, want_conf=True):
+    """Head confidence C [B, H_q] over the critical rows and the N_vis visual heads
+    [B, N_vis] (ascending) of every sample. Returns (vis_heads, conf or None)."""
+    B, Lm, Hq, dh = Q.shape
+    Hkv = K.shape[2]
+    dev = Q.device
+    Ntm = int(N_t_max if N_t_max is not None else (crit_mask.shape[1] if crit_mask is not None
+                                                   else int(text_len.max().item())))
+    vis = torch.empty((B, N_vis), dtype=torch.int32, device=dev)
+    conf = torch.empty((B, Hq), dtype=torch.float32, device=dev) if want_conf else None
+    L = lib()
+    dt = _dtype_code(Q)
+    need = L.provip_visual_heads_workspace_size(B, Lm, Hq, Ntm, N_v, N_vis, algo, dt)
+    if ws is None or ws.numel() < need:
+        ws = workspace(need, dev)
+    rc = L.provip_head_confidence(_ptr(Q), _ptr(K), B, Lm, Hq, Hkv, dh, _i32(text_start),
+                                  _i32(text_len), _u8(crit_mask), Ntm, vis_start, N_v, _i32(seq_len),
+                                  N_vis, dt, algo, _ptr(conf), _ptr(vis), _ptr(ws), ws.numel(),
+                                  _stream(dev))
+    _check(rc, "provip_head_confidence")
+    return vis, conf
+
+
+class VisualHeadsPruneStep:
+    """Pre-allocated outputs + workspace for repeated provip_prune_visual_heads calls."""
+
+    def __init__(self, Q, K, V, hidden, pos, N_t_max, N_v, keep, N_vis, algo=ALGO_AUTO,
+                 want_scores=True, want_conf=True, flags=0, ws=None):
+        B, Lm, Hq, dh = Q.shape
+        self.shape = (B, Lm, Hq, K.shape[2], dh, hidden.shape[2])
+        self.N_t_max, self.N_v, self.keep, self.N_vis, self.algo = int(N_t_max), int(N_v), int(keep), int(N_vis), algo
+        self.flags = int(flags)
+        dev = Q.device
+        self.dtype = _dtype_code(Q)
+        L_out = Lm - N_v + keep
+        self.hidden_out, self.K_out, self.V_out, self.pos_out = _outs(hidden, K, V, pos, B, L_out)
+        self.idx = torch.empty((B, keep), dtype=torch.int32, device=dev)
+        self.seq_len_out = torch.empty(B, dtype=torch.int32, device=dev)
+        self.scores = torch.empty((B, N_v), dtype=torch.float32, device=dev) if want_scores else None
+        self.vis_heads = torch.empty((B, self.N_vis), dtype=torch.int32, device=dev)
+        self.conf = torch.empty((B, Hq), dtype=torch.float32, device=dev) if want_conf else None
+        need = lib().provip_visual_heads_workspace_size(B, Lm, Hq, self.N_t_max, N_v, self.N_vis, algo,
+                                                        self.dtype)
+        self.ws = ws if ws is not None and ws.numel() >= need else workspace(need, dev)
+
+    def __call__(self, Q, K, V, hidden, pos, text_start, text_len, seq_len, vis_start,
+                 crit_mask=None, stream=None):
+        B, Lm, Hq, Hkv, dh, D = self.shape
+        P = pos.shape[0] if pos is not None else 0
+        st = ctypes.c_void_p(stream.cuda_stream) if stream is not None else _stream(Q.device)
+        rc = lib().provip_prune_visual_heads(
+            _ptr(Q), _ptr(K), _ptr(V), _ptr(hidden), B, Lm, Hq, Hkv, dh, D, _i32(text_start),
+            _i32(text_len), _u8(crit_mask), self.N_t_max, vis_start, self.N_v, _i32(seq_len),
+            _i32(pos), P, self.N_vis, self.keep, self.dtype, self.algo, _ptr(self.hidden_out),
+            _ptr(self.K_out), _ptr(self.V_out), _i32(self.pos_out), _ptr(self.idx),
+            _i32(self.seq_len_out), _ptr(self.scores), _ptr(self.vis_heads), _ptr(self.conf),
+            _ptr(self.ws), self.ws.numel(), self.flags, st)
+        _check(rc, "provip_prune_visual_heads")
+        return dict(hidden=self.hidden_out, K=self.K_out, V=self.V_out, pos=self.pos_out,
+                    idx=self.idx, seq_len=self.seq_len_out, scores=self.scores,
+                    vis_heads=self.vis_heads, conf=self.conf)
+
+
+def provip_prune_visual_heads(Q, K, V, hidden, pos, text_start, text_len, seq_len, vis_start, N_v,
+                              keep, N_vis, crit_mask=None, algo=ALGO_AUTO, N_t_max=None):
+    Ntm = int(N_t_max if N_t_max is not None else (crit_mask.shape[1] if crit_mask is not None
+                                                   else int(text_len.max().item())))
+    step = VisualHeadsPruneStep(Q, K, V, hidden, pos, Ntm, N_v, keep, N_vis, algo)
+    return step(Q, K, V, hidden, pos, text_start, text_len, seq_len, vis_start, crit_mask)

@@ -47,6 +47,7 @@ import numpy as np
 import torch
 
 N_SYS = 35
+VISUAL_FOCUS = 12.0  # query offset of a planted visual head (a typical query norm is ~11.3)
 D_HEAD = 128
 SEED_BASE = 20260000
 
@@ -212,8 +213,15 @@ def pre_llm_inputs(w: Workload, device="cpu", seed: int | None = None, batch: in
 
 
 def in_llm_inputs(w: Workload, device="cpu", seed: int | None = None, batch: int | None = None,
-                  with_kv: bool = True):
-    """Inputs of the in-LLM pruning step (Sec. 4.4) at the pruning layer."""
+                  with_kv: bool = True, visual_heads: bool = False, focus: float = VISUAL_FOCUS):
+    """Inputs of the in-LLM pruning step (Sec. 4.4) at the pruning layer.
+
+    visual_heads: the heads of head_list become planted visual heads - on the
+    text rows their queries get `focus` times the unit direction of the summed
+    keys of 16 seeded visual rows of the sample (per key/value group), so their
+    attention concentrates on those tokens (sharp focus on a few visual tokens,
+    the behaviour the paper's head confidence detects). Drawn from a separate
+    stream: every other value is the same as without it."""
     seed = w.seed if seed is None else seed
     B = w.B if batch is None else batch
     tl_all = text_lengths(w, seed)
@@ -257,6 +265,14 @@ def in_llm_inputs(w: Workload, device="cpu", seed: int | None = None, batch: int
             t0 = vis_start + 24
             for p in range(3):
                 pos[p, b, vis_start + nv:L] = t0 + np.arange(L - vis_start - nv)
+        if visual_heads:
+            rv = _rng(seed, 6000 + b)
+            focus_rows = vis_start + rv.choice(nv, size=16, replace=False)
+            t0, t1 = int(text_start[b]), int(text_start[b] + tl[b])
+            for h in heads:
+                g = h // group
+                d = K[b, focus_rows, g].sum(axis=0)
+                Q[b, t0:t1, h] += focus * d / np.linalg.norm(d)
         for arr in (Q, K, V, H):
             if arr is not None:
                 arr[b, L:] = np.nan

@@ -74,6 +74,34 @@ def test_head_scores_validation(L):
     assert b"workspace" in L.provip_last_error()
 
 
+def test_all_heads_null_list_validation(L):
+    hs = lambda heads, n, Hq=8: L.provip_head_scores(
+        FAKE, FAKE, 2, 100, Hq, 4, 128, heads, n, FAKE, FAKE, None, 16, 10, 50, FAKE, 1, 0, FAKE, None, 0, None)
+    assert hs(None, 4) == -1                  # a NULL list means every head: needs H_sel == H_q
+    assert hs(None, 8) == -3                  # accepted; only the workspace is missing
+    assert hs(None, 72, Hq=72) == -1          # more than 64 heads
+
+
+def test_visual_heads_validation(L):
+    conf = lambda nvis, **kw: L.provip_head_confidence(
+        FAKE, FAKE, 2, 100, kw.get("Hq", 8), 4, 128, FAKE, FAKE, None, 16, 10, 50, FAKE, nvis, 1, 0, None,
+        kw.get("out", FAKE), None, 0, None)
+    assert conf(0) == -1                      # N_vis < 1
+    assert conf(9) == -1                      # N_vis > H_q
+    assert conf(2, Hq=72) == -2               # more than 64 heads
+    assert conf(2, out=None) == -1            # vis_heads_out is required
+    assert conf(2) == -3                      # workspace too small
+    need = L.provip_visual_heads_workspace_size(2, 100, 8, 16, 50, 2, 0, 1)
+    assert need > L.provip_head_scores_workspace_size(2, 100, 8, 16, 50, 0, 1)
+    prune = lambda keep, flags=0: L.provip_prune_visual_heads(
+        FAKE, FAKE, FAKE, FAKE, 2, 100, 8, 4, 128, 64, FAKE, FAKE, None, 16, 10, 50, FAKE, None, 0, 2, keep,
+        1, 0, FAKE, FAKE, FAKE, None, FAKE, None, None, None, None, None, 0, flags, None)
+    assert prune(0) == -1                     # keep < 1
+    assert prune(51) == -1                    # keep > N_v
+    assert prune(5, flags=4) == -1            # unknown flag
+    assert prune(5) == -3                     # workspace too small
+
+
 def test_topk_and_compact_validation(L):
     assert L.provip_topk(FAKE, 1, 10, 0, FAKE, None) == -1
     assert L.provip_topk(FAKE, 1, 10, 11, FAKE, None) == -1
