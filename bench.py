@@ -45,6 +45,7 @@ DEFAULT_WORKLOAD = "llava_next_7b_bf16_b8"
 FALLBACK_HBM_GBS = 6800.0
 GRAPH_CHUNK = 100
 N_COPIES = 3
+N_VIS = 6  # visual heads per pruning layer (the paper's setting, Sec. 5.1)
 
 # DRAM traffic of one compaction launch on the default workload, from the ncu
 # capture summarised in profiles/ (null when the kernel source has changed
@@ -180,6 +181,44 @@ def prellm_measure(w, dev, reps=20):
                                 "peak_source": src, "unit": "TFLOP/s", "frac": ach / peak}}
 
 
+def schedule_measure(w, dev, reps=10):
+    """The progressive schedule (Sec. 4.1) on the workload's batch: pre-LLM
+    N_v -> keep_pre, shallow layer keep_pre -> keep with each sample's N_VIS
+    visual heads, middle layer keep -> keep / 2 over every head; one CUDA graph
+    per call, timed back to back (one input set larger than L2)."""
+    import torch
+    from paper_2608_25332_gb300 import synth
+    from paper_2608_25332_gb300.schedule import ProgressiveSchedule
+    cpu = synth.schedule_inputs(w)
+    g = {k: {kk: (vv.to(dev) if isinstance(vv, torch.Tensor) else vv) for kk, vv in v.items()}
+         for k, v in cpu.items()}
+    n3 = w.keep // 2
+    sched = ProgressiveSchedule(w.B, w.N_v, w.D, w.n_t[1], w.L_max, w.H_q, w.H_kv, w.D, w.P, w.keep_pre,
+                                w.keep, n3, min(N_VIS, w.H_q), dtype=w.torch_dtype, device=dev)
+    sh = g["shallow"]
+    call = lambda: sched(g["pre"]["emb_v"], g["pre"]["emb_t"], g["pre"]["text_len"], sh, g["middle"],
+                         sh["vis_start"])
+    for _ in range(3):
+        call()
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    stream = torch.cuda.Stream(device=dev)
+    with torch.cuda.graph(graph, stream=stream):
+        call()
+    graph.replay()
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for _ in range(reps):
+        graph.replay()
+    b.record()
+    torch.cuda.synchronize()
+    us = a.elapsed_time(b) / reps * 1e3
+    return {"workload": w.name, "stages": f"{w.N_v} -> {w.keep_pre} -> {w.keep} -> {n3} visual tokens",
+            "n_vis": min(N_VIS, w.H_q), "us_per_call": us, "samples_per_s": w.B / us * 1e6,
+            "host_syncs": 0}
+
+
 class ClockSampler:
     FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
@@ -263,19 +302,22 @@ def workload_config(w, algo="auto", copies=N_COPIES, input_mb=None):
                        "step's compaction (PROVIP_PRUNE_OVERLAP_PREVIOUS)"}
 
 
-def algorithmic_bytes(w, inp):
+def algorithmic_bytes(w, inp, all_heads=False):
+    """bytes the step must move: keys of the key/value heads the scored heads use
+    and the scored heads' text queries (read once), scores and indices, and the
+    compaction's reads + writes of the surviving rows"""
     import numpy as np
     es = 4 if w.dtype == "f32" else 2
     dh = 128
     seq = inp["seq_len"].cpu().numpy().astype(np.int64)
     tl = inp["text_len"].cpu().numpy().astype(np.int64)
-    heads = inp["head_list"].cpu().numpy()
+    heads = np.arange(w.H_q) if all_heads else inp["head_list"].cpu().numpy()
     group = w.H_q // w.H_kv
     n_kv_used = len(set(int(h) // group for h in heads))
     out_rows = seq - w.keep_pre + w.keep
     row = (w.D + 2 * w.H_kv * dh) * es
     compact = int((2 * out_rows * row).sum() + (2 * out_rows * w.P * 4).sum() + w.B * w.keep * 4)
-    scores = int((seq * n_kv_used * dh * es).sum() + (tl * w.H_sel * dh * es).sum()
+    scores = int((seq * n_kv_used * dh * es).sum() + (tl * len(heads) * dh * es).sum()
                  + w.B * w.keep_pre * 4 + w.B * w.keep * 4)
     return {"compact": compact, "head_topk": scores, "path": compact + scores}
 
@@ -311,7 +353,7 @@ def oracle_step(o, w, samples, vis_start, N_v, keep, threads):
                               o["pos"][:, sel], threads=threads)
 
 
-def cpu_baseline(cpu, w, vis_start, N_v, keep, budget_s=4.0):
+def cpu_baseline(cpu, w, vis_start, N_v, keep, budget_s=12.0):
     """The oracle on the workload's samples, all host cores, repeated until ~budget_s wall."""
     import oracle
     oracle.build()
@@ -325,7 +367,7 @@ def cpu_baseline(cpu, w, vis_start, N_v, keep, budget_s=4.0):
         done += B
         reps += 1
         el = time.perf_counter() - t0
-        if el >= budget_s or reps >= 20:
+        if el >= budget_s or reps >= 400:
             break
     used = min(threads, B)
     return {"value": done / el, "unit": UNIT, "cores": used, "kind": "oracle",
@@ -531,6 +573,35 @@ def run_gb300(args, dist):
 
     t_serial = time_graph(serial_i, reps)
     peak, peak_src = hbm_peak()
+
+    # the next rows on the same batches: shallow-layer pruning with the N_VIS
+    # most confident heads of each sample (confidence over every head), and
+    # the middle-layer variant over every head
+    ab_all = algorithmic_bytes(w, cpu, all_heads=True)
+    vh = P.VisualHeadsPruneStep(g0["Q"], g0["K"], g0["V"], g0["hidden"], g0["pos"], w.n_t[1], nv, keep,
+                                min(N_VIS, w.H_q), algo=algo, want_scores=False, want_conf=False,
+                                flags=P.PRUNE_OVERLAP_PREVIOUS)
+    ah = P.PruneStep(g0["Q"], g0["K"], g0["V"], g0["hidden"], g0["pos"], None, w.n_t[1], nv, keep,
+                     algo=algo, want_scores=False, flags=P.PRUNE_OVERLAP_PREVIOUS)
+
+    def vh_i(i):
+        c = copies[i % len(copies)]
+        vh(c["Q"], c["K"], c["V"], c["hidden"], c["pos"], c["text_start"], c["text_len"], c["seq_len"], vis)
+
+    def ah_i(i):
+        c = copies[i % len(copies)]
+        ah(c["Q"], c["K"], c["V"], c["hidden"], c["pos"], c["text_start"], c["text_len"], c["seq_len"], vis)
+
+    next_rows = {}
+    for name, fn, extra in (("visual_heads", vh_i, {"n_vis": min(N_VIS, w.H_q), "heads_scored": w.H_q}),
+                            ("all_heads", ah_i, {"heads_scored": w.H_q})):
+        t = time_graph(fn, reps)
+        gbs = ab_all["path"] / t / 1e9
+        next_rows[name] = dict(extra, us_per_step=t * 1e6, samples_per_s=w.B / t,
+                               algorithmic_bytes=ab_all["path"], achieved_gbs=gbs, frac=gbs / peak)
+    rc, bits = P.provip_device_status(clear=True)
+    if rc != 0:
+        raise RuntimeError(f"device status {rc} {bits} after the next-row legs")
     ach = ab["compact"] / t_compact / 1e9
     traffic = None
     if COMPACT_TRAFFIC["bytes"] and COMPACT_TRAFFIC["sha1"] == kernel_sha1("compact.cu") and \
@@ -570,6 +641,7 @@ def run_gb300(args, dist):
     e2e_value = aggregate(dist.sum(float(w.B * E)), e2e_sec)
 
     prellm = prellm_measure(w, dev) if dist.rank == 0 else None
+    schedule = schedule_measure(w, dev) if dist.rank == 0 else None
 
     cpu_base = None
     if dist.rank == 0 and dist.world == 1 and not args.no_cpu_baseline:
@@ -594,6 +666,7 @@ def run_gb300(args, dist):
             "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
             "gpu_launches": launches_per_step * K,
             "prellm": prellm,
+            "next_rows": dict(next_rows, schedule=schedule),
             "clocks": clocks,
         }
         print(json.dumps(line))

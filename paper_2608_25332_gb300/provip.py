@@ -211,15 +211,19 @@ def provip_merge(emb_v, keep_idx, want_merged=True):
 
 
 def provip_similarity_reduce(emb_v, emb_t, text_len, keep_pre, crit_mask=None, want_merged=True,
-                             ws=None):
-    """Sec. 4.2-4.3 end to end. Returns dict(idx, merged, p, mask)."""
+                             ws=None, out=None):
+    """Sec. 4.2-4.3 end to end. Returns dict(idx, merged, p, mask); out: the same
+    dict of pre-allocated outputs to write instead."""
     B, Nv, D = emb_v.shape
     Ntm = emb_t.shape[1]
     dev = emb_v.device
-    idx = torch.empty((B, keep_pre), dtype=torch.int32, device=dev)
-    merged = torch.empty((B, keep_pre, D), dtype=emb_v.dtype, device=dev) if want_merged else None
-    p = torch.empty((B, Nv), dtype=torch.float32, device=dev)
-    mask = torch.empty((B, Ntm), dtype=torch.uint8, device=dev)
+    if out is not None:
+        idx, merged, p, mask = out["idx"], out.get("merged"), out["p"], out["mask"]
+    else:
+        idx = torch.empty((B, keep_pre), dtype=torch.int32, device=dev)
+        merged = torch.empty((B, keep_pre, D), dtype=emb_v.dtype, device=dev) if want_merged else None
+        p = torch.empty((B, Nv), dtype=torch.float32, device=dev)
+        mask = torch.empty((B, Ntm), dtype=torch.uint8, device=dev)
     L = lib()
     need = L.provip_similarity_reduce_workspace_size(B, Nv, D, Ntm, keep_pre)
     if ws is None or ws.numel() < need:
@@ -266,8 +270,8 @@ def provip_head_scores(Q, K, head_list, text_start, text_len, seq_len, vis_start
     return scores
 
 
-def _outs(hidden, K, V, pos, B, L_out):
-    dev = hidden.device
+def _outs(hidden, K, V, pos, B, L_out, device=None):
+    dev = hidden.device if device is None else device
     ho = torch.empty((B, L_out) + tuple(hidden.shape[2:]), dtype=hidden.dtype, device=dev)
     ko = torch.empty((B, L_out) + tuple(K.shape[2:]), dtype=K.dtype, device=dev) if K is not None else None
     vo = torch.empty((B, L_out) + tuple(V.shape[2:]), dtype=V.dtype, device=dev) if V is not None else None
@@ -310,16 +314,18 @@ class PruneStep:
     """Pre-allocated outputs + workspace for repeated provip_prune calls (one shape)."""
 
     def __init__(self, Q, K, V, hidden, pos, head_list, N_t_max, N_v, keep, algo=ALGO_AUTO,
-                 want_scores=True, flags=0, ws=None):
+                 want_scores=True, flags=0, ws=None, device=None):
+        """Q, K, V, hidden, pos give the shapes and dtypes (meta tensors are fine
+        with device=...)."""
         B, Lm, Hq, dh = Q.shape
         self.shape = (B, Lm, Hq, K.shape[2], dh, hidden.shape[2])
         self.heads, self.H_sel = _heads_arg(head_list, Q.shape[2])
         self.N_t_max, self.N_v, self.keep, self.algo = int(N_t_max), int(N_v), int(keep), algo
         self.flags = int(flags)
-        dev = Q.device
+        dev = Q.device if device is None else torch.device(device)
         self.dtype = _dtype_code(Q)
         L_out = Lm - N_v + keep
-        self.hidden_out, self.K_out, self.V_out, self.pos_out = _outs(hidden, K, V, pos, B, L_out)
+        self.hidden_out, self.K_out, self.V_out, self.pos_out = _outs(hidden, K, V, pos, B, L_out, dev)
         self.idx = torch.empty((B, keep), dtype=torch.int32, device=dev)
         self.seq_len_out = torch.empty(B, dtype=torch.int32, device=dev)
         self.scores = torch.empty((B, N_v), dtype=torch.float32, device=dev) if want_scores else None
@@ -420,15 +426,17 @@ class VisualHeadsPruneStep:
     """Pre-allocated outputs + workspace for repeated provip_prune_visual_heads calls."""
 
     def __init__(self, Q, K, V, hidden, pos, N_t_max, N_v, keep, N_vis, algo=ALGO_AUTO,
-                 want_scores=True, want_conf=True, flags=0, ws=None):
+                 want_scores=True, want_conf=True, flags=0, ws=None, device=None):
+        """Q, K, V, hidden, pos give the shapes and dtypes (meta tensors are fine
+        with device=...)."""
         B, Lm, Hq, dh = Q.shape
         self.shape = (B, Lm, Hq, K.shape[2], dh, hidden.shape[2])
         self.N_t_max, self.N_v, self.keep, self.N_vis, self.algo = int(N_t_max), int(N_v), int(keep), int(N_vis), algo
         self.flags = int(flags)
-        dev = Q.device
+        dev = Q.device if device is None else torch.device(device)
         self.dtype = _dtype_code(Q)
         L_out = Lm - N_v + keep
-        self.hidden_out, self.K_out, self.V_out, self.pos_out = _outs(hidden, K, V, pos, B, L_out)
+        self.hidden_out, self.K_out, self.V_out, self.pos_out = _outs(hidden, K, V, pos, B, L_out, dev)
         self.idx = torch.empty((B, keep), dtype=torch.int32, device=dev)
         self.seq_len_out = torch.empty(B, dtype=torch.int32, device=dev)
         self.scores = torch.empty((B, N_v), dtype=torch.float32, device=dev) if want_scores else None

@@ -300,3 +300,33 @@ def random_scores(B: int, N: int, seed: int, ties: bool = True) -> torch.Tensor:
         mask = rng.random((B, N)) < 0.33
         s[mask] = pool[rng.integers(0, 5, size=int(mask.sum()))]
     return torch.from_numpy(s)
+
+
+def schedule_inputs(w: Workload, device="cpu", seed: int | None = None, batch: int | None = None):
+    """Inputs of the progressive schedule (Sec. 4.1): the pre-LLM inputs, the
+    shallow pruning layer's inputs (keep_pre visual rows, planted visual heads)
+    and the middle layer's queries over the sequence the shallow layer leaves
+    (L_max - keep_pre + keep rows: 35 system rows, keep visual rows, the text).
+    The middle layer's keys, values, hidden states and position ids are the
+    shallow layer's compacted outputs, so they are not drawn here. Middle-layer
+    queries: N(0, 1) + u_g as at the shallow layer, NaN past the sequence."""
+    seed = w.seed if seed is None else seed
+    B = w.B if batch is None else batch
+    pre = pre_llm_inputs(w, seed=seed, batch=B)
+    shallow = in_llm_inputs(w, seed=seed, batch=B, visual_heads=True)
+    rng = _rng(seed, 3000)
+    rng.choice(w.H_q, size=w.H_sel, replace=False)  # same draws as in_llm_inputs
+    U = np.stack([_unit(rng, D_HEAD) for _ in range(w.H_kv)])
+    L2 = w.L_max - w.keep_pre + w.keep
+    tl = shallow["text_len"].numpy()
+    Q = np.empty((B, L2, w.H_q, D_HEAD), np.float32)
+    for b in range(B):
+        r = _rng(seed, 8000 + b)
+        Q[b] = r.standard_normal((L2, w.H_q, D_HEAD), dtype=np.float32)
+        Q[b] += np.repeat(U, w.H_q // w.H_kv, axis=0)[None]
+        Q[b, N_SYS + w.keep + int(tl[b]):] = np.nan
+    middle = dict(Q=_cast(Q, w.torch_dtype).to(device),
+                  text_start=torch.full((B,), N_SYS + w.keep, dtype=torch.int32).to(device))
+    return dict(pre={k: v.to(device) for k, v in pre.items()},
+                shallow={k: (v.to(device) if isinstance(v, torch.Tensor) else v) for k, v in shallow.items()},
+                middle=middle)
