@@ -60,12 +60,22 @@ extern "C" {
 /* kernel families for provip_head_scores / provip_prune */
 #define PROVIP_ALGO_AUTO 0    /* tensor cores for bf16, CUDA cores for fp32 */
 #define PROVIP_ALGO_SIMT 1    /* CUDA-core FFMA kernels (fp32 and bf16) */
-#define PROVIP_ALGO_TCGEN05 2 /* tcgen05 tensor cores, one pass over K in a cluster per
-                                 (head, sample), logits kept in TMEM (bf16 only); falls
-                                 back to the two-pass form when L_max > 8192 or no
-                                 cluster shape fits */
+#define PROVIP_ALGO_TCGEN05 2 /* tcgen05 tensor cores (bf16 only): the streaming form
+                                 when there are at least as many (sample, head, row
+                                 block) units as SMs, else the cluster form */
 #define PROVIP_ALGO_TCGEN05_TWOPASS 3 /* tcgen05, two kernels: chunk statistics, then
                                          probabilities (bf16 only) */
+#define PROVIP_ALGO_TCGEN05_STREAM 4  /* tcgen05, one CTA per (sample, head, row block)
+                                         streaming that head's keys through a TMA/TMEM
+                                         pipeline: every key, then the visual keys again
+                                         (from L2) (bf16 only) */
+#define PROVIP_ALGO_TCGEN05_CLUSTER 5 /* tcgen05, one pass over K in a cluster per (head,
+                                         sample), logits kept in TMEM (bf16 only); falls
+                                         back to the two-pass form when L_max > 8192 or
+                                         no cluster shape fits */
+/* Different kernel families sum in different orders: results agree within the
+ * floating-point tolerance, and are bit-identical between calls that take the
+ * same family (the same algo and, for PROVIP_ALGO_TCGEN05, the same choice). */
 
 /* bits of the device status word */
 #define PROVIP_DEVSTAT_TIMEOUT 1u  /* a bounded wait gave up */
@@ -315,7 +325,8 @@ int provip_head_confidence(const void *Q, const void *K, int B, int L_max, int H
  * sample over all its text rows (S^vis and v of Sec. 4.4), the top `keep` of v
  * (idx_out [B, keep] ascending, ties to the lower index) and the compaction of
  * provip_compact. One pass over the keys computes the attention statistics of
- * every head; the scores of a sample's visual heads are bit-identical to
+ * every head; with the same kernel family (algo STREAM, CLUSTER or TWOPASS on
+ * both sides) the scores of a sample's visual heads are bit-identical to
  * provip_prune called on that sample alone with head_list = its visual heads.
  * scores_out_or_null [B, N_v], vis_heads_out_or_null [B, N_vis] and
  * conf_out_or_null [B, H_q] receive v, the visual heads and C when non-NULL.

@@ -84,7 +84,16 @@ int resolve_algo(int algo, int dtype) {
   if (algo == PROVIP_ALGO_AUTO) return dtype == PROVIP_BF16 ? PROVIP_ALGO_TCGEN05 : PROVIP_ALGO_SIMT;
   return algo;
 }
-bool is_tc(int algo) { return algo == PROVIP_ALGO_TCGEN05 || algo == PROVIP_ALGO_TCGEN05_TWOPASS; }
+bool is_tc(int algo) {
+  return algo == PROVIP_ALGO_TCGEN05 || algo == PROVIP_ALGO_TCGEN05_TWOPASS ||
+         algo == PROVIP_ALGO_TCGEN05_STREAM || algo == PROVIP_ALGO_TCGEN05_CLUSTER;
+}
+// PROVIP_ALGO_TCGEN05: the streaming form once the (sample, head, row block)
+// units fill the SMs, else the cluster form (spreads one unit over its key chunks)
+int tc_form(int algo, int B, int H_sel, int n_rb, int sms) {
+  if (algo != PROVIP_ALGO_TCGEN05) return algo;
+  return (long long)B * H_sel * n_rb >= sms ? PROVIP_ALGO_TCGEN05_STREAM : PROVIP_ALGO_TCGEN05_CLUSTER;
+}
 int key_chunk(int algo) { return is_tc(algo) ? 128 : 64; }
 int vis_chunk(int algo) { return is_tc(algo) ? 128 : 64; }
 
@@ -110,7 +119,9 @@ size_t hs_ws(Carve& c, int B, int H_sel, const HSShape& s, int N_v, float2** sta
 // head confidence: chunk capacity per row (every chunk layout the resolved
 // path may take) and the workspace it needs
 int conf_stride(const HSShape& sh, int algo) {
-  return algo == PROVIP_ALGO_TCGEN05 ? (sh.n_vc > kFusedMaxChunks ? sh.n_vc : kFusedMaxChunks) : sh.n_vc;
+  return (algo == PROVIP_ALGO_TCGEN05 || algo == PROVIP_ALGO_TCGEN05_CLUSTER)
+             ? (sh.n_vc > kFusedMaxChunks ? sh.n_vc : kFusedMaxChunks)
+             : sh.n_vc;  // TWOPASS, SIMT: n_vc; STREAM uses 1
 }
 struct ConfWs {
   float2* part = nullptr;
@@ -196,6 +207,10 @@ int hs_run(const HSArgs& a, int dtype, int algo, cudaStream_t s, bool overlap = 
            ConfGeom* geom = nullptr) {
   cudaError_t e;
   if (is_tc(algo)) {
+    DevInfo* d;
+    int rc = dev_info(&d);
+    if (rc) return rc;
+    algo = tc_form(algo, a.B, a.H_sel, a.n_rb, d->sms);
     CUtensorMap tq, tk;
     const uint64_t qstride = (uint64_t)a.H_q * a.d_h * 2, kstride = (uint64_t)a.H_kv * a.d_h * 2;
     if (make_tmap_bf16_2d(&tq, a.Q, (uint64_t)a.B * a.L_max, (uint64_t)a.H_q * a.d_h, qstride, 128) ||
@@ -203,7 +218,12 @@ int hs_run(const HSArgs& a, int dtype, int algo, cudaStream_t s, bool overlap = 
       return fail(PROVIP_ERR_CUDA, "head_scores: cuTensorMapEncodeTiled failed");
     bool launched = false;
     e = cudaSuccess;
-    if (algo == PROVIP_ALGO_TCGEN05) e = hs_launch_fused(a, &tq, &tk, s, &launched, overlap, geom);
+    if (algo == PROVIP_ALGO_TCGEN05_STREAM) {
+      e = hs_launch_stream(a, &tq, &tk, s, overlap, geom);
+      launched = true;
+    } else if (algo == PROVIP_ALGO_TCGEN05_CLUSTER) {
+      e = hs_launch_fused(a, &tq, &tk, s, &launched, overlap, geom);
+    }
     if (e == cudaSuccess && !launched) e = hs_launch_tc(a, &tq, &tk, s, geom);
   } else {
     e = hs_launch_simt(a, dtype, s, geom);

@@ -202,6 +202,8 @@ __global__ void __launch_bounds__(kThreads, CPC == 1 ? 3 : (CPC == 2 ? 2 : 1))
   // is stored back in TMEM with mb the running max after its block.
   float mblk[kBlocks];
   float m = -INFINITY, l = 0.f;
+  const float sc = a.scale_log2;
+  const int t_first = ts + rb * kTile;  // every row of the block sits at or after it
   if (warp_live) {
 #pragma unroll
     for (int cb = 0; cb < kBlocks; ++cb) {
@@ -209,21 +211,30 @@ __global__ void __launch_bounds__(kThreads, CPC == 1 ? 3 : (CPC == 2 ? 2 : 1))
       tmem_ld32(tbase + cb * 32, v);
       tc_wait_ld();
       const int k0 = key0 + col0 + cb * 32;
-      float bm = -INFINITY;
+      float mn = m;
+      if (rv) {
+        // keys before the block's first row are causal for every row
+        float bm = -INFINITY;
+        if (k0 + 31 <= t_first) {
 #pragma unroll
-      for (int i = 0; i < 32; ++i) {
-        v[i] = (rv && k0 + i <= t) ? v[i] * a.scale_log2 : -INFINITY;
-        bm = fmaxf(bm, v[i]);
+          for (int i = 0; i < 32; ++i) bm = fmaxf(bm, v[i]);
+        } else {
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            v[i] = k0 + i <= t ? v[i] : -INFINITY;
+            bm = fmaxf(bm, v[i]);
+          }
+        }
+        mn = fmaxf(m, bm * sc);  // sc > 0: the max commutes with the scale
       }
-      const float mn = fmaxf(m, bm);
       if (mn != -INFINITY) {
         float s4[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
         for (int i = 0; i < 32; ++i) {
-          v[i] = exp2f(v[i] - mn);  // exp2f(-inf) = 0 for masked keys
+          v[i] = ex2_approx(fmaf(v[i], sc, -mn));  // 2^-inf = 0 for masked keys
           s4[i & 3] += v[i];
         }
-        l = l * exp2f(m - mn) + ((s4[0] + s4[1]) + (s4[2] + s4[3]));
+        l = l * ex2_approx(m - mn) + ((s4[0] + s4[1]) + (s4[2] + s4[3]));
       } else {
 #pragma unroll
         for (int i = 0; i < 32; ++i) v[i] = 0.f;
@@ -241,8 +252,8 @@ __global__ void __launch_bounds__(kThreads, CPC == 1 ? 3 : (CPC == 2 ? 2 : 1))
     const float2 h0 = halfstat[0][r], h1 = halfstat[1][r];
     const float mm = fmaxf(h0.x, h1.x);
     float ll = 0.f;
-    if (h0.x != -INFINITY) ll += h0.y * exp2f(h0.x - mm);
-    if (h1.x != -INFINITY) ll += h1.y * exp2f(h1.x - mm);
+    if (h0.x != -INFINITY) ll += h0.y * ex2_approx(h0.x - mm);
+    if (h1.x != -INFINITY) ll += h1.y * ex2_approx(h1.x - mm);
     rowstat[r] = make_float2(mm, ll);
   }
   cluster_sync_all();
@@ -259,7 +270,7 @@ __global__ void __launch_bounds__(kThreads, CPC == 1 ? 3 : (CPC == 2 ? 2 : 1))
       if (q < nrank) M = fmaxf(M, st[q].x);
 #pragma unroll
     for (uint32_t q = 0; q < 16; ++q)
-      if (q < nrank && st[q].x != -INFINITY) L += st[q].y * exp2f(st[q].x - M);
+      if (q < nrank && st[q].x != -INFINITY) L += st[q].y * ex2_approx(st[q].x - M);
   }
   const float invL = (rv && L > 0.f) ? 1.f / L : 0.f;
   cluster_arrive();  // done reading the peers' rowstat
@@ -275,14 +286,19 @@ __global__ void __launch_bounds__(kThreads, CPC == 1 ? 3 : (CPC == 2 ? 2 : 1))
     if (k0 + 32 <= a.vis_start || k0 >= a.vis_start + a.N_v) continue;  // warp-uniform
     float v[32];
     if (warp_live) {
-      const float w = (mblk[cb] != -INFINITY) ? exp2f(mblk[cb] - M) * invL : 0.f;
+      const float w = (mblk[cb] != -INFINITY) ? ex2_approx(mblk[cb] - M) * invL : 0.f;
       tmem_ld32(tbase + cb * 32, v);
       tc_wait_ld();
+      if (k0 >= a.vis_start && k0 + 32 <= a.vis_start + a.N_v) {
 #pragma unroll
-      for (int i = 0; i < 32; ++i) {
-        const int k = k0 + i;
-        const bool kv = k >= a.vis_start && k < a.vis_start + a.N_v;
-        v[i] = kv ? v[i] * w : 0.f;
+        for (int i = 0; i < 32; ++i) v[i] *= w;
+      } else {
+#pragma unroll
+        for (int i = 0; i < 32; ++i) {
+          const int k = k0 + i;
+          const bool kv = k >= a.vis_start && k < a.vis_start + a.N_v;
+          v[i] = kv ? v[i] * w : 0.f;
+        }
       }
       if (CONF) {
         const int lo = max(k0, a.vis_start), hi = min(k0 + 32, a.vis_start + a.N_v);

@@ -75,6 +75,10 @@ cudaError_t hs_launch_tc(const HSArgs& a, const CUtensorMap* tmQ, const CUtensor
 cudaError_t hs_launch_fused(const HSArgs& a, const CUtensorMap* tmQ, const CUtensorMap* tmK,
                             cudaStream_t s, bool* launched, bool pdl = false,
                             ConfGeom* geom = nullptr);
+// streaming tcgen05 path: one CTA per (row block x head, sample), keys through
+// a TMA/TMEM pipeline, visual keys read a second time (from L2); no cluster.
+cudaError_t hs_launch_stream(const HSArgs& a, const CUtensorMap* tmQ, const CUtensorMap* tmK,
+                             cudaStream_t s, bool pdl = false, ConfGeom* geom = nullptr);
 // largest number of confidence chunks the one-pass kernel uses (its cluster size)
 constexpr int kFusedMaxChunks = 16;
 // scores[b][i] = sum_u partial[b][u][i] / (H_sel * valid text rows of b)

@@ -25,6 +25,7 @@ ERR_CUDA = -4
 ERR_TIMEOUT = -5
 F32, BF16 = 0, 1
 ALGO_AUTO, ALGO_SIMT, ALGO_TCGEN05, ALGO_TCGEN05_TWOPASS = 0, 1, 2, 3
+ALGO_TCGEN05_STREAM, ALGO_TCGEN05_CLUSTER = 4, 5
 PRUNE_OVERLAP_PREVIOUS = 1
 
 _P = ctypes.c_void_p

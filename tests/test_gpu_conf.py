@@ -79,9 +79,9 @@ def check_conf(conf_gpu, C_ref, rtol, what):
         assert_close_rel(conf_gpu[b], C_ref[b], rtol, f"{what} sample {b}", atol=rtol * 1e-2 * C_ref[b].max())
 
 
+TC_ALGOS = [P.ALGO_TCGEN05_STREAM, P.ALGO_TCGEN05_CLUSTER, P.ALGO_TCGEN05_TWOPASS]
 CASES = [(w.name, a) for w in synth.WORKLOADS
-         for a in ([P.ALGO_SIMT] if w.dtype == "f32" else
-                   [P.ALGO_SIMT, P.ALGO_TCGEN05, P.ALGO_TCGEN05_TWOPASS])]
+         for a in ([P.ALGO_SIMT] if w.dtype == "f32" else [P.ALGO_SIMT] + TC_ALGOS)]
 
 
 @pytest.mark.parametrize("name,algo", CASES)
@@ -106,7 +106,8 @@ def test_confidence_paths_agree_on_the_selection():
     runs = [P.provip_head_confidence(g["Q"], g["K"], g["text_start"], g["text_len"], g["seq_len"],
                                      g["vis_start"], g["N_v"], N_VIS, crit_mask=g["crit_mask"], algo=a,
                                      N_t_max=w.n_t[1])
-            for a in (P.ALGO_TCGEN05, P.ALGO_TCGEN05, P.ALGO_TCGEN05_TWOPASS, P.ALGO_SIMT)]
+            for a in (P.ALGO_TCGEN05, P.ALGO_TCGEN05, P.ALGO_TCGEN05_STREAM, P.ALGO_TCGEN05_CLUSTER,
+                      P.ALGO_TCGEN05_TWOPASS, P.ALGO_SIMT)]
     torch.cuda.synchronize()
     assert torch.equal(runs[0][1], runs[1][1]) and torch.equal(runs[0][0], runs[1][0])
     for vis, _ in runs[2:]:
@@ -121,7 +122,7 @@ def test_uniform_attention_gives_zero_confidence():
     cpu = synth.in_llm_inputs(w, batch=2)
     g = {k: (v.to(DEV) if isinstance(v, torch.Tensor) else v) for k, v in cpu.items()}
     Q = torch.zeros_like(g["Q"])
-    for algo in (P.ALGO_TCGEN05, P.ALGO_TCGEN05_TWOPASS, P.ALGO_SIMT):
+    for algo in (P.ALGO_TCGEN05_STREAM, P.ALGO_TCGEN05_CLUSTER, P.ALGO_TCGEN05_TWOPASS, P.ALGO_SIMT):
         vis, conf = P.provip_head_confidence(Q, g["K"], g["text_start"], g["text_len"], g["seq_len"],
                                              g["vis_start"], g["N_v"], 4, algo=algo, N_t_max=w.n_t[1])
         torch.cuda.synchronize()
@@ -141,16 +142,20 @@ def test_empty_critical_set_selects_the_first_heads():
     assert vis.cpu().tolist() == [[0, 1, 2]] * 2
 
 
-@pytest.mark.parametrize("name", [w.name for w in synth.WORKLOADS])
-def test_prune_visual_heads_end_to_end(name):
+E2E = [(w.name, a) for w in synth.WORKLOADS
+       for a in ([P.ALGO_SIMT] if w.dtype == "f32" else [P.ALGO_TCGEN05_STREAM, P.ALGO_TCGEN05_CLUSTER])]
+
+
+@pytest.mark.parametrize("name,algo", E2E)
+def test_prune_visual_heads_end_to_end(name, algo):
     """Visual heads within the tie band of the oracle's C; v of the chosen heads
     within tolerance of the oracle's; keep set exact outside the band;
-    compaction exact; and bit-identical to provip_prune on each sample alone
-    with head_list = its visual heads."""
+    compaction exact; and bit-identical to provip_prune (same kernel family)
+    on each sample alone with head_list = its visual heads."""
     w, B, cpu, g, mask, C_ref = case(name)
     n_vis = min(N_VIS, w.H_q)
     step = P.VisualHeadsPruneStep(g["Q"], g["K"], g["V"], g["hidden"], g["pos"], w.n_t[1], g["N_v"],
-                                  w.keep, n_vis)
+                                  w.keep, n_vis, algo=algo)
     out = step(g["Q"], g["K"], g["V"], g["hidden"], g["pos"], g["text_start"], g["text_len"],
                g["seq_len"], g["vis_start"], crit_mask=g["crit_mask"])
     torch.cuda.synchronize()
@@ -181,7 +186,7 @@ def test_prune_visual_heads_end_to_end(name):
         one["pos"] = g["pos"][:, b:b + 1].contiguous()
         ref = P.provip_prune(one["Q"], one["K"], one["V"], one["hidden"], one["pos"], vis[b].tolist(),
                              one["text_start"], one["text_len"], one["seq_len"], g["vis_start"], g["N_v"],
-                             w.keep, N_t_max=w.n_t[1])
+                             w.keep, algo=algo, N_t_max=w.n_t[1])
         torch.cuda.synchronize()
         assert torch.equal(ref["scores"][0], out["scores"][b]), f"{name} sample {b}: scores differ"
         assert torch.equal(ref["idx"][0], out["idx"][b])

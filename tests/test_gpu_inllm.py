@@ -66,7 +66,8 @@ def ref_scores(name):
 
 CASES = [(w.name, a) for w in synth.WORKLOADS
          for a in ([P.ALGO_SIMT] if w.dtype == "f32" else
-                   [P.ALGO_SIMT, P.ALGO_TCGEN05, P.ALGO_TCGEN05_TWOPASS])]
+                   [P.ALGO_SIMT, P.ALGO_TCGEN05, P.ALGO_TCGEN05_TWOPASS, P.ALGO_TCGEN05_STREAM,
+                    P.ALGO_TCGEN05_CLUSTER])]
 
 
 @pytest.mark.parametrize("name,algo", CASES)
@@ -169,7 +170,8 @@ def _small_case(seed, B=3, Hq=6, Hkv=2, nsys=5, nv=37, tls=(1, 9, 130), dtype=to
     return dict(Q=Qt, K=Kt, tl=tl, sl=sl, ts=np.full(B, nsys + nv, np.int32), nsys=nsys, nv=nv, Ntm=Ntm)
 
 
-@pytest.mark.parametrize("algo", [P.ALGO_SIMT, P.ALGO_TCGEN05, P.ALGO_TCGEN05_TWOPASS])
+@pytest.mark.parametrize("algo", [P.ALGO_SIMT, P.ALGO_TCGEN05, P.ALGO_TCGEN05_TWOPASS, P.ALGO_TCGEN05_STREAM,
+                                  P.ALGO_TCGEN05_CLUSTER])
 def test_head_scores_ragged_and_masked_rows(algo):
     c = _small_case(7)
     heads = [1, 2, 5]
@@ -200,7 +202,8 @@ def test_head_scores_long_sequences(nv, tl):
     Qn, Kn = c["Q"].float().numpy(), c["K"].float().numpy()
     ref = oracle.head_scores(Qn[0, :c["sl"][0]], Kn[0, :c["sl"][0]], heads,
                              np.arange(c["ts"][0], c["ts"][0] + c["tl"][0]), c["nsys"], c["nv"])
-    for algo in (P.ALGO_TCGEN05, P.ALGO_TCGEN05_TWOPASS, P.ALGO_SIMT):
+    for algo in (P.ALGO_TCGEN05, P.ALGO_TCGEN05_TWOPASS, P.ALGO_SIMT, P.ALGO_TCGEN05_STREAM,
+                 P.ALGO_TCGEN05_CLUSTER):
         s = P.provip_head_scores(Qd, Kd, heads, ts, tlt, sl, c["nsys"], c["nv"], algo=algo, N_t_max=c["Ntm"])
         torch.cuda.synchronize()
         assert_close_rel(s[0].cpu().numpy(), ref, 2e-3, f"long L={c['sl'][0]} algo={algo}")
