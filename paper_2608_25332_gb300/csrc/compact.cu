@@ -24,12 +24,15 @@ namespace provip {
 namespace {
 
 #ifndef PROVIP_COMPACT_SLOTS
-#define PROVIP_COMPACT_SLOTS 6
+#define PROVIP_COMPACT_SLOTS 5
 #endif
 #ifndef PROVIP_COMPACT_CTAS_PER_SM
-#define PROVIP_COMPACT_CTAS_PER_SM 3
+#define PROVIP_COMPACT_CTAS_PER_SM 2
 #endif
-constexpr int kSlotBytes = 8192;
+#ifndef PROVIP_COMPACT_SLOT_BYTES
+#define PROVIP_COMPACT_SLOT_BYTES 8192
+#endif
+constexpr int kSlotBytes = PROVIP_COMPACT_SLOT_BYTES;
 constexpr int kSlots = PROVIP_COMPACT_SLOTS;          // ring of shared-memory slots per CTA
 constexpr int kCtasPerSm = PROVIP_COMPACT_CTAS_PER_SM;
 constexpr int kCompactThreads = 128;

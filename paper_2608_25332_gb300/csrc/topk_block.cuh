@@ -150,7 +150,8 @@ __device__ __forceinline__ void topk_load_partials(const float* P0, int n_part, 
   auto row = [&](int u) -> int { return sel ? (u / n_sel) * H_sel + sel[u % n_sel] : u; };
   auto ld = [&](size_t off) -> float { return CG ? __ldcg(P0 + off) : __ldg(P0 + off); };
   if (n_sum <= 8) {
-    int ro[8];  // row offsets: n_part x N is below 2^31 (N <= 49152, n_part <= 2^15)
+    // up to 8 partial rows: 4 columns per thread, every load issued first
+    int ro[8];
 #pragma unroll
     for (int u = 0; u < 8; ++u) ro[u] = u < n_sum ? row(u) * N : 0;
     for (int i0 = 0; i0 < N; i0 += 4 * nth) {
@@ -176,9 +177,18 @@ __device__ __forceinline__ void topk_load_partials(const float* P0, int n_part, 
       }
     }
   } else {
+    // more rows: per column, groups of 8 loads in flight, added in row order
     for (int i = tid; i < N; i += nth) {
       float s = 0.f;
-      for (int u = 0; u < n_sum; ++u) s += ld((size_t)row(u) * N + i);
+      for (int u0 = 0; u0 < n_sum; u0 += 8) {
+        float t[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u)
+          if (u0 + u < n_sum) t[u] = ld((size_t)row(u0 + u) * N + i);
+#pragma unroll
+        for (int u = 0; u < 8; ++u)
+          if (u0 + u < n_sum) s += t[u];
+      }
       const float v = zero ? 0.f : s / div;
       if (scores_out) scores_out[i] = v;
       keys[i] = float_key(v);
