@@ -75,7 +75,9 @@ extern "C" {
                                          no cluster shape fits */
 /* Different kernel families sum in different orders: results agree within the
  * floating-point tolerance, and are bit-identical between calls that take the
- * same family (the same algo and, for PROVIP_ALGO_TCGEN05, the same choice). */
+ * same family (the same algo and, for PROVIP_ALGO_TCGEN05, the same choice;
+ * the STREAM form has a second order when it also keeps head-confidence
+ * statistics, see provip_prune_visual_heads). */
 
 /* bits of the device status word */
 #define PROVIP_DEVSTAT_TIMEOUT 1u  /* a bounded wait gave up */
@@ -325,9 +327,11 @@ int provip_head_confidence(const void *Q, const void *K, int B, int L_max, int H
  * sample over all its text rows (S^vis and v of Sec. 4.4), the top `keep` of v
  * (idx_out [B, keep] ascending, ties to the lower index) and the compaction of
  * provip_compact. One pass over the keys computes the attention statistics of
- * every head; with the same kernel family (algo STREAM, CLUSTER or TWOPASS on
- * both sides) the scores of a sample's visual heads are bit-identical to
- * provip_prune called on that sample alone with head_list = its visual heads.
+ * every head; with the same kernel family on both sides (algo CLUSTER, TWOPASS
+ * or SIMT) the scores of a sample's visual heads are bit-identical to
+ * provip_prune called on that sample alone with head_list = its visual heads
+ * (the STREAM form sums the columns in another order when it keeps no
+ * confidence statistics, so there they agree to fp32 rounding).
  * scores_out_or_null [B, N_v], vis_heads_out_or_null [B, N_vis] and
  * conf_out_or_null [B, H_q] receive v, the visual heads and C when non-NULL.
  * flags as in provip_prune. Workspace: provip_visual_heads_workspace_size. */

@@ -218,12 +218,13 @@ __global__ void __launch_bounds__(256) hs_reduce_kernel(const HSArgs a, float* s
 
 // Head confidence and visual-head selection (Sec. 4.4), one CTA per sample.
 // C[i] = sum over the confidence rows of (merged M2) / N_v for head-list
-// position i; each warp takes heads i = warp, warp + 8, ...; each lane a
-// strided set of rows, folded by a fixed butterfly, so C is deterministic.
-// The chunk statistics of a row are merged in chunk order with Chan, Golub and
-// LeVeque's pairwise update; chunk c holds the visual columns of
-// [g.lo0 + c * g.w, g.lo0 + (c + 1) * g.w).
-constexpr int kConfThreads = 256;
+// position i; each warp takes heads i = warp, warp + 32, ...; each lane the rows
+// lane, lane + 32, ... in batches of 4 (their loads in flight together), folded
+// by a fixed butterfly, so C is deterministic. The chunk statistics of a row
+// are merged in chunk order with Chan, Golub and LeVeque's pairwise update;
+// chunk c holds the visual columns of [g.lo0 + c * g.w, g.lo0 + (c + 1) * g.w).
+constexpr int kConfThreads = 1024;
+constexpr int kConfBatch = 4;
 __global__ void __launch_bounds__(kConfThreads) conf_select_kernel(const HSArgs a, const ConfGeom g,
                                                                   const ConfArgs c) {
   __shared__ float C[kMaxHeads];
@@ -236,22 +237,38 @@ __global__ void __launch_bounds__(kConfThreads) conf_select_kernel(const HSArgs 
   const int vlo = a.vis_start, vhi = a.vis_start + a.N_v;
   for (int i = warp; i < a.H_sel; i += kConfThreads / 32) {
     float acc = 0.f;
-    for (int j = lane; j < a.N_t_max; j += 32) {
-      if (!hs_row_valid(a, smp, b, j)) continue;
-      if (a.conf_mask != nullptr && a.conf_mask[(size_t)b * a.N_t_max + j] == 0) continue;
-      const float2* st = a.conf_part + (((size_t)b * a.H_sel + i) * a.N_t_max + j) * a.conf_stride;
-      float n = 0.f, mean = 0.f, m2 = 0.f;
+    const float2* base = a.conf_part + ((size_t)b * a.H_sel + i) * a.N_t_max * a.conf_stride;
+    for (int j0 = 0; j0 < a.N_t_max; j0 += 32 * kConfBatch) {
+      bool use[kConfBatch];
+      float n[kConfBatch], mean[kConfBatch], m2[kConfBatch];
+#pragma unroll
+      for (int r = 0; r < kConfBatch; ++r) {
+        const int j = j0 + 32 * r + lane;
+        use[r] = j < a.N_t_max && hs_row_valid(a, smp, b, j) &&
+                 (a.conf_mask == nullptr || a.conf_mask[(size_t)b * a.N_t_max + j] != 0);
+        n[r] = 0.f;
+        mean[r] = 0.f;
+        m2[r] = 0.f;
+      }
       for (int q = 0; q < g.n; ++q) {
         const int lo = max(g.lo0 + q * g.w, vlo), hi = min(g.lo0 + (q + 1) * g.w, vhi);
         if (hi <= lo) continue;
         const float nb = (float)(hi - lo);
-        const float2 v = st[q];
-        const float nn = n + nb, dl = v.x - mean;
-        mean += dl * (nb / nn);
-        m2 += v.y + dl * dl * (n * nb / nn);
-        n = nn;
+        float2 v[kConfBatch];
+#pragma unroll
+        for (int r = 0; r < kConfBatch; ++r)
+          v[r] = use[r] ? base[(size_t)(j0 + 32 * r + lane) * a.conf_stride + q] : make_float2(0.f, 0.f);
+#pragma unroll
+        for (int r = 0; r < kConfBatch; ++r) {
+          const float nn = n[r] + nb, dl = v[r].x - mean[r];
+          mean[r] += dl * (nb / nn);
+          m2[r] += v[r].y + dl * dl * (n[r] * nb / nn);
+          n[r] = nn;
+        }
       }
-      acc += m2 / (float)a.N_v;
+#pragma unroll
+      for (int r = 0; r < kConfBatch; ++r)
+        if (use[r]) acc += m2[r] / (float)a.N_v;
     }
 #pragma unroll
     for (int o = 16; o >= 1; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);

@@ -7,12 +7,18 @@
 //   pass A (chunks 0 .. n_A - 1, every key up to the block's last text row):
 //     S = Q K^T of the chunk, then per row a running max m and sum l of
 //     exp2(s - m) over its causal keys - the row's global (max, sum);
-//   pass B (the n_B chunks of visual keys, vis_start + 128 c ...):
-//     S again (those keys are read a second time, from L2: the chunk was
-//     loaded in pass A moments before), p = exp2(s - M) / L, summed over the
-//     128 rows into partial[b][rb * H_sel + h][col] (warp butterfly
-//     transpose-reduction, then a fixed-order sum over the 4 lane quadrants);
-//     with CONF, each row's mean and M2 of its visual probabilities as well.
+//   pass B (the n_B chunks of visual keys, vis_start + 128 c ...): the
+//     logits again (those keys are read a second time, from L2: the chunk was
+//     loaded in pass A moments before), p = 2^(s - M) / L = 2^(s - c) with
+//     c = M + log2 L, summed over the 128 rows into
+//     partial[b][rb * H_sel + h][col]. Without CONF the MMA computes S^T = K Q^T
+//     (TMEM lane = key), so a key's sum over the rows stays in its thread (two
+//     halves of 64 rows, added in a fixed order); with CONF it computes S (lane
+//     = row) to keep each row's mean and M2 of its visual probabilities as well,
+//     and sums the columns with a warp butterfly transpose-reduction and a
+//     fixed-order sum over the 4 lane quadrants.
+// Rows of the query tile past the block's text rows are zeroed in shared
+// memory before the first MMA, so every logit the workers read is finite.
 // Roles: warp 8 (one lane) issues the TMA loads into a 2-stage ring of key
 // tiles, warp 9 (one lane) issues 8 tcgen05.mma (M = N = 128, K = 16) per
 // chunk into one of two 128-column TMEM accumulators and commits, warps 0-7
@@ -39,6 +45,7 @@ constexpr uint32_t kIdesc = idesc_bf16_f32(128, 128);
 
 struct Ctl {
   uint64_t q_full;
+  uint64_t q_ready;  // rows past the text block zeroed (finite logits)
   uint64_t k_full[kStages];
   uint64_t k_empty[kStages];
   uint64_t acc_full[2];
@@ -76,6 +83,7 @@ __global__ void __launch_bounds__(kThreads, 2)
   __shared__ Ctl ctl;
   __shared__ float2 halfstat[2][kTile];
   __shared__ float red[2][4][kTile];
+  __shared__ __align__(16) float crow[kTile];  // M + log2(L) per row; +inf: not scored
   const int hi = blockIdx.x % a.H_sel, rb = blockIdx.x / a.H_sel;
   const int b = blockIdx.y;
   const int h = a.heads[hi], g = h / (a.H_q / a.H_kv);
@@ -107,6 +115,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     prefetch_tmap(&tmQ);
     prefetch_tmap(&tmK);
     mbar_init(&ctl.q_full, 1);
+    mbar_init(&ctl.q_ready, kWorkerThreads / 32);
     for (int s = 0; s < kStages; ++s) {
       mbar_init(&ctl.k_full[s], 1);
       mbar_init(&ctl.k_empty[s], 1);
@@ -151,7 +160,7 @@ __global__ void __launch_bounds__(kThreads, 2)
   } else if (warp == 9) {
     // ---- MMA issuer ----
     if (lane == 0) {
-      bool live = mbar_wait(&ctl.q_full, 0, a.err);
+      bool live = mbar_wait(&ctl.q_ready, 0, a.err);
       if (!live) ctl.fail = 1;
       const uint32_t qa = smem_u32(qs);
       for (int it = 0; it < n_it && live; ++it) {
@@ -165,10 +174,14 @@ __global__ void __launch_bounds__(kThreads, 2)
         tc_fence_after();
         const uint32_t ka = smem_u32(ks + (size_t)s * kTileBytes);
         const uint32_t acc = ctl.tmem + (uint32_t)(buf * kTile);
+        // pass A: S = Q K^T (lane = text row); pass B without confidence:
+        // S^T = K Q^T (lane = key), so a key's sum over the rows stays in its thread
+        const bool tr = !CONF && it >= nA;
+        const uint32_t opa = tr ? ka : qa, opb = tr ? qa : ka;
 #pragma unroll
         for (int kstep = 0; kstep < 8; ++kstep) {
           const uint32_t off = (kstep >> 2) * kHalfBytes + (kstep & 3) * 32;
-          tc_mma_bf16(acc, smem_desc_sw128(qa + off), smem_desc_sw128(ka + off), kIdesc,
+          tc_mma_bf16(acc, smem_desc_sw128(opa + off), smem_desc_sw128(opb + off), kIdesc,
                       kstep > 0 ? 1u : 0u);
         }
         tc_commit(&ctl.k_empty[s]);
@@ -185,7 +198,20 @@ __global__ void __launch_bounds__(kThreads, 2)
     const uint32_t tbase = ctl.tmem + ((uint32_t)(quad * 32) << 16) + (uint32_t)(half * 64);
     const float sc = a.scale_log2;
     const int t_first = ts + rb * kTile;  // every row of the block sits at or after it
-    bool failed = false;
+    bool failed = !mbar_wait(&ctl.q_full, 0, a.err);
+    {
+      // rows of the query tile past the block's text rows may hold anything
+      // (other samples, padding): zero them, so every logit is finite
+      const int nz = (kTile - rows) * 16;  // 16-byte pieces: 8 per 128-byte row, two halves
+      for (int q = threadIdx.x; q < nz; q += kWorkerThreads) {
+        const int row = rows + q / 16, piece = q % 16;
+        *reinterpret_cast<uint4*>(qs + (piece >> 3) * kHalfBytes + row * 128 + (piece & 7) * 16) =
+            make_uint4(0u, 0u, 0u, 0u);
+      }
+      fence_proxy_async_smem();  // visible to the tensor cores
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&ctl.q_ready);
+    }
     // m: running max of the scaled logits, l: sum of 2^(s - m); c = M + log2(L)
     float m = -INFINITY, l = 0.f, c = 0.f;
     float cn = 0.f, cmean = 0.f, cm2 = 0.f;
@@ -204,6 +230,10 @@ __global__ void __launch_bounds__(kThreads, 2)
         if (h1.x != -INFINITY) L += h1.y * ex2_approx(h1.x - M);
         // p = 2^(s - M) / L = 2^(s - c); L >= 1 (the max term) for a valid row
         c = (rv && L > 0.f) ? M + lg2_approx(L) : 0.f;
+        if (!CONF) {
+          if (half == 0) crow[r] = (rv && L > 0.f) ? c : INFINITY;  // 2^-inf = 0
+          workers_sync();
+        }
       }
       const uint32_t tacc = tbase + (uint32_t)(buf * kTile);
       if (it < nA) {
@@ -236,6 +266,44 @@ __global__ void __launch_bounds__(kThreads, 2)
             m = mn;
           }
         }
+      } else if (!CONF) {
+        // transposed: thread = key kk of the chunk, 64 text rows per warp
+        const int par = (it - nA) & 1;
+        const int kk = quad * 32 + lane, key = a.vis_start + (it - nA) * kTile + kk;
+        const bool all_causal = a.vis_start + (it - nA) * kTile + kTile - 1 <= t_first;
+        float csum = 0.f;
+#pragma unroll
+        for (int cb = 0; cb < 2; ++cb) {
+          const int i0 = half * 64 + cb * 32;  // first row of the block
+          float v[32];
+          tmem_ld32(tacc + cb * 32, v);
+          tc_wait_ld();
+          float s4[4] = {0.f, 0.f, 0.f, 0.f};
+          const float4* cr = reinterpret_cast<const float4*>(crow + i0);
+          if (all_causal) {
+#pragma unroll
+            for (int i4 = 0; i4 < 8; ++i4) {
+              const float4 cc = cr[i4];
+              s4[0] += ex2_approx(fmaf(v[4 * i4 + 0], sc, -cc.x));
+              s4[1] += ex2_approx(fmaf(v[4 * i4 + 1], sc, -cc.y));
+              s4[2] += ex2_approx(fmaf(v[4 * i4 + 2], sc, -cc.z));
+              s4[3] += ex2_approx(fmaf(v[4 * i4 + 3], sc, -cc.w));
+            }
+          } else {
+#pragma unroll
+            for (int i4 = 0; i4 < 8; ++i4) {
+              const float4 cc = cr[i4];
+              const float cv[4] = {cc.x, cc.y, cc.z, cc.w};
+#pragma unroll
+              for (int e = 0; e < 4; ++e) {
+                const int i = 4 * i4 + e;
+                s4[e] += key <= t_first + i0 + i ? ex2_approx(fmaf(v[i], sc, -cv[e])) : 0.f;
+              }
+            }
+          }
+          csum += (s4[0] + s4[1]) + (s4[2] + s4[3]);
+        }
+        red[par][half][kk] = csum;
       } else {
         const int par = (it - nA) & 1;
 #pragma unroll
@@ -299,8 +367,9 @@ __global__ void __launch_bounds__(kThreads, 2)
         workers_sync();  // red[par] complete (red[par ^ 1] is free: read before this barrier)
         const int c = (it - nA) * kTile + threadIdx.x;
         if (threadIdx.x < kTile && c < a.N_v)
-          out[c] = red[par][0][threadIdx.x] + red[par][1][threadIdx.x] + red[par][2][threadIdx.x] +
-                   red[par][3][threadIdx.x];
+          out[c] = CONF ? red[par][0][threadIdx.x] + red[par][1][threadIdx.x] + red[par][2][threadIdx.x] +
+                              red[par][3][threadIdx.x]
+                        : red[par][0][threadIdx.x] + red[par][1][threadIdx.x];
       }
     }
     if (CONF) {

@@ -150,8 +150,9 @@ E2E = [(w.name, a) for w in synth.WORKLOADS
 def test_prune_visual_heads_end_to_end(name, algo):
     """Visual heads within the tie band of the oracle's C; v of the chosen heads
     within tolerance of the oracle's; keep set exact outside the band;
-    compaction exact; and bit-identical to provip_prune (same kernel family)
-    on each sample alone with head_list = its visual heads."""
+    compaction exact; and, for the cluster and CUDA-core forms, bit-identical
+    to provip_prune (same form) on each sample alone with head_list = its
+    visual heads."""
     w, B, cpu, g, mask, C_ref = case(name)
     n_vis = min(N_VIS, w.H_q)
     step = P.VisualHeadsPruneStep(g["Q"], g["K"], g["V"], g["hidden"], g["pos"], w.n_t[1], g["N_v"],
@@ -188,8 +189,16 @@ def test_prune_visual_heads_end_to_end(name, algo):
                              one["text_start"], one["text_len"], one["seq_len"], g["vis_start"], g["N_v"],
                              w.keep, algo=algo, N_t_max=w.n_t[1])
         torch.cuda.synchronize()
-        assert torch.equal(ref["scores"][0], out["scores"][b]), f"{name} sample {b}: scores differ"
-        assert torch.equal(ref["idx"][0], out["idx"][b])
+        if algo == P.ALGO_TCGEN05_STREAM:
+            # the streaming form sums the columns in another order when it keeps
+            # no confidence statistics: agreement to fp32 rounding, not bits
+            assert_close_rel(out["scores"][b].cpu().numpy(), ref["scores"][0].cpu().numpy(), 1e-5,
+                             f"{name} sample {b}: streaming forms")
+            check_topk_band(out["idx"][b].cpu().numpy(), ref["scores"][0].double().cpu().numpy(), w.keep,
+                            1e-5, f"{name} sample {b}: streaming keep set")
+        else:
+            assert torch.equal(ref["scores"][0], out["scores"][b]), f"{name} sample {b}: scores differ"
+            assert torch.equal(ref["idx"][0], out["idx"][b])
 
 
 def test_prune_visual_heads_overlapped_calls_match_serial():
