@@ -219,6 +219,46 @@ def schedule_measure(w, dev, reps=10):
             "host_syncs": 0}
 
 
+def ablation_measure(dev, reps=20):
+    """The ablation of Sec. 5 on LLaVA-1.5-7B (batch of 16, bf16): no pruning
+    before the LLM, 576 visual tokens -> the paper's shallow / middle budgets,
+    visual heads at the shallow layer (critical rows still found). One CUDA
+    graph per call."""
+    import torch
+    from paper_2608_25332_gb300 import synth
+    from paper_2608_25332_gb300.schedule import ProgressiveSchedule
+    out = {}
+    for n2, n3 in synth.ABLATION_BUDGETS:
+        w = synth.ablation_workload(n2)
+        cpu = synth.schedule_inputs(w)
+        g = {k: {kk: (vv.to(dev) if isinstance(vv, torch.Tensor) else vv) for kk, vv in v.items()}
+             for k, v in cpu.items()}
+        sched = ProgressiveSchedule(w.B, w.N_v, w.D, w.n_t[1], w.L_max, w.H_q, w.H_kv, w.D, w.P, w.N_v, n2,
+                                    n3, min(N_VIS, w.H_q), dtype=w.torch_dtype, device=dev, pre_llm=False)
+        sh = g["shallow"]
+        call = lambda: sched(g["pre"]["emb_v"], g["pre"]["emb_t"], g["pre"]["text_len"], sh, g["middle"],
+                             sh["vis_start"])
+        for _ in range(3):
+            call()
+        torch.cuda.synchronize()
+        graph = torch.cuda.CUDAGraph()
+        stream = torch.cuda.Stream(device=dev)
+        with torch.cuda.graph(graph, stream=stream):
+            call()
+        graph.replay()
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        for _ in range(reps):
+            graph.replay()
+        b.record()
+        torch.cuda.synchronize()
+        us = a.elapsed_time(b) / reps * 1e3
+        out[f"{w.N_v}->{n2}->{n3}"] = {"us_per_call": us, "samples_per_s": w.B / us * 1e6}
+    return {"workload": "llava15_7b_bf16_b16 without pre-LLM pruning, visual heads at the shallow layer",
+            "budgets": out}
+
+
 class ClockSampler:
     FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
@@ -642,6 +682,7 @@ def run_gb300(args, dist):
 
     prellm = prellm_measure(w, dev) if dist.rank == 0 else None
     schedule = schedule_measure(w, dev) if dist.rank == 0 else None
+    ablation = ablation_measure(dev) if dist.rank == 0 else None
 
     cpu_base = None
     if dist.rank == 0 and dist.world == 1 and not args.no_cpu_baseline:
@@ -666,7 +707,7 @@ def run_gb300(args, dist):
             "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
             "gpu_launches": launches_per_step * K,
             "prellm": prellm,
-            "next_rows": dict(next_rows, schedule=schedule),
+            "next_rows": dict(next_rows, schedule=schedule, ablation=ablation),
             "clocks": clocks,
         }
         print(json.dumps(line))

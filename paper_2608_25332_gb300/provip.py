@@ -163,13 +163,17 @@ def provip_version() -> int:
 # ---------------------------------------------------------------------------
 # pre-LLM pass
 # ---------------------------------------------------------------------------
-def provip_crit_text(emb_t, text_len, want_r=False):
+def provip_crit_text(emb_t, text_len, want_r=False, out=None, ws=None):
+    """Sec. 4.2: the critical-row mask T [B, N_t_max] (and r when want_r); out: a
+    pre-allocated mask to write, ws: a pre-allocated workspace."""
     B, Ntm, D = emb_t.shape
     dev = emb_t.device
-    mask = torch.empty((B, Ntm), dtype=torch.uint8, device=dev)
+    mask = out if out is not None else torch.empty((B, Ntm), dtype=torch.uint8, device=dev)
     r = torch.empty((B, Ntm), dtype=torch.float32, device=dev) if want_r else None
     L = lib()
-    ws = workspace(L.provip_crit_text_workspace_size(B, Ntm, D), dev)
+    need = L.provip_crit_text_workspace_size(B, Ntm, D)
+    if ws is None or ws.numel() < need:
+        ws = workspace(need, dev)
     rc = L.provip_crit_text(_ptr(emb_t), B, Ntm, D, _i32(text_len), _dtype_code(emb_t), _u8(mask),
                             _ptr(r), _ptr(ws), ws.numel(), _stream(dev))
     _check(rc, "provip_crit_text")

@@ -1,5 +1,6 @@
 """The paper's progressive pruning schedule (Sec. 4.1) on one stream, with no
-host synchronisation between the stages:
+host synchronisation between the stages (and the ablation of Sec. 5 without
+the pre-LLM stage):
 
   1. before the LLM (Sec. 4.2-4.3): N_v -> N1 visual tokens by text-guided
      similarity, pruned tokens merged into their nearest kept token;
@@ -35,24 +36,39 @@ class ProgressiveSchedule:
     """
 
     def __init__(self, B, N_v, D_v, N_t_max, L_max, H_q, H_kv, D, P_ids, N1, N2, N3, N_vis,
-                 dtype=torch.bfloat16, device="cuda", algo=P.ALGO_AUTO):
+                 dtype=torch.bfloat16, device="cuda", algo=P.ALGO_AUTO, pre_llm=True,
+                 shallow_heads="visual"):
+        """pre_llm=False: the ablation without pruning before the LLM (N1 = N_v;
+        the critical text rows T are still found, by provip_crit_text).
+        shallow_heads: "visual" (the N_vis most confident heads of each sample)
+        or "all" (every head) at the shallow layer."""
+        if not pre_llm and N1 != N_v:
+            raise ValueError("without pre-LLM pruning N1 must equal N_v")
+        if shallow_heads not in ("visual", "all"):
+            raise ValueError("shallow_heads is 'visual' or 'all'")
         self.B, self.N_v, self.N_t_max, self.L_max = B, N_v, N_t_max, L_max
         self.N1, self.N2, self.N3, self.N_vis, self.algo = N1, N2, N3, N_vis, algo
+        self.pre_llm, self.shallow_heads = pre_llm, shallow_heads
         dev = torch.device(device)
         L = P.lib()
-        self.idx1 = torch.empty((B, N1), dtype=torch.int32, device=dev)
-        self.merged = torch.empty((B, N1, D_v), dtype=dtype, device=dev)
-        self.p = torch.empty((B, N_v), dtype=torch.float32, device=dev)
+        self.idx1 = torch.empty((B, N1), dtype=torch.int32, device=dev) if pre_llm else None
+        self.merged = torch.empty((B, N1, D_v), dtype=dtype, device=dev) if pre_llm else None
+        self.p = torch.empty((B, N_v), dtype=torch.float32, device=dev) if pre_llm else None
         self.mask = torch.empty((B, N_t_max), dtype=torch.uint8, device=dev)
-        self.ws_pre = P.workspace(L.provip_similarity_reduce_workspace_size(B, N_v, D_v, N_t_max, N1), dev)
+        self.ws_pre = P.workspace(
+            L.provip_similarity_reduce_workspace_size(B, N_v, D_v, N_t_max, N1) if pre_llm
+            else L.provip_crit_text_workspace_size(B, N_t_max, D_v), dev)
         # shallow layer: outputs of provip_prune_visual_heads (shapes given by
         # meta tensors; the buffers live on dev)
         Q1 = torch.empty((B, L_max, H_q, 128), dtype=dtype, device="meta")
         K1 = torch.empty((B, L_max, H_kv, 128), dtype=dtype, device="meta")
         H1 = torch.empty((B, L_max, D), dtype=dtype, device="meta")
         pos1 = torch.empty((P_ids, B, L_max), dtype=torch.int32, device="meta")
-        self.shallow = P.VisualHeadsPruneStep(Q1, K1, K1, H1, pos1, N_t_max, N1, N2, N_vis, algo=algo,
-                                              device=dev)
+        if shallow_heads == "visual":
+            self.shallow = P.VisualHeadsPruneStep(Q1, K1, K1, H1, pos1, N_t_max, N1, N2, N_vis, algo=algo,
+                                                  device=dev)
+        else:
+            self.shallow = P.PruneStep(Q1, K1, K1, H1, pos1, None, N_t_max, N1, N2, algo=algo, device=dev)
         # middle layer: every head over the compacted sequence
         L2 = L_max - N1 + N2
         Q2 = torch.empty((B, L2, H_q, 128), dtype=dtype, device="meta")
@@ -69,12 +85,20 @@ class ProgressiveSchedule:
         pruning layer (L_max - N1 + N2 rows; its keys, values, hidden states,
         position ids and lengths are the shallow layer's compacted outputs).
         Returns the outputs of every stage (device tensors owned by self)."""
-        pre = P.provip_similarity_reduce(emb_v, emb_t, text_len, self.N1, ws=self.ws_pre,
-                                         out=dict(idx=self.idx1, merged=self.merged, p=self.p,
-                                                  mask=self.mask))
+        if self.pre_llm:
+            pre = P.provip_similarity_reduce(emb_v, emb_t, text_len, self.N1, ws=self.ws_pre,
+                                             out=dict(idx=self.idx1, merged=self.merged, p=self.p,
+                                                      mask=self.mask))
+        else:
+            P.provip_crit_text(emb_t, text_len, out=self.mask, ws=self.ws_pre)
+            pre = dict(mask=self.mask)
         s = shallow
-        o1 = self.shallow(s["Q"], s["K"], s["V"], s["hidden"], s["pos"], s["text_start"], text_len,
-                          s["seq_len"], vis_start, crit_mask=self.mask)
+        if self.shallow_heads == "visual":
+            o1 = self.shallow(s["Q"], s["K"], s["V"], s["hidden"], s["pos"], s["text_start"], text_len,
+                              s["seq_len"], vis_start, crit_mask=self.mask)
+        else:
+            o1 = self.shallow(s["Q"], s["K"], s["V"], s["hidden"], s["pos"], s["text_start"], text_len,
+                              s["seq_len"], vis_start)
         o2 = self.middle(middle["Q"], o1["K"], o1["V"], o1["hidden"], o1["pos"], middle["text_start"],
                          text_len, o1["seq_len"], vis_start)
         return dict(pre=pre, shallow=o1, middle=o2)

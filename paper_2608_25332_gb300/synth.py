@@ -41,7 +41,7 @@ for the video workload, whose visual rows are a seeded sorted subset of the
 from __future__ import annotations
 
 import math
-from dataclasses import dataclass, field
+from dataclasses import dataclass, field, replace
 
 import numpy as np
 import torch
@@ -330,3 +330,16 @@ def schedule_inputs(w: Workload, device="cpu", seed: int | None = None, batch: i
     return dict(pre={k: v.to(device) for k, v in pre.items()},
                 shallow={k: (v.to(device) if isinstance(v, torch.Tensor) else v) for k, v in shallow.items()},
                 middle=middle)
+
+
+# The ablation of Sec. 5 (pruning before the LLM disabled) on LLaVA-1.5-7B:
+# all 576 visual tokens reach the shallow pruning layer; visual tokens kept
+# after the shallow and after the middle layer.
+ABLATION_BUDGETS = ((219, 60), (146, 40), (73, 20), (54, 15), (36, 10), (18, 5))
+
+
+def ablation_workload(n_shallow: int, base: str = "llava15_7b_bf16_b16") -> Workload:
+    """The base workload with every visual token at the shallow layer (keep_pre =
+    N_v) and n_shallow kept there; same seeds."""
+    w = BY_NAME[base]
+    return replace(w, name=f"{w.name}_ablation_{n_shallow}", keep_pre=w.N_v, keep=n_shallow)
