@@ -295,9 +295,13 @@ CompactArgs compact_args(const int* idx, int B, int N_v, int keep, const void* h
 }
 
 // similarity pass: workspace partition
-int rel_splits(int N_v) {
-  int n = (N_v + 255) / 256;
-  return n < 1 ? 1 : (n > 32 ? 32 : n);
+// row chunks of the visual-row norm/sum pass: about 400 CTAs over the batch,
+// at least 8 rows each
+int rel_splits(int B, int N_v) {
+  int n = (400 + B - 1) / B;
+  const int by_rows = (N_v + 7) / 8;
+  if (n > by_rows) n = by_rows;
+  return n < 1 ? 1 : n;
 }
 int merge_splits(int B, int N_v, int keep) {
   const int rows = ((N_v + 127) / 128) * B;
@@ -429,7 +433,7 @@ extern "C" int provip_crit_text(const void* emb_t, int B, int N_t_max, int D, co
 }
 
 static size_t relevance_ws(Carve& c, int B, int N_v, int D, int N_t_max, SimWs& w) {
-  const int ns = rel_splits(N_v);
+  const int ns = rel_splits(B, N_v);
   w.inv_v = c.take<float>((size_t)B * N_v);
   w.sum = c.take<float>((size_t)(ns + 1) * B * D);
   w.mu = c.take<float>((size_t)B * N_t_max);
@@ -458,8 +462,7 @@ extern "C" int provip_relevance(const void* emb_v, int B, int N_v, int D, const 
   relevance_ws(c, B, N_v, D, N_t_max, w);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   SimArgs a = sim_args(emb_v, emb_t, text_len, B, N_v, D, N_t_max, dtype, d->status);
-  cudaError_t e = vis_inv_norm_launch(a, w.inv_v, s);
-  if (e == cudaSuccess) e = relevance_launch(a, crit_mask, w.inv_v, p_out, w.sum, w.mu, w.invt, rel_splits(N_v), s);
+  cudaError_t e = relevance_launch(a, crit_mask, w.inv_v, p_out, w.sum, w.mu, w.invt, rel_splits(B, N_v), s);
   return e == cudaSuccess ? PROVIP_OK : cuda_fail(e, "relevance launch");
 }
 
@@ -590,8 +593,7 @@ extern "C" int provip_similarity_reduce(const void* emb_v, int B, int N_v, int D
     e = cudaMemcpyAsync(mask_out_or_null, mask, (size_t)B * N_t_max, cudaMemcpyDeviceToDevice, s);
   }
   float* p = p_out_or_null ? p_out_or_null : w.p;
-  if (e == cudaSuccess) e = vis_inv_norm_launch(a, w.inv_v, s);
-  if (e == cudaSuccess) e = relevance_launch(a, mask, w.inv_v, p, w.sum, w.mu, w.invt, rel_splits(N_v), s);
+  if (e == cudaSuccess) e = relevance_launch(a, mask, w.inv_v, p, w.sum, w.mu, w.invt, rel_splits(B, N_v), s);
   if (e == cudaSuccess) {
     TopkArgs t;
     memset(&t, 0, sizeof(t));

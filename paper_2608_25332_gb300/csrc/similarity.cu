@@ -165,6 +165,127 @@ __global__ void __launch_bounds__(256) vis_sum_kernel(const SimArgs a, const flo
   part[((size_t)z * a.B + b) * a.D + d] = s;
 }
 
+// One read of the visual rows for both the inverse norms and the normalised
+// sum: a CTA per (row chunk z, sample) fetches its rows kNormRows at a time
+// with bulk copies (cp.async.bulk, one thread issuing) into shared memory;
+// warp w takes row w's squared norm (lane-strided 16-byte pieces, then a warp
+// sum) -> inv_v; then every thread adds its 16-byte pieces of the rows, in row
+// order, scaled by their inverse norms -> part[z][b][d].
+constexpr int kNormRows = 8;
+constexpr int kNormThreads = 256;
+constexpr int kNormMaxPieces = 4;  // 16-byte pieces per thread: D x esize <= 16 KiB
+size_t norm_sum_smem(int D, int esize) { return (size_t)kNormRows * D * esize; }
+bool norm_sum_supported(const SimArgs& a) {
+  const int es = a.dtype == 0 ? 4 : 2;
+  return (size_t)a.D * es <= (size_t)kNormMaxPieces * kNormThreads * 16 && (a.D * es) % 16 == 0;
+}
+
+// 8 bf16 of a shared-memory row as fp32 (plain shared load, not the read-only
+// global path)
+__device__ __forceinline__ void unpack8_shared(const uint8_t* p, float* o) {
+  const uint4 u = *reinterpret_cast<const uint4*>(p);
+  const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&u);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const float2 f = __bfloat1622float2(h[i]);
+    o[2 * i] = f.x;
+    o[2 * i + 1] = f.y;
+  }
+}
+
+template <typename T>
+__global__ void __launch_bounds__(kNormThreads) vis_norm_sum_kernel(const SimArgs a, float* inv_v,
+                                                                    float* part, int chunk) {
+  extern __shared__ __align__(128) uint8_t rows[];
+  __shared__ __align__(8) uint64_t bar;
+  __shared__ float inv_s[kNormRows];
+  constexpr int kVec = 16 / (int)sizeof(T);
+  const int z = blockIdx.x, b = blockIdx.y;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int j0 = z * chunk, j1 = min(a.N_v, j0 + chunk);
+  const T* E = static_cast<const T*>(a.emb_v) + (size_t)b * a.N_v * a.D;
+  const uint32_t row_bytes = (uint32_t)a.D * (uint32_t)sizeof(T);
+  const int n_pieces = (int)(row_bytes / 16);
+  float acc[kNormMaxPieces][kVec];
+#pragma unroll
+  for (int k = 0; k < kNormMaxPieces; ++k)
+#pragma unroll
+    for (int e = 0; e < kVec; ++e) acc[k][e] = 0.f;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    fence_mbar_init();
+  }
+  __syncthreads();
+  uint32_t phase = 0;
+  bool ok = true;
+  for (int r0 = j0; r0 < j1; r0 += kNormRows) {
+    const int nb = min(kNormRows, j1 - r0);
+    if (threadIdx.x == 0) {
+      const uint64_t pol = policy_evict_last();  // read again by the relevance Gram
+      mbar_arrive_expect_tx(&bar, (uint32_t)nb * row_bytes);
+      for (int q = 0; q < nb; ++q)
+        bulk_g2s(rows + (size_t)q * row_bytes, E + (size_t)(r0 + q) * a.D, row_bytes, &bar, pol);
+    }
+    if (ok && !mbar_wait(&bar, phase, a.err)) ok = false;
+    phase ^= 1u;
+    if (warp < nb) {
+      const uint8_t* row = rows + (size_t)warp * row_bytes;
+      float sq = 0.f;
+      for (int pc = lane; pc < n_pieces; pc += 32) {
+        float v[8];
+        if constexpr (sizeof(T) == 2) {
+          unpack8_shared(row + (size_t)pc * 16, v);
+#pragma unroll
+          for (int q = 0; q < 8; ++q) sq = fmaf(v[q], v[q], sq);
+        } else {
+          const float4 f = *reinterpret_cast<const float4*>(row + (size_t)pc * 16);
+          sq = fmaf(f.x, f.x, sq);
+          sq = fmaf(f.y, f.y, sq);
+          sq = fmaf(f.z, f.z, sq);
+          sq = fmaf(f.w, f.w, sq);
+        }
+      }
+      sq = warp_sum(sq);
+      const float iv = sq > 0.f ? 1.f / sqrtf(sq) : 0.f;
+      if (lane == 0) {
+        inv_s[warp] = iv;
+        inv_v[(size_t)b * a.N_v + r0 + warp] = iv;
+      }
+    }
+    __syncthreads();
+    for (int q = 0; q < nb; ++q) {
+      const uint8_t* row = rows + (size_t)q * row_bytes;
+      const float w = inv_s[q];
+#pragma unroll
+      for (int k = 0; k < kNormMaxPieces; ++k) {
+        const int pc = k * kNormThreads + (int)threadIdx.x;
+        if (pc >= n_pieces) continue;
+        if constexpr (sizeof(T) == 2) {
+          float v[8];
+          unpack8_shared(row + (size_t)pc * 16, v);
+#pragma unroll
+          for (int e = 0; e < 8; ++e) acc[k][e] = fmaf(v[e], w, acc[k][e]);
+        } else {
+          const float4 f = *reinterpret_cast<const float4*>(row + (size_t)pc * 16);
+          acc[k][0] = fmaf(f.x, w, acc[k][0]);
+          acc[k][1] = fmaf(f.y, w, acc[k][1]);
+          acc[k][2] = fmaf(f.z, w, acc[k][2]);
+          acc[k][3] = fmaf(f.w, w, acc[k][3]);
+        }
+      }
+    }
+    __syncthreads();  // the rows may be refilled
+  }
+  float* out = part + ((size_t)z * a.B + b) * a.D;
+#pragma unroll
+  for (int k = 0; k < kNormMaxPieces; ++k) {
+    const int pc = k * kNormThreads + (int)threadIdx.x;
+    if (pc >= n_pieces) continue;
+#pragma unroll
+    for (int e = 0; e < kVec; ++e) out[pc * kVec + e] = acc[k][e];
+  }
+}
+
 // sum[b][d] = sum over the row chunks z of part[z][b][d] (fixed order)
 __global__ void __launch_bounds__(256) vis_sum_reduce_kernel(const SimArgs a, const float* part,
                                                              int nz, float* sum) {
@@ -402,12 +523,20 @@ __global__ void merge_assign_kernel(const SimArgs a, const int* kpos, int n_spli
 
 // merged[b][a] = (sum of rows j with assign[b][j] == a, ascending j) / count.
 // The member lists come from a counting sort per sample: counts (atomics),
-// exclusive offsets, unordered fill; each kept row's CTA then orders its
-// members by rank (ascending row index, so the sum order is fixed) and sums
-// them with four member rows in flight. A centroid with more members than the
-// sort buffer falls back to scanning assign in windows.
+// exclusive offsets, unordered fill. One CTA per kept row orders its members
+// by rank (ascending row index, so the sum order is fixed), fetches the member
+// rows with bulk copies (cp.async.bulk, one thread issuing) into a ring of
+// shared-memory row slots, kMeanSlots rows per batch, and sums them slot by
+// slot in rank order, each thread over its 16-byte pieces of the row. A
+// centroid with more members than the sort buffer takes them from a scan of
+// assign in windows (ascending by construction).
 constexpr int kMeanThreads = 256;
+constexpr int kMeanWarps = kMeanThreads / 32;
 constexpr int kMeanSort = 1024;
+constexpr int kMeanSlots = 4;
+// 16-byte pieces per thread: D <= 8192 elements
+template <typename T> constexpr int mean_pieces() { return 8192 * (int)sizeof(T) / 16 / kMeanThreads; }
+size_t merge_mean_smem(int D, int esize) { return (size_t)kMeanSlots * D * esize; }
 
 __global__ void merge_count_kernel(const int* assign, int B, int N_v, int keep, int* count) {
   const size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
@@ -469,47 +598,87 @@ __global__ void merge_fill_kernel(const int* assign, int B, int N_v, int keep, c
   members[(size_t)b * N_v + offset[k] + atomicAdd(&cursor[k], 1)] = j;
 }
 
+// the addition of 16 raw bytes of a row to Acc values (8 bf16 or 4 fp32)
+__device__ __forceinline__ void add16(float* acc, const uint4& u, const __nv_bfloat16*) {
+  const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&u);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const float2 f = __bfloat1622float2(h[i]);
+    acc[2 * i] += f.x;
+    acc[2 * i + 1] += f.y;
+  }
+}
+__device__ __forceinline__ void add16(double* acc, const uint4& u, const float*) {
+  acc[0] += (double)__uint_as_float(u.x);
+  acc[1] += (double)__uint_as_float(u.y);
+  acc[2] += (double)__uint_as_float(u.z);
+  acc[3] += (double)__uint_as_float(u.w);
+}
+// 16 bytes of a row from Acc values, rounded to nearest even
+__device__ __forceinline__ void store16(__nv_bfloat16* p, const float* v) {
+  uint4 u;
+  __nv_bfloat162* h = reinterpret_cast<__nv_bfloat162*>(&u);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) h[i] = __floats2bfloat162_rn(v[2 * i], v[2 * i + 1]);
+  *reinterpret_cast<uint4*>(p) = u;
+}
+__device__ __forceinline__ void store16(float* p, const double* v) {
+  *reinterpret_cast<float4*>(p) = make_float4((float)v[0], (float)v[1], (float)v[2], (float)v[3]);
+}
+
 template <typename T, typename Acc>
-__global__ void __launch_bounds__(kMeanThreads) merge_mean_kernel(const SimArgs a, const int* assign,
+__global__ void __launch_bounds__(kMeanThreads, sizeof(T) == 2 ? 4 : 2) merge_mean_kernel(const SimArgs a, const int* assign,
                                                                   const int* count, const int* offset,
                                                                   const int* members_all, int keep,
                                                                   void* merged) {
+  extern __shared__ __align__(128) uint8_t slots[];  // kMeanSlots rows
   __shared__ int members[kMeanSort];
   __shared__ int unsorted[kMeanSort];
+  __shared__ __align__(8) uint64_t bar;
+  __shared__ int wcount[kMeanWarps];
+  constexpr int kVec = 16 / (int)sizeof(T);  // elements per 16-byte piece
+  constexpr int kPieces = mean_pieces<T>();
   const int ap = blockIdx.x, b = blockIdx.y;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const T* E = static_cast<const T*>(a.emb_v) + (size_t)b * a.N_v * a.D;
   T* out = static_cast<T*>(merged) + ((size_t)b * keep + ap) * a.D;
-  constexpr int kMaxQ = 32;  // D <= 8192
-  Acc acc[kMaxQ];
+  const uint32_t row_bytes = (uint32_t)a.D * (uint32_t)sizeof(T);
+  const int n_pieces = a.D / kVec;
+  Acc acc[kPieces][kVec];
 #pragma unroll
-  for (int q = 0; q < kMaxQ; ++q) acc[q] = Acc(0);
+  for (int k = 0; k < kPieces; ++k)
+#pragma unroll
+    for (int e = 0; e < kVec; ++e) acc[k][e] = Acc(0);
   const int n_all = count[(size_t)b * keep + ap];
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    fence_mbar_init();
+  }
+  uint32_t phase = 0;
+  bool ok = true;
+  // adds rows members[0..n) in order: batches of kMeanSlots bulk copies
   auto add_rows = [&](int n) {
-    int m = 0;
-    for (; m + 4 <= n; m += 4) {
-      const T* r0 = E + (size_t)members[m] * a.D;
-      const T* r1 = E + (size_t)members[m + 1] * a.D;
-      const T* r2 = E + (size_t)members[m + 2] * a.D;
-      const T* r3 = E + (size_t)members[m + 3] * a.D;
+    for (int m0 = 0; m0 < n; m0 += kMeanSlots) {
+      const int nb = min(kMeanSlots, n - m0);
+      if (threadIdx.x == 0 && ok) {
+        const uint64_t pol = policy_evict_first();
+        mbar_arrive_expect_tx(&bar, (uint32_t)nb * row_bytes);
+        for (int q = 0; q < nb; ++q)
+          bulk_g2s(slots + (size_t)q * row_bytes, E + (size_t)members[m0 + q] * a.D, row_bytes, &bar, pol);
+      }
+      if (ok && !mbar_wait(&bar, phase, a.err)) ok = false;
+      phase ^= 1u;
+      if (ok) {
+        for (int q = 0; q < nb; ++q) {
+          const uint8_t* row = slots + (size_t)q * row_bytes;
 #pragma unroll
-      for (int q = 0; q < kMaxQ; ++q) {
-        const int d = threadIdx.x + kMeanThreads * q;
-        if (d < a.D) {
-          const float x0 = to_f32(r0[d]), x1 = to_f32(r1[d]), x2 = to_f32(r2[d]), x3 = to_f32(r3[d]);
-          acc[q] += (Acc)x0;
-          acc[q] += (Acc)x1;
-          acc[q] += (Acc)x2;
-          acc[q] += (Acc)x3;
+          for (int k = 0; k < kPieces; ++k) {
+            const int pc = k * kMeanThreads + (int)threadIdx.x;
+            if (pc < n_pieces) add16(acc[k], *reinterpret_cast<const uint4*>(row + (size_t)pc * 16), E);
+          }
         }
       }
-    }
-    for (; m < n; ++m) {
-      const T* r0 = E + (size_t)members[m] * a.D;
-#pragma unroll
-      for (int q = 0; q < kMaxQ; ++q) {
-        const int d = threadIdx.x + kMeanThreads * q;
-        if (d < a.D) acc[q] += (Acc)to_f32(r0[d]);
-      }
+      __syncthreads();  // the slots may be refilled
     }
   };
   if (n_all <= kMeanSort) {
@@ -528,8 +697,6 @@ __global__ void __launch_bounds__(kMeanThreads) merge_mean_kernel(const SimArgs 
   } else {
     // many members: scan assign in windows, members in ascending order
     const int* as = assign + (size_t)b * a.N_v;
-    __shared__ int wcount[kMeanThreads / 32];
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     int base = 0;
     for (int j0 = 0; j0 < a.N_v; j0 += kMeanThreads) {
       const int j = j0 + threadIdx.x;
@@ -538,7 +705,7 @@ __global__ void __launch_bounds__(kMeanThreads) merge_mean_kernel(const SimArgs 
       if (lane == 0) wcount[warp] = __popc(bal);
       __syncthreads();
       int off = 0, tot = 0;
-      for (int w = 0; w < kMeanThreads / 32; ++w) {
+      for (int w = 0; w < kMeanWarps; ++w) {
         off += w < warp ? wcount[w] : 0;
         tot += wcount[w];
       }
@@ -547,21 +714,18 @@ __global__ void __launch_bounds__(kMeanThreads) merge_mean_kernel(const SimArgs 
       base += tot;
       if (base > kMeanSort - kMeanThreads || j0 + kMeanThreads >= a.N_v) {
         add_rows(base);
-        __syncthreads();
         base = 0;
       }
     }
   }
 #pragma unroll
-  for (int q = 0; q < kMaxQ; ++q) {
-    const int d = threadIdx.x + kMeanThreads * q;
-    if (d < a.D) {
-      const Acc v = n_all > 0 ? acc[q] / (Acc)n_all : Acc(0);
-      if constexpr (sizeof(T) == 4)
-        out[d] = (T)v;
-      else
-        out[d] = __float2bfloat16_rn((float)v);
-    }
+  for (int k = 0; k < kPieces; ++k) {
+    const int pc = k * kMeanThreads + (int)threadIdx.x;
+    if (pc >= n_pieces) continue;
+    Acc v[kVec];
+#pragma unroll
+    for (int e = 0; e < kVec; ++e) v[e] = n_all > 0 ? acc[k][e] / (Acc)n_all : Acc(0);
+    store16(out + (size_t)pc * kVec, v);
   }
 }
 
@@ -592,7 +756,7 @@ cudaError_t vis_inv_norm_launch(const SimArgs& a, float* inv_v, cudaStream_t s) 
   return cudaGetLastError();
 }
 
-cudaError_t relevance_launch(const SimArgs& a, const uint8_t* mask, const float* inv_v, float* p,
+cudaError_t relevance_launch(const SimArgs& a, const uint8_t* mask, float* inv_v, float* p,
                              float* ws_sum, float* ws_mu, float* ws_invt, int n_split,
                              cudaStream_t s) {
   const int chunk = (a.N_v + n_split - 1) / n_split;
@@ -602,13 +766,40 @@ cudaError_t relevance_launch(const SimArgs& a, const uint8_t* mask, const float*
   // ws_sum holds n_split partial sums followed by their total
   float* total = ws_sum + (size_t)n_split * a.B * a.D;
   dim3 g4((a.D + 255) / 256, a.B);
+  // the inverse norms of the visual rows and their normalised sum, in one read
+  // where the rows fit the shared-memory batch, else in two passes
+  const bool fused = norm_sum_supported(a);
+  if (fused) {
+    static bool configured[64] = {false};
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (dev >= 0 && dev < 64 && !configured[dev]) {
+      const int lim = kNormMaxPieces * kNormThreads * 16 * kNormRows;
+      cudaError_t e = cudaFuncSetAttribute(vis_norm_sum_kernel<float>,
+                                           cudaFuncAttributeMaxDynamicSharedMemorySize, lim);
+      if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(vis_norm_sum_kernel<__nv_bfloat16>,
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize, lim);
+      if (e != cudaSuccess) return e;
+      configured[dev] = true;
+    }
+    const size_t smem = norm_sum_smem(a.D, a.dtype == 0 ? 4 : 2);
+    dim3 gn(n_split, a.B);
+    if (a.dtype == 0)
+      vis_norm_sum_kernel<float><<<gn, kNormThreads, smem, s>>>(a, inv_v, ws_sum, chunk);
+    else
+      vis_norm_sum_kernel<__nv_bfloat16><<<gn, kNormThreads, smem, s>>>(a, inv_v, ws_sum, chunk);
+  } else {
+    cudaError_t e = vis_inv_norm_launch(a, inv_v, s);
+    if (e != cudaSuccess) return e;
+  }
   if (a.dtype == 0) {
-    vis_sum_kernel<float><<<g1, 256, 0, s>>>(a, inv_v, ws_sum, chunk);
+    if (!fused) vis_sum_kernel<float><<<g1, 256, 0, s>>>(a, inv_v, ws_sum, chunk);
     vis_sum_reduce_kernel<<<g4, 256, 0, s>>>(a, ws_sum, n_split, total);
     text_mu_kernel<float><<<g2, 256, 0, s>>>(a, total, ws_mu, ws_invt);
     relevance_kernel<float><<<g3, 256, 0, s>>>(a, mask, inv_v, ws_mu, ws_invt, p);
   } else {
-    vis_sum_kernel<__nv_bfloat16><<<g1, 256, 0, s>>>(a, inv_v, ws_sum, chunk);
+    if (!fused) vis_sum_kernel<__nv_bfloat16><<<g1, 256, 0, s>>>(a, inv_v, ws_sum, chunk);
     vis_sum_reduce_kernel<<<g4, 256, 0, s>>>(a, ws_sum, n_split, total);
     text_mu_kernel<__nv_bfloat16><<<g2, 256, 0, s>>>(a, total, ws_mu, ws_invt);
     if (relevance_tc_supported(a)) {
@@ -658,11 +849,25 @@ cudaError_t merge_launch(const SimArgs& a, const int* keep_idx, int keep, const 
     merge_offsets_kernel<<<a.B, 1024, 0, s>>>(cnt, keep, off, cur);
     merge_fill_kernel<<<(unsigned)((nb + 255) / 256), 256, 0, s>>>(assign, a.B, a.N_v, keep, off, cur, mem);
     dim3 gm(keep, a.B);
+    static bool configured[64] = {false};
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (dev >= 0 && dev < 64 && !configured[dev]) {
+      cudaError_t e = cudaFuncSetAttribute(merge_mean_kernel<float, double>,
+                                           cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                           (int)merge_mean_smem(8192, 4));
+      if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(merge_mean_kernel<__nv_bfloat16, float>,
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize, (int)merge_mean_smem(8192, 2));
+      if (e != cudaSuccess) return e;
+      configured[dev] = true;
+    }
+    const size_t smem = merge_mean_smem(a.D, a.dtype == 0 ? 4 : 2);
     if (a.dtype == 0)
-      merge_mean_kernel<float, double><<<gm, kMeanThreads, 0, s>>>(a, assign, cnt, off, mem, keep, merged);
+      merge_mean_kernel<float, double><<<gm, kMeanThreads, smem, s>>>(a, assign, cnt, off, mem, keep, merged);
     else
-      merge_mean_kernel<__nv_bfloat16, float><<<gm, kMeanThreads, 0, s>>>(a, assign, cnt, off, mem, keep,
-                                                                          merged);
+      merge_mean_kernel<__nv_bfloat16, float><<<gm, kMeanThreads, smem, s>>>(a, assign, cnt, off, mem, keep,
+                                                                             merged);
   }
   return cudaGetLastError();
 }
