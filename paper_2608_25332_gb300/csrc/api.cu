@@ -408,10 +408,15 @@ extern "C" int provip_device_status(unsigned* bits, int clear) {
 // ===========================================================================
 // pre-LLM pass
 // ===========================================================================
+// the text Gram, in as many K parts as its tcgen05 form uses (bf16)
+static size_t crit_gram_floats(int B, int N_t_max, int D, int dtype) {
+  const int parts = crit_splits(N_t_max, D, dtype);
+  return (size_t)(parts > 0 ? parts : 1) * B * N_t_max * N_t_max;
+}
+
 extern "C" size_t provip_crit_text_workspace_size(int B, int N_t_max, int D) {
-  (void)D;
   Carve c(nullptr);
-  c.take<float>((size_t)B * N_t_max * N_t_max);
+  c.take<float>(crit_gram_floats(B, N_t_max, D, PROVIP_BF16));  // the larger of the two dtypes' needs
   return c.off;
 }
 
@@ -426,7 +431,7 @@ extern "C" int provip_crit_text(const void* emb_t, int B, int N_t_max, int D, co
   DevInfo* d;
   if ((rc = dev_info(&d))) return rc;
   Carve c(ws);
-  float* G = c.take<float>((size_t)B * N_t_max * N_t_max);
+  float* G = c.take<float>(crit_gram_floats(B, N_t_max, D, PROVIP_BF16));
   SimArgs a = sim_args(nullptr, emb_t, text_len, B, 1, D, N_t_max, dtype, d->status);
   cudaError_t e = crit_text_launch(a, mask_out, r_out, G, static_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? PROVIP_OK : cuda_fail(e, "crit_text launch");
@@ -533,7 +538,7 @@ extern "C" int provip_merge(const void* emb_v, int B, int N_v, int D, const int*
 }
 
 static size_t simred_ws(Carve& c, int B, int N_v, int D, int N_t_max, int keep_pre, SimWs& w) {
-  w.G = c.take<float>((size_t)B * N_t_max * N_t_max);
+  w.G = c.take<float>(crit_gram_floats(B, N_t_max, D, PROVIP_BF16));
   w.mask = c.take<uint8_t>((size_t)B * N_t_max);
   w.p = c.take<float>((size_t)B * N_v);
   w.assign = c.take<int>((size_t)B * N_v);

@@ -159,7 +159,8 @@ struct SimArgs {
   int dtype;
   unsigned* err;
 };
-// Sec. 4.2: mask[b][j] (and r) from the text self-similarity. ws: G [B][Ntm][Ntm] f32.
+// Sec. 4.2: mask[b][j] (and r) from the text self-similarity. ws: G, max(1,
+// crit_splits) x [B][Ntm][Ntm] f32.
 cudaError_t crit_text_launch(const SimArgs& a, uint8_t* mask, float* r_out, float* G,
                              cudaStream_t s);
 // inverse L2 norms of every visual row (0 for a zero row): inv_v [B][N_v]
@@ -180,6 +181,10 @@ cudaError_t merge_launch(const SimArgs& a, const int* keep_idx, int keep, const 
 
 // tcgen05 forms of the pre-LLM Grams (bf16), used by the launchers above
 bool crit_gram_tc_supported(const SimArgs& a);
+// K splits of the tcgen05 text Gram (0: not applicable); G holds that many
+// [B][N_t_max][N_t_max] parts (at least one)
+constexpr int kCritMaxSplits = 16;
+int crit_splits(int N_t_max, int D, int dtype);
 cudaError_t crit_gram_tc_launch(const SimArgs& a, float* G, cudaStream_t s);
 bool relevance_tc_supported(const SimArgs& a);
 cudaError_t relevance_tc_launch(const SimArgs& a, const uint8_t* mask, const float* inv_v,

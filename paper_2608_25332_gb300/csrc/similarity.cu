@@ -56,9 +56,29 @@ __global__ void __launch_bounds__(256) crit_gram_kernel(const SimArgs a, float* 
 }
 
 // one CTA per sample: row softmax statistics, column means r, threshold
+// Adds the K parts of the text Gram into part 0, in part order: one thread per
+// element, every part's load issued first.
+constexpr int kCritMaxParts = 16;
+__global__ void __launch_bounds__(256) crit_parts_sum_kernel(float* G, size_t n, int n_parts) {
+  const size_t e = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (e >= n) return;
+  float v[kCritMaxParts];
+#pragma unroll
+  for (int q = 0; q < kCritMaxParts; ++q)
+    if (q < n_parts) v[q] = G[q * n + e];
+  float s = v[0];
+#pragma unroll
+  for (int q = 1; q < kCritMaxParts; ++q)
+    if (q < n_parts) s += v[q];
+  G[e] = s;
+}
+
+// G: the sample Grams [B][Ntm][Ntm]. Up to kFinishSmemNt text rows the sample's
+// Gram is staged in shared memory.
+constexpr int kFinishSmemNt = 128;
 __global__ void __launch_bounds__(256) crit_finish_kernel(const SimArgs a, const float* G,
                                                           uint8_t* mask, float* r_out) {
-  extern __shared__ float sh[];  // rowm[Ntm], rowinv[Ntm], r[Ntm]
+  extern __shared__ float sh[];  // rowm[Ntm], rowinv[Ntm], r[Ntm] (+ G[Ntm][Ntm] when staged)
   float* rowm = sh;
   float* rowinv = sh + a.N_t_max;
   float* rr = sh + 2 * a.N_t_max;
@@ -71,13 +91,35 @@ __global__ void __launch_bounds__(256) crit_finish_kernel(const SimArgs a, const
     n = 0;
   }
   const float* Gb = G + (size_t)b * a.N_t_max * a.N_t_max;
+  const bool staged = a.N_t_max <= kFinishSmemNt;
+  float* Gs = sh + 3 * a.N_t_max;
+  int ld = a.N_t_max;
+  if (staged) {
+    // eight loads in flight per thread
+    for (int e0 = 0; e0 < n * n; e0 += 8 * (int)blockDim.x) {
+      float v[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const int e = e0 + u * (int)blockDim.x + (int)threadIdx.x;
+        if (e < n * n) v[u] = Gb[(size_t)(e / n) * a.N_t_max + (e - (e / n) * n)];
+      }
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const int e = e0 + u * (int)blockDim.x + (int)threadIdx.x;
+        if (e < n * n) Gs[e] = v[u];
+      }
+    }
+    __syncthreads();
+    Gb = Gs;
+    ld = n;
+  }
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   for (int i = warp; i < n; i += 8) {
     float m = -INFINITY;
-    for (int j = lane; j < n; j += 32) m = fmaxf(m, Gb[(size_t)i * a.N_t_max + j]);
+    for (int j = lane; j < n; j += 32) m = fmaxf(m, Gb[(size_t)i * ld + j]);
     m = warp_max(m);
     float z = 0.f;
-    for (int j = lane; j < n; j += 32) z += expf(Gb[(size_t)i * a.N_t_max + j] - m);
+    for (int j = lane; j < n; j += 32) z += expf(Gb[(size_t)i * ld + j] - m);
     z = warp_sum(z);
     if (lane == 0) {
       rowm[i] = m;
@@ -87,7 +129,7 @@ __global__ void __launch_bounds__(256) crit_finish_kernel(const SimArgs a, const
   __syncthreads();
   for (int j = threadIdx.x; j < n; j += blockDim.x) {
     float s = 0.f;
-    for (int i = 0; i < n; ++i) s += expf(Gb[(size_t)i * a.N_t_max + j] - rowm[i]) * rowinv[i];
+    for (int i = 0; i < n; ++i) s += expf(Gb[(size_t)i * ld + j] - rowm[i]) * rowinv[i];
     rr[j] = s / (float)n;
   }
   __syncthreads();
@@ -734,15 +776,32 @@ __global__ void __launch_bounds__(kMeanThreads, sizeof(T) == 2 ? 4 : 2) merge_me
 cudaError_t crit_text_launch(const SimArgs& a, uint8_t* mask, float* r_out, float* G,
                              cudaStream_t s) {
   dim3 g((a.N_t_max + kSimtBN - 1) / kSimtBN, (a.N_t_max + kSimtBM - 1) / kSimtBM, a.B);
+  int parts = 1;
   if (a.dtype == 0) {
     crit_gram_kernel<float><<<g, 256, 0, s>>>(a, G);
   } else if (crit_gram_tc_supported(a)) {
     cudaError_t e = crit_gram_tc_launch(a, G, s);
     if (e != cudaSuccess) return e;
+    parts = crit_splits(a.N_t_max, a.D, a.dtype);
+    static_assert(kCritMaxSplits <= kCritMaxParts, "text Gram parts");
+    const size_t n = (size_t)a.B * a.N_t_max * a.N_t_max;
+    if (parts > 1) crit_parts_sum_kernel<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(G, n, parts);
   } else {
     crit_gram_kernel<__nv_bfloat16><<<g, 256, 0, s>>>(a, G);
   }
-  crit_finish_kernel<<<a.B, 256, 3 * a.N_t_max * sizeof(float), s>>>(a, G, mask, r_out);
+  static bool configured[64] = {false};
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev >= 0 && dev < 64 && !configured[dev]) {
+    const int lim = (3 * kFinishSmemNt + kFinishSmemNt * kFinishSmemNt) * (int)sizeof(float);
+    cudaError_t e = cudaFuncSetAttribute(crit_finish_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, lim);
+    if (e != cudaSuccess) return e;
+    configured[dev] = true;
+  }
+  size_t smem = 3 * (size_t)a.N_t_max * sizeof(float);
+  if (a.N_t_max <= kFinishSmemNt) smem += (size_t)a.N_t_max * a.N_t_max * sizeof(float);
+  (void)parts;
+  crit_finish_kernel<<<a.B, 256, smem, s>>>(a, G, mask, r_out);
   return cudaGetLastError();
 }
 

@@ -278,17 +278,20 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (threadIdx.x < 32) tmem_dealloc(pipe.tmem, Cfg<kRelBN>::kTmemCols);
 }
 
-// G = E_t E_t^T for one sample (<= 128 text rows): written to G[b] as fp32 for
-// the softmax/column-mean step of Sec. 4.2.
+// G = E_t E_t^T for one sample (<= 128 text rows), split over K: CTA x of
+// sample b sums the K slices [x * ks_per, (x + 1) * ks_per) and writes its part
+// to G[x][b] as fp32; the softmax/column-mean step of Sec. 4.2 adds the parts
+// in split order.
 constexpr int kCritBN = 128;
 
 __global__ void __launch_bounds__(kThreads, 1)
     crit_gram_tc(const __grid_constant__ CUtensorMap mapT, const int* text_len, int N_t_max, int D,
-                 float* G, unsigned* err) {
+                 int B, int ks_per, float* G, unsigned* err) {
   extern __shared__ uint8_t smem_raw[];
   __shared__ Pipe pipe;
   const int b = blockIdx.z;
-  const int n_k = (D + kBK - 1) / kBK;
+  const int k0 = blockIdx.x * ks_per;
+  const int n_k = min(ks_per, (D + kBK - 1) / kBK - k0);
   const uint32_t sbase = smem_u32(smem_raw);
   uint8_t* stages = smem_raw + (((sbase + 1023u) & ~1023u) - sbase);
   if (threadIdx.x == 0) {
@@ -307,7 +310,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0) {
       RowSrc ra{nullptr, b * N_t_max, kBM};
       RowSrc rb{nullptr, b * N_t_max, kCritBN};
-      producer<kCritBN>(pipe, stages, &mapT, &mapT, ra, false, rb, false, 1, n_k, err);
+      producer<kCritBN>(pipe, stages, &mapT, &mapT, ra, false, rb, false, 1, n_k, err, k0);
     }
   } else if (warp == 1) {
     if (lane == 0) mma_issuer<kCritBN>(pipe, stages, 1, n_k, err);
@@ -317,7 +320,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_wait(&pipe.acc_full[0], 0, err);
     tc_fence_after();
     const uint32_t taddr = pipe.tmem + ((uint32_t)(quad * 32) << 16);
-    float* g = G + ((size_t)b * N_t_max + r) * N_t_max;
+    float* g = G + (((size_t)blockIdx.x * B + b) * N_t_max + r) * N_t_max;
 #pragma unroll 1
     for (int cb = 0; cb < kCritBN / 32; ++cb) {
       float v[32];
@@ -446,7 +449,17 @@ cudaError_t relevance_tc_launch(const SimArgs& a, const uint8_t* mask, const flo
 
 namespace provip {
 
-bool crit_gram_tc_supported(const SimArgs& a) { return a.dtype == 1 && a.N_t_max <= kBM && a.D % 8 == 0; }
+bool crit_gram_tc_supported(const SimArgs& a) { return crit_splits(a.N_t_max, a.D, a.dtype) > 0; }
+
+// K parts of the text Gram: 0 when the tcgen05 form does not apply; every part
+// owns ceil(n_k / parts) slices of 64 (the last one possibly fewer)
+int crit_splits(int N_t_max, int D, int dtype) {
+  if (dtype != 1 || N_t_max > kBM || D % 8) return 0;
+  const int n_k = (D + kBK - 1) / kBK;
+  const int ns = n_k < kCritMaxSplits ? n_k : kCritMaxSplits;
+  const int per = (n_k + ns - 1) / ns;
+  return (n_k + per - 1) / per;
+}
 
 cudaError_t crit_gram_tc_launch(const SimArgs& a, float* G, cudaStream_t s) {
   static bool smem_set[64] = {false};
@@ -458,7 +471,10 @@ cudaError_t crit_gram_tc_launch(const SimArgs& a, float* G, cudaStream_t s) {
   CUtensorMap mapT;
   if (make_tmap_bf16_2d(&mapT, a.emb_t, (uint64_t)a.B * a.N_t_max, (uint64_t)a.D, (uint64_t)a.D * 2, 128))
     return cudaErrorInvalidValue;
-  crit_gram_tc<<<dim3(1, 1, a.B), kThreads, smem, s>>>(mapT, a.text_len, a.N_t_max, a.D, G, a.err);
+  const int parts = crit_splits(a.N_t_max, a.D, a.dtype);
+  const int n_k = (a.D + kBK - 1) / kBK, per = (n_k + parts - 1) / parts;
+  crit_gram_tc<<<dim3(parts, 1, a.B), kThreads, smem, s>>>(mapT, a.text_len, a.N_t_max, a.D, a.B, per, G,
+                                                          a.err);
   return cudaGetLastError();
 }
 

@@ -84,10 +84,11 @@ __device__ __forceinline__ void load_rows(uint8_t* dst, const CUtensorMap* map, 
 
 // Producer: for each N tile t in [0, n_tiles), all K slices.
 template <int BN>
+// k0: first K slice (a split-K part starts past the others' slices)
 __device__ __forceinline__ void producer(Pipe& p, uint8_t* stages, const CUtensorMap* mapA,
                                          const CUtensorMap* mapB, const RowSrc& a, bool gatherA,
                                          const RowSrc& b, bool gatherB, int n_tiles, int n_k,
-                                         unsigned* err) {
+                                         unsigned* err, int k0 = 0) {
   int it = 0;
   for (int t = 0; t < n_tiles && !p.fail; ++t) {
     for (int kb = 0; kb < n_k; ++kb, ++it) {
@@ -100,8 +101,8 @@ __device__ __forceinline__ void producer(Pipe& p, uint8_t* stages, const CUtenso
       uint8_t* sa = stages + (size_t)s * Cfg<BN>::kStageBytes;
       uint8_t* sb = sa + kABytes;
       mbar_arrive_expect_tx(&p.full[s], Cfg<BN>::kStageBytes);
-      load_rows(sa, mapA, a, 0, kBM, kb * kBK, &p.full[s], gatherA);
-      load_rows(sb, mapB, b, t * BN, BN, kb * kBK, &p.full[s], gatherB);
+      load_rows(sa, mapA, a, 0, kBM, (k0 + kb) * kBK, &p.full[s], gatherA);
+      load_rows(sb, mapB, b, t * BN, BN, (k0 + kb) * kBK, &p.full[s], gatherB);
     }
   }
 }
