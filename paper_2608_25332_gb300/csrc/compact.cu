@@ -14,7 +14,10 @@
 // (global -> shared, completion on the slot's mbarrier) and, once it lands, a
 // cp.async.bulk store (shared -> global, bulk group). A slot is refilled as soon
 // as the store that drained it has finished reading, so up to kSlots - 1 loads
-// and a store are in flight per CTA. The other warps copy the position ids.
+// and a store are in flight per CTA. The other warps copy the position ids and,
+// with 16-byte vector loads and stores (a warp per row), the rows of tensors
+// whose rows are at most 2 KiB (the K/V rows of a GQA layer with few key/value
+// heads), which per-row bulk copies would move inefficiently.
 // Every wait is bounded; a timeout sets the device error word and the CTA
 // drains what it issued before returning.
 #include "common.cuh"
@@ -37,6 +40,13 @@ constexpr int kSlots = PROVIP_COMPACT_SLOTS;          // ring of shared-memory s
 constexpr int kCtasPerSm = PROVIP_COMPACT_CTAS_PER_SM;
 constexpr int kCompactThreads = 128;
 constexpr size_t kCompactSmem = (size_t)kSlots * kSlotBytes;
+// tensors with rows of at most this many bytes are copied by the helper warps
+// with vector loads and stores (per-row bulk copies would cost more than they
+// move)
+#ifndef PROVIP_COMPACT_SMALL_ROW
+#define PROVIP_COMPACT_SMALL_ROW 2048
+#endif
+constexpr int kSmallRow = PROVIP_COMPACT_SMALL_ROW;
 
 __device__ __forceinline__ int src_row(const CompactArgs& a, int b, int r, bool& ok) {
   if (r < a.vis_start) return r;
@@ -75,12 +85,15 @@ __device__ __forceinline__ void phase_row(const CompactArgs& a, int phase, long 
 }
 
 __global__ void __launch_bounds__(kCompactThreads) compact_kernel(const CompactArgs a, int np0,
-                                                                   int np1, int np2) {
+                                                                   int np1, int np2, int small) {
   extern __shared__ __align__(128) uint8_t slots[];
   __shared__ __align__(8) uint64_t bars[kSlots];
   __shared__ char* ring_dst[kSlots];
   __shared__ uint32_t ring_bytes[kSlots];
-  const int NP = np0 + np1 + np2;
+  // items per output row: the pieces of the bulk-copied tensors (at least one,
+  // so that rows are spread over CTAs even when every tensor is small)
+  const int NB = np0 + np1 + np2;
+  const int NP = NB > 0 ? NB : 1;
   long long rows[2] = {(long long)a.B * (a.L_out - a.keep), (long long)a.B * a.keep};
   long long beg[2], fin[2];
   for (int ph = 0; ph < 2; ++ph) {
@@ -103,7 +116,7 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(const CompactA
   }
   __syncthreads();
 
-  if (threadIdx.x == 0) {
+  if (threadIdx.x == 0 && NB > 0) {
     const uint64_t pol = policy_evict_first();
     int phase = 0;
     long long next = beg[0];
@@ -187,13 +200,17 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(const CompactA
       for (int j = i; j < loaded; ++j) mbar_wait(&bars[j % kSlots], (uint32_t)(j / kSlots) & 1u, a.err);
     }
     bulk_wait<0>();
-  } else if (a.pos != nullptr && threadIdx.x >= 32) {
-    // position ids of the rows whose first item lies in this CTA's ranges
-    const int nth = blockDim.x - 32;
+  } else if (threadIdx.x >= 32 && (a.pos != nullptr || small != 0)) {
+    // rows whose first item lies in this CTA's ranges: their position ids, and
+    // the rows of the small tensors (16-byte vector copies, a warp per row)
+    // a thread per row for the position ids alone, a warp per row with small tensors
+    const int lane = small ? (int)(threadIdx.x & 31) : 0;
+    const int worker = small ? (int)(threadIdx.x >> 5) - 1 : (int)threadIdx.x - 32;
+    const int n_workers = small ? kCompactThreads / 32 - 1 : kCompactThreads - 32;
     for (int ph = 0; ph < 2; ++ph) {
       if (ph == 1) pdl_wait();
       const long long r0 = (beg[ph] + NP - 1) / NP, r1 = (fin[ph] + NP - 1) / NP;
-      for (long long row = r0 + (threadIdx.x - 32); row < r1; row += nth) {
+      for (long long row = r0 + worker; row < r1; row += n_workers) {
         int b, r;
         phase_row(a, ph, row, b, r);
         const int sl = a.seq_len[b];
@@ -201,8 +218,23 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(const CompactA
         bool ok = true;
         const int sr = src_row(a, b, r, ok);
         if (!ok) continue;
-        for (int p = 0; p < a.P; ++p)
-          a.pos_out[((size_t)p * a.B + b) * a.L_out + r] = a.pos[((size_t)p * a.B + b) * a.L_max + sr];
+        if (a.pos != nullptr)
+          for (int p = lane; p < a.P; p += 32)
+            a.pos_out[((size_t)p * a.B + b) * a.L_out + r] = a.pos[((size_t)p * a.B + b) * a.L_max + sr];
+        for (int t = 0; t < a.n_tensors; ++t) {
+          if (!(small & (1 << t))) continue;
+          const long long rb = a.row_bytes[t];
+          const uint4* src = reinterpret_cast<const uint4*>(a.src[t] + ((long long)b * a.L_max + sr) * rb);
+          uint4* dst = reinterpret_cast<uint4*>(a.dst[t] + ((long long)b * a.L_out + r) * rb);
+          const int n16 = (int)(rb / 16);
+          uint4 v[kSmallRow / 16 / 32];
+#pragma unroll
+          for (int k = 0; k < kSmallRow / 16 / 32; ++k)
+            if (lane + 32 * k < n16) v[k] = __ldcs(src + lane + 32 * k);
+#pragma unroll
+          for (int k = 0; k < kSmallRow / 16 / 32; ++k)
+            if (lane + 32 * k < n16) __stcs(dst + lane + 32 * k, v[k]);
+        }
       }
     }
   }
@@ -221,9 +253,15 @@ cudaError_t compact_launch(const CompactArgs& a, int num_sms, cudaStream_t s, bo
     configured[dev] = true;
   }
   int np[3] = {0, 0, 0};
-  for (int t = 0; t < a.n_tensors; ++t)
-    np[t] = (int)((a.row_bytes[t] + kSlotBytes - 1) / kSlotBytes);
-  const long long total = (long long)a.B * a.L_out * (np[0] + np[1] + np[2]);
+  int small = 0;
+  for (int t = 0; t < a.n_tensors; ++t) {
+    if (a.row_bytes[t] <= kSmallRow)
+      small |= 1 << t;
+    else
+      np[t] = (int)((a.row_bytes[t] + kSlotBytes - 1) / kSlotBytes);
+  }
+  const int nb = np[0] + np[1] + np[2];
+  const long long total = (long long)a.B * a.L_out * (nb > 0 ? nb : 1);
   long long grid = (long long)kCtasPerSm * num_sms;
   if (grid > total) grid = total > 0 ? total : 1;
   cudaLaunchConfig_t cfg = {};
@@ -236,7 +274,7 @@ cudaError_t compact_launch(const CompactArgs& a, int num_sms, cudaStream_t s, bo
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = pdl ? 1 : 0;
-  return cudaLaunchKernelEx(&cfg, compact_kernel, a, np[0], np[1], np[2]);
+  return cudaLaunchKernelEx(&cfg, compact_kernel, a, np[0], np[1], np[2], small);
 }
 
 }  // namespace provip
