@@ -61,7 +61,9 @@ def parse_args(argv=None):
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
-    ap.add_argument("--algo", default="auto", choices=["auto", "simt", "tcgen05"])
+    ap.add_argument("--algo", default="auto", choices=["auto", "simt", "tcgen05", "stream", "cluster"],
+                    help="head-score kernel form (auto: tcgen05 for bf16, and the streaming form when "
+                         "several single-sample streams run concurrently)")
     ap.add_argument("--e2e-steps", type=int, default=20)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--copies", type=int, default=N_COPIES, help="rotating device copies of the inputs")
@@ -69,7 +71,7 @@ def parse_args(argv=None):
                     help="time only the pre-LLM pass (provip_similarity_reduce) and print its JSON")
     ap.add_argument("--prellm-reps", type=int, default=20)
     ap.add_argument("--streams", type=int, default=None,
-                    help="independent sample streams run concurrently (default: 10 for single-sample "
+                    help="independent sample streams run concurrently (default: 20 for single-sample "
                          "batches, else 1)")
     return ap.parse_args(argv)
 
@@ -502,7 +504,12 @@ def run_gb300(args, dist):
     # each rank prunes its own shard of samples (seeded by rank)
     cpu = synth.in_llm_inputs(w, seed=w.seed + 1000 * dist.rank)
     vis, nv, keep = cpu["vis_start"], cpu["N_v"], cpu["keep"]
-    algo = {"auto": P.ALGO_AUTO, "simt": P.ALGO_SIMT, "tcgen05": P.ALGO_TCGEN05}[args.algo]
+    S = args.streams if args.streams is not None else (20 if w.B == 1 else 1)
+    # many concurrent single-sample streams: the streaming head-score form uses
+    # less SM time per sample than the cluster form (at a higher latency)
+    algo_name = "stream" if (args.algo == "auto" and S > 1 and w.dtype == "bf16") else args.algo
+    algo = {"auto": P.ALGO_AUTO, "simt": P.ALGO_SIMT, "tcgen05": P.ALGO_TCGEN05,
+            "stream": P.ALGO_TCGEN05_STREAM, "cluster": P.ALGO_TCGEN05_CLUSTER}[algo_name]
     copies = []
     n_copies = max(1, args.copies)
     for _ in range(n_copies):
@@ -519,7 +526,6 @@ def run_gb300(args, dist):
     # fill the GPU with one dependent chain): stream s takes steps s, s + S, ...
     # on its own input copies and its own outputs and workspace; lane 0 is the
     # step and copies above.
-    S = args.streams if args.streams is not None else (10 if w.B == 1 else 1)
     if S < 1 or GRAPH_CHUNK % S or args.steps % S:
         raise SystemExit(f"--streams {S} must divide --steps and {GRAPH_CHUNK}")
     lanes = [(copies, step)]
@@ -640,7 +646,8 @@ def run_gb300(args, dist):
 
     # kernels per step: one-pass head scores (tcgen05, L_max <= 8192), top-k,
     # compaction; the two-pass and CUDA-core forms launch two head kernels
-    launches_per_step = 3 if (args.algo in ("auto", "tcgen05") and w.dtype == "bf16" and w.L_max <= 8192) else 4
+    launches_per_step = 3 if (algo_name in ("auto", "tcgen05", "stream", "cluster") and w.dtype == "bf16"
+                              and w.L_max <= 8192) else 4
     reps = max(1, min(20, K // GRAPH_CHUNK))
     t_compact = time_graph(compact_i, reps)
     t_head = time_graph(head_topk_i, reps)
@@ -731,7 +738,7 @@ def run_gb300(args, dist):
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": dist.world, "steps": K,
             "warmup": args.warmup, "ms_per_step": 1e3 * max_sec / K, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
-            "config": dict(workload_config(w, args.algo, len(copies),
+            "config": dict(workload_config(w, algo_name, len(copies),
                                            sum(v.numel() * v.element_size() for v in pin.values()) / 1e6),
                            streams=S,
                            **({"concurrency": f"{S} streams of independent batches run concurrently, each "
