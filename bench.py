@@ -71,7 +71,7 @@ def parse_args(argv=None):
                     help="time only the pre-LLM pass (provip_similarity_reduce) and print its JSON")
     ap.add_argument("--prellm-reps", type=int, default=20)
     ap.add_argument("--streams", type=int, default=None,
-                    help="independent sample streams run concurrently (default: 20 for single-sample "
+                    help="independent sample streams run concurrently (default: 25 for single-sample "
                          "batches, else 1)")
     return ap.parse_args(argv)
 
@@ -504,7 +504,7 @@ def run_gb300(args, dist):
     # each rank prunes its own shard of samples (seeded by rank)
     cpu = synth.in_llm_inputs(w, seed=w.seed + 1000 * dist.rank)
     vis, nv, keep = cpu["vis_start"], cpu["N_v"], cpu["keep"]
-    S = args.streams if args.streams is not None else (20 if w.B == 1 else 1)
+    S = args.streams if args.streams is not None else (25 if w.B == 1 else 1)
     # many concurrent single-sample streams: the streaming head-score form uses
     # less SM time per sample than the cluster form (at a higher latency)
     algo_name = "stream" if (args.algo == "auto" and S > 1 and w.dtype == "bf16") else args.algo

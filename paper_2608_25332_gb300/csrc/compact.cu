@@ -40,6 +40,10 @@ constexpr int kSlots = PROVIP_COMPACT_SLOTS;          // ring of shared-memory s
 constexpr int kCtasPerSm = PROVIP_COMPACT_CTAS_PER_SM;
 constexpr int kCompactThreads = 128;
 constexpr size_t kCompactSmem = (size_t)kSlots * kSlotBytes;
+#ifndef PROVIP_COMPACT_MIN_CTA_KIB
+#define PROVIP_COMPACT_MIN_CTA_KIB 160
+#endif
+constexpr long long kMinCtaBytes = (long long)PROVIP_COMPACT_MIN_CTA_KIB * 1024;
 // tensors with rows of at most this many bytes are copied by the helper warps
 // with vector loads and stores (per-row bulk copies would cost more than they
 // move)
@@ -263,6 +267,11 @@ cudaError_t compact_launch(const CompactArgs& a, int num_sms, cudaStream_t s, bo
   const int nb = np[0] + np[1] + np[2];
   const long long total = (long long)a.B * a.L_out * (nb > 0 ? nb : 1);
   long long grid = (long long)kCtasPerSm * num_sms;
+  // small problems: at least kMinCtaBytes of rows per CTA, so that every CTA's
+  // pipeline fills (and kernels running beside it keep the SMs it does not need)
+  const long long row_sum = a.row_bytes[0] + a.row_bytes[1] + a.row_bytes[2];
+  const long long by_bytes = ((long long)a.B * a.L_out * row_sum + kMinCtaBytes - 1) / kMinCtaBytes;
+  if (grid > by_bytes) grid = by_bytes;
   if (grid > total) grid = total > 0 ? total : 1;
   cudaLaunchConfig_t cfg = {};
   cudaLaunchAttribute attr[1];
