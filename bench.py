@@ -694,32 +694,81 @@ def run_gb300(args, dist):
         traffic = COMPACT_TRAFFIC["bytes"]
     path_gbs = ab["path"] * K / max_sec / 1e9  # per GPU
 
-    # e2e: host buffers through the C ABI, H2D + prune + D2H per step
+    # e2e: host buffers through the C ABI. Every step copies its inputs from
+    # pinned host memory and its outputs back to pinned host memory inside the
+    # timed region; two device buffer sets (each with its own outputs) alternate
+    # so that the copies of one step overlap the pruning of the other (a stream
+    # per copy direction and one for the kernels, ordered by events).
     pin = {k: v.pin_memory() for k, v in cpu.items() if isinstance(v, torch.Tensor)}
-    dbuf = {k: torch.empty_like(v, device=dev) for k, v in pin.items()}
-    host_out = {k: torch.empty(v.shape, dtype=v.dtype, pin_memory=True)
-                for k, v in (("hidden", step.hidden_out), ("K", step.K_out), ("V", step.V_out),
-                             ("pos", step.pos_out), ("idx", step.idx), ("seq_len", step.seq_len_out))}
+    out_keys = ("hidden", "K", "V", "pos", "idx", "seq_len")
+    e2e_sets = []
+    for j in range(2):
+        db = {k: torch.empty_like(v, device=dev) for k, v in pin.items()}
+        st_j = step if j == 0 else P.PruneStep(db["Q"], db["K"], db["V"], db["hidden"], db["pos"], cpu["head_list"],
+                                              w.n_t[1], nv, keep, algo=algo, want_scores=False,
+                                              flags=P.PRUNE_OVERLAP_PREVIOUS)
+        outs_j = {"hidden": st_j.hidden_out, "K": st_j.K_out, "V": st_j.V_out, "pos": st_j.pos_out,
+                  "idx": st_j.idx, "seq_len": st_j.seq_len_out}
+        ho = {k: torch.empty(outs_j[k].shape, dtype=outs_j[k].dtype, pin_memory=True) for k in out_keys}
+        ev = {n: torch.cuda.Event() for n in ("comp", "d2h")}
+        e2e_sets.append((db, st_j, ho, ev))
     h2d = sum(v.numel() * v.element_size() for v in pin.values())
-    d2h = sum(v.numel() * v.element_size() for v in host_out.values())
+    d2h = sum(v.numel() * v.element_size() for v in e2e_sets[0][2].values())
+    s_comp, s_d2h = (torch.cuda.Stream(device=dev) for _ in range(2))
+    # the input copies are spread over N_H2D streams (copy engines) by size
+    N_H2D = 2
+    s_h2ds = [torch.cuda.Stream(device=dev) for _ in range(N_H2D)]
+    by_size = sorted(pin, key=lambda k: -pin[k].numel() * pin[k].element_size())
+    h2d_parts = [by_size[i::N_H2D] for i in range(N_H2D)]
+    for j in range(2):
+        e2e_sets[j][3]["h2d_parts"] = [torch.cuda.Event() for _ in range(N_H2D)]
+    fresh = [True, True]
 
-    def e2e_step():
-        for k, v in pin.items():
-            dbuf[k].copy_(v, non_blocking=True)
-        r = step(dbuf["Q"], dbuf["K"], dbuf["V"], dbuf["hidden"], dbuf["pos"], dbuf["text_start"],
-                 dbuf["text_len"], dbuf["seq_len"], vis)
-        for k in host_out:
-            host_out[k].copy_(r[k], non_blocking=True)
+    def e2e_step(n):
+        j = n % 2
+        db, st_j, ho, ev = e2e_sets[j]
+        for s_h2d, keys, e_part in zip(s_h2ds, h2d_parts, ev["h2d_parts"]):
+            with torch.cuda.stream(s_h2d):
+                if not fresh[j]:
+                    s_h2d.wait_event(ev["comp"])  # the set's inputs were consumed by step n - 2
+                for k in keys:
+                    db[k].copy_(pin[k], non_blocking=True)
+                e_part.record(s_h2d)
+        with torch.cuda.stream(s_comp):
+            for e_part in ev["h2d_parts"]:
+                s_comp.wait_event(e_part)
+            if not fresh[j]:
+                s_comp.wait_event(ev["d2h"])  # step n - 2's outputs have left this set
+            r = st_j(db["Q"], db["K"], db["V"], db["hidden"], db["pos"], db["text_start"], db["text_len"],
+                     db["seq_len"], vis, stream=s_comp)
+            ev["comp"].record(s_comp)
+        with torch.cuda.stream(s_d2h):
+            s_d2h.wait_event(ev["comp"])
+            for k in out_keys:
+                ho[k].copy_(r[k], non_blocking=True)
+            ev["d2h"].record(s_d2h)
+        fresh[j] = False
 
-    for _ in range(2):
-        e2e_step()
+    def e2e_run(first, n_steps):
+        main = torch.cuda.current_stream(dev)
+        start = torch.cuda.Event()
+        start.record(main)
+        for st_ in (*s_h2ds, s_comp, s_d2h):
+            st_.wait_event(start)
+        for n in range(first, first + n_steps):
+            e2e_step(n)
+        for st_ in (*s_h2ds, s_comp, s_d2h):
+            done = torch.cuda.Event()
+            done.record(st_)
+            main.wait_event(done)
+
+    e2e_run(0, 4)
     torch.cuda.synchronize()
     E = max(1, args.e2e_steps)
     a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     dist.barrier()
     a.record()
-    for _ in range(E):
-        e2e_step()
+    e2e_run(4, E)
     b.record()
     torch.cuda.synchronize()
     e2e_sec = dist.max(a.elapsed_time(b) / 1e3)
