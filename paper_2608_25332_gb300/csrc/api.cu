@@ -542,7 +542,7 @@ static size_t simred_ws(Carve& c, int B, int N_v, int D, int N_t_max, int keep_p
   w.mask = c.take<uint8_t>((size_t)B * N_t_max);
   w.p = c.take<float>((size_t)B * N_v);
   w.assign = c.take<int>((size_t)B * N_v);
-  SimWs r, m;
+  SimWs r;
   relevance_ws(c, B, N_v, D, N_t_max, r);
   const int ns = merge_ws_splits(B, N_v, keep_pre);
   w.inv_v = r.inv_v;
@@ -553,7 +553,6 @@ static size_t simred_ws(Carve& c, int B, int N_v, int D, int N_t_max, int keep_p
   w.bidx = c.take<int>((size_t)ns * B * N_v);
   w.pruned = c.take<int>((size_t)B * N_v);
   w.perm = c.take<uint16_t>((size_t)B * N_v * D);
-  (void)m;
   return c.off;
 }
 

@@ -136,3 +136,13 @@ def test_workspace_sizes_grow_with_the_problem(L):
     assert L.provip_prune_workspace_size(8, 1091, 8, 96, 960, 2, 1) == a
     assert L.provip_similarity_reduce_workspace_size(1, 9216, 3584, 128, 2304) > \
         L.provip_relevance_workspace_size(1, 9216, 3584, 128)
+
+
+def test_schedule_rejects_inconsistent_stages():
+    """The progressive schedule validates its stage arguments before touching
+    the GPU."""
+    from paper_2608_25332_gb300.schedule import ProgressiveSchedule
+    with pytest.raises(ValueError):  # without pre-LLM pruning every visual token reaches the LLM
+        ProgressiveSchedule(2, 576, 4096, 128, 739, 32, 32, 4096, 1, 288, 73, 20, 6, pre_llm=False)
+    with pytest.raises(ValueError):
+        ProgressiveSchedule(2, 576, 4096, 128, 739, 32, 32, 4096, 1, 576, 73, 20, 6, shallow_heads="some")
