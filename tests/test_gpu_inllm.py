@@ -124,20 +124,23 @@ def test_fused_and_standalone_scores_are_identical():
     assert torch.equal(idx2, out["idx"])
 
 
-def test_overlapped_calls_match_serial_calls():
+@pytest.mark.parametrize("algo", ["ALGO_AUTO", "ALGO_TCGEN05_STREAM", "ALGO_TCGEN05_CLUSTER"])
+@pytest.mark.parametrize("name", ["llava_next_7b_bf16_b8", "video_gqa_bf16_b1"])
+def test_overlapped_calls_match_serial_calls(name, algo):
     """PROVIP_PRUNE_OVERLAP_PREVIOUS: back-to-back calls on three different batches
-    sharing one workspace give the same bits as calls separated by a sync."""
-    name = "llava_next_7b_bf16_b8"
+    sharing one workspace give the same bits as calls separated by a sync, for
+    each tensor-core form of the head scores."""
+    algo = getattr(P, algo)
     w, cpu, g0 = inputs(name)
     batches = [g0] + [{k: (v.to(DEV) if isinstance(v, torch.Tensor) else v)
                        for k, v in synth.in_llm_inputs(w, seed=w.seed + 77 + i).items()} for i in range(2)]
     ws = P.workspace(P.lib().provip_prune_workspace_size(w.B, w.L_max, w.H_sel, w.n_t[1], w.keep_pre,
-                                                         P.ALGO_AUTO, P.BF16), DEV)
+                                                         algo, P.BF16), DEV)
     def run(flags, sync):
         outs = []
         for c in batches:
             st = P.PruneStep(c["Q"], c["K"], c["V"], c["hidden"], c["pos"], c["head_list"], w.n_t[1], c["N_v"],
-                             c["keep"], flags=flags, ws=ws)
+                             c["keep"], algo=algo, flags=flags, ws=ws)
             outs.append(st(c["Q"], c["K"], c["V"], c["hidden"], c["pos"], c["text_start"], c["text_len"],
                            c["seq_len"], c["vis_start"]))
             if sync:
