@@ -440,7 +440,10 @@ extern "C" int provip_crit_text(const void* emb_t, int B, int N_t_max, int D, co
 static size_t relevance_ws(Carve& c, int B, int N_v, int D, int N_t_max, SimWs& w) {
   const int ns = rel_splits(B, N_v);
   w.inv_v = c.take<float>((size_t)B * N_v);
-  w.sum = c.take<float>((size_t)(ns + 1) * B * D);
+  // the split column sums of the CUDA-core form, or the cosines and tile sums
+  // of the tensor-core form
+  const size_t sum_f = (size_t)(ns + 1) * B * D, fused_f = relevance_fused_floats(B, N_v, N_t_max);
+  w.sum = c.take<float>(sum_f > fused_f ? sum_f : fused_f);
   w.mu = c.take<float>((size_t)B * N_t_max);
   w.invt = c.take<float>((size_t)B * N_t_max);
   return c.off;
@@ -467,7 +470,8 @@ extern "C" int provip_relevance(const void* emb_v, int B, int N_v, int D, const 
   relevance_ws(c, B, N_v, D, N_t_max, w);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   SimArgs a = sim_args(emb_v, emb_t, text_len, B, N_v, D, N_t_max, dtype, d->status);
-  cudaError_t e = relevance_launch(a, crit_mask, w.inv_v, p_out, w.sum, w.mu, w.invt, rel_splits(B, N_v), s);
+  cudaError_t e =
+      relevance_launch(a, crit_mask, w.inv_v, p_out, w.sum, w.mu, w.invt, rel_splits(B, N_v), d->sms, s);
   return e == cudaSuccess ? PROVIP_OK : cuda_fail(e, "relevance launch");
 }
 
@@ -597,7 +601,8 @@ extern "C" int provip_similarity_reduce(const void* emb_v, int B, int N_v, int D
     e = cudaMemcpyAsync(mask_out_or_null, mask, (size_t)B * N_t_max, cudaMemcpyDeviceToDevice, s);
   }
   float* p = p_out_or_null ? p_out_or_null : w.p;
-  if (e == cudaSuccess) e = relevance_launch(a, mask, w.inv_v, p, w.sum, w.mu, w.invt, rel_splits(B, N_v), s);
+  if (e == cudaSuccess)
+    e = relevance_launch(a, mask, w.inv_v, p, w.sum, w.mu, w.invt, rel_splits(B, N_v), d->sms, s);
   if (e == cudaSuccess) {
     TopkArgs t;
     memset(&t, 0, sizeof(t));

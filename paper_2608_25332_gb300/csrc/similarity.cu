@@ -817,7 +817,10 @@ cudaError_t vis_inv_norm_launch(const SimArgs& a, float* inv_v, cudaStream_t s) 
 
 cudaError_t relevance_launch(const SimArgs& a, const uint8_t* mask, float* inv_v, float* p,
                              float* ws_sum, float* ws_mu, float* ws_invt, int n_split,
-                             cudaStream_t s) {
+                             int num_sms, cudaStream_t s) {
+  // bf16 with at most 128 text rows: one tensor-core read of the visual rows
+  // (norms, cosines and de-meaning sums) and a small max kernel
+  if (relevance_tc_supported(a)) return relevance_tc_launch(a, mask, inv_v, p, ws_sum, num_sms, s);
   const int chunk = (a.N_v + n_split - 1) / n_split;
   dim3 g1((a.D + 255) / 256, a.B, n_split);
   dim3 g2((a.N_t_max + 7) / 8, a.B);
@@ -861,11 +864,6 @@ cudaError_t relevance_launch(const SimArgs& a, const uint8_t* mask, float* inv_v
     if (!fused) vis_sum_kernel<__nv_bfloat16><<<g1, 256, 0, s>>>(a, inv_v, ws_sum, chunk);
     vis_sum_reduce_kernel<<<g4, 256, 0, s>>>(a, ws_sum, n_split, total);
     text_mu_kernel<__nv_bfloat16><<<g2, 256, 0, s>>>(a, total, ws_mu, ws_invt);
-    if (relevance_tc_supported(a)) {
-      cudaError_t e = cudaGetLastError();
-      if (e != cudaSuccess) return e;
-      return relevance_tc_launch(a, mask, inv_v, ws_mu, ws_invt, p, s);
-    }
     relevance_kernel<__nv_bfloat16><<<g3, 256, 0, s>>>(a, mask, inv_v, ws_mu, ws_invt, p);
   }
   return cudaGetLastError();

@@ -7,11 +7,10 @@
 //   epilogue scales a column by 1/|e_k| and keeps, per row, the running (max,
 //   first index) over the kept positions in ascending order, so ties go to the
 //   lower kept position. The (N_v - N1) x N1 matrix never leaves the SM.
-// relevance_tc: the text x visual cosine Gram fused with the de-meaned column
-//   max: p_j = max_{i in T} (<t_i, v_j> / |t_i| / |v_j| - mu_i) for a 128-column
-//   block of visual rows (A = the <= 128 text rows of the sample, B = 128
-//   consecutive visual rows), the max over rows taken with a warp butterfly and
-//   a fixed-order combine of the four epilogue warps.
+// relevance_fused_tc: the visual x text cosine Gram with the row norms of both
+//   operands taken from the same shared-memory stages, so the visual rows are
+//   read once for |v_j|, the cosines and the de-meaning sums (p_j itself is
+//   formed by a small second kernel once every tile's sums are known).
 #include "common.cuh"
 #include "kernels.h"
 #include "tc_gemm.cuh"
@@ -186,37 +185,77 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (threadIdx.x < 32) tmem_dealloc(pipe.tmem, Cfg<kMergeBN>::kTmemCols);
 }
 
-struct RelTcArgs {
+// relevance_fused_tc: one read of the visual rows gives, per 128-row tile of
+// sample b,
+//   * |v_j|^-1 (from the shared-memory stages the MMA consumes: each epilogue
+//     thread sums the squares of its row's 64 elements per K slice) and
+//     |t_i|^-1 for the text rows (same, on the text stage),
+//   * the cosines Y[b][j][i] = <v_j, t_i> |t_i|^-1 |v_j|^-1 (A = the visual
+//     rows, B = the text rows; thread = TMEM lane = visual row j),
+//   * the tile's column sums part[b][tile][i] = sum_j Y[b][j][i] (warp
+//     butterfly, then the four lane quadrants in order).
+// relevance_finish_kernel then forms mu_i = (sum of the tile sums in tile
+// order) / N_v and p_j = max_{i in T} (Y[b][j][i] - mu_i) (Sec. 4.3).
+struct RelFusedArgs {
   int B, N_v, D, N_t_max;
-  const int* text_len;
-  const uint8_t* mask;  // [B][N_t_max]
-  const float* inv_v;   // [B][N_v]
-  const float* mu;      // [B][N_t_max]
-  const float* invt;    // [B][N_t_max]
-  float* p;             // [B][N_v]
+  int NT;        // text rows in the MMA (N_t_max rounded up to 16)
+  int n_vt;      // 128-row visual tiles per sample
+  int n_stages;  // shared-memory ring depth
+  float* inv_v;  // [B][N_v]
+  float* Y;      // [B][N_v][NT]
+  float* part;   // [B][n_vt][NT]
   unsigned* err;
 };
 
-constexpr int kRelBN = 128;
+constexpr int kRelMaxStages = 8;
 
-__global__ void __launch_bounds__(kThreads, 1)
-    relevance_tc(const RelTcArgs a, const __grid_constant__ CUtensorMap mapT,
-                 const __grid_constant__ CUtensorMap mapV) {
+struct RelPipe {
+  uint64_t full[kRelMaxStages];
+  uint64_t empty[kRelMaxStages];
+  uint64_t acc_full;
+  uint32_t tmem;
+  volatile int fail;
+};
+
+// sum of squares of the 8 bf16 values of a 16-byte chunk, two chains
+__device__ __forceinline__ void sumsq8(const uint4 u, float& s0, float& s1) {
+  const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const float lo = __uint_as_float(w[q] << 16), hi = __uint_as_float(w[q] & 0xffff0000u);
+    s0 = fmaf(lo, lo, s0);
+    s1 = fmaf(hi, hi, s1);
+  }
+}
+
+__global__ void __launch_bounds__(kThreads, 2)
+    relevance_fused_tc(const RelFusedArgs a, const __grid_constant__ CUtensorMap mapV,
+                       const __grid_constant__ CUtensorMap mapT) {
   extern __shared__ uint8_t smem_raw[];
-  __shared__ Pipe pipe;
-  __shared__ float red[4][kRelBN];
-  const int b = blockIdx.z;
-  const int n0 = blockIdx.x * kRelBN;
+  __shared__ RelPipe pipe;
+  __shared__ float s_invt[kBM];
+  __shared__ float red[4][kBM];
+  const int b = blockIdx.y, tile = blockIdx.x;
+  const int n0 = tile * kBM;
   const int n_k = (a.D + kBK - 1) / kBK;
+  const int NS = a.n_stages;
+  const uint32_t st_bytes = (uint32_t)kABytes + (uint32_t)a.NT * 128u;
+  const uint32_t tcols = a.NT <= 32 ? 32u : (a.NT <= 64 ? 64u : 128u);
   const uint32_t sbase = smem_u32(smem_raw);
   uint8_t* stages = smem_raw + (((sbase + 1023u) & ~1023u) - sbase);
   if (threadIdx.x == 0) {
-    prefetch_tmap(&mapT);
     prefetch_tmap(&mapV);
-    pipe_init(pipe);
+    prefetch_tmap(&mapT);
+    for (int s = 0; s < NS; ++s) {
+      mbar_init(&pipe.full[s], 1);
+      mbar_init(&pipe.empty[s], 5);  // the MMA commit + one arrival per epilogue warp
+    }
+    mbar_init(&pipe.acc_full, 1);
+    pipe.fail = 0;
+    fence_mbar_init();
   }
   if (threadIdx.x < 32) {
-    tmem_alloc(&pipe.tmem, Cfg<kRelBN>::kTmemCols);
+    tmem_alloc(&pipe.tmem, tcols);
     tmem_relinquish();
   }
   tc_fence_before();
@@ -225,34 +264,98 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (warp == 0) {
     if (lane == 0) {
-      RowSrc ra{nullptr, b * a.N_t_max, kBM};
-      RowSrc rb{nullptr, b * a.N_v + n0, kRelBN};
-      producer<kRelBN>(pipe, stages, &mapT, &mapV, ra, false, rb, false, 1, n_k, a.err);
+      for (int kb = 0; kb < n_k; ++kb) {
+        const int s = kb % NS;
+        const uint32_t ph = (uint32_t)(kb / NS) & 1u;
+        if (pipe.fail || !mbar_wait(&pipe.empty[s], ph ^ 1u, a.err)) {
+          pipe.fail = 1;
+          break;
+        }
+        uint8_t* sa = stages + (size_t)s * st_bytes;
+        mbar_arrive_expect_tx(&pipe.full[s], st_bytes);
+        // rows past the sample's last visual row belong to the next sample (or
+        // lie past the tensor and read as zeros): computed, never stored
+        tma_load_2d(sa, &mapV, kb * kBK, b * a.N_v + n0, &pipe.full[s]);
+        tma_load_2d(sa + kABytes, &mapT, kb * kBK, b * a.N_t_max, &pipe.full[s]);
+      }
     }
   } else if (warp == 1) {
-    if (lane == 0) mma_issuer<kRelBN>(pipe, stages, 1, n_k, a.err);
+    if (lane == 0) {
+      const uint32_t idesc = idesc_bf16_f32(kBM, a.NT);
+      for (int kb = 0; kb < n_k; ++kb) {
+        const int s = kb % NS;
+        const uint32_t ph = (uint32_t)(kb / NS) & 1u;
+        if (pipe.fail || !mbar_wait(&pipe.full[s], ph, a.err)) {
+          pipe.fail = 1;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t sa = smem_u32(stages + (size_t)s * st_bytes);
+        const uint32_t sb = sa + kABytes;
+#pragma unroll
+        for (int k = 0; k < kBK / 16; ++k)
+          tc_mma_bf16(pipe.tmem, smem_desc_sw128(sa + k * 32), smem_desc_sw128(sb + k * 32), idesc,
+                      (kb > 0 || k > 0) ? 1u : 0u);
+        tc_commit(&pipe.empty[s]);
+      }
+      tc_commit(&pipe.acc_full);  // arrives once every MMA above has completed
+    }
   } else {
     const int quad = warp & 3;
     const int r = quad * 32 + lane;
-    const int tl = min(max(a.text_len[b], 0), a.N_t_max);
-    const bool rv = r < tl && a.mask[(size_t)b * a.N_t_max + r] != 0;
-    const float it = rv ? a.invt[(size_t)b * a.N_t_max + r] : 0.f;
-    const float m = rv ? a.mu[(size_t)b * a.N_t_max + r] : 0.f;
-    mbar_wait(&pipe.acc_full[0], 0, a.err);
+    const bool has_t = r < a.NT;
+    float v0 = 0.f, v1 = 0.f, t0 = 0.f, t1 = 0.f;
+    for (int kb = 0; kb < n_k; ++kb) {
+      const int s = kb % NS;
+      const uint32_t ph = (uint32_t)(kb / NS) & 1u;
+      if (pipe.fail || !mbar_wait(&pipe.full[s], ph, a.err)) {
+        pipe.fail = 1;
+        break;
+      }
+      // row r's 128 bytes, the 16-byte chunks taken in a per-row rotated order
+      // so that the eight rows of a swizzle atom hit distinct banks (the sum of
+      // squares does not depend on the chunk order)
+      const uint8_t* ra = stages + (size_t)s * st_bytes + r * 128;
+#pragma unroll
+      for (int c = 0; c < 8; ++c)
+        sumsq8(*reinterpret_cast<const uint4*>(ra + (((c + r) & 7) << 4)), v0, v1);
+      if (has_t) {
+        const uint8_t* rt = ra + kABytes;
+#pragma unroll
+        for (int c = 0; c < 8; ++c)
+          sumsq8(*reinterpret_cast<const uint4*>(rt + (((c + r) & 7) << 4)), t0, t1);
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&pipe.empty[s]);
+    }
+    const float sqt = t0 + t1, sqv = v0 + v1;
+    s_invt[r] = has_t && sqt > 0.f ? 1.f / sqrtf(sqt) : 0.f;
+    const float iv = sqv > 0.f ? 1.f / sqrtf(sqv) : 0.f;
+    const int j = n0 + r;
+    const bool rv = j < a.N_v;
+    asm volatile("bar.sync 1, 128;" ::: "memory");  // s_invt complete (epilogue warps)
+    const bool ok = mbar_wait(&pipe.acc_full, 0, a.err) && !pipe.fail;
     tc_fence_after();
+    if (rv && ok) a.inv_v[(size_t)b * a.N_v + j] = iv;
     const uint32_t taddr = pipe.tmem + ((uint32_t)(quad * 32) << 16);
+    float* yrow = a.Y + ((size_t)b * a.N_v + (rv ? j : 0)) * a.NT;
 #pragma unroll 1
-    for (int cb = 0; cb < kRelBN / 32; ++cb) {
+    for (int cb = 0; cb * 32 < a.NT; ++cb) {
       float v[32];
       tmem_ld32(taddr + cb * 32, v);
       tc_wait_ld();
 #pragma unroll
-      for (int i = 0; i < 32; ++i) {
-        const int j = n0 + cb * 32 + i;
-        const float iv = j < a.N_v ? a.inv_v[(size_t)b * a.N_v + j] : 0.f;
-        v[i] = rv ? v[i] * it * iv - m : -INFINITY;
+      for (int i = 0; i < 32; ++i) v[i] = v[i] * s_invt[cb * 32 + i] * iv;
+      if (rv && ok) {
+#pragma unroll
+        for (int q = 0; q < 8; ++q)
+          if (cb * 32 + q * 4 < a.NT)
+            *reinterpret_cast<float4*>(yrow + cb * 32 + q * 4) =
+                make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
       }
-      // butterfly max over the 32 rows of the warp: lane ends with column `lane`
+#pragma unroll
+      for (int i = 0; i < 32; ++i) v[i] = rv ? v[i] : 0.f;
+      // butterfly sum over the 32 rows of the warp: lane ends with column `lane`
 #pragma unroll
       for (int sh = 16; sh >= 1; sh >>= 1) {
         const bool upper = (lane & sh) != 0;
@@ -260,22 +363,52 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int i = 0; i < sh; ++i) {
           const float keep = upper ? v[i + sh] : v[i];
           const float send = upper ? v[i] : v[i + sh];
-          v[i] = fmaxf(keep, __shfl_xor_sync(0xffffffffu, send, sh));
+          v[i] = keep + __shfl_xor_sync(0xffffffffu, send, sh);
         }
       }
       red[quad][cb * 32 + lane] = v[0];
     }
     tc_fence_before();
-    // combine the four lane quadrants (epilogue warps only: named barrier)
     asm volatile("bar.sync 1, 128;" ::: "memory");
     const int c = threadIdx.x - 64;
-    const int j = n0 + c;
-    if (j < a.N_v && !pipe.fail)
-      a.p[(size_t)b * a.N_v + j] = fmaxf(fmaxf(red[0][c], red[1][c]), fmaxf(red[2][c], red[3][c]));
+    if (c < a.NT && ok)
+      a.part[((size_t)b * a.n_vt + tile) * a.NT + c] = (red[0][c] + red[1][c]) + (red[2][c] + red[3][c]);
   }
   tc_fence_before();
   __syncthreads();
-  if (threadIdx.x < 32) tmem_dealloc(pipe.tmem, Cfg<kRelBN>::kTmemCols);
+  if (threadIdx.x < 32) tmem_dealloc(pipe.tmem, tcols);
+}
+
+// mu_i from the tile sums (tile order), then p_j = max over the critical rows
+// of Y[b][j][i] - mu_i; an empty T gives -inf
+__global__ void __launch_bounds__(256) relevance_finish_kernel(const RelFusedArgs a, const int* text_len,
+                                                               const uint8_t* mask, float* p) {
+  __shared__ float mu[kBM];
+  __shared__ int valid[kBM];
+  const int b = blockIdx.y;
+  const int tl = min(max(text_len[b], 0), a.N_t_max);
+  for (int c = threadIdx.x; c < a.NT; c += blockDim.x) {
+    const bool v = c < tl && mask[(size_t)b * a.N_t_max + c] != 0;
+    float s = 0.f;
+    if (v)
+      for (int t = 0; t < a.n_vt; ++t) s += a.part[((size_t)b * a.n_vt + t) * a.NT + c];
+    mu[c] = s / (float)a.N_v;
+    valid[c] = v;
+  }
+  __syncthreads();
+  const int j = blockIdx.x * blockDim.x + threadIdx.x;
+  if (j >= a.N_v) return;
+  const float4* y = reinterpret_cast<const float4*>(a.Y + ((size_t)b * a.N_v + j) * a.NT);
+  float best = -INFINITY;
+  for (int q = 0; q < a.NT / 4; ++q) {
+    const float4 f = y[q];
+    const int c = q * 4;
+    if (valid[c]) best = fmaxf(best, f.x - mu[c]);
+    if (valid[c + 1]) best = fmaxf(best, f.y - mu[c + 1]);
+    if (valid[c + 2]) best = fmaxf(best, f.z - mu[c + 2]);
+    if (valid[c + 3]) best = fmaxf(best, f.w - mu[c + 3]);
+  }
+  p[(size_t)b * a.N_v + j] = best;
 }
 
 // G = E_t E_t^T for one sample (<= 128 text rows), split over K: CTA x of
@@ -416,32 +549,45 @@ cudaError_t merge_argmax_tc_launch(const SimArgs& a, const int* keep_idx, int ke
 
 bool relevance_tc_supported(const SimArgs& a) { return a.dtype == 1 && a.N_t_max <= kBM && a.D % 8 == 0; }
 
-cudaError_t relevance_tc_launch(const SimArgs& a, const uint8_t* mask, const float* inv_v,
-                                const float* mu, const float* invt, float* p, cudaStream_t s) {
+static int rel_nt(int N_t_max) { return (N_t_max + 15) / 16 * 16; }
+
+size_t relevance_fused_floats(int B, int N_v, int N_t_max) {
+  const int NT = rel_nt(N_t_max), n_vt = (N_v + kBM - 1) / kBM;
+  return (size_t)B * N_v * NT + (size_t)B * n_vt * NT;
+}
+
+cudaError_t relevance_tc_launch(const SimArgs& a, const uint8_t* mask, float* inv_v, float* p, float* ws,
+                                int num_sms, cudaStream_t s) {
   static bool smem_set[64] = {false};
   int dev = 0;
   cudaGetDevice(&dev);
-  const size_t smem = Cfg<kRelBN>::kStagesBytes + 1024;
-  cudaError_t e = set_smem(relevance_tc, smem, &smem_set[dev < 64 ? dev : 0]);
+  constexpr size_t kSmemMax = 200 * 1024;
+  cudaError_t e = set_smem(relevance_fused_tc, kSmemMax, &smem_set[dev < 64 ? dev : 0]);
   if (e != cudaSuccess) return e;
-  CUtensorMap mapT, mapV;
-  if (make_tmap_bf16_2d(&mapT, a.emb_t, (uint64_t)a.B * a.N_t_max, (uint64_t)a.D, (uint64_t)a.D * 2, 128) ||
-      make_tmap_bf16_2d(&mapV, a.emb_v, (uint64_t)a.B * a.N_v, (uint64_t)a.D, (uint64_t)a.D * 2, 128))
-    return cudaErrorInvalidValue;
-  RelTcArgs r;
+  RelFusedArgs r;
   r.B = a.B;
   r.N_v = a.N_v;
   r.D = a.D;
   r.N_t_max = a.N_t_max;
-  r.text_len = a.text_len;
-  r.mask = mask;
+  r.NT = rel_nt(a.N_t_max);
+  r.n_vt = (a.N_v + kBM - 1) / kBM;
   r.inv_v = inv_v;
-  r.mu = mu;
-  r.invt = invt;
-  r.p = p;
+  r.Y = ws;
+  r.part = ws + (size_t)a.B * a.N_v * r.NT;
   r.err = a.err;
-  dim3 grid((a.N_v + kRelBN - 1) / kRelBN, 1, a.B);
-  relevance_tc<<<grid, kThreads, smem, s>>>(r, mapT, mapV);
+  // one CTA per SM when the tiles do not fill the GPU (deeper ring), else two
+  const size_t st_bytes = (size_t)kABytes + (size_t)r.NT * 128;
+  const size_t budget = (long long)a.B * r.n_vt <= num_sms ? kSmemMax - 1024 : 110 * 1024 - 1024;
+  int ns = (int)(budget / st_bytes);
+  r.n_stages = ns > kRelMaxStages ? kRelMaxStages : (ns < 2 ? 2 : ns);
+  const size_t smem = (size_t)r.n_stages * st_bytes + 1024;
+  CUtensorMap mapV, mapT;
+  if (make_tmap_bf16_2d(&mapV, a.emb_v, (uint64_t)a.B * a.N_v, (uint64_t)a.D, (uint64_t)a.D * 2, kBM) ||
+      make_tmap_bf16_2d(&mapT, a.emb_t, (uint64_t)a.B * a.N_t_max, (uint64_t)a.D, (uint64_t)a.D * 2,
+                        (uint32_t)r.NT))
+    return cudaErrorInvalidValue;
+  relevance_fused_tc<<<dim3(r.n_vt, a.B), kThreads, smem, s>>>(r, mapV, mapT);
+  relevance_finish_kernel<<<dim3((a.N_v + 255) / 256, a.B), 256, 0, s>>>(r, a.text_len, mask, p);
   return cudaGetLastError();
 }
 

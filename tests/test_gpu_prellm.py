@@ -132,3 +132,17 @@ def test_merge_matches_oracle(name):
             mem = np.flatnonzero(a_gpu == a)
             expect = Ev[mem].mean(axis=0)
             np.testing.assert_allclose(mg[a], expect, rtol=8e-3, atol=1e-6)
+
+
+@pytest.mark.parametrize("name", [w.name for w in synth.WORKLOADS])
+def test_reduce_merge_agrees_with_the_merge_call(name):
+    """The merge inside provip_similarity_reduce takes its inverse norms from the
+    relevance kernel; the stand-alone merge computes its own. On the same kept
+    set both give the same centroids, apart from rows whose nearest kept row is
+    a near tie that the two fp32 norm orders may break differently."""
+    w, cpu, g = inputs(name)
+    res = P.provip_similarity_reduce(g["emb_v"], g["emb_t"], g["text_len"], w.keep_pre, want_merged=True)
+    _, merged = P.provip_merge(g["emb_v"], res["idx"])
+    torch.cuda.synchronize()
+    same = (res["merged"] == merged).all(dim=2).float().mean().item()
+    assert same >= 0.98, f"{name}: only {same:.3f} of the merged rows agree"
