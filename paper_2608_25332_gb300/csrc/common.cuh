@@ -83,6 +83,16 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, unsign
   }
 }
 
+// Lane 0 waits on the mbarrier for the whole warp (one poller instead of 32);
+// the warp barrier that follows orders the other lanes after it. Returns the
+// wait's result in every lane.
+__device__ __forceinline__ bool warp_mbar_wait(uint64_t* bar, uint32_t parity, unsigned* err) {
+  bool ok = true;
+  if ((threadIdx.x & 31) == 0) ok = mbar_wait(bar, parity, err);
+  __syncwarp();
+  return __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+}
+
 // ---------------------------------------------------------------------------
 // bulk (1-D) TMA copies
 // ---------------------------------------------------------------------------

@@ -190,9 +190,10 @@ cudaError_t crit_gram_tc_launch(const SimArgs& a, float* G, cudaStream_t s);
 bool relevance_tc_supported(const SimArgs& a);
 // workspace floats of the tensor-core relevance (cosines + per-tile sums)
 size_t relevance_fused_floats(int B, int N_v, int N_t_max);
-// writes inv_v and p; ws holds relevance_fused_floats(...) floats
-cudaError_t relevance_tc_launch(const SimArgs& a, const uint8_t* mask, float* inv_v, float* p, float* ws,
-                                int num_sms, cudaStream_t s);
+// reads the text rows' inverse norms inv_t [B][N_t_max]; writes inv_v and p;
+// ws holds relevance_fused_floats(...) floats
+cudaError_t relevance_tc_launch(const SimArgs& a, const uint8_t* mask, const float* inv_t, float* inv_v,
+                                float* p, float* ws, int num_sms, cudaStream_t s);
 bool merge_tc_supported(const SimArgs& a, int keep, int n_split);
 cudaError_t merge_argmax_tc_launch(const SimArgs& a, const int* keep_idx, int keep,
                                    const float* inv_v, const int* kpos, int* pruned, void* perm,

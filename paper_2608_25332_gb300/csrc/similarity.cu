@@ -818,9 +818,14 @@ cudaError_t vis_inv_norm_launch(const SimArgs& a, float* inv_v, cudaStream_t s) 
 cudaError_t relevance_launch(const SimArgs& a, const uint8_t* mask, float* inv_v, float* p,
                              float* ws_sum, float* ws_mu, float* ws_invt, int n_split,
                              int num_sms, cudaStream_t s) {
-  // bf16 with at most 128 text rows: one tensor-core read of the visual rows
-  // (norms, cosines and de-meaning sums) and a small max kernel
-  if (relevance_tc_supported(a)) return relevance_tc_launch(a, mask, inv_v, p, ws_sum, num_sms, s);
+  // bf16 with at most 128 text rows: the text rows' inverse norms, one
+  // tensor-core read of the visual rows (norms, cosines and de-meaning sums)
+  // and a small max kernel
+  if (relevance_tc_supported(a)) {
+    const size_t rows = (size_t)a.B * a.N_t_max;
+    inv_norm_kernel<__nv_bfloat16><<<(unsigned)((rows + 7) / 8), 256, 0, s>>>(a.emb_t, rows, a.D, ws_invt);
+    return relevance_tc_launch(a, mask, ws_invt, inv_v, p, ws_sum, num_sms, s);
+  }
   const int chunk = (a.N_v + n_split - 1) / n_split;
   dim3 g1((a.D + 255) / 256, a.B, n_split);
   dim3 g2((a.N_t_max + 7) / 8, a.B);

@@ -186,12 +186,12 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 // relevance_fused_tc: one read of the visual rows gives, per 128-row tile of
-// sample b,
-//   * |v_j|^-1 (from the shared-memory stages the MMA consumes: each epilogue
-//     thread sums the squares of its row's 64 elements per K slice) and
-//     |t_i|^-1 for the text rows (same, on the text stage),
-//   * the cosines Y[b][j][i] = <v_j, t_i> |t_i|^-1 |v_j|^-1 (A = the visual
-//     rows, B = the text rows; thread = TMEM lane = visual row j),
+// sample b (A = the 128 visual rows, B = [the same 128 visual rows ; the text
+// rows], both already adjacent in the stage, so one MMA of N = 128 + NT),
+//   * |v_j|^2 from the diagonal of the visual x visual block (thread = TMEM
+//     lane = visual row j reads its own column),
+//   * the cosines Y[b][j][i] = <v_j, t_i> |t_i|^-1 |v_j|^-1 (|t_i|^-1 from a
+//     separate pass over the text rows),
 //   * the tile's column sums part[b][tile][i] = sum_j Y[b][j][i] (warp
 //     butterfly, then the four lane quadrants in order).
 // relevance_finish_kernel then forms mu_i = (sum of the tile sums in tile
@@ -201,6 +201,7 @@ struct RelFusedArgs {
   int NT;        // text rows in the MMA (N_t_max rounded up to 16)
   int n_vt;      // 128-row visual tiles per sample
   int n_stages;  // shared-memory ring depth
+  const float* inv_t;  // [B][N_t_max]
   float* inv_v;  // [B][N_v]
   float* Y;      // [B][N_v][NT]
   float* part;   // [B][n_vt][NT]
@@ -208,6 +209,7 @@ struct RelFusedArgs {
 };
 
 constexpr int kRelMaxStages = 8;
+constexpr uint32_t kRelTmemCols = 256;  // 128 visual + <= 128 text columns
 
 struct RelPipe {
   uint64_t full[kRelMaxStages];
@@ -216,17 +218,6 @@ struct RelPipe {
   uint32_t tmem;
   volatile int fail;
 };
-
-// sum of squares of the 8 bf16 values of a 16-byte chunk, two chains
-__device__ __forceinline__ void sumsq8(const uint4 u, float& s0, float& s1) {
-  const uint32_t w[4] = {u.x, u.y, u.z, u.w};
-#pragma unroll
-  for (int q = 0; q < 4; ++q) {
-    const float lo = __uint_as_float(w[q] << 16), hi = __uint_as_float(w[q] & 0xffff0000u);
-    s0 = fmaf(lo, lo, s0);
-    s1 = fmaf(hi, hi, s1);
-  }
-}
 
 __global__ void __launch_bounds__(kThreads, 2)
     relevance_fused_tc(const RelFusedArgs a, const __grid_constant__ CUtensorMap mapV,
@@ -240,7 +231,6 @@ __global__ void __launch_bounds__(kThreads, 2)
   const int n_k = (a.D + kBK - 1) / kBK;
   const int NS = a.n_stages;
   const uint32_t st_bytes = (uint32_t)kABytes + (uint32_t)a.NT * 128u;
-  const uint32_t tcols = a.NT <= 32 ? 32u : (a.NT <= 64 ? 64u : 128u);
   const uint32_t sbase = smem_u32(smem_raw);
   uint8_t* stages = smem_raw + (((sbase + 1023u) & ~1023u) - sbase);
   if (threadIdx.x == 0) {
@@ -248,14 +238,14 @@ __global__ void __launch_bounds__(kThreads, 2)
     prefetch_tmap(&mapT);
     for (int s = 0; s < NS; ++s) {
       mbar_init(&pipe.full[s], 1);
-      mbar_init(&pipe.empty[s], 5);  // the MMA commit + one arrival per epilogue warp
+      mbar_init(&pipe.empty[s], 1);
     }
     mbar_init(&pipe.acc_full, 1);
     pipe.fail = 0;
     fence_mbar_init();
   }
   if (threadIdx.x < 32) {
-    tmem_alloc(&pipe.tmem, tcols);
+    tmem_alloc(&pipe.tmem, kRelTmemCols);
     tmem_relinquish();
   }
   tc_fence_before();
@@ -281,7 +271,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     }
   } else if (warp == 1) {
     if (lane == 0) {
-      const uint32_t idesc = idesc_bf16_f32(kBM, a.NT);
+      const uint32_t idesc = idesc_bf16_f32(kBM, kBM + a.NT);
       for (int kb = 0; kb < n_k; ++kb) {
         const int s = kb % NS;
         const uint32_t ph = (uint32_t)(kb / NS) & 1u;
@@ -291,10 +281,9 @@ __global__ void __launch_bounds__(kThreads, 2)
         }
         tc_fence_after();
         const uint32_t sa = smem_u32(stages + (size_t)s * st_bytes);
-        const uint32_t sb = sa + kABytes;
 #pragma unroll
         for (int k = 0; k < kBK / 16; ++k)
-          tc_mma_bf16(pipe.tmem, smem_desc_sw128(sa + k * 32), smem_desc_sw128(sb + k * 32), idesc,
+          tc_mma_bf16(pipe.tmem, smem_desc_sw128(sa + k * 32), smem_desc_sw128(sa + k * 32), idesc,
                       (kb > 0 || k > 0) ? 1u : 0u);
         tc_commit(&pipe.empty[s]);
       }
@@ -303,46 +292,26 @@ __global__ void __launch_bounds__(kThreads, 2)
   } else {
     const int quad = warp & 3;
     const int r = quad * 32 + lane;
-    const bool has_t = r < a.NT;
-    float v0 = 0.f, v1 = 0.f, t0 = 0.f, t1 = 0.f;
-    for (int kb = 0; kb < n_k; ++kb) {
-      const int s = kb % NS;
-      const uint32_t ph = (uint32_t)(kb / NS) & 1u;
-      if (pipe.fail || !mbar_wait(&pipe.full[s], ph, a.err)) {
-        pipe.fail = 1;
-        break;
-      }
-      // row r's 128 bytes, the 16-byte chunks taken in a per-row rotated order
-      // so that the eight rows of a swizzle atom hit distinct banks (the sum of
-      // squares does not depend on the chunk order)
-      const uint8_t* ra = stages + (size_t)s * st_bytes + r * 128;
-#pragma unroll
-      for (int c = 0; c < 8; ++c)
-        sumsq8(*reinterpret_cast<const uint4*>(ra + (((c + r) & 7) << 4)), v0, v1);
-      if (has_t) {
-        const uint8_t* rt = ra + kABytes;
-#pragma unroll
-        for (int c = 0; c < 8; ++c)
-          sumsq8(*reinterpret_cast<const uint4*>(rt + (((c + r) & 7) << 4)), t0, t1);
-      }
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&pipe.empty[s]);
-    }
-    const float sqt = t0 + t1, sqv = v0 + v1;
-    s_invt[r] = has_t && sqt > 0.f ? 1.f / sqrtf(sqt) : 0.f;
-    const float iv = sqv > 0.f ? 1.f / sqrtf(sqv) : 0.f;
     const int j = n0 + r;
     const bool rv = j < a.N_v;
+    s_invt[r] = r < a.N_t_max ? a.inv_t[(size_t)b * a.N_t_max + r] : 0.f;
     asm volatile("bar.sync 1, 128;" ::: "memory");  // s_invt complete (epilogue warps)
-    const bool ok = mbar_wait(&pipe.acc_full, 0, a.err) && !pipe.fail;
+    const bool ok = warp_mbar_wait(&pipe.acc_full, 0, a.err) && !pipe.fail;
     tc_fence_after();
-    if (rv && ok) a.inv_v[(size_t)b * a.N_v + j] = iv;
     const uint32_t taddr = pipe.tmem + ((uint32_t)(quad * 32) << 16);
+    float v[32];
+    // |v_j|^2: column j of the visual block, i.e. element `lane` of the warp's 32 columns
+    tmem_ld32(taddr + (uint32_t)(quad * 32), v);
+    tc_wait_ld();
+    float sqv = 0.f;
+#pragma unroll
+    for (int i = 0; i < 32; ++i) sqv = i == lane ? v[i] : sqv;
+    const float iv = sqv > 0.f ? 1.f / sqrtf(sqv) : 0.f;
+    if (rv && ok) a.inv_v[(size_t)b * a.N_v + j] = iv;
     float* yrow = a.Y + ((size_t)b * a.N_v + (rv ? j : 0)) * a.NT;
 #pragma unroll 1
     for (int cb = 0; cb * 32 < a.NT; ++cb) {
-      float v[32];
-      tmem_ld32(taddr + cb * 32, v);
+      tmem_ld32(taddr + (uint32_t)(kBM + cb * 32), v);
       tc_wait_ld();
 #pragma unroll
       for (int i = 0; i < 32; ++i) v[i] = v[i] * s_invt[cb * 32 + i] * iv;
@@ -376,11 +345,11 @@ __global__ void __launch_bounds__(kThreads, 2)
   }
   tc_fence_before();
   __syncthreads();
-  if (threadIdx.x < 32) tmem_dealloc(pipe.tmem, tcols);
+  if (threadIdx.x < 32) tmem_dealloc(pipe.tmem, kRelTmemCols);
 }
 
 // mu_i from the tile sums (tile order), then p_j = max over the critical rows
-// of Y[b][j][i] - mu_i; an empty T gives -inf
+// of Y[b][j][i] - mu_i; an empty T gives -inf. Loads go out eight at a time.
 __global__ void __launch_bounds__(256) relevance_finish_kernel(const RelFusedArgs a, const int* text_len,
                                                                const uint8_t* mask, float* p) {
   __shared__ float mu[kBM];
@@ -390,8 +359,17 @@ __global__ void __launch_bounds__(256) relevance_finish_kernel(const RelFusedArg
   for (int c = threadIdx.x; c < a.NT; c += blockDim.x) {
     const bool v = c < tl && mask[(size_t)b * a.N_t_max + c] != 0;
     float s = 0.f;
-    if (v)
-      for (int t = 0; t < a.n_vt; ++t) s += a.part[((size_t)b * a.n_vt + t) * a.NT + c];
+    if (v) {
+      const float* col = a.part + (size_t)b * a.n_vt * a.NT + c;
+      for (int t0 = 0; t0 < a.n_vt; t0 += 8) {
+        float x[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) x[u] = t0 + u < a.n_vt ? col[(size_t)(t0 + u) * a.NT] : 0.f;
+#pragma unroll
+        for (int u = 0; u < 8; ++u)
+          if (t0 + u < a.n_vt) s += x[u];
+      }
+    }
     mu[c] = s / (float)a.N_v;
     valid[c] = v;
   }
@@ -400,13 +378,20 @@ __global__ void __launch_bounds__(256) relevance_finish_kernel(const RelFusedArg
   if (j >= a.N_v) return;
   const float4* y = reinterpret_cast<const float4*>(a.Y + ((size_t)b * a.N_v + j) * a.NT);
   float best = -INFINITY;
-  for (int q = 0; q < a.NT / 4; ++q) {
-    const float4 f = y[q];
-    const int c = q * 4;
-    if (valid[c]) best = fmaxf(best, f.x - mu[c]);
-    if (valid[c + 1]) best = fmaxf(best, f.y - mu[c + 1]);
-    if (valid[c + 2]) best = fmaxf(best, f.z - mu[c + 2]);
-    if (valid[c + 3]) best = fmaxf(best, f.w - mu[c + 3]);
+  for (int q0 = 0; q0 < a.NT / 4; q0 += 8) {
+    float4 f[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u)
+      if (q0 + u < a.NT / 4) f[u] = y[q0 + u];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      if (q0 + u >= a.NT / 4) break;
+      const int c = (q0 + u) * 4;
+      if (valid[c]) best = fmaxf(best, f[u].x - mu[c]);
+      if (valid[c + 1]) best = fmaxf(best, f[u].y - mu[c + 1]);
+      if (valid[c + 2]) best = fmaxf(best, f[u].z - mu[c + 2]);
+      if (valid[c + 3]) best = fmaxf(best, f[u].w - mu[c + 3]);
+    }
   }
   p[(size_t)b * a.N_v + j] = best;
 }
@@ -556,8 +541,8 @@ size_t relevance_fused_floats(int B, int N_v, int N_t_max) {
   return (size_t)B * N_v * NT + (size_t)B * n_vt * NT;
 }
 
-cudaError_t relevance_tc_launch(const SimArgs& a, const uint8_t* mask, float* inv_v, float* p, float* ws,
-                                int num_sms, cudaStream_t s) {
+cudaError_t relevance_tc_launch(const SimArgs& a, const uint8_t* mask, const float* inv_t, float* inv_v,
+                                float* p, float* ws, int num_sms, cudaStream_t s) {
   static bool smem_set[64] = {false};
   int dev = 0;
   cudaGetDevice(&dev);
@@ -571,6 +556,7 @@ cudaError_t relevance_tc_launch(const SimArgs& a, const uint8_t* mask, float* in
   r.N_t_max = a.N_t_max;
   r.NT = rel_nt(a.N_t_max);
   r.n_vt = (a.N_v + kBM - 1) / kBM;
+  r.inv_t = inv_t;
   r.inv_v = inv_v;
   r.Y = ws;
   r.part = ws + (size_t)a.B * a.N_v * r.NT;
