@@ -198,7 +198,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     const uint32_t tbase = ctl.tmem + ((uint32_t)(quad * 32) << 16) + (uint32_t)(half * 64);
     const float sc = a.scale_log2;
     const int t_first = ts + rb * kTile;  // every row of the block sits at or after it
-    bool failed = !mbar_wait(&ctl.q_full, 0, a.err);
+    bool failed = !warp_mbar_wait(&ctl.q_full, 0, a.err);  // warp-uniform from here on
     {
       // rows of the query tile past the block's text rows may hold anything
       // (other samples, padding): zero them, so every logit is finite
@@ -217,7 +217,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     float cn = 0.f, cmean = 0.f, cm2 = 0.f;
     for (int it = 0; it < n_it; ++it) {
       const int buf = it & 1;
-      if (!failed) failed = !mbar_wait(&ctl.acc_full[buf], (uint32_t)(it >> 1) & 1u, a.err);
+      if (!failed) failed = !warp_mbar_wait(&ctl.acc_full[buf], (uint32_t)(it >> 1) & 1u, a.err);
       tc_fence_after();
       if (it == nA) {
         // the row's global (max, sum) from the two column halves
