@@ -1,0 +1,148 @@
+"""GPU parity on the degenerate and boundary cases of the method, against the
+oracle: the smallest and largest keep sizes (one kept token, nothing pruned),
+one text row (T falls back to every row), zero-norm and duplicated visual rows
+(cosine 0 by reading, exact cosine ties), row counts that leave ragged tiles,
+text padding that holds NaN (so any read of it shows), and both dtypes.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2608_25332_gb300 import provip as P
+from parity import assert_close_rel, check_mask_band, check_topk_band, rtol_for
+
+pytestmark = pytest.mark.gpu
+
+DEV = "cuda:0"
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    import __graft_entry__
+    __graft_entry__.build()
+    yield
+    rc, bits = P.provip_device_status(clear=True)
+    assert rc == 0 and bits == 0, f"device status {rc} {bits}"
+
+
+def _pre_case(seed, B, N_v, D, tls, dtype):
+    rng = np.random.default_rng(seed)
+    Ntm = max(tls)
+    Ev = rng.standard_normal((B, N_v, D)).astype(np.float32)
+    Ev[:, 3] = 0.0               # zero norm: cosine 0 against everything
+    Ev[:, 7] = Ev[:, 5]          # an exact duplicate: ties in every cosine
+    Ev[:, 11] *= 40.0            # scale does not change a cosine
+    Et = rng.standard_normal((B, Ntm, D)).astype(np.float32)
+    for b, t in enumerate(tls):
+        Et[b, t:] = np.nan       # padding past each sample's text rows
+    td = torch.bfloat16 if dtype == "bf16" else torch.float32
+    ev, et = torch.from_numpy(Ev).to(td), torch.from_numpy(Et).to(td)
+    return ev, et, np.array(tls, np.int32)
+
+
+def _ulp(x, dtype):
+    x = np.abs(x)
+    if dtype == "f32":
+        return np.spacing(x.astype(np.float32)).astype(np.float64)
+    return 2.0 ** (np.floor(np.log2(np.maximum(x, 1e-30))) - 7)
+
+
+@pytest.mark.parametrize("dtype,B,N_v,D,tls,keep_pre", [
+    ("bf16", 3, 37, 64, (1, 5, 17), 1),      # one kept token: every row merges into it
+    ("bf16", 3, 37, 64, (1, 5, 17), 36),     # one pruned token
+    ("bf16", 2, 37, 64, (3, 8), 37),         # nothing pruned: merged rows are the rows
+    ("bf16", 2, 300, 128, (128, 33), 100),   # 128 text rows (the tensor-core limit), tiles 128+128+44
+    ("bf16", 2, 200, 136, (129, 2), 50),     # 129 text rows: the CUDA-core relevance
+    ("f32", 2, 37, 64, (1, 9), 10),
+])
+def test_similarity_reduce_edge_cases(dtype, B, N_v, D, tls, keep_pre):
+    ev, et, tl = _pre_case(17, B, N_v, D, tls, dtype)
+    rt = rtol_for(dtype)
+    res = P.provip_similarity_reduce(ev.to(DEV), et.to(DEV), torch.from_numpy(tl).to(DEV), keep_pre,
+                                     want_merged=True)
+    torch.cuda.synchronize()
+    Evn = ev.float().numpy().astype(np.float64)
+    Etn = et.float().numpy().astype(np.float64)
+    full = 0
+    for b in range(B):
+        n = int(tl[b])
+        r_ref, T = oracle.crit_text(Etn[b, :n])
+        mask = res["mask"][b].cpu().numpy()
+        check_mask_band(mask[:n], r_ref, rt, f"T[{b}]")
+        assert not mask[n:].any()
+        if n == 1:
+            assert mask[0] == 1, "a single text row is critical"
+        if not np.array_equal(mask[:n].astype(bool), T.astype(bool)):
+            continue
+        p_ref = oracle.relevance(Etn[b, :n], T, Evn[b])
+        assert_close_rel(res["p"][b].cpu().numpy(), p_ref, 0.0, f"p[{b}]", atol=rt)
+        idx = res["idx"][b].cpu().numpy()
+        check_topk_band(idx, p_ref, keep_pre, rt, f"keep[{b}]")
+        if not np.array_equal(idx, oracle.topk(p_ref, keep_pre)):
+            continue
+        a_ref, mg_ref = oracle.merge(Evn[b], idx)
+        mg = res["merged"][b].float().cpu().numpy().astype(np.float64)
+        err = np.abs(mg - mg_ref)
+        rows_ok = np.all(err <= _ulp(mg_ref, dtype) * 1.0001 + 1e-37, axis=1)
+        if keep_pre == N_v:
+            # nothing merged: every output row is its input row, bit for bit
+            assert torch.equal(res["merged"][b].cpu(), ev[b][torch.from_numpy(idx).long()])
+        else:
+            # a near-tie between two kept rows may move a pruned row; all other
+            # centroids are the oracle's within one output ulp
+            assert rows_ok.mean() >= 0.9, f"merged[{b}]: {np.flatnonzero(~rows_ok)} beyond one ulp"
+        full += 1
+    assert full >= 1, "no sample reached the merge comparison"
+
+
+def _in_llm_case(seed, B, nsys, nv, tls, Hq=4, Hkv=2, D=256, P_=3):
+    rng = np.random.default_rng(seed)
+    Ntm = max(tls)
+    Lm = nsys + nv + Ntm
+    Q = rng.standard_normal((B, Lm, Hq, 128)).astype(np.float32)
+    K = rng.standard_normal((B, Lm, Hkv, 128)).astype(np.float32)
+    V = rng.standard_normal((B, Lm, Hkv, 128)).astype(np.float32)
+    H = rng.standard_normal((B, Lm, D)).astype(np.float32)
+    tl = np.array(tls, np.int32)
+    sl = (nsys + nv + tl).astype(np.int32)
+    for b in range(B):
+        Q[b, sl[b]:] = np.nan
+        K[b, sl[b]:] = np.nan
+    pos = rng.integers(0, 1 << 20, (P_, B, Lm)).astype(np.int32)
+    bf = lambda x: torch.from_numpy(x).to(torch.bfloat16)
+    return dict(Q=bf(Q), K=bf(K), V=bf(V), H=bf(H), pos=torch.from_numpy(pos), tl=tl, sl=sl,
+                ts=np.full(B, nsys + nv, np.int32), nsys=nsys, nv=nv, Ntm=Ntm)
+
+
+@pytest.mark.parametrize("keep", [1, 37])
+@pytest.mark.parametrize("algo", ["ALGO_AUTO", "ALGO_TCGEN05_STREAM", "ALGO_SIMT"])
+def test_prune_single_keep_and_identity(keep, algo):
+    """keep = 1 keeps the single best visual token; keep = N_v is the identity
+    gather (every row in place, the sequence unchanged)."""
+    c = _in_llm_case(23, B=3, nsys=5, nv=37, tls=(1, 9, 130))
+    heads = [0, 3]
+    g = {k: c[k].to(DEV) for k in ("Q", "K", "V", "H", "pos")}
+    ts, tl, sl = (torch.from_numpy(x).to(DEV) for x in (c["ts"], c["tl"], c["sl"]))
+    out = P.provip_prune(g["Q"], g["K"], g["V"], g["H"], g["pos"], heads, ts, tl, sl, c["nsys"], c["nv"], keep,
+                         algo=getattr(P, algo), N_t_max=c["Ntm"])
+    torch.cuda.synchronize()
+    Qn, Kn = c["Q"].float().numpy(), c["K"].float().numpy()
+    for b in range(3):
+        slb = int(c["sl"][b])
+        ref = oracle.head_scores(Qn[b, :slb], Kn[b, :slb], heads, np.arange(c["ts"][b], c["ts"][b] + c["tl"][b]),
+                                 c["nsys"], c["nv"])
+        assert_close_rel(out["scores"][b].cpu().numpy(), ref, 2e-3, f"scores[{b}]")
+        idx = out["idx"][b].cpu().numpy()
+        check_topk_band(idx, ref, keep, 2e-3, f"keep[{b}]")
+        if keep == c["nv"]:
+            assert idx.tolist() == list(range(c["nv"]))
+        n = int(out["seq_len"][b])
+        assert n == slb - c["nv"] + keep
+        src = oracle.compact_map(slb, c["nsys"], c["nv"], idx)
+        for key, src_t in (("hidden", c["H"]), ("K", c["K"]), ("V", c["V"])):
+            got = out[key][b, :n].cpu().view(torch.int16).numpy()
+            exp = oracle.gather_rows(src_t[b].view(torch.int16).numpy(), src)
+            np.testing.assert_array_equal(got, exp)
+        for p in range(c["pos"].shape[0]):
+            np.testing.assert_array_equal(out["pos"][p, b, :n].cpu().numpy(), c["pos"][p, b].numpy()[src])
