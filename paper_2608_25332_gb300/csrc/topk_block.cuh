@@ -177,21 +177,35 @@ __device__ __forceinline__ void topk_load_partials(const float* P0, int n_part, 
       }
     }
   } else {
-    // more rows: per column, groups of 8 loads in flight, added in row order
-    for (int i = tid; i < N; i += nth) {
-      float s = 0.f;
+    // more rows: 4 columns per thread, groups of 8 rows with the 32 loads of a
+    // group issued first, each column's sum taken in row order
+    for (int i0 = 0; i0 < N; i0 += 4 * nth) {
+      float s[4] = {0.f, 0.f, 0.f, 0.f};
       for (int u0 = 0; u0 < n_sum; u0 += 8) {
-        float t[8];
+        int ro[8];
 #pragma unroll
-        for (int u = 0; u < 8; ++u)
-          if (u0 + u < n_sum) t[u] = ld((size_t)row(u0 + u) * N + i);
+        for (int u = 0; u < 8; ++u) ro[u] = u0 + u < n_sum ? row(u0 + u) * N : 0;
+        float t[4][8];
 #pragma unroll
-        for (int u = 0; u < 8; ++u)
-          if (u0 + u < n_sum) s += t[u];
+        for (int c = 0; c < 4; ++c) {
+          const int i = i0 + c * nth + tid;
+#pragma unroll
+          for (int u = 0; u < 8; ++u) t[c][u] = (u0 + u < n_sum && i < N) ? ld((size_t)ro[u] + i) : 0.f;
+        }
+#pragma unroll
+        for (int c = 0; c < 4; ++c)
+#pragma unroll
+          for (int u = 0; u < 8; ++u)
+            if (u0 + u < n_sum) s[c] += t[c][u];
       }
-      const float v = zero ? 0.f : s / div;
-      if (scores_out) scores_out[i] = v;
-      keys[i] = float_key(v);
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        const int i = i0 + c * nth + tid;
+        if (i >= N) continue;
+        const float v = zero ? 0.f : s[c] / div;
+        if (scores_out) scores_out[i] = v;
+        keys[i] = float_key(v);
+      }
     }
   }
 }
