@@ -244,3 +244,36 @@ def test_compact_bit_exact(name):
         for p in range(w.P):
             np.testing.assert_array_equal(out["pos"][p, b, :n].cpu().numpy(),
                                           oracle.gather_rows(cpu["pos"][p, b].numpy(), src))
+
+
+@pytest.mark.parametrize("name,lanes", [("llava_next_7b_bf16_b8", 2), ("video_gqa_bf16_b1", 5)])
+def test_concurrent_lanes_match_serial_calls(name, lanes):
+    """The bench's multi-stream configuration: independent batches on their own
+    streams, each with its own outputs and workspace, several steps per lane,
+    running at the same time, give the bits of the same calls made serially."""
+    w = synth.BY_NAME[name]
+    batches = [{k: (v.to(DEV) if isinstance(v, torch.Tensor) else v)
+                for k, v in synth.in_llm_inputs(w, seed=w.seed + 31 * i).items()} for i in range(lanes)]
+    steps = [P.PruneStep(c["Q"], c["K"], c["V"], c["hidden"], c["pos"], c["head_list"], w.n_t[1], c["N_v"],
+                         c["keep"], algo=P.ALGO_TCGEN05_STREAM, flags=P.PRUNE_OVERLAP_PREVIOUS) for c in batches]
+
+    def call(i, stream=None):
+        c = batches[i]
+        return steps[i](c["Q"], c["K"], c["V"], c["hidden"], c["pos"], c["text_start"], c["text_len"],
+                        c["seq_len"], c["vis_start"], stream=stream)
+
+    serial = []
+    for i in range(lanes):
+        o = call(i)
+        torch.cuda.synchronize()
+        serial.append({k: v.clone() for k, v in o.items() if v is not None})
+    streams = [torch.cuda.Stream(device=DEV) for _ in range(lanes)]
+    for rep in range(4):
+        for i in range(lanes):
+            call(i, streams[i])
+    torch.cuda.synchronize()
+    for i in range(lanes):
+        for k, v in serial[i].items():
+            got = getattr(steps[i], {"hidden": "hidden_out", "K": "K_out", "V": "V_out", "pos": "pos_out",
+                                     "idx": "idx", "seq_len": "seq_len_out", "scores": "scores"}[k])
+            assert torch.equal(got, v), f"{name} lane {i}: {k} differs under concurrency"
