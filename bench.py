@@ -354,7 +354,7 @@ def workload_config(w, algo="auto", copies=N_COPIES, input_mb=None):
             "H_q": w.H_q, "H_kv": w.H_kv, "H_sel": w.H_sel, "D": w.D, "algo": algo,
             "l2": f"inputs larger than L2: {copies} rotating device copies of "
                   f"{input_mb if input_mb is not None else 286:.0f} MB",
-            "timing": f"CUDA graphs of {GRAPH_CHUNK} steps, events on the launching stream",
+            "timing": f"CUDA graphs of {GRAPH_CHUNK} steps per stream, events on the launching stream",
             "overlap": "independent batches: each step's head scores may start under the previous "
                        "step's compaction (PROVIP_PRUNE_OVERLAP_PREVIOUS)"}
 
@@ -550,8 +550,12 @@ def run_gb300(args, dist):
     # fill the GPU with one dependent chain): stream s takes steps s, s + S, ...
     # on its own input copies and its own outputs and workspace; lane 0 is the
     # step and copies above.
-    if S < 1 or GRAPH_CHUNK % S or args.steps % S:
-        raise SystemExit(f"--streams {S} must divide --steps and {GRAPH_CHUNK}")
+    if S < 1 or args.steps % S:
+        raise SystemExit(f"--streams {S} must divide --steps")
+    # graphs of GRAPH_CHUNK steps per stream: with many short single-sample
+    # chains, a small graph would spend a visible part of its time filling and
+    # draining the streams
+    chunk = GRAPH_CHUNK * S
     lanes = [(copies, step)]
     for s_ in range(1, S):
         cpu_s = synth.in_llm_inputs(w, seed=w.seed + 1000 * dist.rank + 7 * s_)
@@ -597,12 +601,12 @@ def run_gb300(args, dist):
     if rc != 0:
         raise RuntimeError(f"device status {rc} {bits} after warm-up")
 
-    # graphs of up to GRAPH_CHUNK steps (the step index picks the input copy)
+    # graphs of up to `chunk` steps (the step index picks the input copy)
     K = args.steps
     sizes = []
     left = K
     while left > 0:
-        n = min(GRAPH_CHUNK, left)
+        n = min(chunk, left)
         sizes.append(n)
         left -= n
     graphs = {}
@@ -612,6 +616,12 @@ def run_gb300(args, dist):
         with torch.cuda.graph(g, stream=stream):
             run_steps(n)
         graphs[n] = g
+    torch.cuda.synchronize()
+    # one untimed replay of each graph: the first launch of a freshly captured
+    # graph (upload, cold instruction and address-translation caches) runs
+    # slower than the ones after it
+    for g in graphs.values():
+        g.replay()
     torch.cuda.synchronize()
 
     sampler = ClockSampler(visible_device_index(dist.local_rank) if dist.rank == 0 else None)
@@ -663,6 +673,8 @@ def run_gb300(args, dist):
         with torch.cuda.graph(g, stream=stream):
             for i in range(GRAPH_CHUNK):
                 fn(i)
+        torch.cuda.synchronize()
+        g.replay()  # untimed first launch
         torch.cuda.synchronize()
         a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         a.record()
