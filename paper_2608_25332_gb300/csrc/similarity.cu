@@ -568,17 +568,23 @@ __global__ void merge_assign_kernel(const SimArgs a, const int* kpos, int n_spli
 // exclusive offsets, unordered fill. One CTA per kept row orders its members
 // by rank (ascending row index, so the sum order is fixed), fetches the member
 // rows with bulk copies (cp.async.bulk, one thread issuing) into a ring of
-// shared-memory row slots, kMeanSlots rows per batch, and sums them slot by
-// slot in rank order, each thread over its 16-byte pieces of the row. A
-// centroid with more members than the sort buffer takes them from a scan of
-// assign in windows (ascending by construction).
-constexpr int kMeanThreads = 256;
-constexpr int kMeanWarps = kMeanThreads / 32;
-constexpr int kMeanSort = 1024;
-constexpr int kMeanSlots = 4;
-// 16-byte pieces per thread: D <= 8192 elements
-template <typename T> constexpr int mean_pieces() { return 8192 * (int)sizeof(T) / 16 / kMeanThreads; }
-size_t merge_mean_smem(int D, int esize) { return (size_t)kMeanSlots * D * esize; }
+// shared-memory row slots, SLOTS rows per batch, and sums them slot by slot in
+// rank order, each thread over its 16-byte pieces of the row. A centroid with
+// more members than the sort buffer takes them from a scan of assign in
+// windows (ascending by construction). Each CTA is a short chain of dependent
+// steps, so the configuration is chosen for CTAs resident per SM: rows of at
+// most 8 KiB take 128 threads with 4 pieces each (8 CTAs per SM), longer rows
+// 256 threads (up to 8192 elements).
+template <int THR, int PIECES, int SLOTS, int SORT, int MINB>
+struct MeanCfg {
+  static constexpr int kThreads = THR, kWarps = THR / 32, kPieces = PIECES, kSlots = SLOTS, kSort = SORT,
+                       kMinBlocks = MINB;
+};
+using MeanSmall = MeanCfg<128, 4, 3, 256, 8>;       // row bytes <= 128 * 4 * 16
+using MeanBf16 = MeanCfg<256, 4, 4, 1024, 4>;       // bf16 rows <= 8192 elements
+using MeanF32 = MeanCfg<256, 8, 4, 1024, 2>;        // fp32 rows <= 8192 elements
+constexpr int kMeanSmallRowBytes = 128 * 4 * 16;
+template <typename C> size_t merge_mean_smem(int row_bytes) { return (size_t)C::kSlots * row_bytes; }
 
 __global__ void merge_count_kernel(const int* assign, int B, int N_v, int keep, int* count) {
   const size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
@@ -668,18 +674,19 @@ __device__ __forceinline__ void store16(float* p, const double* v) {
   *reinterpret_cast<float4*>(p) = make_float4((float)v[0], (float)v[1], (float)v[2], (float)v[3]);
 }
 
-template <typename T, typename Acc>
-__global__ void __launch_bounds__(kMeanThreads, sizeof(T) == 2 ? 4 : 2) merge_mean_kernel(const SimArgs a, const int* assign,
-                                                                  const int* count, const int* offset,
-                                                                  const int* members_all, int keep,
-                                                                  void* merged) {
+template <typename T, typename Acc, typename C>
+__global__ void __launch_bounds__(C::kThreads, C::kMinBlocks)
+    merge_mean_kernel(const SimArgs a, const int* assign, const int* count, const int* offset,
+                      const int* members_all, int keep, void* merged) {
+  constexpr int kMeanThreads = C::kThreads, kMeanWarps = C::kWarps, kMeanSort = C::kSort,
+                kMeanSlots = C::kSlots;
   extern __shared__ __align__(128) uint8_t slots[];  // kMeanSlots rows
   __shared__ int members[kMeanSort];
   __shared__ int unsorted[kMeanSort];
   __shared__ __align__(8) uint64_t bar;
   __shared__ int wcount[kMeanWarps];
   constexpr int kVec = 16 / (int)sizeof(T);  // elements per 16-byte piece
-  constexpr int kPieces = mean_pieces<T>();
+  constexpr int kPieces = C::kPieces;
   const int ap = blockIdx.x, b = blockIdx.y;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const T* E = static_cast<const T*>(a.emb_v) + (size_t)b * a.N_v * a.D;
@@ -915,21 +922,33 @@ cudaError_t merge_launch(const SimArgs& a, const int* keep_idx, int keep, const 
     int dev = 0;
     cudaGetDevice(&dev);
     if (dev >= 0 && dev < 64 && !configured[dev]) {
-      cudaError_t e = cudaFuncSetAttribute(merge_mean_kernel<float, double>,
+      cudaError_t e = cudaFuncSetAttribute(merge_mean_kernel<float, double, MeanF32>,
                                            cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                           (int)merge_mean_smem(8192, 4));
+                                           (int)merge_mean_smem<MeanF32>(8192 * 4));
       if (e == cudaSuccess)
-        e = cudaFuncSetAttribute(merge_mean_kernel<__nv_bfloat16, float>,
-                                 cudaFuncAttributeMaxDynamicSharedMemorySize, (int)merge_mean_smem(8192, 2));
+        e = cudaFuncSetAttribute(merge_mean_kernel<__nv_bfloat16, float, MeanBf16>,
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)merge_mean_smem<MeanBf16>(8192 * 2));
       if (e != cudaSuccess) return e;
       configured[dev] = true;
     }
-    const size_t smem = merge_mean_smem(a.D, a.dtype == 0 ? 4 : 2);
-    if (a.dtype == 0)
-      merge_mean_kernel<float, double><<<gm, kMeanThreads, smem, s>>>(a, assign, cnt, off, mem, keep, merged);
-    else
-      merge_mean_kernel<__nv_bfloat16, float><<<gm, kMeanThreads, smem, s>>>(a, assign, cnt, off, mem, keep,
-                                                                             merged);
+    const int row_bytes = a.D * (a.dtype == 0 ? 4 : 2);
+    if (row_bytes <= kMeanSmallRowBytes) {
+      const size_t smem = merge_mean_smem<MeanSmall>(row_bytes);
+      if (a.dtype == 0)
+        merge_mean_kernel<float, double, MeanSmall><<<gm, MeanSmall::kThreads, smem, s>>>(a, assign, cnt, off, mem,
+                                                                                        keep, merged);
+      else
+        merge_mean_kernel<__nv_bfloat16, float, MeanSmall><<<gm, MeanSmall::kThreads, smem, s>>>(
+            a, assign, cnt, off, mem, keep, merged);
+    } else if (a.dtype == 0) {
+      merge_mean_kernel<float, double, MeanF32><<<gm, MeanF32::kThreads, merge_mean_smem<MeanF32>(row_bytes), s>>>(
+          a, assign, cnt, off, mem, keep, merged);
+    } else {
+      merge_mean_kernel<__nv_bfloat16, float, MeanBf16>
+          <<<gm, MeanBf16::kThreads, merge_mean_smem<MeanBf16>(row_bytes), s>>>(a, assign, cnt, off, mem, keep,
+                                                                              merged);
+    }
   }
   return cudaGetLastError();
 }
