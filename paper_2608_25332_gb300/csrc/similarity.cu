@@ -698,7 +698,9 @@ __global__ void __launch_bounds__(C::kThreads, C::kMinBlocks)
   for (int k = 0; k < kPieces; ++k)
 #pragma unroll
     for (int e = 0; e < kVec; ++e) acc[k][e] = Acc(0);
+  // count and offset issued together: the member list depends on both
   const int n_all = count[(size_t)b * keep + ap];
+  const int off0 = offset[(size_t)b * keep + ap];
   if (threadIdx.x == 0) {
     mbar_init(&bar, 1);
     fence_mbar_init();
@@ -731,7 +733,7 @@ __global__ void __launch_bounds__(C::kThreads, C::kMinBlocks)
     }
   };
   if (n_all <= kMeanSort) {
-    const int* src = members_all + (size_t)b * a.N_v + offset[(size_t)b * keep + ap];
+    const int* src = members_all + (size_t)b * a.N_v + off0;
     for (int m = threadIdx.x; m < n_all; m += kMeanThreads) unsorted[m] = src[m];
     __syncthreads();
     // rank = number of smaller row indices (they are distinct)

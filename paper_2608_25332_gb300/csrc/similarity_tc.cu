@@ -65,7 +65,16 @@ __global__ void __launch_bounds__(256) gather_perm_kernel(const __nv_bfloat16* E
   const uint4* src = reinterpret_cast<const uint4*>(E + ((size_t)b * N_v + j) * D);
   uint4* dst = reinterpret_cast<uint4*>(perm + ((size_t)b * N_v + r) * D);
   const int nvec = D / 8;
-  for (int v = lane; v < nvec; v += 32) dst[v] = __ldg(src + v);
+  // four 16-byte loads in flight per lane before their stores
+  int v = lane;
+  for (; v + 96 < nvec; v += 128) {
+    const uint4 x0 = __ldg(src + v), x1 = __ldg(src + v + 32), x2 = __ldg(src + v + 64), x3 = __ldg(src + v + 96);
+    dst[v] = x0;
+    dst[v + 32] = x1;
+    dst[v + 64] = x2;
+    dst[v + 96] = x3;
+  }
+  for (; v < nvec; v += 32) dst[v] = __ldg(src + v);
 }
 
 struct MergeTcArgs {
