@@ -790,7 +790,12 @@ extern "C" int provip_prune(const void* Q, const void* K, const void* V, const v
   CompactArgs ca = compact_args(idx_out, B, N_v, keep, hidden, D, K, V, H_kv, d_h, pos, P, seq_len,
                                 L_max, vis_start, dtype, hidden_out, K_out, V_out, pos_out,
                                 seq_len_out, d->status);
-  cudaError_t e = compact_launch(ca, d->sms, static_cast<cudaStream_t>(stream), true);
+  // the next step's head scores overlap this compaction: the deeper ring only
+  // beside the streaming form
+  const int form = tc_form(resolve_algo(algo, dtype), B, H_sel, hs_shape(L_max, N_t_max, N_v, algo).n_rb,
+                           d->sms);
+  cudaError_t e = compact_launch(ca, d->sms, static_cast<cudaStream_t>(stream), true,
+                                 form == PROVIP_ALGO_TCGEN05_STREAM);
   return e == cudaSuccess ? PROVIP_OK : cuda_fail(e, "prune compact");
 }
 
@@ -919,7 +924,11 @@ extern "C" int provip_prune_visual_heads(
   CompactArgs ca = compact_args(idx_out, B, N_v, keep, hidden, D, K, V, H_kv, d_h, pos, P, seq_len,
                                 L_max, vis_start, dtype, hidden_out, K_out, V_out, pos_out,
                                 seq_len_out, d->status);
-  cudaError_t e = compact_launch(ca, d->sms, static_cast<cudaStream_t>(stream), true);
+  // every head is scored: the streaming form unless the units are fewer than the SMs
+  const int form = tc_form(resolve_algo(algo, dtype), B, H_q, hs_shape(L_max, N_t_max, N_v, algo).n_rb,
+                           d->sms);
+  cudaError_t e = compact_launch(ca, d->sms, static_cast<cudaStream_t>(stream), true,
+                                 form == PROVIP_ALGO_TCGEN05_STREAM);
   return e == cudaSuccess ? PROVIP_OK : cuda_fail(e, "prune_visual_heads compact");
 }
 

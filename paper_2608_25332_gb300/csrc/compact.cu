@@ -14,7 +14,8 @@
 // (global -> shared, completion on the slot's mbarrier) and, once it lands, a
 // cp.async.bulk store (shared -> global, bulk group). A slot is refilled as soon
 // as the store that drained it has finished reading, so up to kSlots - 1 loads
-// and a store are in flight per CTA. The other warps copy the position ids and,
+// and a store are in flight per CTA (kSlots = 5, or 6 when the rows fill every
+// CTA slot of the GPU and the caller allows it). The other warps copy the position ids and,
 // with 16-byte vector loads and stores (a warp per row), the rows of tensors
 // whose rows are at most 2 KiB (the K/V rows of a GQA layer with few key/value
 // heads), which per-row bulk copies would move inefficiently.
@@ -29,6 +30,9 @@ namespace {
 #ifndef PROVIP_COMPACT_SLOTS
 #define PROVIP_COMPACT_SLOTS 5
 #endif
+#ifndef PROVIP_COMPACT_DEEP_SLOTS
+#define PROVIP_COMPACT_DEEP_SLOTS 6
+#endif
 #ifndef PROVIP_COMPACT_CTAS_PER_SM
 #define PROVIP_COMPACT_CTAS_PER_SM 2
 #endif
@@ -36,10 +40,15 @@ namespace {
 #define PROVIP_COMPACT_SLOT_BYTES 8192
 #endif
 constexpr int kSlotBytes = PROVIP_COMPACT_SLOT_BYTES;
-constexpr int kSlots = PROVIP_COMPACT_SLOTS;          // ring of shared-memory slots per CTA
+// ring of shared-memory slots per CTA: the short ring when the compaction does
+// not fill every CTA slot of the GPU (small batches, many of them running side
+// by side) or when the caller's previous kernel needs room beside it; the deep
+// one otherwise (more bytes in flight per CTA; two such CTAs and a streaming
+// head-score CTA of the next step still fit an SM's shared memory)
+constexpr int kSlotsShort = PROVIP_COMPACT_SLOTS;
+constexpr int kSlotsDeep = PROVIP_COMPACT_DEEP_SLOTS;
 constexpr int kCtasPerSm = PROVIP_COMPACT_CTAS_PER_SM;
 constexpr int kCompactThreads = 128;
-constexpr size_t kCompactSmem = (size_t)kSlots * kSlotBytes;
 #ifndef PROVIP_COMPACT_MIN_CTA_KIB
 #define PROVIP_COMPACT_MIN_CTA_KIB 160
 #endif
@@ -88,6 +97,7 @@ __device__ __forceinline__ void phase_row(const CompactArgs& a, int phase, long 
   }
 }
 
+template <int kSlots>
 __global__ void __launch_bounds__(kCompactThreads) compact_kernel(const CompactArgs a, int np0,
                                                                    int np1, int np2, int small) {
   extern __shared__ __align__(128) uint8_t slots[];
@@ -246,13 +256,17 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(const CompactA
 
 }  // namespace
 
-cudaError_t compact_launch(const CompactArgs& a, int num_sms, cudaStream_t s, bool pdl) {
+cudaError_t compact_launch(const CompactArgs& a, int num_sms, cudaStream_t s, bool pdl, bool allow_deep) {
   static bool configured[64] = {false};
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev >= 0 && dev < 64 && !configured[dev]) {
-    cudaError_t e = cudaFuncSetAttribute(compact_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)kCompactSmem);
+    cudaError_t e = cudaFuncSetAttribute(compact_kernel<kSlotsShort>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)((size_t)kSlotsShort * kSlotBytes));
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(compact_kernel<kSlotsDeep>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               (int)((size_t)kSlotsDeep * kSlotBytes));
     if (e != cudaSuccess) return e;
     configured[dev] = true;
   }
@@ -271,19 +285,21 @@ cudaError_t compact_launch(const CompactArgs& a, int num_sms, cudaStream_t s, bo
   // pipeline fills (and kernels running beside it keep the SMs it does not need)
   const long long row_sum = a.row_bytes[0] + a.row_bytes[1] + a.row_bytes[2];
   const long long by_bytes = ((long long)a.B * a.L_out * row_sum + kMinCtaBytes - 1) / kMinCtaBytes;
+  const bool deep = allow_deep && by_bytes >= grid;  // the rows fill every CTA slot
   if (grid > by_bytes) grid = by_bytes;
   if (grid > total) grid = total > 0 ? total : 1;
   cudaLaunchConfig_t cfg = {};
   cudaLaunchAttribute attr[1];
   cfg.gridDim = dim3((unsigned)grid);
   cfg.blockDim = dim3(kCompactThreads);
-  cfg.dynamicSmemBytes = kCompactSmem;
+  cfg.dynamicSmemBytes = (size_t)(deep ? kSlotsDeep : kSlotsShort) * kSlotBytes;
   cfg.stream = s;
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = pdl ? 1 : 0;
-  return cudaLaunchKernelEx(&cfg, compact_kernel, a, np[0], np[1], np[2], small);
+  return deep ? cudaLaunchKernelEx(&cfg, compact_kernel<kSlotsDeep>, a, np[0], np[1], np[2], small)
+              : cudaLaunchKernelEx(&cfg, compact_kernel<kSlotsShort>, a, np[0], np[1], np[2], small);
 }
 
 }  // namespace provip

@@ -146,7 +146,10 @@ struct CompactArgs {
 };
 // pdl: launched as a programmatic dependent of the previous kernel on the
 // stream; rows that do not depend on idx are copied before waiting for it.
-cudaError_t compact_launch(const CompactArgs& a, int num_sms, cudaStream_t s, bool pdl = false);
+// allow_deep: the deeper slot ring may be used (it leaves room for a streaming
+// head-score CTA per SM, not for the cluster form's larger one)
+cudaError_t compact_launch(const CompactArgs& a, int num_sms, cudaStream_t s, bool pdl = false,
+                           bool allow_deep = true);
 
 // ---------------------------------------------------------------------------
 // pre-LLM similarity pass (Sec. 4.2-4.3)
