@@ -166,7 +166,7 @@ def prellm_measure(w, dev, reps=20):
     n_T = first["mask"].sum(dim=1).double().cpu()  # |T| per sample
     assign_only = lambda: P.provip_merge(g["emb_v"], idx, want_merged=False)
 
-    def t(f):
+    def t_eager(f):
         for _ in range(3):
             f()
         torch.cuda.synchronize()
@@ -178,7 +178,27 @@ def prellm_measure(w, dev, reps=20):
         torch.cuda.synchronize()
         return a.elapsed_time(b) / reps * 1e3
 
+    def t(f):
+        # device time: reps calls in one CUDA graph, replayed once untimed, then timed
+        for _ in range(3):
+            f()
+        torch.cuda.synchronize()
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=torch.cuda.Stream(device=dev)):
+            for _ in range(reps):
+                f()
+        graph.replay()
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        for _ in range(3):
+            graph.replay()
+        b.record()
+        torch.cuda.synchronize()
+        return a.elapsed_time(b) / (3 * reps) * 1e3
+
     us_full, us_assign = t(full), t(assign_only)
+    us_eager = t_eager(full)
     flops = 2.0 * w.D * (w.N_v - w.keep_pre) * w.keep_pre * w.B
     peak, src = bf16_peak()
     ach = flops / us_assign / 1e6
@@ -188,6 +208,9 @@ def prellm_measure(w, dev, reps=20):
     k1_peak, k1_src = bf16_peak(sustained=True)
     k1_ach = k1_flops / us_full / 1e6
     return {"workload": w.name, "us_per_call": us_full, "samples_per_s": w.B / us_full * 1e6,
+            "timing": "CUDA graphs of the calls (device time); us_per_call_eager: the same calls "
+                      "launched one by one from Python",
+            "us_per_call_eager": us_eager,
             "k1": {"flops": k1_flops, "achieved": k1_ach, "peak": k1_peak, "peak_source": k1_src,
                    "unit": "TFLOP/s", "frac": k1_ach / k1_peak,
                    "note": "the whole pass (text Gram, relevance, top-k, gather, merge Gram, "
