@@ -74,16 +74,22 @@ __global__ void __launch_bounds__(256) crit_parts_sum_kernel(float* G, size_t n,
 }
 
 // G: the sample Grams [B][Ntm][Ntm]. Up to kFinishSmemNt text rows the sample's
-// Gram is staged in shared memory.
+// Gram is staged in shared memory. One CTA of 1024 threads per sample: a warp
+// per row for the softmax statistics, then the column sums of the softmax in
+// kFinishThreads / n row groups whose partial sums are added in group order.
 constexpr int kFinishSmemNt = 128;
-__global__ void __launch_bounds__(256) crit_finish_kernel(const SimArgs a, const float* G,
-                                                          uint8_t* mask, float* r_out) {
-  extern __shared__ float sh[];  // rowm[Ntm], rowinv[Ntm], r[Ntm] (+ G[Ntm][Ntm] when staged)
+constexpr int kFinishThreads = 1024;
+__global__ void __launch_bounds__(kFinishThreads) crit_finish_kernel(const SimArgs a, const float* G,
+                                                                     uint8_t* mask, float* r_out) {
+  // rowm[Ntm], rowinv[Ntm], r[Ntm], part[kFinishThreads] (+ G[Ntm][Ntm] when staged)
+  extern __shared__ float sh[];
   float* rowm = sh;
   float* rowinv = sh + a.N_t_max;
   float* rr = sh + 2 * a.N_t_max;
-  __shared__ float wsum[8];
-  __shared__ int wcnt[8];
+  float* part = sh + 3 * a.N_t_max;
+  __shared__ float wsum[kFinishThreads / 32];
+  __shared__ int wcnt[kFinishThreads / 32];
+  constexpr int kWarps = kFinishThreads / 32;
   const int b = blockIdx.x;
   int n = a.text_len[b];
   if (n < 0 || n > a.N_t_max) {
@@ -92,7 +98,7 @@ __global__ void __launch_bounds__(256) crit_finish_kernel(const SimArgs a, const
   }
   const float* Gb = G + (size_t)b * a.N_t_max * a.N_t_max;
   const bool staged = a.N_t_max <= kFinishSmemNt;
-  float* Gs = sh + 3 * a.N_t_max;
+  float* Gs = part + kFinishThreads;
   int ld = a.N_t_max;
   if (staged) {
     // eight loads in flight per thread
@@ -114,7 +120,7 @@ __global__ void __launch_bounds__(256) crit_finish_kernel(const SimArgs a, const
     ld = n;
   }
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  for (int i = warp; i < n; i += 8) {
+  for (int i = warp; i < n; i += kWarps) {
     float m = -INFINITY;
     for (int j = lane; j < n; j += 32) m = fmaxf(m, Gb[(size_t)i * ld + j]);
     m = warp_max(m);
@@ -127,20 +133,37 @@ __global__ void __launch_bounds__(256) crit_finish_kernel(const SimArgs a, const
     }
   }
   __syncthreads();
-  for (int j = threadIdx.x; j < n; j += blockDim.x) {
-    float s = 0.f;
-    for (int i = 0; i < n; ++i) s += expf(Gb[(size_t)i * ld + j] - rowm[i]) * rowinv[i];
-    rr[j] = s / (float)n;
+  if (n > 0 && n <= kFinishThreads) {
+    // column j of row group g: rows g, g + groups, ... (in order)
+    const int groups = kFinishThreads / n;
+    const int g = threadIdx.x / n, j = threadIdx.x - g * n;
+    if (g < groups) {
+      float s = 0.f;
+      for (int i = g; i < n; i += groups) s += expf(Gb[(size_t)i * ld + j] - rowm[i]) * rowinv[i];
+      part[g * n + j] = s;
+    }
+    __syncthreads();
+    for (int jj = threadIdx.x; jj < n; jj += blockDim.x) {
+      float s = 0.f;
+      for (int g2 = 0; g2 < groups; ++g2) s += part[g2 * n + jj];
+      rr[jj] = s / (float)n;
+    }
+  } else {
+    for (int j = threadIdx.x; j < n; j += blockDim.x) {
+      float s = 0.f;
+      for (int i = 0; i < n; ++i) s += expf(Gb[(size_t)i * ld + j] - rowm[i]) * rowinv[i];
+      rr[j] = s / (float)n;
+    }
   }
   __syncthreads();
   // mean(r), fixed-order block sum
-  float part = 0.f;
-  for (int j = threadIdx.x; j < n; j += blockDim.x) part += rr[j];
-  part = warp_sum(part);
-  if (lane == 0) wsum[warp] = part;
+  float pt = 0.f;
+  for (int j = threadIdx.x; j < n; j += blockDim.x) pt += rr[j];
+  pt = warp_sum(pt);
+  if (lane == 0) wsum[warp] = pt;
   __syncthreads();
   float tot = 0.f;
-  for (int w = 0; w < 8; ++w) tot += wsum[w];
+  for (int w = 0; w < kWarps; ++w) tot += wsum[w];
   const float mean = n > 0 ? tot / (float)n : 0.f;
   int c = 0;
   for (int j = threadIdx.x; j < n; j += blockDim.x) c += rr[j] > mean;
@@ -148,7 +171,7 @@ __global__ void __launch_bounds__(256) crit_finish_kernel(const SimArgs a, const
   if (lane == 0) wcnt[warp] = c;
   __syncthreads();
   int cnt = 0;
-  for (int w = 0; w < 8; ++w) cnt += wcnt[w];
+  for (int w = 0; w < kWarps; ++w) cnt += wcnt[w];
   for (int j = threadIdx.x; j < a.N_t_max; j += blockDim.x) {
     const bool in = j < n && (cnt == 0 || rr[j] > mean);
     mask[(size_t)b * a.N_t_max + j] = in ? 1 : 0;
@@ -802,15 +825,17 @@ cudaError_t crit_text_launch(const SimArgs& a, uint8_t* mask, float* r_out, floa
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev >= 0 && dev < 64 && !configured[dev]) {
-    const int lim = (3 * kFinishSmemNt + kFinishSmemNt * kFinishSmemNt) * (int)sizeof(float);
+    const int lim = (3 * kFinishSmemNt + kFinishThreads + kFinishSmemNt * kFinishSmemNt) * (int)sizeof(float);
     cudaError_t e = cudaFuncSetAttribute(crit_finish_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, lim);
     if (e != cudaSuccess) return e;
     configured[dev] = true;
   }
-  size_t smem = 3 * (size_t)a.N_t_max * sizeof(float);
+  size_t smem = (3 * (size_t)a.N_t_max + kFinishThreads) * sizeof(float);
   if (a.N_t_max <= kFinishSmemNt) smem += (size_t)a.N_t_max * a.N_t_max * sizeof(float);
+  if (smem > (size_t)(3 * kFinishSmemNt + kFinishThreads + kFinishSmemNt * kFinishSmemNt) * sizeof(float))
+    return cudaErrorInvalidValue;  // N_t_max beyond what the shared-memory layout holds
   (void)parts;
-  crit_finish_kernel<<<a.B, 256, smem, s>>>(a, G, mask, r_out);
+  crit_finish_kernel<<<a.B, kFinishThreads, smem, s>>>(a, G, mask, r_out);
   return cudaGetLastError();
 }
 
