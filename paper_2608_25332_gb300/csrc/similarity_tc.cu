@@ -358,7 +358,7 @@ __global__ void __launch_bounds__(kThreads, 2)
 }
 
 // mu_i from the tile sums (tile order), then p_j = max over the critical rows
-// of Y[b][j][i] - mu_i; an empty T gives -inf. Loads go out eight at a time.
+// of Y[b][j][i] - mu_i; an empty T gives -inf. Loads go out 32 at a time.
 __global__ void __launch_bounds__(256) relevance_finish_kernel(const RelFusedArgs a, const int* text_len,
                                                                const uint8_t* mask, float* p) {
   __shared__ float mu[kBM];
@@ -370,12 +370,12 @@ __global__ void __launch_bounds__(256) relevance_finish_kernel(const RelFusedArg
     float s = 0.f;
     if (v) {
       const float* col = a.part + (size_t)b * a.n_vt * a.NT + c;
-      for (int t0 = 0; t0 < a.n_vt; t0 += 8) {
-        float x[8];
+      for (int t0 = 0; t0 < a.n_vt; t0 += 32) {
+        float x[32];
 #pragma unroll
-        for (int u = 0; u < 8; ++u) x[u] = t0 + u < a.n_vt ? col[(size_t)(t0 + u) * a.NT] : 0.f;
+        for (int u = 0; u < 32; ++u) x[u] = t0 + u < a.n_vt ? col[(size_t)(t0 + u) * a.NT] : 0.f;
 #pragma unroll
-        for (int u = 0; u < 8; ++u)
+        for (int u = 0; u < 32; ++u)
           if (t0 + u < a.n_vt) s += x[u];
       }
     }
@@ -387,13 +387,13 @@ __global__ void __launch_bounds__(256) relevance_finish_kernel(const RelFusedArg
   if (j >= a.N_v) return;
   const float4* y = reinterpret_cast<const float4*>(a.Y + ((size_t)b * a.N_v + j) * a.NT);
   float best = -INFINITY;
-  for (int q0 = 0; q0 < a.NT / 4; q0 += 8) {
-    float4 f[8];
+  for (int q0 = 0; q0 < a.NT / 4; q0 += 32) {  // NT <= 128: one batch
+    float4 f[32];
 #pragma unroll
-    for (int u = 0; u < 8; ++u)
+    for (int u = 0; u < 32; ++u)
       if (q0 + u < a.NT / 4) f[u] = y[q0 + u];
 #pragma unroll
-    for (int u = 0; u < 8; ++u) {
+    for (int u = 0; u < 32; ++u) {
       if (q0 + u >= a.NT / 4) break;
       const int c = (q0 + u) * 4;
       if (valid[c]) best = fmaxf(best, f[u].x - mu[c]);
@@ -437,10 +437,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0) {
       RowSrc ra{nullptr, b * N_t_max, kBM};
       RowSrc rb{nullptr, b * N_t_max, kCritBN};
-      producer<kCritBN>(pipe, stages, &mapT, &mapT, ra, false, rb, false, 1, n_k, err, k0);
+      // both operands are the same text rows: one load per K slice
+      producer<kCritBN>(pipe, stages, &mapT, &mapT, ra, false, rb, false, 1, n_k, err, k0, true);
     }
   } else if (warp == 1) {
-    if (lane == 0) mma_issuer<kCritBN>(pipe, stages, 1, n_k, err);
+    if (lane == 0) mma_issuer<kCritBN>(pipe, stages, 1, n_k, err, true);
   } else {
     const int quad = warp & 3;
     const int r = quad * 32 + lane;

@@ -84,11 +84,12 @@ __device__ __forceinline__ void load_rows(uint8_t* dst, const CUtensorMap* map, 
 
 // Producer: for each N tile t in [0, n_tiles), all K slices.
 template <int BN>
-// k0: first K slice (a split-K part starts past the others' slices)
+// k0: first K slice (a split-K part starts past the others' slices); b_is_a:
+// the B operand is the A tile itself (a Gram of one row block), loaded once
 __device__ __forceinline__ void producer(Pipe& p, uint8_t* stages, const CUtensorMap* mapA,
                                          const CUtensorMap* mapB, const RowSrc& a, bool gatherA,
                                          const RowSrc& b, bool gatherB, int n_tiles, int n_k,
-                                         unsigned* err, int k0 = 0) {
+                                         unsigned* err, int k0 = 0, bool b_is_a = false) {
   int it = 0;
   for (int t = 0; t < n_tiles && !p.fail; ++t) {
     for (int kb = 0; kb < n_k; ++kb, ++it) {
@@ -100,9 +101,9 @@ __device__ __forceinline__ void producer(Pipe& p, uint8_t* stages, const CUtenso
       }
       uint8_t* sa = stages + (size_t)s * Cfg<BN>::kStageBytes;
       uint8_t* sb = sa + kABytes;
-      mbar_arrive_expect_tx(&p.full[s], Cfg<BN>::kStageBytes);
+      mbar_arrive_expect_tx(&p.full[s], b_is_a ? (uint32_t)kABytes : (uint32_t)Cfg<BN>::kStageBytes);
       load_rows(sa, mapA, a, 0, kBM, (k0 + kb) * kBK, &p.full[s], gatherA);
-      load_rows(sb, mapB, b, t * BN, BN, (k0 + kb) * kBK, &p.full[s], gatherB);
+      if (!b_is_a) load_rows(sb, mapB, b, t * BN, BN, (k0 + kb) * kBK, &p.full[s], gatherB);
     }
   }
 }
@@ -110,7 +111,7 @@ __device__ __forceinline__ void producer(Pipe& p, uint8_t* stages, const CUtenso
 // MMA issuer.
 template <int BN>
 __device__ __forceinline__ void mma_issuer(Pipe& p, uint8_t* stages, int n_tiles, int n_k,
-                                           unsigned* err) {
+                                           unsigned* err, bool b_is_a = false) {
   int it = 0;
   for (int t = 0; t < n_tiles; ++t) {
     const int buf = t & 1;
@@ -127,7 +128,7 @@ __device__ __forceinline__ void mma_issuer(Pipe& p, uint8_t* stages, int n_tiles
       }
       tc_fence_after();
       const uint32_t sa = smem_u32(stages + (size_t)s * Cfg<BN>::kStageBytes);
-      const uint32_t sb = sa + kABytes;
+      const uint32_t sb = b_is_a ? sa : sa + kABytes;
 #pragma unroll
       for (int k = 0; k < kBK / 16; ++k)
         tc_mma_bf16(acc_addr, smem_desc_sw128(sa + k * 32), smem_desc_sw128(sb + k * 32),
