@@ -460,25 +460,48 @@ __global__ void __launch_bounds__(256) relevance_kernel(const SimArgs a, const u
 // ---------------------------------------------------------------------------
 // Sec. 4.3 merge
 // ---------------------------------------------------------------------------
-// kept-position map: pos[b][j] = a if j == keep[b][a], else -1
-__global__ void keep_pos_kernel(const int* keep_idx, int keep, int B, int N_v, int* kpos,
-                                unsigned* err) {
-  const size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (i < (size_t)B * N_v) kpos[i] = -1;
-}
-__global__ void keep_scatter_kernel(const int* keep_idx, int keep, int B, int N_v, int* kpos,
-                                    unsigned* err) {
-  const size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (i >= (size_t)B * keep) return;
-  const int b = (int)(i / keep), a = (int)(i - (size_t)b * keep);
-  const int j = keep_idx[i];
-  if (j < 0 || j >= N_v || (a > 0 && keep_idx[i - 1] >= j)) {
-    set_error(err, kErrBadDeviceArg);
-    return;
+// Per sample (one CTA of 1024 threads): the kept-position map kpos[b][j] =
+// a if j == keep[b][a], else -1, and, when `pruned` is given, the rows not
+// kept in ascending order, pruned[b][0 .. N_v - keep) (ballot compaction).
+__global__ void __launch_bounds__(1024) merge_index_kernel(const int* keep_idx, int keep, int N_v, int* kpos,
+                                                           int* pruned, unsigned* err) {
+  __shared__ int warp_tot[32];
+  const int b = blockIdx.x;
+  int* kp = kpos + (size_t)b * N_v;
+  const int* ki = keep_idx + (size_t)b * keep;
+  for (int j = threadIdx.x; j < N_v; j += blockDim.x) kp[j] = -1;
+  __syncthreads();
+  for (int q = threadIdx.x; q < keep; q += blockDim.x) {
+    const int j = ki[q];
+    if (j < 0 || j >= N_v || (q > 0 && ki[q - 1] >= j)) {
+      set_error(err, kErrBadDeviceArg);
+      continue;
+    }
+    kp[j] = q;
   }
-  kpos[(size_t)b * N_v + j] = a;
+  if (pruned == nullptr) return;
+  __syncthreads();  // the map is complete (global writes of this block)
+  const int n_pruned = N_v - keep;
+  int* out = pruned + (size_t)b * n_pruned;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+  int base = 0;
+  for (int j0 = 0; j0 < N_v; j0 += blockDim.x) {
+    const int j = j0 + threadIdx.x;
+    const bool pr = j < N_v && kp[j] < 0;
+    const unsigned bal = __ballot_sync(0xffffffffu, pr);
+    if (lane == 0) warp_tot[warp] = __popc(bal);
+    __syncthreads();
+    int off = 0, tot = 0;
+    for (int w = 0; w < nw; ++w) {
+      off += w < warp ? warp_tot[w] : 0;
+      tot += warp_tot[w];
+    }
+    const int pos = base + off + __popc(bal & ((1u << lane) - 1u));
+    if (pr && pos < n_pruned) out[pos] = j;
+    base += tot;
+    __syncthreads();
+  }
 }
-
 __device__ __forceinline__ bool better(float v, int i, float bv, int bi) {
   return v > bv || (v == bv && i < bi);
 }
@@ -609,26 +632,35 @@ using MeanF32 = MeanCfg<256, 8, 4, 1024, 2>;        // fp32 rows <= 8192 element
 constexpr int kMeanSmallRowBytes = 128 * 4 * 16;
 template <typename C> size_t merge_mean_smem(int row_bytes) { return (size_t)C::kSlots * row_bytes; }
 
-__global__ void merge_count_kernel(const int* assign, int B, int N_v, int keep, int* count) {
-  const size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (i >= (size_t)B * N_v) return;
-  const int b = (int)(i / N_v);
-  const int ap = assign[i];
-  if (ap >= 0 && ap < keep) atomicAdd(&count[(size_t)b * keep + ap], 1);
-}
-
-// exclusive scan of count[b][0..keep) -> offset[b][..], cursor[b][..] = 0
-__global__ void __launch_bounds__(1024) merge_offsets_kernel(const int* count, int keep, int* offset,
-                                                              int* cursor) {
+// Counting sort of one sample's rows by centroid (one CTA of 1024 threads):
+// count[b][a] = rows assigned to a, offset[b][.] its exclusive scan, and
+// members[b][offset[a] ..] the rows of a in no particular order (the means
+// rank them). The block-wide barriers order the phases (global memory of this
+// block only).
+__global__ void __launch_bounds__(1024) merge_sort_kernel(const int* assign, int N_v, int keep, int* count,
+                                                          int* offset, int* cursor, int* members) {
   __shared__ uint32_t warp_tot[32];
   __shared__ uint32_t carry;
   const int b = blockIdx.x;
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int* as = assign + (size_t)b * N_v;
+  int* cnt = count + (size_t)b * keep;
+  int* off = offset + (size_t)b * keep;
+  int* cur = cursor + (size_t)b * keep;
+  for (int q = threadIdx.x; q < keep; q += blockDim.x) {
+    cnt[q] = 0;
+    cur[q] = 0;
+  }
   if (threadIdx.x == 0) carry = 0;
   __syncthreads();
+  for (int j = threadIdx.x; j < N_v; j += blockDim.x) {
+    const int ap = as[j];
+    if (ap >= 0 && ap < keep) atomicAdd(&cnt[ap], 1);
+  }
+  __syncthreads();
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   for (int a0 = 0; a0 < keep; a0 += 1024) {
     const int ap = a0 + threadIdx.x;
-    const uint32_t v = ap < keep ? (uint32_t)count[(size_t)b * keep + ap] : 0u;
+    const uint32_t v = ap < keep ? (uint32_t)cnt[ap] : 0u;
     uint32_t incl = v;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
@@ -648,25 +680,15 @@ __global__ void __launch_bounds__(1024) merge_offsets_kernel(const int* count, i
       warp_tot[lane] = ti - t;
     }
     __syncthreads();
-    if (ap < keep) {
-      offset[(size_t)b * keep + ap] = (int)(carry + warp_tot[warp] + incl - v);
-      cursor[(size_t)b * keep + ap] = 0;
-    }
+    if (ap < keep) off[ap] = (int)(carry + warp_tot[warp] + incl - v);
     __syncthreads();
     if (threadIdx.x == 1023) carry += warp_tot[31] + incl;
     __syncthreads();
   }
-}
-
-__global__ void merge_fill_kernel(const int* assign, int B, int N_v, int keep, const int* offset,
-                                  int* cursor, int* members) {
-  const size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (i >= (size_t)B * N_v) return;
-  const int b = (int)(i / N_v), j = (int)(i - (size_t)b * N_v);
-  const int ap = assign[i];
-  if (ap < 0 || ap >= keep) return;
-  const size_t k = (size_t)b * keep + ap;
-  members[(size_t)b * N_v + offset[k] + atomicAdd(&cursor[k], 1)] = j;
+  for (int j = threadIdx.x; j < N_v; j += blockDim.x) {
+    const int ap = as[j];
+    if (ap >= 0 && ap < keep) members[(size_t)b * N_v + off[ap] + atomicAdd(&cur[ap], 1)] = j;
+  }
 }
 
 // the addition of 16 raw bytes of a row to Acc values (8 bf16 or 4 fp32)
@@ -915,11 +937,11 @@ cudaError_t merge_launch(const SimArgs& a, const int* keep_idx, int keep, const 
   // read by merge_argmax_kernel and merge_assign_kernel (same index only).
   int* kpos = assign;
   const size_t nb = (size_t)a.B * a.N_v;
-  keep_pos_kernel<<<(unsigned)((nb + 255) / 256), 256, 0, s>>>(keep_idx, keep, a.B, a.N_v, kpos, a.err);
-  const size_t nk = (size_t)a.B * keep;
-  keep_scatter_kernel<<<(unsigned)((nk + 255) / 256), 256, 0, s>>>(keep_idx, keep, a.B, a.N_v, kpos, a.err);
   const int tc_split = merge_tc_split(a.B, a.N_v, keep, num_sms);
-  if (ws_pruned != nullptr && ws_perm != nullptr && merge_tc_supported(a, keep, tc_split)) {
+  const bool tc = ws_pruned != nullptr && ws_perm != nullptr && merge_tc_supported(a, keep, tc_split);
+  // the kept-position map, and the pruned rows for the tensor-core Gram
+  merge_index_kernel<<<a.B, 1024, 0, s>>>(keep_idx, keep, a.N_v, kpos, tc ? ws_pruned : nullptr, a.err);
+  if (tc) {
     cudaError_t e = merge_argmax_tc_launch(a, keep_idx, keep, inv_v, kpos, ws_pruned, ws_perm, tc_split,
                                            ws_best, ws_bidx, s);
     if (e != cudaSuccess) return e;
@@ -940,10 +962,7 @@ cudaError_t merge_launch(const SimArgs& a, const int* keep_idx, int keep, const 
     int* off = cnt + (size_t)a.B * keep;
     int* cur = off + (size_t)a.B * keep;
     int* mem = reinterpret_cast<int*>(ws_best);
-    cudaMemsetAsync(cnt, 0, (size_t)a.B * keep * sizeof(int), s);
-    merge_count_kernel<<<(unsigned)((nb + 255) / 256), 256, 0, s>>>(assign, a.B, a.N_v, keep, cnt);
-    merge_offsets_kernel<<<a.B, 1024, 0, s>>>(cnt, keep, off, cur);
-    merge_fill_kernel<<<(unsigned)((nb + 255) / 256), 256, 0, s>>>(assign, a.B, a.N_v, keep, off, cur, mem);
+    merge_sort_kernel<<<a.B, 1024, 0, s>>>(assign, a.N_v, keep, cnt, off, cur, mem);
     dim3 gm(keep, a.B);
     static bool configured[64] = {false};
     int dev = 0;

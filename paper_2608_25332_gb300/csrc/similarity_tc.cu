@@ -20,33 +20,6 @@ namespace {
 
 using namespace tcg;
 
-// pruned[b][0..N_v - keep): the visual rows not in keep, ascending (kpos < 0)
-__global__ void __launch_bounds__(1024) pruned_list_kernel(const int* kpos, int N_v, int* pruned,
-                                                            int n_pruned) {
-  __shared__ int warp_tot[32];
-  const int b = blockIdx.x;
-  const int* kp = kpos + (size_t)b * N_v;
-  int* out = pruned + (size_t)b * n_pruned;
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
-  int base = 0;
-  for (int j0 = 0; j0 < N_v; j0 += blockDim.x) {
-    const int j = j0 + threadIdx.x;
-    const bool pr = j < N_v && kp[j] < 0;
-    const unsigned bal = __ballot_sync(0xffffffffu, pr);
-    if (lane == 0) warp_tot[warp] = __popc(bal);
-    __syncthreads();
-    int off = 0, tot = 0;
-    for (int w = 0; w < nw; ++w) {
-      off += w < warp ? warp_tot[w] : 0;
-      tot += warp_tot[w];
-    }
-    const int pos = base + off + __popc(bal & ((1u << lane) - 1u));
-    if (pr && pos < n_pruned) out[pos] = j;
-    base += tot;
-    __syncthreads();
-  }
-}
-
 // perm[b] = rows of E_v[b] reordered as [pruned rows (ascending) | kept rows
 // (keep order)], so that the Gram reads both operands as contiguous tiles.
 // One warp per output row, 16-byte vectors.
@@ -515,8 +488,7 @@ cudaError_t merge_argmax_tc_launch(const SimArgs& a, const int* keep_idx, int ke
   const size_t smem = merge_tc_smem();
   cudaError_t e = set_smem(merge_argmax_tc, smem, &smem_set[dev < 64 ? dev : 0]);
   if (e != cudaSuccess) return e;
-  const int n_pruned = a.N_v - keep;
-  pruned_list_kernel<<<a.B, 1024, 0, s>>>(kpos, a.N_v, pruned, n_pruned);
+  const int n_pruned = a.N_v - keep;  // pruned: the rows not kept, ascending (merge_index_kernel)
   dim3 gg((a.N_v + 7) / 8, a.B);
   gather_perm_kernel<<<gg, 256, 0, s>>>(static_cast<const __nv_bfloat16*>(a.emb_v), pruned, keep_idx,
                                         n_pruned, keep, a.N_v, a.D, static_cast<__nv_bfloat16*>(perm),
