@@ -11,12 +11,14 @@
 //     logits again (those keys are read a second time, from L2: the chunk was
 //     loaded in pass A moments before), p = 2^(s - M) / L = 2^(s - c) with
 //     c = M + log2 L, summed over the 128 rows into
-//     partial[b][rb * H_sel + h][col]. Without CONF the MMA computes S^T = K Q^T
-//     (TMEM lane = key), so a key's sum over the rows stays in its thread (two
-//     halves of 64 rows, added in a fixed order); with CONF it computes S (lane
-//     = row) to keep each row's mean and M2 of its visual probabilities as well,
-//     and sums the columns with a warp butterfly transpose-reduction and a
-//     fixed-order sum over the 4 lane quadrants.
+//     partial[b][rb * H_sel + h][col]. Pass B computes S^T = K Q^T (TMEM lane =
+//     key), so a key's sum over the rows stays in its thread (two halves of 64
+//     rows, added in a fixed order).
+// With CONF, pass A also keeps, per row, the count, mean and M2 (Chan, Golub
+// and LeVeque) of 2^(s - m) over its visual keys, rescaled whenever the
+// running max m rises (mean by 2^(m_old - m_new), M2 by its square); at the
+// switch to pass B the two column halves are brought to the row max M and
+// merged, and mean / L, M2 / L^2 are those of the visual probabilities p.
 // Rows of the query tile past the block's text rows are zeroed in shared
 // memory before the first MMA, so every logit the workers read is finite.
 // Roles: warp 8 (one lane) issues the TMA loads into a 2-stage ring of key
@@ -82,6 +84,7 @@ __global__ void __launch_bounds__(kThreads, 2)
   extern __shared__ uint8_t smem_raw[];
   __shared__ Ctl ctl;
   __shared__ float2 halfstat[2][kTile];
+  __shared__ float4 halfconf[CONF ? 2 : 1][CONF ? kTile : 1];  // (count, mean, M2, max) per half
   __shared__ float red[2][4][kTile];
   __shared__ __align__(16) float crow[kTile];  // M + log2(L) per row; +inf: not scored
   const int hi = blockIdx.x % a.H_sel, rb = blockIdx.x / a.H_sel;
@@ -174,9 +177,9 @@ __global__ void __launch_bounds__(kThreads, 2)
         tc_fence_after();
         const uint32_t ka = smem_u32(ks + (size_t)s * kTileBytes);
         const uint32_t acc = ctl.tmem + (uint32_t)(buf * kTile);
-        // pass A: S = Q K^T (lane = text row); pass B without confidence:
-        // S^T = K Q^T (lane = key), so a key's sum over the rows stays in its thread
-        const bool tr = !CONF && it >= nA;
+        // pass A: S = Q K^T (lane = text row); pass B: S^T = K Q^T (lane =
+        // key), so a key's sum over the rows stays in its thread
+        const bool tr = it >= nA;
         const uint32_t opa = tr ? ka : qa, opb = tr ? qa : ka;
 #pragma unroll
         for (int kstep = 0; kstep < 8; ++kstep) {
@@ -230,10 +233,28 @@ __global__ void __launch_bounds__(kThreads, 2)
         if (h1.x != -INFINITY) L += h1.y * ex2_approx(h1.x - M);
         // p = 2^(s - M) / L = 2^(s - c); L >= 1 (the max term) for a valid row
         c = (rv && L > 0.f) ? M + lg2_approx(L) : 0.f;
-        if (!CONF) {
-          if (half == 0) crow[r] = (rv && L > 0.f) ? c : INFINITY;  // 2^-inf = 0
+        if (CONF) {
+          // each half's statistics at the row max M, merged in half order, then
+          // those of p = x / L; written for the rows of T
+          halfconf[half][r] = make_float4(cn, cmean, cm2, m);
           workers_sync();
+          if (half == 0 && rv && L > 0.f &&
+              (a.conf_mask == nullptr || a.conf_mask[(size_t)b * a.N_t_max + j] != 0)) {
+            float n = 0.f, mean = 0.f, m2 = 0.f;
+#pragma unroll
+            for (int q = 0; q < 2; ++q) {
+              const float4 hc = halfconf[q][r];
+              if (hc.x > 0.f) {
+                const float f = ex2_approx(hc.w - M);
+                chan_merge(n, mean, m2, hc.x, hc.y * f, hc.z * f * f);
+              }
+            }
+            a.conf_part[(((size_t)b * a.H_sel + hi) * a.N_t_max + j) * a.conf_stride] =
+                make_float2(mean / L, m2 / (L * L));
+          }
         }
+        if (half == 0) crow[r] = (rv && L > 0.f) ? c : INFINITY;  // 2^-inf = 0
+        workers_sync();
       }
       const uint32_t tacc = tbase + (uint32_t)(buf * kTile);
       if (it < nA) {
@@ -260,13 +281,52 @@ __global__ void __launch_bounds__(kThreads, 2)
             if (mn != -INFINITY) {
               float s4[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-              for (int i = 0; i < 32; ++i) s4[i & 3] += ex2_approx(fmaf(v[i], sc, -mn));
-              l = l * ex2_approx(m - mn) + ((s4[0] + s4[1]) + (s4[2] + s4[3]));
+              for (int i = 0; i < 32; ++i) {
+                v[i] = ex2_approx(fmaf(v[i], sc, -mn));
+                s4[i & 3] += v[i];
+              }
+              const float rs = ex2_approx(m - mn);
+              l = l * rs + ((s4[0] + s4[1]) + (s4[2] + s4[3]));
+              if (CONF) {
+                // the visual keys of this block: [vlo, vhi) relative to k0
+                const int vlo = max(a.vis_start - k0, 0), vhi = min(a.vis_start + a.N_v - k0, 32);
+                if (cn > 0.f) {
+                  cmean *= rs;
+                  cm2 *= rs * rs;
+                }
+                if (vlo == 0 && vhi == 32) {
+                  // every key of the block is visual (the common case)
+                  float q4[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+                  for (int i = 0; i < 32; ++i) q4[i & 3] += v[i];
+                  const float mb = ((q4[0] + q4[1]) + (q4[2] + q4[3])) * (1.f / 32.f);
+                  float d4[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+                  for (int i = 0; i < 32; ++i) {
+                    const float d = v[i] - mb;
+                    d4[i & 3] = fmaf(d, d, d4[i & 3]);
+                  }
+                  chan_merge(cn, cmean, cm2, 32.f, mb, (d4[0] + d4[1]) + (d4[2] + d4[3]));
+                } else if (vlo < vhi) {
+                  const float nb = (float)(vhi - vlo);
+                  float q4[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+                  for (int i = 0; i < 32; ++i) q4[i & 3] += (i >= vlo && i < vhi) ? v[i] : 0.f;
+                  const float mb = ((q4[0] + q4[1]) + (q4[2] + q4[3])) / nb;
+                  float d4[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+                  for (int i = 0; i < 32; ++i) {
+                    const float d = (i >= vlo && i < vhi) ? v[i] - mb : 0.f;
+                    d4[i & 3] = fmaf(d, d, d4[i & 3]);
+                  }
+                  chan_merge(cn, cmean, cm2, nb, mb, (d4[0] + d4[1]) + (d4[2] + d4[3]));
+                }
+              }
             }
             m = mn;
           }
         }
-      } else if (!CONF) {
+      } else {
         // transposed: thread = key kk of the chunk, 64 text rows per warp
         const int par = (it - nA) & 1;
         const int kk = quad * 32 + lane, key = a.vis_start + (it - nA) * kTile + kk;
@@ -304,59 +364,6 @@ __global__ void __launch_bounds__(kThreads, 2)
           csum += (s4[0] + s4[1]) + (s4[2] + s4[3]);
         }
         red[par][half][kk] = csum;
-      } else {
-        const int par = (it - nA) & 1;
-#pragma unroll
-        for (int cb = 0; cb < 2; ++cb) {
-          const int vc0 = (it - nA) * kTile + half * 64 + cb * 32;  // first visual column
-          if (vc0 >= a.N_v) {  // warp-uniform
-            red[par][quad][half * 64 + cb * 32 + lane] = 0.f;
-            continue;
-          }
-          float v[32];
-          tmem_ld32(tacc + cb * 32, v);
-          tc_wait_ld();
-          if (!rv) {
-#pragma unroll
-            for (int i = 0; i < 32; ++i) v[i] = 0.f;
-          } else if (vc0 + 32 <= a.N_v && a.vis_start + vc0 + 31 <= t_first) {
-#pragma unroll
-            for (int i = 0; i < 32; ++i) v[i] = ex2_approx(fmaf(v[i], sc, -c));
-          } else {
-#pragma unroll
-            for (int i = 0; i < 32; ++i) {
-              const bool kv = vc0 + i < a.N_v && a.vis_start + vc0 + i <= t;
-              v[i] = kv ? ex2_approx(fmaf(v[i], sc, -c)) : 0.f;
-            }
-          }
-          if (CONF) {
-            const int nbi = min(32, a.N_v - vc0);
-            const float nb = (float)nbi;
-            float s4[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-            for (int i = 0; i < 32; ++i) s4[i & 3] += v[i];  // zero past N_v
-            const float mb = ((s4[0] + s4[1]) + (s4[2] + s4[3])) / nb;
-            float q4[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-            for (int i = 0; i < 32; ++i) {
-              const float d = i < nbi ? v[i] - mb : 0.f;
-              q4[i & 3] += d * d;
-            }
-            chan_merge(cn, cmean, cm2, nb, mb, (q4[0] + q4[1]) + (q4[2] + q4[3]));
-          }
-          // butterfly transpose-reduction: lane ends with the sum of column `lane`
-#pragma unroll
-          for (int sh = 16; sh >= 1; sh >>= 1) {
-            const bool upper = (lane & sh) != 0;
-#pragma unroll
-            for (int i = 0; i < sh; ++i) {
-              const float keep = upper ? v[i + sh] : v[i];
-              const float send = upper ? v[i] : v[i + sh];
-              v[i] = keep + __shfl_xor_sync(0xffffffffu, send, sh);
-            }
-          }
-          red[par][quad][half * 64 + cb * 32 + lane] = v[0];
-        }
       }
       // the accumulator may be overwritten
       tc_fence_before();
@@ -367,25 +374,7 @@ __global__ void __launch_bounds__(kThreads, 2)
         workers_sync();  // red[par] complete (red[par ^ 1] is free: read before this barrier)
         const int c = (it - nA) * kTile + threadIdx.x;
         if (threadIdx.x < kTile && c < a.N_v)
-          out[c] = CONF ? red[par][0][threadIdx.x] + red[par][1][threadIdx.x] + red[par][2][threadIdx.x] +
-                              red[par][3][threadIdx.x]
-                        : red[par][0][threadIdx.x] + red[par][1][threadIdx.x];
-      }
-    }
-    if (CONF) {
-      // merge the two column halves of each row; counts from the column ranges
-      halfstat[half][r] = make_float2(cmean, cm2);
-      workers_sync();
-      if (half == 0 && rv && (a.conf_mask == nullptr || a.conf_mask[(size_t)b * a.N_t_max + j] != 0)) {
-        float n0 = 0.f, n1 = 0.f;
-        for (int c = 0; c < nB; ++c) {
-          n0 += (float)max(0, min(64, a.N_v - c * kTile));
-          n1 += (float)max(0, min(64, a.N_v - c * kTile - 64));
-        }
-        const float2 s0 = halfstat[0][r], s1 = halfstat[1][r];
-        float n = n0, mean = s0.x, m2 = s0.y;
-        if (n1 > 0.f) chan_merge(n, mean, m2, n1, s1.x, s1.y);
-        a.conf_part[(((size_t)b * a.H_sel + hi) * a.N_t_max + j) * a.conf_stride] = make_float2(mean, m2);
+          out[c] = red[par][0][threadIdx.x] + red[par][1][threadIdx.x];
       }
     }
   }
