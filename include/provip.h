@@ -75,9 +75,8 @@ extern "C" {
                                          no cluster shape fits */
 /* Different kernel families sum in different orders: results agree within the
  * floating-point tolerance, and are bit-identical between calls that take the
- * same family (the same algo and, for PROVIP_ALGO_TCGEN05, the same choice;
- * the STREAM form has a second order when it also keeps head-confidence
- * statistics, see provip_prune_visual_heads). */
+ * same family (the same algo and, for PROVIP_ALGO_TCGEN05, the same choice),
+ * with or without head-confidence statistics. */
 
 /* bits of the device status word */
 #define PROVIP_DEVSTAT_TIMEOUT 1u  /* a bounded wait gave up */
@@ -327,11 +326,9 @@ int provip_head_confidence(const void *Q, const void *K, int B, int L_max, int H
  * sample over all its text rows (S^vis and v of Sec. 4.4), the top `keep` of v
  * (idx_out [B, keep] ascending, ties to the lower index) and the compaction of
  * provip_compact. One pass over the keys computes the attention statistics of
- * every head; with the same kernel family on both sides (algo CLUSTER, TWOPASS
- * or SIMT) the scores of a sample's visual heads are bit-identical to
- * provip_prune called on that sample alone with head_list = its visual heads
- * (the STREAM form sums the columns in another order when it keeps no
- * confidence statistics, so there they agree to fp32 rounding).
+ * every head; with the same kernel family on both sides (algo STREAM, CLUSTER,
+ * TWOPASS or SIMT) the scores of a sample's visual heads are bit-identical to
+ * provip_prune called on that sample alone with head_list = its visual heads.
  * scores_out_or_null [B, N_v], vis_heads_out_or_null [B, N_vis] and
  * conf_out_or_null [B, H_q] receive v, the visual heads and C when non-NULL.
  * flags as in provip_prune. Workspace: provip_visual_heads_workspace_size. */
