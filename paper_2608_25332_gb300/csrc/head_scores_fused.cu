@@ -308,10 +308,18 @@ __global__ void __launch_bounds__(kThreads, CPC == 1 ? 3 : (CPC == 2 ? 2 : 1))
         for (int i = 0; i < 32; ++i) s4[i & 3] += v[i];  // zero outside the visual range
         const float mb = ((s4[0] + s4[1]) + (s4[2] + s4[3])) / nb;
         float q4[4] = {0.f, 0.f, 0.f, 0.f};
+        if (lo == k0 && hi == k0 + 32) {  // every column of the block is visual
 #pragma unroll
-        for (int i = 0; i < 32; ++i) {
-          const float d = (k0 + i >= lo && k0 + i < hi) ? v[i] - mb : 0.f;
-          q4[i & 3] += d * d;
+          for (int i = 0; i < 32; ++i) {
+            const float d = v[i] - mb;
+            q4[i & 3] = fmaf(d, d, q4[i & 3]);
+          }
+        } else {
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            const float d = (k0 + i >= lo && k0 + i < hi) ? v[i] - mb : 0.f;
+            q4[i & 3] = fmaf(d, d, q4[i & 3]);
+          }
         }
         const float n = cn + nb, dl = mb - cmean;
         cmean += dl * (nb / n);
