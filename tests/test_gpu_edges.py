@@ -54,6 +54,7 @@ def _ulp(x, dtype):
     ("bf16", 2, 37, 64, (3, 8), 37),         # nothing pruned: merged rows are the rows
     ("bf16", 2, 300, 128, (128, 33), 100),   # 128 text rows (the tensor-core limit), tiles 128+128+44
     ("bf16", 2, 200, 136, (129, 2), 50),     # 129 text rows: the CUDA-core relevance
+    ("bf16", 2, 150, 136, (40, 7), 60),      # D = 136: the last K slice of the tensor-core Grams is partial
     ("f32", 2, 37, 64, (1, 9), 10),
 ])
 def test_similarity_reduce_edge_cases(dtype, B, N_v, D, tls, keep_pre):
