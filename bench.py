@@ -713,6 +713,15 @@ def run_gb300(args, dist):
                               and w.L_max <= 8192) else 4
     reps = max(1, min(20, K // GRAPH_CHUNK))
     t_compact = time_graph(compact_i, reps)
+    # context for the fraction: torch's copy_ (the operation the HBM peak was
+    # measured with, there over 2 GiB) on the same bytes (half read, half
+    # written), its source rotating over three buffers as the inputs do, timed
+    # the same way
+    n_el = ab["compact"] // 4  # bf16 elements read (= written)
+    copy_src = [torch.empty(n_el, dtype=torch.bfloat16, device=dev).fill_(1.0) for _ in range(3)]
+    copy_dst = torch.empty(n_el, dtype=torch.bfloat16, device=dev)
+    t_copy = time_graph(lambda i: copy_dst.copy_(copy_src[i % 3]), reps)
+    del copy_src, copy_dst
     t_head = time_graph(head_topk_i, reps)
 
     def serial_i(i):
@@ -862,7 +871,12 @@ def run_gb300(args, dist):
             "roofline": {"bound": "hbm", "kernel": "compact_kernel", "achieved": ach, "peak": peak,
                          "peak_source": peak_src, "unit": "GB/s", "frac": ach / peak,
                          "traffic": traffic, "algorithmic_bytes": ab["compact"],
-                         "duration_us": t_compact * 1e6},
+                         "duration_us": t_compact * 1e6,
+                         "copy_same_bytes": {"duration_us": t_copy * 1e6,
+                                             "frac": ab["compact"] / t_copy / 1e9 / peak,
+                                             "note": "torch copy_ (the operation the peak was measured "
+                                                     "with, over 2 GiB) on the same bytes, timed the "
+                                                     "same way"}},
             "path": {"algorithmic_bytes": ab["path"], "achieved_gbs": path_gbs, "frac": path_gbs / peak,
                      "head_topk_us": t_head * 1e6, "head_topk_bytes": ab["head_topk"],
                      "compact_us": t_compact * 1e6,
