@@ -595,9 +595,17 @@ def run_gb300(args, dist):
         st(c["Q"], c["K"], c["V"], c["hidden"], c["pos"], c["text_start"], c["text_len"], c["seq_len"], vis,
            stream=lane_streams[i % S] if S > 1 else None)
 
+    # one stream: with --algo auto, the head-score form the library picks for a
+    # single stream (the streaming form above is chosen for concurrent ones)
+    single_algo = P.ALGO_AUTO if args.algo == "auto" else algo
+    step_one = step if single_algo == algo else P.PruneStep(
+        g0["Q"], g0["K"], g0["V"], g0["hidden"], g0["pos"], g0["head_list"], w.n_t[1], nv, keep,
+        algo=single_algo, want_scores=False, flags=P.PRUNE_OVERLAP_PREVIOUS)
+
     def do_step_single(i):
         c = copies[i % len(copies)]
-        step(c["Q"], c["K"], c["V"], c["hidden"], c["pos"], c["text_start"], c["text_len"], c["seq_len"], vis)
+        step_one(c["Q"], c["K"], c["V"], c["hidden"], c["pos"], c["text_start"], c["text_len"], c["seq_len"],
+                 vis)
 
     def run_steps(n):
         # n consecutive steps; with S > 1, fork onto the lane streams and join
@@ -881,7 +889,8 @@ def run_gb300(args, dist):
                      "head_topk_us": t_head * 1e6, "head_topk_bytes": ab["head_topk"],
                      "compact_us": t_compact * 1e6,
                      "step_us_without_overlap": t_serial * 1e6,
-                     **({"single_stream": {"value": w.B / t_single, "ms_per_step": t_single * 1e3,
+                     **({"single_stream": {"algo": "auto" if single_algo == P.ALGO_AUTO else algo_name,
+                                           "value": w.B / t_single, "ms_per_step": t_single * 1e3,
                                            "frac": ab["path"] / t_single / 1e9 / peak}}
                         if t_single else {})},
             "cpu_baseline": cpu_base,
