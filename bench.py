@@ -848,14 +848,22 @@ def run_gb300(args, dist):
     e2e_run(0, 4)
     torch.cuda.synchronize()
     E = max(1, args.e2e_steps)
-    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    dist.barrier()
-    a.record()
-    e2e_run(4, E)
-    b.record()
-    torch.cuda.synchronize()
-    e2e_sec = dist.max(a.elapsed_time(b) / 1e3)
-    e2e_value = aggregate(dist.sum(float(w.B * E)), e2e_sec)
+    # three timed runs of E steps each, the median reported: the host copies
+    # share the machine's memory system with other jobs, so a single run can be
+    # an outlier
+    e2e_runs = []
+    first = 4
+    for _ in range(3):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        dist.barrier()
+        a.record()
+        e2e_run(first, E)
+        b.record()
+        torch.cuda.synchronize()
+        first += E
+        e2e_sec = dist.max(a.elapsed_time(b) / 1e3)
+        e2e_runs.append(aggregate(dist.sum(float(w.B * E)), e2e_sec))
+    e2e_value = sorted(e2e_runs)[1]
 
     prellm = prellm_measure(w, dev) if dist.rank == 0 else None
     schedule = schedule_measure(w, dev) if dist.rank == 0 else None
@@ -894,7 +902,8 @@ def run_gb300(args, dist):
                                            "frac": ab["path"] / t_single / 1e9 / peak}}
                         if t_single else {})},
             "cpu_baseline": cpu_base,
-            "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+            "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                    "runs": e2e_runs, "note": f"median of 3 timed runs of {E} steps"},
             "gpu_launches": launches_per_step * K,
             "prellm": prellm,
             "next_rows": dict(next_rows, schedule=schedule, ablation=ablation),
