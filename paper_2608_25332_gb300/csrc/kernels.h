@@ -198,8 +198,9 @@ size_t relevance_fused_floats(int B, int N_v, int N_t_max);
 cudaError_t relevance_tc_launch(const SimArgs& a, const uint8_t* mask, const float* inv_t, float* inv_v,
                                 float* p, float* ws, int num_sms, cudaStream_t s);
 bool merge_tc_supported(const SimArgs& a, int keep, int n_split);
+// pruned: the rows not kept, ascending ([B][N_v - keep], from merge_index_kernel)
 cudaError_t merge_argmax_tc_launch(const SimArgs& a, const int* keep_idx, int keep,
-                                   const float* inv_v, const int* kpos, int* pruned, void* perm,
+                                   const float* inv_v, const int* pruned, void* perm,
                                    int n_split, float* ws_best, int* ws_bidx, cudaStream_t s);
 // N split of the tcgen05 merge Gram (fewest waves x tiles per CTA) and its upper bound
 int merge_tc_split(int B, int N_v, int keep, int num_sms);

@@ -7,10 +7,11 @@
 //   epilogue scales a column by 1/|e_k| and keeps, per row, the running (max,
 //   first index) over the kept positions in ascending order, so ties go to the
 //   lower kept position. The (N_v - N1) x N1 matrix never leaves the SM.
-// relevance_fused_tc: the visual x text cosine Gram with the row norms of both
-//   operands taken from the same shared-memory stages, so the visual rows are
-//   read once for |v_j|, the cosines and the de-meaning sums (p_j itself is
-//   formed by a small second kernel once every tile's sums are known).
+// relevance_fused_tc: the visual x [visual ; text] Gram of a 128-row visual
+//   tile, one read of the visual rows giving |v_j|^2 (the diagonal of the
+//   visual block), the cosines and the de-meaning sums (p_j itself is formed by
+//   a small second kernel once every tile's sums are known).
+// crit_gram_tc: the text Gram E_t E_t^T, split over K.
 #include "common.cuh"
 #include "kernels.h"
 #include "tc_gemm.cuh"
@@ -480,7 +481,7 @@ bool merge_tc_supported(const SimArgs& a, int keep, int n_split) {
 }
 
 cudaError_t merge_argmax_tc_launch(const SimArgs& a, const int* keep_idx, int keep, const float* inv_v,
-                                   const int* kpos, int* pruned, void* perm, int n_split,
+                                   const int* pruned, void* perm, int n_split,
                                    float* ws_best, int* ws_bidx, cudaStream_t s) {
   static bool smem_set[64] = {false};
   int dev = 0;
