@@ -146,3 +146,12 @@ def test_schedule_rejects_inconsistent_stages():
         ProgressiveSchedule(2, 576, 4096, 128, 739, 32, 32, 4096, 1, 288, 73, 20, 6, pre_llm=False)
     with pytest.raises(ValueError):
         ProgressiveSchedule(2, 576, 4096, 128, 739, 32, 32, 4096, 1, 576, 73, 20, 6, shallow_heads="some")
+
+
+def test_missing_library_fails_loudly(tmp_path, monkeypatch):
+    """No fallback: with the compiled library absent, the first call raises."""
+    from paper_2608_25332_gb300 import provip
+    monkeypatch.setattr(provip, "_lib", None)
+    monkeypatch.setattr(provip, "LIB_PATH", str(tmp_path / "libprovip.so"))
+    with pytest.raises(provip.ProvipError, match="not built"):
+        provip.lib()
