@@ -147,3 +147,53 @@ def test_prune_single_keep_and_identity(keep, algo):
             np.testing.assert_array_equal(got, exp)
         for p in range(c["pos"].shape[0]):
             np.testing.assert_array_equal(out["pos"][p, b, :n].cpu().numpy(), c["pos"][p, b].numpy()[src])
+
+
+def _random_case(rng):
+    B = int(rng.integers(1, 5))
+    Hkv = int(rng.choice([1, 2, 4]))
+    Hq = Hkv * int(rng.choice([1, 2, 4]))
+    H_sel = int(rng.integers(1, Hq + 1))
+    nsys = int(rng.integers(0, 40))
+    nv = int(rng.integers(8, 700))
+    tls = tuple(int(x) for x in rng.integers(0, 260, B))
+    keep = int(rng.integers(1, nv + 1))
+    heads = sorted(rng.choice(Hq, H_sel, replace=False).tolist())
+    return B, Hkv, Hq, heads, nsys, nv, tls, keep
+
+
+@pytest.mark.parametrize("seed", range(8))
+def test_prune_random_shapes(seed):
+    """Seeded random shapes (batch, GQA ratio, selected heads, prefix, visual
+    count, ragged text lengths including zero rows, keep) for every tensor-core
+    form and the automatic choice: scores, keep sets and compaction against the
+    oracle."""
+    rng = np.random.default_rng(1000 + seed)
+    B, Hkv, Hq, heads, nsys, nv, tls, keep = _random_case(rng)
+    c = _in_llm_case(2000 + seed, B=B, nsys=nsys, nv=nv, tls=tls, Hq=Hq, Hkv=Hkv, D=128 * int(rng.integers(1, 9)))
+    Qn, Kn = c["Q"].float().numpy(), c["K"].float().numpy()
+    g = {k: c[k].to(DEV) for k in ("Q", "K", "V", "H", "pos")}
+    ts, tl, sl = (torch.from_numpy(x).to(DEV) for x in (c["ts"], c["tl"], c["sl"]))
+    for algo in (P.ALGO_AUTO, P.ALGO_TCGEN05_STREAM, P.ALGO_TCGEN05_CLUSTER, P.ALGO_TCGEN05_TWOPASS):
+        out = P.provip_prune(g["Q"], g["K"], g["V"], g["H"], g["pos"], heads, ts, tl, sl, nsys, nv, keep,
+                             algo=algo, N_t_max=c["Ntm"])
+        torch.cuda.synchronize()
+        what = f"seed {seed} (B={B} Hq={Hq} Hkv={Hkv} heads={heads} nsys={nsys} nv={nv} tl={tls} keep={keep}) algo {algo}"
+        for b in range(B):
+            slb = int(c["sl"][b])
+            if tls[b] == 0:
+                ref = np.zeros(nv)  # no text rows: nothing to score
+                assert np.all(out["scores"][b].cpu().numpy() == 0.0), what
+            else:
+                ref = oracle.head_scores(Qn[b, :slb], Kn[b, :slb], heads,
+                                         np.arange(c["ts"][b], c["ts"][b] + c["tl"][b]), nsys, nv)
+                assert_close_rel(out["scores"][b].cpu().numpy(), ref, 2e-3, what + f" scores[{b}]")
+            idx = out["idx"][b].cpu().numpy()
+            check_topk_band(idx, ref, keep, 2e-3, what + f" keep[{b}]")
+            n = int(out["seq_len"][b])
+            assert n == slb - nv + keep, what
+            src = oracle.compact_map(slb, nsys, nv, idx)
+            for key, src_t in (("hidden", c["H"]), ("K", c["K"]), ("V", c["V"])):
+                np.testing.assert_array_equal(out[key][b, :n].cpu().view(torch.int16).numpy(),
+                                              oracle.gather_rows(src_t[b].view(torch.int16).numpy(), src),
+                                              err_msg=what + f" {key}[{b}]")
