@@ -26,7 +26,7 @@ def _lib():
     assert rc == 0 and bits == 0, f"device status {rc} {bits}"
 
 
-def _pre_case(seed, B, N_v, D, tls, dtype):
+def _pre_case(seed, B, N_v, D, tls, dtype, smooth_text=False):
     rng = np.random.default_rng(seed)
     Ntm = max(tls)
     Ev = rng.standard_normal((B, N_v, D)).astype(np.float32)
@@ -34,6 +34,10 @@ def _pre_case(seed, B, N_v, D, tls, dtype):
     Ev[:, 7] = Ev[:, 5]          # an exact duplicate: ties in every cosine
     Ev[:, 11] *= 40.0            # scale does not change a cosine
     Et = rng.standard_normal((B, Ntm, D)).astype(np.float32)
+    if smooth_text:
+        # text logits of standard deviation 1/16 (the scale of LLM token
+        # embeddings): a smooth softmax, so r and T are well separated
+        Et *= 0.25 / D ** 0.25
     for b, t in enumerate(tls):
         Et[b, t:] = np.nan       # padding past each sample's text rows
     td = torch.bfloat16 if dtype == "bf16" else torch.float32
@@ -59,6 +63,26 @@ def _ulp(x, dtype):
 ])
 def test_similarity_reduce_edge_cases(dtype, B, N_v, D, tls, keep_pre):
     ev, et, tl = _pre_case(17, B, N_v, D, tls, dtype)
+    _check_reduce(ev, et, tl, keep_pre, dtype, f"edge {dtype} B={B} N_v={N_v} D={D} tl={tls} keep={keep_pre}")
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_similarity_reduce_random_shapes(seed):
+    """Seeded random pre-LLM shapes: batch, visual count, width, ragged text
+    lengths (one row included), keep_pre, both dtypes."""
+    rng = np.random.default_rng(3000 + seed)
+    dtype = "f32" if seed % 3 == 2 else "bf16"
+    B = int(rng.integers(1, 5))
+    N_v = int(rng.integers(20, 600))
+    D = 8 * int(rng.integers(4, 64))
+    tls = tuple(int(x) for x in rng.integers(1, 129, B))
+    keep_pre = int(rng.integers(1, N_v + 1))
+    ev, et, tl = _pre_case(4000 + seed, B, N_v, D, tls, dtype, smooth_text=True)
+    _check_reduce(ev, et, tl, keep_pre, dtype, f"seed {seed} {dtype} B={B} N_v={N_v} D={D} tl={tls} keep={keep_pre}")
+
+
+def _check_reduce(ev, et, tl, keep_pre, dtype, what):
+    B, N_v = ev.shape[0], ev.shape[1]
     rt = rtol_for(dtype)
     res = P.provip_similarity_reduce(ev.to(DEV), et.to(DEV), torch.from_numpy(tl).to(DEV), keep_pre,
                                      want_merged=True)
@@ -70,16 +94,16 @@ def test_similarity_reduce_edge_cases(dtype, B, N_v, D, tls, keep_pre):
         n = int(tl[b])
         r_ref, T = oracle.crit_text(Etn[b, :n])
         mask = res["mask"][b].cpu().numpy()
-        check_mask_band(mask[:n], r_ref, rt, f"T[{b}]")
+        check_mask_band(mask[:n], r_ref, rt, f"{what} T[{b}]")
         assert not mask[n:].any()
         if n == 1:
             assert mask[0] == 1, "a single text row is critical"
         if not np.array_equal(mask[:n].astype(bool), T.astype(bool)):
             continue
         p_ref = oracle.relevance(Etn[b, :n], T, Evn[b])
-        assert_close_rel(res["p"][b].cpu().numpy(), p_ref, 0.0, f"p[{b}]", atol=rt)
+        assert_close_rel(res["p"][b].cpu().numpy(), p_ref, 0.0, f"{what} p[{b}]", atol=rt)
         idx = res["idx"][b].cpu().numpy()
-        check_topk_band(idx, p_ref, keep_pre, rt, f"keep[{b}]")
+        check_topk_band(idx, p_ref, keep_pre, rt, f"{what} keep[{b}]")
         if not np.array_equal(idx, oracle.topk(p_ref, keep_pre)):
             continue
         a_ref, mg_ref = oracle.merge(Evn[b], idx)
@@ -92,9 +116,9 @@ def test_similarity_reduce_edge_cases(dtype, B, N_v, D, tls, keep_pre):
         else:
             # a near-tie between two kept rows may move a pruned row; all other
             # centroids are the oracle's within one output ulp
-            assert rows_ok.mean() >= 0.9, f"merged[{b}]: {np.flatnonzero(~rows_ok)} beyond one ulp"
+            assert rows_ok.mean() >= 0.9, f"{what} merged[{b}]: {np.flatnonzero(~rows_ok)} beyond one ulp"
         full += 1
-    assert full >= 1, "no sample reached the merge comparison"
+    assert full >= 1, f"{what}: no sample reached the merge comparison"
 
 
 def _in_llm_case(seed, B, nsys, nv, tls, Hq=4, Hkv=2, D=256, P_=3):
