@@ -249,3 +249,46 @@ def test_all_heads_prune_matches_oracle(name):
                                    cpu["vis_start"], cpu["N_v"])
         assert_close_rel(a["scores"][b].cpu().numpy(), v_ref, rt, f"{name} all heads sample {b}")
         check_topk_band(a["idx"][b].cpu().numpy(), v_ref, g["keep"], rt, f"{name} keep sample {b}")
+
+
+@pytest.mark.parametrize("seed", range(5))
+def test_confidence_random_shapes(seed):
+    """Seeded random shapes for head confidence and the visual heads: batch,
+    GQA ratio, heads, prefix, visual count (ragged against the 128-key tiles),
+    ragged text lengths with a random critical-row mask, N_vis; every form."""
+    rng = np.random.default_rng(5000 + seed)
+    B = int(rng.integers(1, 4))
+    Hkv = int(rng.choice([1, 2, 4]))
+    Hq = Hkv * int(rng.choice([2, 4]))
+    nsys = int(rng.integers(0, 40))
+    nv = int(rng.integers(16, 600))
+    tls = rng.integers(1, 200, B).astype(np.int32)
+    n_vis = int(rng.integers(1, Hq + 1))
+    Ntm = int(tls.max())
+    Lm = nsys + nv + Ntm
+    Q = rng.standard_normal((B, Lm, Hq, 128)).astype(np.float32)
+    K = rng.standard_normal((B, Lm, Hkv, 128)).astype(np.float32)
+    Q[:, :, 0] *= 3.0  # one sharp query head: confidences spread out
+    sl = (nsys + nv + tls).astype(np.int32)
+    ts = np.full(B, nsys + nv, np.int32)
+    mask = (rng.random((B, Ntm)) < 0.5).astype(np.uint8)
+    for b in range(B):
+        Q[b, sl[b]:] = np.nan
+        K[b, sl[b]:] = np.nan
+        mask[b, tls[b]:] = 0
+        if mask[b].sum() == 0:
+            mask[b, 0] = 1
+    Qt, Kt = torch.from_numpy(Q).to(torch.bfloat16), torch.from_numpy(K).to(torch.bfloat16)
+    Qn, Kn = Qt.float().numpy(), Kt.float().numpy()
+    C_ref = np.stack([oracle.head_confidence(Qn[b, :sl[b]], Kn[b, :sl[b]], ts[b] + np.flatnonzero(mask[b]), nsys, nv)
+                      for b in range(B)])
+    g = [torch.from_numpy(x).to(DEV) for x in (ts, tls, sl, mask)]
+    for algo in (P.ALGO_TCGEN05_STREAM, P.ALGO_TCGEN05_CLUSTER, P.ALGO_TCGEN05_TWOPASS, P.ALGO_SIMT):
+        vis, conf = P.provip_head_confidence(Qt.to(DEV), Kt.to(DEV), g[0], g[1], g[2], nsys, nv, n_vis,
+                                             crit_mask=g[3], algo=algo, N_t_max=Ntm)
+        torch.cuda.synchronize()
+        what = f"seed {seed} (B={B} Hq={Hq} Hkv={Hkv} nsys={nsys} nv={nv} tl={tls.tolist()} n_vis={n_vis}) algo {algo}"
+        check_conf(conf.cpu().numpy(), C_ref, 2e-3, what + " C")
+        vis = vis.cpu().numpy()
+        for b in range(B):
+            check_topk_band(vis[b], C_ref[b], n_vis, 2e-3, what + f" visual heads sample {b}")
