@@ -1,12 +1,13 @@
 // Pre-LLM pass (Sec. 4.3) on 5th-generation tensor cores (bf16).
 //
 // merge_argmax_tc: the pruned x kept cosine Gram fused with the row argmax.
-//   A = the pruned visual rows of a 128-row M tile, B = the kept rows of a range
-//   of 256-row N tiles, read as contiguous tiles of a per-sample copy of E_v
-//   permuted to [pruned | kept] by one bandwidth-bound gather pass. The
-//   epilogue scales a column by 1/|e_k| and keeps, per row, the running (max,
-//   first index) over the kept positions in ascending order, so ties go to the
-//   lower kept position. The (N_v - N1) x N1 matrix never leaves the SM.
+//   A = the pruned visual rows of two 128-row M tiles, B = the kept rows of a
+//   range of 256-row N tiles shared by both, read as contiguous tiles of a
+//   per-sample copy of E_v permuted to [pruned | kept] by one bandwidth-bound
+//   gather pass. The epilogue scales a column by 1/|e_k| and keeps, per row,
+//   the running (max, first index) over the kept positions in ascending order,
+//   so ties go to the lower kept position. The (N_v - N1) x N1 matrix never
+//   leaves the SM.
 // relevance_fused_tc: the visual x [visual ; text] Gram of a 128-row visual
 //   tile, one read of the visual rows giving |v_j|^2 (the diagonal of the
 //   visual block), the cosines and the de-meaning sums (p_j itself is formed by
@@ -66,14 +67,36 @@ struct MergeTcArgs {
 
 constexpr int kMergeBN = 256;
 constexpr int kMergeMaxKeep = 2560;  // kept rows handled by one split (shared index table)
+constexpr int kMergeStages = 3;
+constexpr int kMergeBBytes = kMergeBN * kBK * 2;                 // 32 KiB
+constexpr int kMergeStageBytes = 2 * kABytes + kMergeBBytes;     // A0 | A1 | B: 64 KiB
+constexpr uint32_t kMergeTmemCols = 2 * kMergeBN;                // one accumulator per M tile
 
+struct MergePipe {
+  uint64_t full[kMergeStages];
+  uint64_t empty[kMergeStages];
+  uint64_t acc_full;
+  uint64_t acc_empty;
+  uint32_t tmem;
+  volatile int fail;
+};
+
+// One CTA owns two 128-row M tiles of pruned rows (A0, A1) and sweeps its range
+// of 256-row N tiles of kept rows; each stage holds A0, A1 and one B tile, and
+// two MMAs (M = 128, N <= 256) share that B tile, so a stage carries 64 KiB for
+// 8.4 MFLOP instead of 48 KiB for 4.2 MFLOP with a single M tile. The two
+// accumulators fill the 512 TMEM columns: the epilogue of an N tile runs
+// between that tile's last MMA and the next tile's first (the producer keeps
+// loading meanwhile). The last N tile's MMA is only as wide as its kept rows
+// (rounded up to 16).
 __global__ void __launch_bounds__(kThreads, 1)
     merge_argmax_tc(const MergeTcArgs a, const __grid_constant__ CUtensorMap mapE) {
   extern __shared__ uint8_t smem_raw[];
-  __shared__ Pipe pipe;
-  __shared__ int sidx_a[kBM];
+  __shared__ MergePipe pipe;
+  __shared__ int sidx_a[2 * kBM];
   const int b = blockIdx.z, split = blockIdx.y;
-  const int m0 = blockIdx.x * kBM;
+  const int m0 = blockIdx.x * 2 * kBM;
+  const bool has1 = m0 + kBM < a.n_pruned;  // the second M tile holds pruned rows
   const int n_tiles_all = (a.keep + kMergeBN - 1) / kMergeBN;
   const int t0 = (int)((long long)n_tiles_all * split / a.n_split);
   const int t1 = (int)((long long)n_tiles_all * (split + 1) / a.n_split);
@@ -84,88 +107,163 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   const uint32_t sbase = smem_u32(smem_raw);
   uint8_t* stages = smem_raw + (((sbase + 1023u) & ~1023u) - sbase);
-  int* sidx_b = reinterpret_cast<int*>(stages + Cfg<kMergeBN>::kStagesBytes);
-  float* skinv = reinterpret_cast<float*>(sidx_b + kMergeMaxKeep);
+  float* skinv = reinterpret_cast<float*>(stages + (size_t)kMergeStages * kMergeStageBytes);
 
-  const int* pr = a.pruned + (size_t)b * a.n_pruned;
-  const int* kp = a.keep_idx + (size_t)b * a.keep;
-  for (int r = threadIdx.x; r < kBM; r += blockDim.x) sidx_a[r] = m0 + r < a.n_pruned ? pr[m0 + r] : 0;
-  for (int q = threadIdx.x; q < n_keep; q += blockDim.x) {
-    int j = kp[a0 + q];
-    if (j < 0 || j >= a.N_v) {
-      set_error(a.err, kErrBadDeviceArg);
-      j = 0;
-    }
-    sidx_b[q] = j;
-    skinv[q] = a.inv_v[(size_t)b * a.N_v + j];
-  }
   if (threadIdx.x == 0) {
     prefetch_tmap(&mapE);
-    pipe_init(pipe);
+    for (int s = 0; s < kMergeStages; ++s) {
+      mbar_init(&pipe.full[s], 1);
+      mbar_init(&pipe.empty[s], 1);
+    }
+    mbar_init(&pipe.acc_full, 1);
+    mbar_init(&pipe.acc_empty, 4);  // one arrival per epilogue warp
+    pipe.fail = 0;
+    fence_mbar_init();
   }
   if (threadIdx.x < 32) {
-    tmem_alloc(&pipe.tmem, Cfg<kMergeBN>::kTmemCols);
+    tmem_alloc(&pipe.tmem, kMergeTmemCols);
     tmem_relinquish();
   }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
 
+  // N columns of tile t: 256, or the kept rows of a ragged last tile rounded up to 16
+  auto tile_cols = [&](int t) { return min(kMergeBN, (n_keep - t * kMergeBN + 15) / 16 * 16); };
+
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (n_tiles > 0) {
     if (warp == 0) {
       if (lane == 0) {
-        // operands are contiguous rows of the permuted copy: [pruned | kept]
-        RowSrc ra{nullptr, b * a.N_v + m0, kBM};
-        RowSrc rb{nullptr, b * a.N_v + a.n_pruned + a0, n_tiles * kMergeBN};
-        producer<kMergeBN>(pipe, stages, &mapE, &mapE, ra, false, rb, false, n_tiles, n_k, a.err);
+        // operands are contiguous rows of the permuted copy [pruned | kept];
+        // rows past a tile's valid rows are computed and never used
+        const int row_a = b * a.N_v + m0;
+        const int row_b = b * a.N_v + a.n_pruned + a0;
+        int it = 0;
+        for (int t = 0; t < n_tiles && !pipe.fail; ++t) {
+          const bool b_hi = tile_cols(t) > kBM;  // the tile's second 128-row box is used
+          const uint32_t tx = (uint32_t)((has1 ? 2 : 1) * kABytes + (b_hi ? 2 : 1) * kABytes);
+          for (int kb = 0; kb < n_k; ++kb, ++it) {
+            const int s = it % kMergeStages;
+            const uint32_t ph = (uint32_t)(it / kMergeStages) & 1u;
+            if (pipe.fail || !mbar_wait(&pipe.empty[s], ph ^ 1u, a.err)) {
+              pipe.fail = 1;
+              break;
+            }
+            uint8_t* sa = stages + (size_t)s * kMergeStageBytes;
+            uint8_t* sb = sa + 2 * kABytes;
+            const int x = kb * kBK;
+            mbar_arrive_expect_tx(&pipe.full[s], tx);
+            tma_load_2d(sa, &mapE, x, row_a, &pipe.full[s]);
+            if (has1) tma_load_2d(sa + kABytes, &mapE, x, row_a + kBM, &pipe.full[s]);
+            tma_load_2d(sb, &mapE, x, row_b + t * kMergeBN, &pipe.full[s]);
+            if (b_hi) tma_load_2d(sb + kABytes, &mapE, x, row_b + t * kMergeBN + kBM, &pipe.full[s]);
+          }
+        }
       }
     } else if (warp == 1) {
-      if (lane == 0) mma_issuer<kMergeBN>(pipe, stages, n_tiles, n_k, a.err);
+      if (lane == 0) {
+        int it = 0;
+        for (int t = 0; t < n_tiles; ++t) {
+          if (!pipe.fail && !mbar_wait(&pipe.acc_empty, ((uint32_t)t & 1u) ^ 1u, a.err)) pipe.fail = 1;
+          const uint32_t idesc = idesc_bf16_f32(kBM, tile_cols(t));
+          for (int kb = 0; kb < n_k; ++kb, ++it) {
+            const int s = it % kMergeStages;
+            const uint32_t ph = (uint32_t)(it / kMergeStages) & 1u;
+            if (pipe.fail || !mbar_wait(&pipe.full[s], ph, a.err)) {
+              pipe.fail = 1;
+              break;
+            }
+            tc_fence_after();
+            const uint32_t sa = smem_u32(stages + (size_t)s * kMergeStageBytes);
+            const uint32_t sb = sa + 2 * kABytes;
+#pragma unroll
+            for (int k = 0; k < kBK / 16; ++k) {
+              const uint32_t acc = (kb > 0 || k > 0) ? 1u : 0u;
+              const uint64_t bd = smem_desc_sw128(sb + k * 32);
+              tc_mma_bf16(pipe.tmem, smem_desc_sw128(sa + k * 32), bd, idesc, acc);
+              if (has1) tc_mma_bf16(pipe.tmem + kMergeBN, smem_desc_sw128(sa + kABytes + k * 32), bd, idesc, acc);
+            }
+            tc_commit(&pipe.empty[s]);
+          }
+          tc_commit(&pipe.acc_full);  // arrives when every MMA above has completed
+          if (pipe.fail) break;
+        }
+      }
     } else {
-      // epilogue: row r of the M tile, running (max, first index) over the range
+      // the epilogue warps fill the index tables while the first stages load
+      const int* pr = a.pruned + (size_t)b * a.n_pruned;
+      const int* kp = a.keep_idx + (size_t)b * a.keep;
+      const int et = threadIdx.x - 64;
+      for (int r = et; r < 2 * kBM; r += 128) sidx_a[r] = m0 + r < a.n_pruned ? pr[m0 + r] : 0;
+      for (int q = et; q < n_keep; q += 128) {
+        int j = kp[a0 + q];
+        if (j < 0 || j >= a.N_v) {
+          set_error(a.err, kErrBadDeviceArg);
+          j = 0;
+        }
+        skinv[q] = a.inv_v[(size_t)b * a.N_v + j];
+      }
+      asm volatile("bar.sync 1, 128;" ::: "memory");  // tables complete (epilogue warps)
+      // epilogue: row r of each M tile, running (max, first index) over the range
       const int quad = warp & 3;
       const int r = quad * 32 + lane;
-      const bool rv = m0 + r < a.n_pruned;
-      float best = -INFINITY;
-      int bidx = 0x7fffffff;
+      float best0 = -INFINITY, best1 = -INFINITY;
+      int bidx0 = 0x7fffffff, bidx1 = 0x7fffffff;
+      bool ok = true;
       for (int t = 0; t < n_tiles; ++t) {
-        const int buf = t & 1;
-        mbar_wait(&pipe.acc_full[buf], (uint32_t)(t >> 1) & 1u, a.err);
+        ok = warp_mbar_wait(&pipe.acc_full, (uint32_t)t & 1u, a.err) && !pipe.fail;
+        if (!ok) break;
         tc_fence_after();
-        const uint32_t taddr = pipe.tmem + ((uint32_t)(quad * 32) << 16) + (uint32_t)(buf * kMergeBN);
+        const uint32_t taddr = pipe.tmem + ((uint32_t)(quad * 32) << 16);
+        const int ncb = (tile_cols(t) + 31) / 32;
 #pragma unroll 1
-        for (int cb = 0; cb < kMergeBN / 32; ++cb) {
-          float v[32];
-          tmem_ld32(taddr + cb * 32, v);
+        for (int cb = 0; cb < ncb; ++cb) {
+          float v0[32], v1[32];
+          tmem_ld32(taddr + cb * 32, v0);
+          if (has1) tmem_ld32(taddr + kMergeBN + cb * 32, v1);
           tc_wait_ld();
           const int q0 = t * kMergeBN + cb * 32;  // position within the range
 #pragma unroll
           for (int i = 0; i < 32; ++i) {
             const int q = q0 + i;
             if (q < n_keep) {
-              const float x = v[i] * skinv[q];
-              if (x > best) {
-                best = x;
-                bidx = a0 + q;
+              const float sk = skinv[q];
+              const float x0 = v0[i] * sk;
+              if (x0 > best0) {
+                best0 = x0;
+                bidx0 = a0 + q;
+              }
+              if (has1) {
+                const float x1 = v1[i] * sk;
+                if (x1 > best1) {
+                  best1 = x1;
+                  bidx1 = a0 + q;
+                }
               }
             }
           }
         }
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive(&pipe.acc_empty[buf]);
+        if (lane == 0) mbar_arrive(&pipe.acc_empty);
       }
-      if (rv && !pipe.fail) {
-        const size_t o = ((size_t)split * a.B + b) * a.N_v + sidx_a[r];
-        a.ws_best[o] = best;
-        a.ws_bidx[o] = bidx;
+      if (ok && !pipe.fail) {
+        const size_t o = ((size_t)split * a.B + b) * a.N_v;
+        if (m0 + r < a.n_pruned) {
+          a.ws_best[o + sidx_a[r]] = best0;
+          a.ws_bidx[o + sidx_a[r]] = bidx0;
+        }
+        if (m0 + kBM + r < a.n_pruned) {
+          a.ws_best[o + sidx_a[kBM + r]] = best1;
+          a.ws_bidx[o + sidx_a[kBM + r]] = bidx1;
+        }
       }
     }
   }
   tc_fence_before();
   __syncthreads();
-  if (threadIdx.x < 32) tmem_dealloc(pipe.tmem, Cfg<kMergeBN>::kTmemCols);
+  if (threadIdx.x < 32) tmem_dealloc(pipe.tmem, kMergeTmemCols);
 }
 
 // relevance_fused_tc: one read of the visual rows gives, per 128-row tile of
@@ -409,10 +507,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (warp == 0) {
     if (lane == 0) {
-      RowSrc ra{nullptr, b * N_t_max, kBM};
-      RowSrc rb{nullptr, b * N_t_max, kCritBN};
+      RowSrc ra{b * N_t_max, kBM};
+      RowSrc rb{b * N_t_max, kCritBN};
       // both operands are the same text rows: one load per K slice
-      producer<kCritBN>(pipe, stages, &mapT, &mapT, ra, false, rb, false, 1, n_k, err, k0, true);
+      producer<kCritBN>(pipe, stages, &mapT, &mapT, ra, rb, 1, n_k, err, k0, true);
     }
   } else if (warp == 1) {
     if (lane == 0) mma_issuer<kCritBN>(pipe, stages, 1, n_k, err, true);
@@ -452,11 +550,11 @@ cudaError_t set_smem(K kernel, size_t bytes, bool* done) {
 }  // namespace
 
 size_t merge_tc_smem() {
-  return Cfg<kMergeBN>::kStagesBytes + 1024 + (size_t)kMergeMaxKeep * (sizeof(int) + sizeof(float));
+  return (size_t)kMergeStages * kMergeStageBytes + 1024 + (size_t)kMergeMaxKeep * sizeof(float);
 }
 
 int merge_tc_split(int B, int N_v, int keep, int num_sms) {
-  const int m_tiles = B * ((N_v - keep + kBM - 1) / kBM);
+  const int m_tiles = B * ((N_v - keep + 2 * kBM - 1) / (2 * kBM));  // CTAs: pairs of M tiles
   const int n_tiles = (keep + kMergeBN - 1) / kMergeBN;
   int best = 1;
   long long best_cost = -1;
@@ -510,7 +608,7 @@ cudaError_t merge_argmax_tc_launch(const SimArgs& a, const int* keep_idx, int ke
   m.ws_best = ws_best;
   m.ws_bidx = ws_bidx;
   m.err = a.err;
-  dim3 grid((n_pruned + kBM - 1) / kBM, n_split, a.B);
+  dim3 grid((n_pruned + 2 * kBM - 1) / (2 * kBM), n_split, a.B);
   merge_argmax_tc<<<grid, kThreads, smem, s>>>(m, mapE);
   return cudaGetLastError();
 }

@@ -1,8 +1,7 @@
 // Warp-specialised tcgen05 "NT" Gram core for the pre-LLM pass (Sec. 4.3):
 //   D[M x N] = A[M x K] * B[N x K]^T, bf16 operands, fp32 accumulation in TMEM,
-// with A and B rows fetched by 2-D TMA (128-byte swizzle), either as a block of
-// consecutive rows or gathered by row index with tile::gather4 (boxes one row
-// high, four rows per instruction).
+// with A and B fetched by 2-D TMA (128-byte swizzle) as blocks of consecutive
+// rows (boxes of 128 rows).
 //
 // One CTA owns one 128-row M tile and sweeps a range of BN-column N tiles
 // (BN = 128 or 256):
@@ -39,16 +38,6 @@ struct Cfg {
   static constexpr uint32_t kTmemCols = 2 * BN;  // two accumulators
 };
 
-__device__ __forceinline__ void tma_gather4(void* smem_dst, const CUtensorMap* map, int x, int r0,
-                                            int r1, int r2, int r3, uint64_t* bar) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.tile::gather4.mbarrier::complete_tx::bytes "
-      "[%0], [%1, {%2, %3, %4, %5, %6}], [%7];" ::"r"(smem_u32(smem_dst)),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(r0), "r"(r1), "r"(r2), "r"(r3),
-      "r"(smem_u32(bar))
-      : "memory");
-}
-
 struct Pipe {
   uint64_t full[kStages];
   uint64_t empty[kStages];
@@ -58,28 +47,18 @@ struct Pipe {
   volatile int fail;
 };
 
-// Row source of an operand: either rows base + r (contiguous) or rows idx[r].
+// Row source of an operand: rows base + r, r < count (rows >= count are loaded
+// but their results are masked by the caller).
 struct RowSrc {
-  const int* idx;  // in shared memory, or null for contiguous rows
-  int base;        // first row (contiguous) or offset added to idx[r]
-  int count;       // valid rows; rows >= count load row `base` (masked later)
-  __device__ __forceinline__ int row(int r) const {
-    const int rr = r < count ? r : 0;
-    return idx ? base + idx[rr] : base + rr;
-  }
+  int base;   // first row
+  int count;  // valid rows
 };
 
-// Loads rows [r0, r0 + nrows) of an operand for K slice x into a 128-B-row tile.
+// Loads rows [r0, r0 + nrows) of an operand for K slice x into a 128-B-row tile,
+// in boxes of 128 rows (the tensor map's box height).
 __device__ __forceinline__ void load_rows(uint8_t* dst, const CUtensorMap* map, const RowSrc& src,
-                                          int r0, int nrows, int x, uint64_t* bar, bool gather) {
-  if (gather) {
-    for (int r = 0; r < nrows; r += 4)
-      tma_gather4(dst + r * 128, map, x, src.row(r0 + r), src.row(r0 + r + 1), src.row(r0 + r + 2),
-                  src.row(r0 + r + 3), bar);
-  } else {
-    // contiguous: boxes of 128 rows (the tensor map's box height)
-    for (int r = 0; r < nrows; r += 128) tma_load_2d(dst + r * 128, map, x, src.base + r0 + r, bar);
-  }
+                                          int r0, int nrows, int x, uint64_t* bar) {
+  for (int r = 0; r < nrows; r += 128) tma_load_2d(dst + r * 128, map, x, src.base + r0 + r, bar);
 }
 
 // Producer: for each N tile t in [0, n_tiles), all K slices.
@@ -87,9 +66,9 @@ template <int BN>
 // k0: first K slice (a split-K part starts past the others' slices); b_is_a:
 // the B operand is the A tile itself (a Gram of one row block), loaded once
 __device__ __forceinline__ void producer(Pipe& p, uint8_t* stages, const CUtensorMap* mapA,
-                                         const CUtensorMap* mapB, const RowSrc& a, bool gatherA,
-                                         const RowSrc& b, bool gatherB, int n_tiles, int n_k,
-                                         unsigned* err, int k0 = 0, bool b_is_a = false) {
+                                         const CUtensorMap* mapB, const RowSrc& a, const RowSrc& b,
+                                         int n_tiles, int n_k, unsigned* err, int k0 = 0,
+                                         bool b_is_a = false) {
   int it = 0;
   for (int t = 0; t < n_tiles && !p.fail; ++t) {
     for (int kb = 0; kb < n_k; ++kb, ++it) {
@@ -102,8 +81,8 @@ __device__ __forceinline__ void producer(Pipe& p, uint8_t* stages, const CUtenso
       uint8_t* sa = stages + (size_t)s * Cfg<BN>::kStageBytes;
       uint8_t* sb = sa + kABytes;
       mbar_arrive_expect_tx(&p.full[s], b_is_a ? (uint32_t)kABytes : (uint32_t)Cfg<BN>::kStageBytes);
-      load_rows(sa, mapA, a, 0, kBM, (k0 + kb) * kBK, &p.full[s], gatherA);
-      if (!b_is_a) load_rows(sb, mapB, b, t * BN, BN, (k0 + kb) * kBK, &p.full[s], gatherB);
+      load_rows(sa, mapA, a, 0, kBM, (k0 + kb) * kBK, &p.full[s]);
+      if (!b_is_a) load_rows(sb, mapB, b, t * BN, BN, (k0 + kb) * kBK, &p.full[s]);
     }
   }
 }
