@@ -760,13 +760,66 @@ def run_gb300(args, dist):
         c = copies[i % len(copies)]
         ah(c["Q"], c["K"], c["V"], c["hidden"], c["pos"], c["text_start"], c["text_len"], c["seq_len"], vis)
 
+    def time_lanes(make, reps):
+        # the same steps on the S concurrent streams of the headline: one step
+        # object per lane (own outputs and workspace) over that lane's inputs,
+        # graphs of GRAPH_CHUNK steps per stream; seconds per step (one batch)
+        objs = [make(cs[0]) for cs, _ in lanes]
+
+        def run(n):
+            main = torch.cuda.current_stream(dev)
+            ev = torch.cuda.Event()
+            ev.record(main)
+            for ls in lane_streams:
+                ls.wait_event(ev)
+            for i in range(n):
+                cs = lanes[i % S][0]
+                c = cs[(i // S) % len(cs)]
+                objs[i % S](c["Q"], c["K"], c["V"], c["hidden"], c["pos"], c["text_start"], c["text_len"],
+                            c["seq_len"], vis, stream=lane_streams[i % S])
+            for ls in lane_streams:
+                e2 = torch.cuda.Event()
+                e2.record(ls)
+                main.wait_event(e2)
+
+        run(3 * S)
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            run(GRAPH_CHUNK * S)
+        torch.cuda.synchronize()
+        g.replay()  # untimed first launch
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        for _ in range(reps):
+            g.replay()
+        b.record()
+        torch.cuda.synchronize()
+        return a.elapsed_time(b) / 1e3 / (reps * GRAPH_CHUNK * S)
+
+    def make_vh(c):
+        return P.VisualHeadsPruneStep(c["Q"], c["K"], c["V"], c["hidden"], c["pos"], w.n_t[1], nv, keep,
+                                      min(N_VIS, w.H_q), algo=algo, want_scores=False, want_conf=False,
+                                      flags=P.PRUNE_OVERLAP_PREVIOUS)
+
+    def make_ah(c):
+        return P.PruneStep(c["Q"], c["K"], c["V"], c["hidden"], c["pos"], None, w.n_t[1], nv, keep,
+                           algo=algo, want_scores=False, flags=P.PRUNE_OVERLAP_PREVIOUS)
+
     next_rows = {}
-    for name, fn, extra in (("visual_heads", vh_i, {"n_vis": min(N_VIS, w.H_q), "heads_scored": w.H_q}),
-                            ("all_heads", ah_i, {"heads_scored": w.H_q})):
+    for name, fn, make, extra in (
+            ("visual_heads", vh_i, make_vh, {"n_vis": min(N_VIS, w.H_q), "heads_scored": w.H_q}),
+            ("all_heads", ah_i, make_ah, {"heads_scored": w.H_q})):
         t = time_graph(fn, reps)
         gbs = ab_all["path"] / t / 1e9
         next_rows[name] = dict(extra, us_per_step=t * 1e6, samples_per_s=w.B / t,
                                algorithmic_bytes=ab_all["path"], achieved_gbs=gbs, frac=gbs / peak)
+        if S > 1:
+            tc = time_lanes(make, reps)
+            gc = ab_all["path"] / tc / 1e9
+            next_rows[name]["streams"] = dict(streams=S, us_per_step=tc * 1e6, samples_per_s=w.B / tc,
+                                              achieved_gbs=gc, frac=gc / peak)
     rc, bits = P.provip_device_status(clear=True)
     if rc != 0:
         raise RuntimeError(f"device status {rc} {bits} after the next-row legs")
