@@ -88,17 +88,27 @@ def _cos_argmax_band(Ev, rows, keep, assign_gpu, tol):
 
 @pytest.mark.parametrize("name", [w.name for w in synth.WORKLOADS])
 def test_merge_matches_oracle(name):
+    """The whole batch in one call (the launch configuration the benchmark
+    times: several kept-row splits, ragged last tiles), each sample with the
+    oracle's own keep set; the first and last samples checked against the
+    oracle."""
     w, cpu, g = inputs(name)
-    b = 0
-    Ev = f64(cpu["emb_v"][b])
-    n = int(cpu["text_len"][b])
-    _, m_ref = oracle.crit_text(f64(cpu["emb_t"][b, :n]))
-    keep = oracle.topk(oracle.relevance(f64(cpu["emb_t"][b, :n]), m_ref, Ev), w.keep_pre)
-    assign, merged = P.provip_merge(g["emb_v"][b:b + 1].contiguous(), torch.from_numpy(keep[None]).to(DEV))
+    keeps = []
+    for b in range(w.B):
+        n = int(cpu["text_len"][b])
+        Et = f64(cpu["emb_t"][b, :n])
+        _, m_ref = oracle.crit_text(Et)
+        keeps.append(oracle.topk(oracle.relevance(Et, m_ref, f64(cpu["emb_v"][b])), w.keep_pre))
+    assign, merged = P.provip_merge(g["emb_v"], torch.from_numpy(np.stack(keeps)).to(DEV))
     torch.cuda.synchronize()
-    a_gpu = assign[0].cpu().numpy()
+    for b in sorted({0, w.B - 1}):
+        _check_merge_sample(w, f64(cpu["emb_v"][b]), keeps[b], assign[b].cpu().numpy(),
+                            merged[b].float().cpu().numpy().astype(np.float64), f"{name}[{b}]")
+
+
+def _check_merge_sample(w, Ev, keep, a_gpu, mg, what):
     pruned = np.setdiff1d(np.arange(w.N_v), keep)
-    assert np.array_equal(a_gpu[keep], np.arange(w.keep_pre)), "kept rows must be their own centroid"
+    assert np.array_equal(a_gpu[keep], np.arange(w.keep_pre)), f"{what}: kept rows must be their own centroid"
     exact = w.N_v <= 1000
     if exact:
         a_ref, mg_ref = oracle.merge(Ev, keep)
@@ -116,8 +126,7 @@ def test_merge_matches_oracle(name):
     same = a_gpu[rows] == a_ref[rows]
     if not same.all():
         _cos_argmax_band(Ev, rows[~same], keep, a_gpu, tol)
-    assert same.mean() > 0.95
-    mg = merged[0].float().cpu().numpy().astype(np.float64)
+    assert same.mean() > 0.95, what
     if exact:
         # centroids whose member set is identical: within one output ulp
         ok = np.array([np.array_equal(np.flatnonzero(a_gpu == a), np.flatnonzero(a_ref == a))
@@ -125,7 +134,7 @@ def test_merge_matches_oracle(name):
         ulp = np.spacing(np.abs(mg_ref).astype(np.float32)).astype(np.float64) if w.dtype == "f32" else \
             2.0 ** (np.floor(np.log2(np.maximum(np.abs(mg_ref), 1e-30))) - 7)
         err = np.abs(mg - mg_ref)
-        assert np.all(err[ok] <= ulp[ok] * 1.0001 + 1e-37), "merged rows beyond one ulp"
+        assert np.all(err[ok] <= ulp[ok] * 1.0001 + 1e-37), f"{what}: merged rows beyond one ulp"
     else:
         # at full size: every merged row is the mean of its GPU-assigned members
         for a in np.random.default_rng(6).choice(w.keep_pre, 16, replace=False):
