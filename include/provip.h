@@ -102,6 +102,15 @@ int provip_version(void);
  * PROVIP_ERR_INVALID_ARG if BAD_ARG is set, PROVIP_OK otherwise. */
 int provip_device_status(unsigned *bits, int clear);
 
+/* Failure-detection self test: enqueues one CTA on `stream` whose first thread
+ * waits, through the same bounded wait every kernel of the library uses, on an
+ * mbarrier that nothing ever completes. After the wait budget (2 s) the wait
+ * gives up, sets PROVIP_DEVSTAT_TIMEOUT in the device status word and the
+ * kernel returns, so the context stays usable; provip_device_status() then
+ * reports PROVIP_ERR_TIMEOUT. Returns PROVIP_OK once launched, or
+ * PROVIP_ERR_CUDA. */
+int provip_selftest_wait_timeout(void *stream);
+
 /* ------------------------------------------------------------------------
  * Pre-LLM pass (Sec. 4.2-4.3)
  * ---------------------------------------------------------------------- */

@@ -7,6 +7,7 @@
 #include <string.h>
 
 #include "../../include/provip.h"
+#include "common.cuh"
 #include "kernels.h"
 
 using namespace provip;
@@ -402,6 +403,28 @@ extern "C" int provip_device_status(unsigned* bits, int clear) {
   if (bits) *bits = v;
   if (v & PROVIP_DEVSTAT_TIMEOUT) return PROVIP_ERR_TIMEOUT;
   if (v & PROVIP_DEVSTAT_BAD_ARG) return PROVIP_ERR_INVALID_ARG;
+  return PROVIP_OK;
+}
+
+namespace {
+// one thread waits on an mbarrier whose single expected arrival never comes
+__global__ void selftest_wait_kernel(unsigned* err) {
+  __shared__ uint64_t bar;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    fence_mbar_init();
+    mbar_wait(&bar, 0, err);  // gives up after the wait budget and sets kErrTimeout
+  }
+}
+}  // namespace
+
+extern "C" int provip_selftest_wait_timeout(void* stream) {
+  DevInfo* d;
+  int rc = dev_info(&d);
+  if (rc) return rc;
+  selftest_wait_kernel<<<1, 32, 0, static_cast<cudaStream_t>(stream)>>>(d->status);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_fail(e, "selftest_wait_kernel launch");
   return PROVIP_OK;
 }
 

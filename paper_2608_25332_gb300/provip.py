@@ -23,6 +23,7 @@ ERR_UNSUPPORTED = -2
 ERR_WORKSPACE = -3
 ERR_CUDA = -4
 ERR_TIMEOUT = -5
+DEVSTAT_TIMEOUT, DEVSTAT_BAD_ARG = 1, 2  # bits of the device status word
 F32, BF16 = 0, 1
 ALGO_AUTO, ALGO_SIMT, ALGO_TCGEN05, ALGO_TCGEN05_TWOPASS = 0, 1, 2, 3
 ALGO_TCGEN05_STREAM, ALGO_TCGEN05_CLUSTER = 4, 5
@@ -38,6 +39,7 @@ _SIGS = {
     "provip_last_error": (ctypes.c_char_p, []),
     "provip_version": (_I, []),
     "provip_device_status": (_I, [_P, _I]),
+    "provip_selftest_wait_timeout": (_I, [_P]),
     "provip_crit_text_workspace_size": (_Z, [_I, _I, _I]),
     "provip_crit_text": (_I, [_P, _I, _I, _I, _P, _I, _P, _P, _P, _Z, _P]),
     "provip_relevance_workspace_size": (_Z, [_I, _I, _I, _I]),
@@ -154,6 +156,13 @@ def provip_device_status(clear: bool = True):
     bits = ctypes.c_uint(0)
     rc = lib().provip_device_status(ctypes.byref(bits), 1 if clear else 0)
     return rc, bits.value
+
+
+def provip_selftest_wait_timeout(device="cuda:0"):
+    """Enqueues the failure-detection self test: a bounded wait that nothing
+    completes gives up after 2 s and sets the TIMEOUT bit of the device status
+    word (read it with provip_device_status)."""
+    _check(lib().provip_selftest_wait_timeout(_stream(torch.device(device))), "provip_selftest_wait_timeout")
 
 
 def provip_version() -> int:
