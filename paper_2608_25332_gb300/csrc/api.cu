@@ -6,6 +6,9 @@
 #include <stdio.h>
 #include <string.h>
 
+#include <atomic>
+#include <mutex>
+
 #include "../../include/provip.h"
 #include "common.cuh"
 #include "kernels.h"
@@ -32,27 +35,35 @@ int cuda_fail(cudaError_t e, const char* where) {
 }
 
 struct DevInfo {
-  bool init = false;
+  std::atomic<bool> init{false};  // set (release) once sms and status are written
   int sms = 0;
   unsigned* status = nullptr;
 };
 DevInfo g_dev[64];
+std::mutex g_dev_mu;  // serialises the first lookup of each device
 
-// per-device facts, looked up once with that device current
+// per-device facts, looked up once with that device current (safe from several
+// host threads: the first caller fills them under the lock, later ones read them
+// after an acquire of `init`)
 int dev_info(DevInfo** out) {
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
   if (dev < 0 || dev >= 64) return fail(PROVIP_ERR_UNSUPPORTED, "device ordinal %d >= 64", dev);
   DevInfo& d = g_dev[dev];
-  if (!d.init) {
-    e = cudaDeviceGetAttribute(&d.sms, cudaDevAttrMultiProcessorCount, dev);
-    if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceGetAttribute");
-    void* p = nullptr;
-    e = cudaGetSymbolAddress(&p, g_provip_status);
-    if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress(status)");
-    d.status = static_cast<unsigned*>(p);
-    d.init = true;
+  if (!d.init.load(std::memory_order_acquire)) {
+    std::lock_guard<std::mutex> lock(g_dev_mu);
+    if (!d.init.load(std::memory_order_relaxed)) {
+      int sms = 0;
+      e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+      if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceGetAttribute");
+      void* p = nullptr;
+      e = cudaGetSymbolAddress(&p, g_provip_status);
+      if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress(status)");
+      d.sms = sms;
+      d.status = static_cast<unsigned*>(p);
+      d.init.store(true, std::memory_order_release);
+    }
   }
   *out = &d;
   return PROVIP_OK;

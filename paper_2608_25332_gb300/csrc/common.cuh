@@ -10,6 +10,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <atomic>  // host-side one-time launch configuration flags
+
 namespace provip {
 
 // ---------------------------------------------------------------------------

@@ -257,7 +257,7 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(const CompactA
 }  // namespace
 
 cudaError_t compact_launch(const CompactArgs& a, int num_sms, cudaStream_t s, bool pdl, bool allow_deep) {
-  static bool configured[64] = {false};
+  static std::atomic<bool> configured[64];  // per device, zero-initialised
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev >= 0 && dev < 64 && !configured[dev]) {

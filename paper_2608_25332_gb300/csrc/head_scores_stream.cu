@@ -387,7 +387,7 @@ __global__ void __launch_bounds__(kThreads, 2)
 template <bool CONF>
 cudaError_t launch(const HSArgs& a, const CUtensorMap* tmQ, const CUtensorMap* tmK, cudaStream_t s,
                    bool pdl) {
-  static bool configured[64] = {false};
+  static std::atomic<bool> configured[64];  // per device, zero-initialised
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev >= 0 && dev < 64 && !configured[dev]) {

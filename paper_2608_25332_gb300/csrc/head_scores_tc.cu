@@ -280,7 +280,7 @@ __global__ void __launch_bounds__(kTcThreads) hs_probs_tc(const HSArgs a,
 cudaError_t hs_launch_tc(const HSArgs& a, const CUtensorMap* tmQ, const CUtensorMap* tmK,
                          cudaStream_t s, ConfGeom* geom) {
   if (geom) *geom = ConfGeom{a.vis_start, kTile, a.n_vc};
-  static bool configured[64] = {false};
+  static std::atomic<bool> configured[64];  // per device, zero-initialised
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev >= 0 && dev < 64 && !configured[dev]) {

@@ -843,7 +843,7 @@ cudaError_t crit_text_launch(const SimArgs& a, uint8_t* mask, float* r_out, floa
   } else {
     crit_gram_kernel<__nv_bfloat16><<<g, 256, 0, s>>>(a, G);
   }
-  static bool configured[64] = {false};
+  static std::atomic<bool> configured[64];  // per device, zero-initialised
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev >= 0 && dev < 64 && !configured[dev]) {
@@ -893,7 +893,7 @@ cudaError_t relevance_launch(const SimArgs& a, const uint8_t* mask, float* inv_v
   // where the rows fit the shared-memory batch, else in two passes
   const bool fused = norm_sum_supported(a);
   if (fused) {
-    static bool configured[64] = {false};
+    static std::atomic<bool> configured[64];  // per device, zero-initialised
     int dev = 0;
     cudaGetDevice(&dev);
     if (dev >= 0 && dev < 64 && !configured[dev]) {
@@ -964,7 +964,7 @@ cudaError_t merge_launch(const SimArgs& a, const int* keep_idx, int keep, const 
     int* mem = reinterpret_cast<int*>(ws_best);
     merge_sort_kernel<<<a.B, 1024, 0, s>>>(assign, a.N_v, keep, cnt, off, cur, mem);
     dim3 gm(keep, a.B);
-    static bool configured[64] = {false};
+    static std::atomic<bool> configured[64];  // per device, zero-initialised
     int dev = 0;
     cudaGetDevice(&dev);
     if (dev >= 0 && dev < 64 && !configured[dev]) {

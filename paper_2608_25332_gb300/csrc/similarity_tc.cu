@@ -540,10 +540,10 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 template <typename K>
-cudaError_t set_smem(K kernel, size_t bytes, bool* done) {
-  if (*done) return cudaSuccess;
+cudaError_t set_smem(K kernel, size_t bytes, std::atomic<bool>* done) {
+  if (done->load()) return cudaSuccess;
   cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
-  if (e == cudaSuccess) *done = true;
+  if (e == cudaSuccess) done->store(true);  // idempotent: concurrent first calls may both set it
   return e;
 }
 
@@ -581,7 +581,7 @@ bool merge_tc_supported(const SimArgs& a, int keep, int n_split) {
 cudaError_t merge_argmax_tc_launch(const SimArgs& a, const int* keep_idx, int keep, const float* inv_v,
                                    const int* pruned, void* perm, int n_split,
                                    float* ws_best, int* ws_bidx, cudaStream_t s) {
-  static bool smem_set[64] = {false};
+  static std::atomic<bool> smem_set[64];  // per device, zero-initialised
   int dev = 0;
   cudaGetDevice(&dev);
   const size_t smem = merge_tc_smem();
@@ -624,7 +624,7 @@ size_t relevance_fused_floats(int B, int N_v, int N_t_max) {
 
 cudaError_t relevance_tc_launch(const SimArgs& a, const uint8_t* mask, const float* inv_t, float* inv_v,
                                 float* p, float* ws, int num_sms, cudaStream_t s) {
-  static bool smem_set[64] = {false};
+  static std::atomic<bool> smem_set[64];  // per device, zero-initialised
   int dev = 0;
   cudaGetDevice(&dev);
   constexpr size_t kSmemMax = 200 * 1024;
@@ -675,7 +675,7 @@ int crit_splits(int N_t_max, int D, int dtype) {
 }
 
 cudaError_t crit_gram_tc_launch(const SimArgs& a, float* G, cudaStream_t s) {
-  static bool smem_set[64] = {false};
+  static std::atomic<bool> smem_set[64];  // per device, zero-initialised
   int dev = 0;
   cudaGetDevice(&dev);
   const size_t smem = Cfg<kCritBN>::kStagesBytes + 1024;

@@ -158,7 +158,7 @@ __global__ void __launch_bounds__(kRankThreads) topk_rank_kernel(const TopkArgs 
 }  // namespace
 
 cudaError_t topk_launch(const TopkArgs& a, cudaStream_t s, bool pdl) {
-  static bool configured[64] = {false};
+  static std::atomic<bool> configured[64];  // per device, zero-initialised
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev >= 0 && dev < 64 && !configured[dev]) {
