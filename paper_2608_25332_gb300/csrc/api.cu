@@ -9,6 +9,8 @@
 #include <atomic>
 #include <mutex>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "../../include/provip.h"
 #include "common.cuh"
 #include "kernels.h"
@@ -21,6 +23,16 @@ __device__ unsigned int g_provip_status;
 namespace {
 
 thread_local char g_last_error[512] = {0};
+
+// An NVTX range named after the entry point for the duration of the host call,
+// so that a profiler timeline attributes the kernels each call enqueues to the
+// call (header-only NVTX: a no-op unless a profiling tool is attached).
+struct NvtxRange {
+  explicit NvtxRange(const char* name) { nvtxRangePushA(name); }
+  ~NvtxRange() { nvtxRangePop(); }
+  NvtxRange(const NvtxRange&) = delete;
+  NvtxRange& operator=(const NvtxRange&) = delete;
+};
 
 int fail(int code, const char* fmt, ...) {
   va_list ap;
@@ -457,6 +469,7 @@ extern "C" size_t provip_crit_text_workspace_size(int B, int N_t_max, int D) {
 extern "C" int provip_crit_text(const void* emb_t, int B, int N_t_max, int D, const int* text_len,
                                 int dtype, uint8_t* mask_out, float* r_out, void* ws,
                                 size_t ws_bytes, void* stream) {
+  NvtxRange nvtx_range("provip_crit_text");
   int rc = sim_validate_common(emb_t, B, N_t_max, D, dtype, "crit_text");
   if (rc) return rc;
   if (!text_len || !mask_out) return fail(PROVIP_ERR_INVALID_ARG, "crit_text: null text_len/mask_out");
@@ -492,6 +505,7 @@ extern "C" size_t provip_relevance_workspace_size(int B, int N_v, int D, int N_t
 extern "C" int provip_relevance(const void* emb_v, int B, int N_v, int D, const void* emb_t,
                                 const int* text_len, int N_t_max, const uint8_t* crit_mask,
                                 int dtype, float* p_out, void* ws, size_t ws_bytes, void* stream) {
+  NvtxRange nvtx_range("provip_relevance");
   int rc = sim_validate_common(emb_v, B, N_v, D, dtype, "relevance");
   if (rc) return rc;
   if ((rc = sim_validate_common(emb_t, B, N_t_max, D, dtype, "relevance"))) return rc;
@@ -510,6 +524,7 @@ extern "C" int provip_relevance(const void* emb_v, int B, int N_v, int D, const 
 }
 
 extern "C" int provip_topk(const float* scores, int B, int N, int k, int* idx_out, void* stream) {
+  NvtxRange nvtx_range("provip_topk");
   if (!scores || !idx_out) return fail(PROVIP_ERR_INVALID_ARG, "topk: null pointer");
   if (B < 1 || N < 1 || k < 1 || k > N) return fail(PROVIP_ERR_INVALID_ARG, "topk: need 1 <= k <= N");
   if (N > kTopkMaxN) return fail(PROVIP_ERR_UNSUPPORTED, "topk: N > %d", kTopkMaxN);
@@ -557,6 +572,7 @@ static int merge_validate(const void* emb_v, int B, int N_v, int D, const int* k
 extern "C" int provip_merge(const void* emb_v, int B, int N_v, int D, const int* keep_idx, int keep,
                             int dtype, int* assign_out, void* merged_out, void* ws, size_t ws_bytes,
                             void* stream) {
+  NvtxRange nvtx_range("provip_merge");
   int rc = merge_validate(emb_v, B, N_v, D, keep_idx, keep, dtype, assign_out);
   if (rc) return rc;
   if ((rc = check_ws(provip_merge_workspace_size(B, N_v, D, keep), ws, ws_bytes, "merge"))) return rc;
@@ -607,6 +623,7 @@ extern "C" int provip_similarity_reduce(const void* emb_v, int B, int N_v, int D
                                         int* idx_out, void* merged_out_or_null,
                                         float* p_out_or_null, uint8_t* mask_out_or_null, void* ws,
                                         size_t ws_bytes, void* stream) {
+  NvtxRange nvtx_range("provip_similarity_reduce");
   int rc = sim_validate_common(emb_v, B, N_v, D, dtype, "similarity_reduce");
   if (rc) return rc;
   if ((rc = sim_validate_common(emb_t, B, N_t_max, D, dtype, "similarity_reduce"))) return rc;
@@ -673,6 +690,7 @@ extern "C" int provip_head_scores(const void* Q, const void* K, int B, int L_max
                                   const int* text_len, const uint8_t* row_mask_or_null, int N_t_max,
                                   int vis_start, int N_v, const int* seq_len, int dtype, int algo,
                                   float* scores, void* ws, size_t ws_bytes, void* stream) {
+  NvtxRange nvtx_range("provip_head_scores");
   algo = resolve_algo(algo, dtype);
   int rc = hs_validate(Q, K, B, L_max, H_q, H_kv, d_h, head_list, H_sel, text_start, text_len,
                        N_t_max, vis_start, N_v, seq_len, dtype, algo);
@@ -702,6 +720,7 @@ extern "C" int provip_compact(const int* idx, int B, int N_v, int keep, const vo
                               int P, const int* seq_len, int L_max, int vis_start, int dtype,
                               void* hidden_out, void* K_out, void* V_out, int* pos_out,
                               int* seq_len_out, void* stream) {
+  NvtxRange nvtx_range("provip_compact");
   int rc = compact_validate(idx, B, N_v, keep, hidden, D, K, V, H_kv, d_h, pos, P, seq_len, L_max,
                             vis_start, dtype, hidden_out, K_out, V_out, pos_out);
   if (rc) return rc;
@@ -720,6 +739,7 @@ extern "C" int provip_topk_compact(const float* scores, int B, int N_v, int keep
                                    int vis_start, int dtype, void* hidden_out, void* K_out,
                                    void* V_out, int* pos_out, int* idx_out, int* seq_len_out,
                                    void* stream) {
+  NvtxRange nvtx_range("provip_topk_compact");
   if (!scores || !idx_out) return fail(PROVIP_ERR_INVALID_ARG, "topk_compact: null scores/idx_out");
   int rc = compact_validate(idx_out, B, N_v, keep, hidden, D, K, V, H_kv, d_h, pos, P, seq_len,
                             L_max, vis_start, dtype, hidden_out, K_out, V_out, pos_out);
@@ -790,6 +810,7 @@ extern "C" int provip_head_topk(const void* Q, const void* K, int B, int L_max, 
                                 int vis_start, int N_v, const int* seq_len, int keep, int dtype,
                                 int algo, int* idx_out, float* scores_out_or_null, void* ws,
                                 size_t ws_bytes, void* stream) {
+  NvtxRange nvtx_range("provip_head_topk");
   return head_topk_impl(Q, K, B, L_max, H_q, H_kv, d_h, head_list, H_sel, text_start, text_len,
                         row_mask_or_null, N_t_max, vis_start, N_v, seq_len, keep, dtype, algo,
                         idx_out, scores_out_or_null, ws, ws_bytes, stream, false);
@@ -803,6 +824,7 @@ extern "C" int provip_prune(const void* Q, const void* K, const void* V, const v
                             int algo, void* hidden_out, void* K_out, void* V_out, int* pos_out,
                             int* idx_out, int* seq_len_out, float* scores_out_or_null, void* ws,
                             size_t ws_bytes, unsigned flags, void* stream) {
+  NvtxRange nvtx_range("provip_prune");
   // validate both halves before enqueueing anything
   if (flags & ~(unsigned)PROVIP_PRUNE_OVERLAP_PREVIOUS) return fail(PROVIP_ERR_INVALID_ARG, "prune: unknown flags 0x%x", flags);
   int rc = hs_validate(Q, K, B, L_max, H_q, H_kv, d_h, head_list, H_sel, text_start, text_len,
@@ -925,6 +947,7 @@ extern "C" int provip_head_confidence(const void* Q, const void* K, int B, int L
                                       int N_v, const int* seq_len, int N_vis, int dtype, int algo,
                                       float* conf_out_or_null, int* vis_heads_out, void* ws,
                                       size_t ws_bytes, void* stream) {
+  NvtxRange nvtx_range("provip_head_confidence");
   if (!vis_heads_out) return fail(PROVIP_ERR_INVALID_ARG, "head_confidence: null vis_heads_out");
   return visual_heads_impl(Q, K, B, L_max, H_q, H_kv, d_h, text_start, text_len, crit_mask_or_null,
                            N_t_max, vis_start, N_v, seq_len, N_vis, 0, dtype, algo,
@@ -940,6 +963,7 @@ extern "C" int provip_prune_visual_heads(
     void* V_out, int* pos_out, int* idx_out, int* seq_len_out, float* scores_out_or_null,
     int* vis_heads_out_or_null, float* conf_out_or_null, void* ws, size_t ws_bytes,
     unsigned flags, void* stream) {
+  NvtxRange nvtx_range("provip_prune_visual_heads");
   if (flags & ~(unsigned)PROVIP_PRUNE_OVERLAP_PREVIOUS)
     return fail(PROVIP_ERR_INVALID_ARG, "prune_visual_heads: unknown flags 0x%x", flags);
   if (keep < 1) return fail(PROVIP_ERR_INVALID_ARG, "prune_visual_heads: keep %d < 1", keep);
@@ -981,23 +1005,25 @@ static constexpr size_t kNoAllocScratchBytes = (size_t)PROVIP_NOALLOC_SCRATCH_BY
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
 // Device address of the array on each device. In host code the symbol only
 // names a host-side stand-in, so a kernel must be given this address, looked up
-// with the device current.
-static void* g_noalloc_addr[64];
+// with the device current. Published with a release store: host threads making
+// their first call on a device at the same moment may both look it up (the
+// same value), and a reader that sees it non-null sees a complete lookup.
+static std::atomic<void*> g_noalloc_addr[64];
 
 static int noalloc_scratch_addr(void** out) {
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return cuda_fail(e, "head_scores_noalloc: cudaGetDevice");
   if (dev < 0 || dev >= 64) return fail(PROVIP_ERR_UNSUPPORTED, "head_scores_noalloc: device %d >= 64", dev);
-  if (g_noalloc_addr[dev] == nullptr) {
-    void* p = nullptr;
+  void* p = g_noalloc_addr[dev].load(std::memory_order_acquire);
+  if (p == nullptr) {
     e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
     if (e != cudaSuccess || p == nullptr)
       return cuda_fail(e != cudaSuccess ? e : cudaErrorInvalidSymbol,
                        "head_scores_noalloc: cudaGetSymbolAddress(scratch)");
-    g_noalloc_addr[dev] = p;
+    g_noalloc_addr[dev].store(p, std::memory_order_release);
   }
-  *out = g_noalloc_addr[dev];
+  *out = p;
   return PROVIP_OK;
 }
 
@@ -1007,6 +1033,7 @@ extern "C" int provip_head_scores_noalloc(const void* Q, const void* K, int B, i
                                           const uint8_t* row_mask_or_null, int N_t_max,
                                           int vis_start, int N_v, const int* seq_len, int dtype,
                                           int algo, float* scores, void* stream) {
+  NvtxRange nvtx_range("provip_head_scores_noalloc");
   const int ralgo = resolve_algo(algo, dtype);
   int rc = hs_validate(Q, K, B, L_max, H_q, H_kv, d_h, head_list, H_sel, text_start, text_len,
                        N_t_max, vis_start, N_v, seq_len, dtype, ralgo);

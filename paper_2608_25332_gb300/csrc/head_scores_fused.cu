@@ -26,6 +26,8 @@
 // attention matrix never leaves the SM. The host sizes the dynamic shared
 // memory so that the CTAs an SM can hold never ask for more than its 512 TMEM
 // columns (a tcgen05.alloc that has to wait inside a cluster could deadlock).
+#include <mutex>
+
 #include "common.cuh"
 #include "kernels.h"
 
@@ -383,12 +385,18 @@ __global__ void __launch_bounds__(kThreads, CPC == 1 ? 3 : (CPC == 2 ? 2 : 1))
     asm volatile("griddepcontrol.wait;" ::: "memory");
 }
 
+// One-time launch facts per (device, CPC, CONF): whether the kernel can be
+// configured at all (state: 0 not yet checked, 1 usable, -1 not) and, per
+// cluster size, whether such a cluster can be placed (0 unknown, 1 yes, -1 no).
+// Each is worked out under g_cfg_mu and published with a release store, so a
+// host thread that reads a non-zero value also sees the kernel attributes set
+// before it; threads racing on a first call wait for the one doing the setup.
 struct FusedCfg {
-  bool checked = false;
-  bool usable = false;
-  signed char clusters_ok[17] = {0};  // per cluster size: 0 unknown, 1 placeable, -1 not
+  std::atomic<int> state;
+  std::atomic<int> clusters_ok[17];
 };
-FusedCfg g_cfg[64][3][2];
+FusedCfg g_cfg[64][3][2];  // static storage: every field starts at zero
+std::mutex g_cfg_mu;
 
 template <int CPC, bool CONF>
 cudaError_t launch_cpc(const HSArgs& a, const CUtensorMap* tmQ, const CUtensorMap* tmK, int C,
@@ -403,7 +411,7 @@ cudaError_t launch_cpc(const HSArgs& a, const CUtensorMap* tmQ, const CUtensorMa
   int dev = 0;
   cudaGetDevice(&dev);
   const int slot = CPC == 1 ? 0 : (CPC == 2 ? 1 : 2);
-  FusedCfg& fc = g_cfg[dev < 64 ? dev : 0][slot][CONF ? 1 : 0];
+  FusedCfg& fc = g_cfg[dev >= 0 && dev < 64 ? dev : 0][slot][CONF ? 1 : 0];
   cudaLaunchConfig_t cfg = {};
   cudaLaunchAttribute attr[3];
   cfg.gridDim = dim3((unsigned)C, (unsigned)(a.H_sel * a.n_rb), (unsigned)a.B);
@@ -422,32 +430,40 @@ cudaError_t launch_cpc(const HSArgs& a, const CUtensorMap* tmQ, const CUtensorMa
   attr[2].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 2;
-  if (!fc.checked) {
-    fc.checked = true;
-    cudaError_t e = cudaFuncSetAttribute(hs_fused_tc<CPC, CONF>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e == cudaSuccess) e = cudaFuncSetAttribute(hs_fused_tc<CPC, CONF>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
-    if (e != cudaSuccess) {
-      cudaGetLastError();
-      return cudaSuccess;  // not usable: the caller takes the two-kernel path
+  int state = fc.state.load(std::memory_order_acquire);
+  if (state == 0) {
+    std::lock_guard<std::mutex> lock(g_cfg_mu);
+    state = fc.state.load(std::memory_order_relaxed);
+    if (state == 0) {
+      bool usable = false;
+      cudaError_t e = cudaFuncSetAttribute(hs_fused_tc<CPC, CONF>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+      if (e == cudaSuccess) e = cudaFuncSetAttribute(hs_fused_tc<CPC, CONF>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+      if (e == cudaSuccess) {
+        int per = 0;
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per, hs_fused_tc<CPC, CONF>, kThreads, smem);
+        usable = e == cudaSuccess && per >= 1 && per * CPC * kTile <= 512;
+      }
+      if (e != cudaSuccess) cudaGetLastError();  // not usable: the caller takes the two-kernel path
+      state = usable ? 1 : -1;
+      fc.state.store(state, std::memory_order_release);
     }
-    int per = 0;
-    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per, hs_fused_tc<CPC, CONF>, kThreads, smem);
-    if (e != cudaSuccess || per < 1 || per * CPC * kTile > 512) {
-      cudaGetLastError();
-      return cudaSuccess;
-    }
-    fc.usable = true;
   }
-  if (!fc.usable) return cudaSuccess;
+  if (state < 0) return cudaSuccess;
   // a cluster of C CTAs must be placeable on this GPU (checked once per size)
   if (C < 1 || C > 16) return cudaSuccess;
-  if (fc.clusters_ok[C] == 0) {
-    int nclusters = 0;
-    cudaError_t q = cudaOccupancyMaxActiveClusters(&nclusters, hs_fused_tc<CPC, CONF>, &cfg);
-    if (q != cudaSuccess) cudaGetLastError();
-    fc.clusters_ok[C] = (q == cudaSuccess && nclusters >= 1) ? 1 : -1;
+  int placeable = fc.clusters_ok[C].load(std::memory_order_acquire);
+  if (placeable == 0) {
+    std::lock_guard<std::mutex> lock(g_cfg_mu);
+    placeable = fc.clusters_ok[C].load(std::memory_order_relaxed);
+    if (placeable == 0) {
+      int nclusters = 0;
+      cudaError_t q = cudaOccupancyMaxActiveClusters(&nclusters, hs_fused_tc<CPC, CONF>, &cfg);
+      if (q != cudaSuccess) cudaGetLastError();
+      placeable = (q == cudaSuccess && nclusters >= 1) ? 1 : -1;
+      fc.clusters_ok[C].store(placeable, std::memory_order_release);
+    }
   }
-  if (fc.clusters_ok[C] < 0) return cudaSuccess;
+  if (placeable < 0) return cudaSuccess;
   if (pdl) cfg.numAttrs = 3;
   cudaError_t e = cudaLaunchKernelEx(&cfg, hs_fused_tc<CPC, CONF>, a, *tmQ, *tmK);
   if (e == cudaSuccess) *launched = true;

@@ -47,8 +47,14 @@ def _both(w, g, algo):
 
 def test_noalloc_matches_workspace_version_twice():
     # first call: LLaVA-1.5-7B shapes, ragged text lengths; second: the video GQA
-    # workload (different shape, so the shared scratch holds the first call's data)
+    # workload (different shape, so the shared scratch holds the first call's data);
+    # then the same LLaVA-1.5 shapes with the streaming and two-pass tcgen05
+    # forms forced (the tiny batch would otherwise take the cluster form) and the
+    # CUDA-core form, so that every kernel form that uses the scratch is checked
+    # against the workspace version
     for name, batch, algo in (("llava15_7b_bf16_b16", 4, P.ALGO_AUTO), ("video_gqa_bf16_b1", None, P.ALGO_AUTO),
+                              ("llava15_7b_bf16_b16", 4, P.ALGO_TCGEN05_STREAM),
+                              ("llava15_7b_bf16_b16", 4, P.ALGO_TCGEN05_TWOPASS),
                               ("llava15_7b_bf16_b16", 4, P.ALGO_SIMT)):
         w, g = _inputs(name, batch)
         ref, got = _both(w, g, algo)
