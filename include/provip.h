@@ -167,14 +167,16 @@ int provip_merge(const void *emb_v, int B, int N_v, int D, const int *keep_idx, 
 /* The whole pre-LLM pass: critical text tokens (unless crit_mask_or_null is
  * given), relevance p, top keep_pre of p (idx_out, ascending), and the merge
  * (when merged_out_or_null is given). p_out_or_null / mask_out_or_null
- * receive the intermediate p [B, N_v] and T mask [B, N_t_max] when non-NULL. */
+ * receive the intermediate p [B, N_v] and T mask [B, N_t_max] when non-NULL;
+ * assign_out_or_null [B, N_v] int32 receives the merge's assignment (as
+ * provip_merge's assign_out) when non-NULL and the merge runs. */
 size_t provip_similarity_reduce_workspace_size(int B, int N_v, int D, int N_t_max, int keep_pre);
 int provip_similarity_reduce(const void *emb_v, int B, int N_v, int D, const void *emb_t,
                              const int *text_len, int N_t_max,
                              const uint8_t *crit_mask_or_null, int keep_pre, int dtype,
-                             int *idx_out, void *merged_out_or_null, float *p_out_or_null,
-                             uint8_t *mask_out_or_null, void *ws, size_t ws_bytes,
-                             void *stream);
+                             int *idx_out, void *merged_out_or_null, int *assign_out_or_null,
+                             float *p_out_or_null, uint8_t *mask_out_or_null, void *ws,
+                             size_t ws_bytes, void *stream);
 
 /* ------------------------------------------------------------------------
  * In-LLM head-aware pruning (Sec. 4.4)
@@ -279,15 +281,24 @@ int provip_head_topk(const void *Q, const void *K, int B, int L_max, int H_q, in
  * dependents (the compaction copies the rows that do not depend on the kept
  * indices while the selection finishes).
  *
- * flags: 0, or PROVIP_PRUNE_OVERLAP_PREVIOUS - the call's head-score kernel may
- * start while the kernel before it on the stream (typically the previous
- * call's compaction) is still running; it waits for that kernel only before
- * it completes (its workspace writes do not conflict with the previous
- * call's kernels, which have consumed the workspace by then). Pass it only when this call's Q and K were not written
- * by the kernel launched just before it on the stream (for instance when
- * pruning a stream of independent batches); other kernels in between (e.g. the
- * LLM layers that produce Q/K) make the flag harmless. */
+ * flags: 0, or a combination of the two below.
+ * PROVIP_PRUNE_OVERLAP_PREVIOUS - the call's head-score kernel may start while
+ * the kernel before it on the stream (typically the previous call's
+ * compaction) is still running; it waits for that kernel only before it
+ * completes (its workspace writes do not conflict with the previous call's
+ * kernels, which have consumed the workspace by then). Pass it only when this
+ * call's Q and K were not written by the kernel launched just before it on the
+ * stream (for instance when pruning a stream of independent batches); other
+ * kernels in between (e.g. the LLM layers that produce Q/K) make the flag
+ * harmless. */
 #define PROVIP_PRUNE_OVERLAP_PREVIOUS 1u
+/* PROVIP_PRUNE_CONCURRENT - the caller runs other calls at the same time
+ * on other streams (e.g. several independent batches side by side). The
+ * compaction then takes only as many CTAs as the call's rows fill (at least
+ * 160 KiB of rows each) and leaves the remaining SMs to the concurrent calls;
+ * without the flag it spreads over every SM, which finishes a call that runs
+ * alone soonest. Results are the same either way. */
+#define PROVIP_PRUNE_CONCURRENT 2u
 size_t provip_prune_workspace_size(int B, int L_max, int H_sel, int N_t_max, int N_v, int algo,
                                    int dtype);
 int provip_prune(const void *Q, const void *K, const void *V, const void *hidden, int B,

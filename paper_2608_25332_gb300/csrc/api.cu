@@ -621,8 +621,9 @@ extern "C" int provip_similarity_reduce(const void* emb_v, int B, int N_v, int D
                                         const int* text_len, int N_t_max,
                                         const uint8_t* crit_mask_or_null, int keep_pre, int dtype,
                                         int* idx_out, void* merged_out_or_null,
-                                        float* p_out_or_null, uint8_t* mask_out_or_null, void* ws,
-                                        size_t ws_bytes, void* stream) {
+                                        int* assign_out_or_null, float* p_out_or_null,
+                                        uint8_t* mask_out_or_null, void* ws, size_t ws_bytes,
+                                        void* stream) {
   NvtxRange nvtx_range("provip_similarity_reduce");
   int rc = sim_validate_common(emb_v, B, N_v, D, dtype, "similarity_reduce");
   if (rc) return rc;
@@ -666,7 +667,8 @@ extern "C" int provip_similarity_reduce(const void* emb_v, int B, int N_v, int D
     e = topk_launch(t, s);
   }
   if (e == cudaSuccess && merged_out_or_null)
-    e = merge_launch(a, idx_out, keep_pre, w.inv_v, w.assign, merged_out_or_null, w.best, w.bidx,
+    e = merge_launch(a, idx_out, keep_pre, w.inv_v, assign_out_or_null ? assign_out_or_null : w.assign,
+                     merged_out_or_null, w.best, w.bidx,
                      merge_splits(B, N_v, keep_pre), w.pruned,
                      dtype == PROVIP_BF16 ? w.perm : nullptr, d->sms, s);
   return e == cudaSuccess ? PROVIP_OK : cuda_fail(e, "similarity_reduce launch");
@@ -826,7 +828,8 @@ extern "C" int provip_prune(const void* Q, const void* K, const void* V, const v
                             size_t ws_bytes, unsigned flags, void* stream) {
   NvtxRange nvtx_range("provip_prune");
   // validate both halves before enqueueing anything
-  if (flags & ~(unsigned)PROVIP_PRUNE_OVERLAP_PREVIOUS) return fail(PROVIP_ERR_INVALID_ARG, "prune: unknown flags 0x%x", flags);
+  if (flags & ~(unsigned)(PROVIP_PRUNE_OVERLAP_PREVIOUS | PROVIP_PRUNE_CONCURRENT))
+    return fail(PROVIP_ERR_INVALID_ARG, "prune: unknown flags 0x%x", flags);
   int rc = hs_validate(Q, K, B, L_max, H_q, H_kv, d_h, head_list, H_sel, text_start, text_len,
                        N_t_max, vis_start, N_v, seq_len, dtype, resolve_algo(algo, dtype));
   if (rc) return rc;
@@ -851,7 +854,7 @@ extern "C" int provip_prune(const void* Q, const void* K, const void* V, const v
   const int form = tc_form(resolve_algo(algo, dtype), B, H_sel, hs_shape(L_max, N_t_max, N_v, algo).n_rb,
                            d->sms);
   cudaError_t e = compact_launch(ca, d->sms, static_cast<cudaStream_t>(stream), true,
-                                 form == PROVIP_ALGO_TCGEN05_STREAM);
+                                 form == PROVIP_ALGO_TCGEN05_STREAM, (flags & PROVIP_PRUNE_CONCURRENT) != 0);
   return e == cudaSuccess ? PROVIP_OK : cuda_fail(e, "prune compact");
 }
 
@@ -964,7 +967,7 @@ extern "C" int provip_prune_visual_heads(
     int* vis_heads_out_or_null, float* conf_out_or_null, void* ws, size_t ws_bytes,
     unsigned flags, void* stream) {
   NvtxRange nvtx_range("provip_prune_visual_heads");
-  if (flags & ~(unsigned)PROVIP_PRUNE_OVERLAP_PREVIOUS)
+  if (flags & ~(unsigned)(PROVIP_PRUNE_OVERLAP_PREVIOUS | PROVIP_PRUNE_CONCURRENT))
     return fail(PROVIP_ERR_INVALID_ARG, "prune_visual_heads: unknown flags 0x%x", flags);
   if (keep < 1) return fail(PROVIP_ERR_INVALID_ARG, "prune_visual_heads: keep %d < 1", keep);
   int rc = compact_validate(idx_out ? idx_out : reinterpret_cast<int*>(16), B, N_v, keep, hidden, D,
@@ -986,7 +989,7 @@ extern "C" int provip_prune_visual_heads(
   const int form = tc_form(resolve_algo(algo, dtype), B, H_q, hs_shape(L_max, N_t_max, N_v, algo).n_rb,
                            d->sms);
   cudaError_t e = compact_launch(ca, d->sms, static_cast<cudaStream_t>(stream), true,
-                                 form == PROVIP_ALGO_TCGEN05_STREAM);
+                                 form == PROVIP_ALGO_TCGEN05_STREAM, (flags & PROVIP_PRUNE_CONCURRENT) != 0);
   return e == cudaSuccess ? PROVIP_OK : cuda_fail(e, "prune_visual_heads compact");
 }
 

@@ -60,6 +60,12 @@ constexpr long long kMinCtaBytes = (long long)PROVIP_COMPACT_MIN_CTA_KIB * 1024;
 #define PROVIP_COMPACT_SMALL_ROW 2048
 #endif
 constexpr int kSmallRow = PROVIP_COMPACT_SMALL_ROW;
+// 16-byte pieces a helper lane holds in flight (the K and V rows of 1 KiB of a
+// GQA layer with four key/value heads in one round trip)
+constexpr int kSmallPieces = 4;
+// bytes of rows per CTA below which a compaction that runs alone uses fewer
+// CTAs than two per SM
+constexpr long long kMinCtaBytesAlone = 16 * 1024;
 
 __device__ __forceinline__ int src_row(const CompactArgs& a, int b, int r, bool& ok) {
   if (r < a.vis_start) return r;
@@ -235,19 +241,44 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(const CompactA
         if (a.pos != nullptr)
           for (int p = lane; p < a.P; p += 32)
             a.pos_out[((size_t)p * a.B + b) * a.L_out + r] = a.pos[((size_t)p * a.B + b) * a.L_max + sr];
-        for (int t = 0; t < a.n_tensors; ++t) {
-          if (!(small & (1 << t))) continue;
-          const long long rb = a.row_bytes[t];
-          const uint4* src = reinterpret_cast<const uint4*>(a.src[t] + ((long long)b * a.L_max + sr) * rb);
-          uint4* dst = reinterpret_cast<uint4*>(a.dst[t] + ((long long)b * a.L_out + r) * rb);
-          const int n16 = (int)(rb / 16);
-          uint4 v[kSmallRow / 16 / 32];
+        // the row's pieces of every small tensor, as one list of 16-byte
+        // pieces: all of a lane's loads are issued before its stores (one
+        // memory round trip per row, not one per tensor)
+        const uint4 *s0 = nullptr, *s1 = nullptr, *s2 = nullptr;
+        uint4 *d0 = nullptr, *d1 = nullptr, *d2 = nullptr;
+        int n0 = 0, n1 = 0, n2 = 0;
+        if (small & 1) {
+          const long long rb = a.row_bytes[0];
+          s0 = reinterpret_cast<const uint4*>(a.src[0] + ((long long)b * a.L_max + sr) * rb);
+          d0 = reinterpret_cast<uint4*>(a.dst[0] + ((long long)b * a.L_out + r) * rb);
+          n0 = (int)(rb / 16);
+        }
+        if (small & 2) {
+          const long long rb = a.row_bytes[1];
+          s1 = reinterpret_cast<const uint4*>(a.src[1] + ((long long)b * a.L_max + sr) * rb);
+          d1 = reinterpret_cast<uint4*>(a.dst[1] + ((long long)b * a.L_out + r) * rb);
+          n1 = (int)(rb / 16);
+        }
+        if (small & 4) {
+          const long long rb = a.row_bytes[2];
+          s2 = reinterpret_cast<const uint4*>(a.src[2] + ((long long)b * a.L_max + sr) * rb);
+          d2 = reinterpret_cast<uint4*>(a.dst[2] + ((long long)b * a.L_out + r) * rb);
+          n2 = (int)(rb / 16);
+        }
+        const int tot = n0 + n1 + n2;
+        for (int q0 = 0; q0 < tot; q0 += 32 * kSmallPieces) {
+          uint4 v[kSmallPieces];
 #pragma unroll
-          for (int k = 0; k < kSmallRow / 16 / 32; ++k)
-            if (lane + 32 * k < n16) v[k] = __ldcs(src + lane + 32 * k);
+          for (int j = 0; j < kSmallPieces; ++j) {
+            const int q = q0 + lane + 32 * j;
+            if (q < tot)
+              v[j] = __ldcs(q < n0 ? s0 + q : (q < n0 + n1 ? s1 + (q - n0) : s2 + (q - n0 - n1)));
+          }
 #pragma unroll
-          for (int k = 0; k < kSmallRow / 16 / 32; ++k)
-            if (lane + 32 * k < n16) __stcs(dst + lane + 32 * k, v[k]);
+          for (int j = 0; j < kSmallPieces; ++j) {
+            const int q = q0 + lane + 32 * j;
+            if (q < tot) __stcs(q < n0 ? d0 + q : (q < n0 + n1 ? d1 + (q - n0) : d2 + (q - n0 - n1)), v[j]);
+          }
         }
       }
     }
@@ -256,7 +287,8 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(const CompactA
 
 }  // namespace
 
-cudaError_t compact_launch(const CompactArgs& a, int num_sms, cudaStream_t s, bool pdl, bool allow_deep) {
+cudaError_t compact_launch(const CompactArgs& a, int num_sms, cudaStream_t s, bool pdl, bool allow_deep,
+                           bool concurrent) {
   static std::atomic<bool> configured[64];  // per device, zero-initialised
   int dev = 0;
   cudaGetDevice(&dev);
@@ -281,12 +313,17 @@ cudaError_t compact_launch(const CompactArgs& a, int num_sms, cudaStream_t s, bo
   const int nb = np[0] + np[1] + np[2];
   const long long total = (long long)a.B * a.L_out * (nb > 0 ? nb : 1);
   long long grid = (long long)kCtasPerSm * num_sms;
-  // small problems: at least kMinCtaBytes of rows per CTA, so that every CTA's
-  // pipeline fills (and kernels running beside it keep the SMs it does not need)
+  // Alone, the compaction spreads over every SM (a small problem is bound by
+  // the latency of each CTA's few copies, so more CTAs finish it sooner). With
+  // concurrent calls on other streams, a small problem takes at least
+  // kMinCtaBytes of rows per CTA, so that every CTA's pipeline fills and the
+  // kernels running beside it keep the SMs it does not need.
   const long long row_sum = a.row_bytes[0] + a.row_bytes[1] + a.row_bytes[2];
-  const long long by_bytes = ((long long)a.B * a.L_out * row_sum + kMinCtaBytes - 1) / kMinCtaBytes;
+  const long long bytes = (long long)a.B * a.L_out * row_sum;
+  const long long by_bytes = (bytes + kMinCtaBytes - 1) / kMinCtaBytes;
   const bool deep = allow_deep && by_bytes >= grid;  // the rows fill every CTA slot
-  if (grid > by_bytes) grid = by_bytes;
+  const long long cap = concurrent ? by_bytes : (bytes + kMinCtaBytesAlone - 1) / kMinCtaBytesAlone;
+  if (grid > cap) grid = cap;
   if (grid > total) grid = total > 0 ? total : 1;
   cudaLaunchConfig_t cfg = {};
   cudaLaunchAttribute attr[1];

@@ -13,15 +13,18 @@
 //      e = exp2(s - mb) goes back into TMEM with tcgen05.st, mb being the
 //      running max after that block (kept per block); the two halves' (m, l)
 //      are combined in shared memory;
-//   3. after a cluster barrier, reads every peer's (m, l) for its row through
-//      distributed shared memory and forms the row's global max M and sum L;
+//   3. pushes its (m, l) of each row into every cluster CTA's shared memory
+//      (remote stores into the key-tile region, free once every CTA's MMAs
+//      are done: a split cluster barrier around pass 1 guarantees it), and
+//      after one cluster barrier forms the row's global max M and sum L from
+//      its own shared memory;
 //   4. turns its visual columns into probabilities p = e * exp2(mb - M) / L and
 //      sums them over the 128 rows (warp butterfly transpose-reduction, then a
 //      fixed-order sum over the 4 warps) into partial[b][rb * H_sel + h][col];
 //      the CONF variant also keeps, per row, the mean and M2 of its visual
 //      probabilities (head confidence) and writes them per cluster rank;
-//   5. waits on a second cluster barrier (peers may still read its shared
-//      memory) and frees its TMEM.
+//   5. frees its TMEM (no CTA touches another's shared memory after the
+//      barrier of step 3).
 // Every key is read from HBM once and every logit is exponentiated once; the
 // attention matrix never leaves the SM. The host sizes the dynamic shared
 // memory so that the CTAs an SM can hold never ask for more than its 512 TMEM
@@ -54,8 +57,8 @@ __device__ __forceinline__ void cluster_sync_all() {
   asm volatile("barrier.cluster.arrive.release.aligned;\n\t"
                "barrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
-__device__ __forceinline__ void cluster_arrive() {
-  asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+__device__ __forceinline__ void cluster_arrive_relaxed() {
+  asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
 }
 __device__ __forceinline__ void cluster_wait() {
   asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
@@ -64,12 +67,11 @@ __device__ __forceinline__ void cluster_wait() {
 __device__ __forceinline__ void pdl_trigger() {
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 }
-__device__ __forceinline__ float2 ld_peer_f2(const float2* local, uint32_t rank) {
+// stores v at the address of `local` in the shared memory of cluster CTA `rank`
+__device__ __forceinline__ void st_peer_f2(float2* local, uint32_t rank, float2 v) {
   uint32_t raddr;
   asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(raddr) : "r"(smem_u32(local)), "r"(rank));
-  float2 v;
-  asm volatile("ld.shared::cluster.v2.f32 {%0, %1}, [%2];" : "=f"(v.x), "=f"(v.y) : "r"(raddr) : "memory");
-  return v;
+  asm volatile("st.shared::cluster.v2.f32 [%0], {%1, %2};" ::"r"(raddr), "f"(v.x), "f"(v.y) : "memory");
 }
 __device__ __forceinline__ void tmem_st32(uint32_t taddr, const float* v) {
   asm volatile(
@@ -114,7 +116,6 @@ __global__ void __launch_bounds__(kThreads, CPC == 1 ? 3 : (CPC == 2 ? 2 : 1))
   constexpr uint32_t kCols = CPC * kTile;  // 128, 256 or 512: a power of two
   extern __shared__ uint8_t smem_raw[];
   __shared__ Ctl ctl;
-  __shared__ float2 rowstat[kTile];
   __shared__ float2 halfstat[2][kTile];
   __shared__ float red[4][kCols];
   const uint32_t rank = cluster_rank(), nrank = cluster_size();
@@ -152,8 +153,8 @@ __global__ void __launch_bounds__(kThreads, CPC == 1 ? 3 : (CPC == 2 ? 2 : 1))
       tma_load_2d(ks + c * kTileBytes + kHalfBytes, &tmK, xk + 64, yk, &ctl.tma_bar);
     }
   }
-  __syncwarp();
-  if (threadIdx.x < 32) {
+  // warp 1 allocates the tensor memory while thread 0 issues the loads
+  if (threadIdx.x >= 32 && threadIdx.x < 64) {
     tmem_alloc(&ctl.tmem, kCols);
     tmem_relinquish();
   }
@@ -186,6 +187,9 @@ __global__ void __launch_bounds__(kThreads, CPC == 1 ? 3 : (CPC == 2 ? 2 : 1))
   __syncwarp();
   const bool good = mbar_wait(&ctl.mma_bar, 0, a.err) && ctl.fail == 0;
   tc_fence_after();
+  // this CTA's MMAs have read its Q and K tiles: from the matching wait on,
+  // peers may write their row statistics into the key-tile region
+  cluster_arrive_relaxed();
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int quad = warp & 3, half = warp >> 2;  // TMEM lanes 32*quad.., columns of this half
@@ -249,24 +253,31 @@ __global__ void __launch_bounds__(kThreads, CPC == 1 ? 3 : (CPC == 2 ? 2 : 1))
   }
   halfstat[half][r] = make_float2(rv ? m : -INFINITY, rv ? l : 0.f);
   __syncthreads();
+  // every CTA of the cluster has finished its MMAs (and so has started): its
+  // key-tile region may receive the row statistics of the whole cluster,
+  // recv[rank][row] = that CTA's (max, sum) of the row over its keys
+  float2* recv = reinterpret_cast<float2*>(ks);
+  cluster_wait();
   if (half == 0) {
-    // the CTA's (max, sum) of the row from its two column halves
+    // the CTA's (max, sum) of the row from its two column halves, pushed to
+    // every CTA of the cluster (remote stores, made visible by the barrier)
     const float2 h0 = halfstat[0][r], h1 = halfstat[1][r];
     const float mm = fmaxf(h0.x, h1.x);
     float ll = 0.f;
     if (h0.x != -INFINITY) ll += h0.y * ex2_approx(h0.x - mm);
     if (h1.x != -INFINITY) ll += h1.y * ex2_approx(h1.x - mm);
-    rowstat[r] = make_float2(mm, ll);
+    const float2 st = make_float2(mm, ll);
+    for (uint32_t q = 0; q < nrank; ++q) st_peer_f2(&recv[rank * kTile + r], q, st);
   }
   cluster_sync_all();
 
-  // global (max, sum) of the row over the cluster: all peer loads issued first
+  // global (max, sum) of the row over the cluster, from local shared memory
   float M = -INFINITY, L = 0.f;
   if (rv) {
     float2 st[16];
 #pragma unroll
     for (uint32_t q = 0; q < 16; ++q)
-      if (q < nrank) st[q] = ld_peer_f2(&rowstat[r], q);
+      if (q < nrank) st[q] = recv[q * kTile + r];
 #pragma unroll
     for (uint32_t q = 0; q < 16; ++q)
       if (q < nrank) M = fmaxf(M, st[q].x);
@@ -275,7 +286,6 @@ __global__ void __launch_bounds__(kThreads, CPC == 1 ? 3 : (CPC == 2 ? 2 : 1))
       if (q < nrank && st[q].x != -INFINITY) L += st[q].y * ex2_approx(st[q].x - M);
   }
   const float invL = (rv && L > 0.f) ? 1.f / L : 0.f;
-  cluster_arrive();  // done reading the peers' rowstat
 
   // pass 2: probabilities of the visual columns, summed over the rows; with
   // CONF, the row's mean and M2 over this warp's visual columns as well (the
@@ -373,8 +383,7 @@ __global__ void __launch_bounds__(kThreads, CPC == 1 ? 3 : (CPC == 2 ? 2 : 1))
   }
   tc_fence_before();
   __syncthreads();
-  if (threadIdx.x < 32) tmem_dealloc(ctl.tmem, kCols);
-  cluster_wait();  // every peer has read this CTA's rowstat
+  if (threadIdx.x >= 32 && threadIdx.x < 64) tmem_dealloc(ctl.tmem, kCols);  // the allocating warp
   // When this grid is a programmatic dependent of the previous call's
   // compaction (independent batches), one CTA waits for that kernel before
   // exiting, so that this grid - and therefore the top-k that follows it and

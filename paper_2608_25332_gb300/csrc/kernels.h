@@ -147,9 +147,11 @@ struct CompactArgs {
 // pdl: launched as a programmatic dependent of the previous kernel on the
 // stream; rows that do not depend on idx are copied before waiting for it.
 // allow_deep: the deeper slot ring may be used (it leaves room for a streaming
-// head-score CTA per SM, not for the cluster form's larger one)
+// head-score CTA per SM, not for the cluster form's larger one). concurrent:
+// other calls run beside this one on other streams, so a small problem takes
+// only the CTAs its bytes fill (otherwise it spreads over every SM).
 cudaError_t compact_launch(const CompactArgs& a, int num_sms, cudaStream_t s, bool pdl = false,
-                           bool allow_deep = true);
+                           bool allow_deep = true, bool concurrent = false);
 
 // ---------------------------------------------------------------------------
 // pre-LLM similarity pass (Sec. 4.2-4.3)

@@ -1,9 +1,10 @@
 // Per-sample top-k kernels (Sec. 4.3 top N1 of p, Sec. 4.4 top N2 of v): ties
 // to the lower index, ascending output. Up to 512 scores: exact ranks in a
 // cluster of CTAs per sample (topk_rank_kernel, built for latency). Larger N:
-// one CTA per sample (about 4 keys per thread, 128 to 1024 threads), the N
-// scores held in shared memory as order-preserving keys, selected by
-// topk_block_select (topk_block.cuh).
+// one CTA per sample selecting on order-preserving keys (topk_block.cuh: a
+// digit histogram over the keys' actual range, usually one pass, then exact
+// ranks of the few candidates left) - up to 16384 keys held in registers, 4 to
+// 32 per thread (topk_reg_kernel), more in shared memory (topk_kernel).
 //
 // When fed head partials (the in-LLM path), the kernel first sums them per
 // column in a fixed order and divides by (heads x valid text rows): the same
@@ -33,25 +34,29 @@ __device__ __forceinline__ int block_count_rows(const TopkArgs& a, int b) {
 }
 
 // keys[0..N) of sample b (and, when so is set, the scores) from the scores or
-// the head partials; every thread of the block takes part
-__device__ __forceinline__ void load_sample_keys(const TopkArgs& a, int b, uint32_t* keys,
-                                                 float* so) {
+// the head partials, with the thread's min and max key; every thread of the
+// block takes part. The keys are visible to the block after its next barrier.
+__device__ __forceinline__ void load_sample_keys(const TopkArgs& a, int b, uint32_t* keys, float* so,
+                                                 uint32_t& mn, uint32_t& mx) {
   const int N = a.N;
+  mn = 0xffffffffu;
+  mx = 0u;
   if (a.partial != nullptr) {
     __shared__ int sel[kMaxHeads];
-    if (a.sel != nullptr)
-      for (int q = threadIdx.x; q < a.n_sel; q += blockDim.x) sel[q] = a.sel[(size_t)b * a.n_sel + q];
-    const int nrows = block_count_rows(a, b);  // synchronises the block
-    const float nh = (float)(a.sel != nullptr ? a.n_sel : a.H_sel);
-    topk_load_partials<false>(a.partial + (size_t)b * a.n_part * N, a.n_part, N, nh * (float)nrows,
-                              nrows <= 0, so, keys, a.sel != nullptr ? sel : nullptr, a.n_sel,
-                              a.H_sel);
-  } else {
-    for (int i = threadIdx.x; i < N; i += blockDim.x) {
-      const float v = a.scores[(size_t)b * N + i];
-      if (so) so[i] = v;
-      keys[i] = float_key(v);
+    int nrows;
+    if (a.row_mask == nullptr && a.sel == nullptr) {
+      // every text row counts: no block-wide count needed
+      nrows = min(max(a.text_len[b], 0), a.N_t_max);
+    } else {
+      if (a.sel != nullptr)
+        for (int q = threadIdx.x; q < a.n_sel; q += blockDim.x) sel[q] = a.sel[(size_t)b * a.n_sel + q];
+      nrows = block_count_rows(a, b);  // synchronises the block (sel is visible after it)
     }
+    const float nh = (float)(a.sel != nullptr ? a.n_sel : a.H_sel);
+    topk_load_partials(a.partial + (size_t)b * a.n_part * N, a.n_part, N, nh * (float)nrows, nrows <= 0, so,
+                       keys, mn, mx, a.sel != nullptr ? sel : nullptr, a.n_sel, a.H_sel);
+  } else {
+    topk_load_scores(a.scores + (size_t)b * N, N, so, keys, mn, mx);
   }
 }
 
@@ -63,13 +68,133 @@ __global__ void __launch_bounds__(kTopkMaxThreads) topk_kernel(const TopkArgs a)
   // compaction has completed too)
   asm volatile("griddepcontrol.wait;" ::: "memory");
   const int b = blockIdx.x;
-  load_sample_keys(a, b, keys, a.scores_out ? a.scores_out + (size_t)b * a.N : nullptr);
-  __syncthreads();
+  for (int q = threadIdx.x; q < kSelectBins; q += blockDim.x) sh.hist[0][q] = 0;
+  uint32_t mn, mx, lo, hi;
+  load_sample_keys(a, b, keys, a.scores_out ? a.scores_out + (size_t)b * a.N : nullptr, mn, mx);
+  topk_block_range(mn, mx, sh, lo, hi);  // its barrier also publishes the keys and the cleared histogram
   // The scores are in shared memory now: the next kernel (the compaction, and
   // through it the next call's head scores, which rewrite the partials) may
   // start. idx is only read by the compaction after this grid completes.
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-  topk_block_select(keys, a.N, a.k, a.idx_out + (size_t)b * a.k, sh);
+  topk_block_select(keys, a.N, a.k, lo, hi, a.idx_out + (size_t)b * a.k, sh);
+}
+
+// Thread t's KPT keys (indices t * KPT + c, c < KPT; 0 past N) from the scores
+// or the head partials (the same sums, in the same order, as
+// load_sample_keys), with the thread's min and max key. Every load of a group
+// of partial rows is issued before the first sum.
+template <int KPT>
+__device__ __forceinline__ void load_keys_reg(const TopkArgs& a, int b, uint32_t (&key)[KPT],
+                                              uint32_t& mn, uint32_t& mx) {
+  const int N = a.N, i0 = threadIdx.x * KPT;
+  float v[KPT];
+  if (a.partial != nullptr) {
+    __shared__ int sel[kMaxHeads];
+    int nrows;
+    if (a.row_mask == nullptr && a.sel == nullptr) {
+      nrows = min(max(a.text_len[b], 0), a.N_t_max);
+    } else {
+      if (a.sel != nullptr)
+        for (int q = threadIdx.x; q < a.n_sel; q += blockDim.x) sel[q] = a.sel[(size_t)b * a.n_sel + q];
+      nrows = block_count_rows(a, b);  // synchronises the block (sel is visible after it)
+    }
+    const int n_sum = a.sel != nullptr ? (a.n_part / a.H_sel) * a.n_sel : a.n_part;
+    const float div = (float)(a.sel != nullptr ? a.n_sel : a.H_sel) * (float)nrows;
+    const float* P0 = a.partial + (size_t)b * a.n_part * N;
+    // N % 4 == 0 and an aligned base: every row and every thread's columns start
+    // on 16 bytes, and a group of 4 columns lies wholly below N or wholly past it
+    const bool vec = (N & 3) == 0 && (reinterpret_cast<uintptr_t>(P0) & 15u) == 0;
+    constexpr int G = KPT >= 16 ? 2 : 32 / KPT;  // rows per group: 32 to 64 loads in flight
+    float s[KPT];
+#pragma unroll
+    for (int c = 0; c < KPT; ++c) s[c] = 0.f;
+    for (int u0 = 0; u0 < n_sum; u0 += G) {
+      int ro[G];
+#pragma unroll
+      for (int u = 0; u < G; ++u) {
+        const int uu = u0 + u;
+        ro[u] = uu < n_sum ? (a.sel != nullptr ? (uu / a.n_sel) * a.H_sel + sel[uu % a.n_sel] : uu) * N : 0;
+      }
+      float t[KPT][G];
+      if (vec) {
+        // 16-byte loads of the thread's KPT consecutive columns
+#pragma unroll
+        for (int u = 0; u < G; ++u)
+#pragma unroll
+          for (int c4 = 0; c4 < KPT / 4; ++c4) {
+            float4 f = make_float4(0.f, 0.f, 0.f, 0.f);
+            if (u0 + u < n_sum && i0 + 4 * c4 < N)
+              f = __ldg(reinterpret_cast<const float4*>(P0 + (size_t)ro[u] + i0) + c4);
+            t[4 * c4 + 0][u] = f.x;
+            t[4 * c4 + 1][u] = f.y;
+            t[4 * c4 + 2][u] = f.z;
+            t[4 * c4 + 3][u] = f.w;
+          }
+      } else {
+#pragma unroll
+        for (int c = 0; c < KPT; ++c)
+#pragma unroll
+          for (int u = 0; u < G; ++u)
+            t[c][u] = (u0 + u < n_sum && i0 + c < N) ? __ldg(P0 + (size_t)ro[u] + i0 + c) : 0.f;
+      }
+#pragma unroll
+      for (int c = 0; c < KPT; ++c)
+#pragma unroll
+        for (int u = 0; u < G; ++u)
+          if (u0 + u < n_sum) s[c] += t[c][u];
+    }
+#pragma unroll
+    for (int c = 0; c < KPT; ++c) v[c] = nrows <= 0 ? 0.f : s[c] / div;
+  } else {
+    const float* src = a.scores + (size_t)b * N;
+    if ((N & 3) == 0 && (reinterpret_cast<uintptr_t>(src) & 15u) == 0) {
+#pragma unroll
+      for (int c4 = 0; c4 < KPT / 4; ++c4) {
+        float4 f = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (i0 + 4 * c4 < N) f = __ldg(reinterpret_cast<const float4*>(src + i0) + c4);
+        v[4 * c4 + 0] = f.x;
+        v[4 * c4 + 1] = f.y;
+        v[4 * c4 + 2] = f.z;
+        v[4 * c4 + 3] = f.w;
+      }
+    } else {
+#pragma unroll
+      for (int c = 0; c < KPT; ++c) v[c] = i0 + c < N ? __ldg(src + i0 + c) : 0.f;
+    }
+  }
+  float* so = a.scores_out ? a.scores_out + (size_t)b * N : nullptr;
+  mn = 0xffffffffu;
+  mx = 0u;
+#pragma unroll
+  for (int c = 0; c < KPT; ++c) {
+    key[c] = 0u;
+    if (i0 + c < N) {
+      if (so) so[i0 + c] = v[c];
+      key[c] = float_key(v[c]);
+      mn = min(mn, key[c]);
+      mx = max(mx, key[c]);
+    }
+  }
+}
+
+// Up to 16384 keys: they stay in registers, 4 to 32 per thread (at most 512
+// threads, so a thread may hold 128 registers), thread t owning the contiguous
+// indices [t * KPT, t * KPT + KPT).
+constexpr int kRegMaxThreads = 512;
+template <int KPT>
+__global__ void __launch_bounds__(kRegMaxThreads) topk_reg_kernel(const TopkArgs a) {
+  __shared__ TopkShared sh;
+  // a programmatic dependent: wait for the kernel that writes the scores
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  const int b = blockIdx.x;
+  for (int q = threadIdx.x; q < kSelectBins; q += blockDim.x) sh.hist[0][q] = 0;
+  uint32_t key[KPT], mn, mx, lo, hi;
+  load_keys_reg<KPT>(a, b, key, mn, mx);
+  topk_block_range(mn, mx, sh, lo, hi);  // its barrier also publishes the cleared histogram
+  // the scores are consumed: the next kernel may start (it waits for this
+  // grid's completion before reading idx)
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  topk_block_select_reg<KPT>(key, a.N, a.k, lo, hi, a.idx_out + (size_t)b * a.k, sh);
 }
 
 // Small N (<= kRankUseMaxN): selection by exact ranks, for latency. A cluster of
@@ -113,7 +238,8 @@ __global__ void __launch_bounds__(kRankThreads) topk_rank_kernel(const TopkArgs 
   const uint32_t crank = cluster_ctarank();
   const int b = blockIdx.y, N = a.N;
   // one CTA of the cluster writes the scores
-  load_sample_keys(a, b, keys, (a.scores_out && crank == 0) ? a.scores_out + (size_t)b * N : nullptr);
+  uint32_t mn, mx;
+  load_sample_keys(a, b, keys, (a.scores_out && crank == 0) ? a.scores_out + (size_t)b * N : nullptr, mn, mx);
   __syncthreads();
   for (int j = threadIdx.x; j < N; j += kRankThreads)
     ck[j] = ((unsigned long long)keys[j] << 32) | (unsigned long long)(~(uint32_t)j);
@@ -194,6 +320,18 @@ cudaError_t topk_launch(const TopkArgs& a, cudaStream_t s, bool pdl) {
     cfg.attrs = rattr;
     cfg.numAttrs = pdl ? 2 : 1;
     return cudaLaunchKernelEx(&cfg, topk_rank_kernel, a);
+  }
+  if (a.N <= 32 * kRegMaxThreads) {
+    // keys in registers: 4, 8, 16 or 32 per thread, 128 to 512 threads
+    const int kpt = a.N <= 4 * kRegMaxThreads ? 4
+                    : (a.N <= 8 * kRegMaxThreads ? 8 : (a.N <= 16 * kRegMaxThreads ? 16 : 32));
+    int nt = ((a.N + kpt - 1) / kpt + 31) / 32 * 32;
+    cfg.blockDim = dim3((unsigned)(nt < 128 ? 128 : nt));
+    cfg.dynamicSmemBytes = 0;
+    if (kpt == 4) return cudaLaunchKernelEx(&cfg, topk_reg_kernel<4>, a);
+    if (kpt == 8) return cudaLaunchKernelEx(&cfg, topk_reg_kernel<8>, a);
+    if (kpt == 16) return cudaLaunchKernelEx(&cfg, topk_reg_kernel<16>, a);
+    return cudaLaunchKernelEx(&cfg, topk_reg_kernel<32>, a);
   }
   return cudaLaunchKernelEx(&cfg, topk_kernel, a);
 }

@@ -2,124 +2,217 @@
 // 4.4 top N2): ties broken toward the lower index, indices in ascending order.
 // Used by the top-k kernel. Any block size that is a multiple of 32 (<= 1024) works.
 //
-// keys[0..N) are order-preserving uint32 keys (float_key). An 8-bit MSD radix
-// select (4 passes of a 256-bin shared histogram, one increment per group of
-// lanes with the same digit) finds the exact key T of the k-th largest and how
-// many keys equal to T are taken (need_eq); one block scan of packed
-// (greater, equal) counts in index order then gives every selected element its
-// slot #(greater before i) + min(#(equal before i), need_eq).
+// keys[0..N) are order-preserving uint32 keys (float_key). The select narrows
+// an inclusive key range [lo, hi] that holds the k-th largest key, starting
+// from the block's min and max. Each pass takes the 11 bits of the keys below
+// the leading bits that lo and hi share (a digit: every key of the range maps
+// to one of at most 2048 bins, and at least half of the bins span the range),
+// builds a shared histogram of the digits, and one warp finds the bin that
+// holds the k-th largest key; the range becomes that bin's keys. A range of
+// one key value ends the search, and so does a bin of at most kSmallCand keys:
+// they are gathered and one warp ranks them exactly by (key, lower index
+// first). Spread-out keys take one pass; a 32-bit range needs at most three.
+// The threshold key T and how many keys equal to T are taken (need_eq) then
+// give every selected element its output slot, #(greater before i) +
+// min(#(equal before i), need_eq), from counts of (greater, equal) in index
+// order scanned within warps and then across them.
 #pragma once
 
 #include "common.cuh"
 
 namespace provip {
 
+constexpr int kSelectBins = 2048;  // one 11-bit digit
+constexpr int kSmallCand = 32;
+
 struct TopkShared {
-  int hist[256];
-  uint32_t warp_tot[32];
-  uint32_t prefix;
-  int rem;
+  __align__(16) int hist[2][kSelectBins];  // double-buffered: the next pass's is cleared during this one
+  uint32_t wmin[32], wmax[32];
+  uint32_t wcnt[32];         // packed (greater << 16 | equal) counts per warp
+  int sel, above, cnt;       // chosen bin, keys above it in the range, keys in it
+  int ncand;
+  __align__(16) uint32_t ckey[kSmallCand];
+  __align__(16) int cidx[kSmallCand];
 };
 
-// exclusive block scan of one uint32 per thread
-__device__ __forceinline__ uint32_t topk_block_exclusive_scan(uint32_t v, uint32_t* warp_tot) {
+// Min and max of the block's keys. Every thread passes its own partial min and
+// max; the result is valid in every thread after the call (one barrier).
+__device__ __forceinline__ void topk_block_range(uint32_t mn, uint32_t mx, TopkShared& sh,
+                                                 uint32_t& lo, uint32_t& hi) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
-  uint32_t incl = v;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    mn = min(mn, __shfl_xor_sync(0xffffffffu, mn, o));
+    mx = max(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+  }
+  if (lane == 0) {
+    sh.wmin[warp] = mn;
+    sh.wmax[warp] = mx;
+  }
+  __syncthreads();
+  mn = lane < nw ? sh.wmin[lane] : 0xffffffffu;
+  mx = lane < nw ? sh.wmax[lane] : 0u;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    mn = min(mn, __shfl_xor_sync(0xffffffffu, mn, o));
+    mx = max(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+  }
+  lo = mn;
+  hi = mx;
+}
+
+// In descending bin order over hist[0..kSelectBins) (bins past the digit's
+// range are zero), the bin where the count from the top first reaches rem:
+// writes sh.sel, sh.above (keys in higher bins) and sh.cnt (keys in the bin).
+// Every thread sums a segment of BPT consecutive bins (16-byte loads), a block
+// scan of the segment counts finds the segment that holds the bin, and its
+// thread walks it. Called by every thread; two barriers.
+__device__ __forceinline__ void topk_block_find_bin(const int* hist, int rem, TopkShared& sh) {
+  const int tid = threadIdx.x, nth = blockDim.x, lane = tid & 31, warp = tid >> 5;
+  // bins per thread: 4, 8 or 16 (blocks of at least 128 threads)
+  const int bpt = nth >= kSelectBins / 4 ? 4 : (nth >= kSelectBins / 8 ? 8 : 16);
+  const int top = kSelectBins - tid * bpt;  // this thread's bins are [top - bpt, top)
+  int h[16];
+  int tot = 0;
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    if (q * 4 < bpt && top - q * 4 - 4 >= 0) {
+      const int4 v = *reinterpret_cast<const int4*>(hist + top - q * 4 - 4);
+      h[q * 4 + 0] = v.w;  // descending: the highest bin first
+      h[q * 4 + 1] = v.z;
+      h[q * 4 + 2] = v.y;
+      h[q * 4 + 3] = v.x;
+    } else {
+      h[q * 4 + 0] = h[q * 4 + 1] = h[q * 4 + 2] = h[q * 4 + 3] = 0;
+    }
+    tot += (h[q * 4 + 0] + h[q * 4 + 1]) + (h[q * 4 + 2] + h[q * 4 + 3]);
+  }
+  int incl = tot;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int y = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += y;
+  }
+  if (lane == 31) sh.wcnt[warp] = (uint32_t)incl;
+  __syncthreads();
+  int before = lane < warp ? (int)sh.wcnt[lane] : 0;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) before += __shfl_xor_sync(0xffffffffu, before, o);
+  const int excl = before + incl - tot;
+  if (excl < rem && rem <= excl + tot) {
+    int cum = excl;
+#pragma unroll
+    for (int q = 0; q < 16; ++q) {
+      if (q < bpt && cum + h[q] >= rem) {
+        sh.sel = top - 1 - q;
+        sh.above = cum;
+        sh.cnt = h[q];
+        break;
+      }
+      cum += h[q];
+    }
+  }
+  __syncthreads();
+}
+
+// Exact rank of the rem-th largest of the nc <= kSmallCand candidates (key,
+// index) in shared memory: the threshold key T and how many keys equal to T
+// are taken. Lane l ranks candidate l against all of them, read with 16-byte
+// broadcast loads; every warp that calls it gets the same answer.
+__device__ __forceinline__ void topk_warp_rank(const TopkShared& sh, int nc, int rem, uint32_t& T,
+                                               int& need_eq) {
+  const int lane = threadIdx.x & 31;
+  const uint32_t ku = lane < nc ? sh.ckey[lane] : 0u;
+  const int ki = lane < nc ? sh.cidx[lane] : 0x7fffffff;
+  int rank = 0;
+#pragma unroll
+  for (int q = 0; q < kSmallCand / 4; ++q) {
+    const uint4 kv = reinterpret_cast<const uint4*>(sh.ckey)[q];
+    const int4 iv = reinterpret_cast<const int4*>(sh.cidx)[q];
+    // branch-free: (j < nc) & (key_j > key or (key_j == key and idx_j < idx))
+    rank += (int)((4 * q + 0 < nc) & ((kv.x > ku) | ((kv.x == ku) & (iv.x < ki))));
+    rank += (int)((4 * q + 1 < nc) & ((kv.y > ku) | ((kv.y == ku) & (iv.y < ki))));
+    rank += (int)((4 * q + 2 < nc) & ((kv.z > ku) | ((kv.z == ku) & (iv.z < ki))));
+    rank += (int)((4 * q + 3 < nc) & ((kv.w > ku) | ((kv.w == ku) & (iv.w < ki))));
+  }
+  const unsigned hit = __ballot_sync(0xffffffffu, lane < nc && rank == rem - 1);
+  T = __shfl_sync(0xffffffffu, ku, hit ? __ffs(hit) - 1 : 0);
+  const unsigned gt = __ballot_sync(0xffffffffu, lane < nc && ku > T);
+  need_eq = rem - __popc(gt);
+}
+
+// Selects the k largest of keys[0..N) (shared memory) into out[0..k), given the
+// keys' min lo and max hi. Must be called by every thread of the block; keys
+// and sh.hist[0] (cleared) must be visible (synced).
+__device__ __forceinline__ void topk_block_select(const uint32_t* keys, int N, int k, uint32_t lo,
+                                                  uint32_t hi, int* out, TopkShared& sh) {
+  const int tid = threadIdx.x, nth = blockDim.x, lane = tid & 31, warp = tid >> 5;
+  int rem = k;  // keys still to take from [lo, hi]
+  int buf = 0;
+  uint32_t T = lo;
+  int need_eq = rem;
+  for (int pass = 0; pass < 4; ++pass) {  // three passes at most (see above)
+    if (lo == hi) {  // one key value left: take rem of it
+      T = lo;
+      need_eq = rem;
+      break;
+    }
+    const int hb = 31 - __clz(lo ^ hi);  // highest bit where lo and hi differ
+    const int shift = hb > 10 ? hb - 10 : 0;
+    const uint32_t base = lo >> shift;  // digits (key >> shift) - base < kSelectBins
+    int* hist = sh.hist[buf];
+    for (int q = tid; q < kSelectBins; q += nth) sh.hist[buf ^ 1][q] = 0;
+    for (int i = tid; i < N; i += nth) {
+      const uint32_t u = keys[i];
+      if (u >= lo && u <= hi) atomicAdd(&hist[(u >> shift) - base], 1);
+    }
+    if (tid == 0) sh.ncand = 0;
+    __syncthreads();
+    topk_block_find_bin(hist, rem, sh);
+    const uint32_t b0 = (base + (uint32_t)sh.sel) << shift;  // <= hi
+    const int cnt = sh.cnt;
+    rem -= sh.above;
+    lo = max(lo, b0);
+    hi = min(hi, b0 + ((1u << shift) - 1u));
+    buf ^= 1;
+    if (lo != hi && cnt <= kSmallCand) {
+      // few candidates: gather them and rank them exactly in one warp
+      for (int i = tid; i < N; i += nth) {
+        const uint32_t u = keys[i];
+        if (u >= lo && u <= hi) {
+          const int p = atomicAdd(&sh.ncand, 1);
+          if (p < kSmallCand) {
+            sh.ckey[p] = u;
+            sh.cidx[p] = i;
+          }
+        }
+      }
+      __syncthreads();
+      topk_warp_rank(sh, min(sh.ncand, kSmallCand), rem, T, need_eq);
+      break;
+    }
+  }
+  // output slots in index order: thread t owns the keys [t * ipt, t * ipt + ipt)
+  const int ipt = (N + nth - 1) / nth;
+  const int beg = min(N, tid * ipt), end = min(N, beg + ipt);
+  uint32_t cnt = 0;  // greater << 16 | equal (N <= 65535)
+  for (int i = beg; i < end; ++i) {
+    const uint32_t u = keys[i];
+    cnt += (u > T ? 0x10000u : 0u) + (u == T ? 1u : 0u);
+  }
+  uint32_t incl = cnt;
 #pragma unroll
   for (int o = 1; o < 32; o <<= 1) {
     const uint32_t y = __shfl_up_sync(0xffffffffu, incl, o);
     if (lane >= o) incl += y;
   }
-  if (lane == 31) warp_tot[warp] = incl;
+  if (lane == 31) sh.wcnt[warp] = incl;
   __syncthreads();
-  if (warp == 0) {
-    const uint32_t t = lane < nw ? warp_tot[lane] : 0u;
-    uint32_t ti = t;
+  uint32_t before = lane < warp ? sh.wcnt[lane] : 0u;  // the lower warps' totals
 #pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const uint32_t y = __shfl_up_sync(0xffffffffu, ti, o);
-      if (lane >= o) ti += y;
-    }
-    warp_tot[lane] = ti - t;
-  }
-  __syncthreads();
-  const uint32_t r = warp_tot[warp] + incl - v;
-  __syncthreads();  // warp_tot may be reused by the caller
-  return r;
-}
-
-// one shared-histogram increment per group of lanes holding the same digit
-// (scores share their leading bytes, so plain per-lane atomics would serialise)
-__device__ __forceinline__ void topk_hist_add(int* hist, uint32_t digit, bool active) {
-  const unsigned act = __ballot_sync(0xffffffffu, active);
-  if (!active) return;
-  const unsigned peers = __match_any_sync(act, digit);
-  if ((threadIdx.x & 31) == __ffs(peers) - 1) atomicAdd(&hist[digit], __popc(peers));
-}
-
-// Selects the k largest of keys[0..N) (shared memory) into out[0..k).
-// Must be called by every thread of the block; keys must be visible (synced).
-__device__ __forceinline__ void topk_block_select(const uint32_t* keys, int N, int k, int* out,
-                                                  TopkShared& sh) {
-  const int tid = threadIdx.x, nth = blockDim.x;
-  uint32_t prefix = 0, pmask = 0;
-  int rem = k;
-  const int iters = (N + nth - 1) / nth;
-  for (int shift = 24; shift >= 0; shift -= 8) {
-    for (int q = tid; q < 256; q += nth) sh.hist[q] = 0;
-    __syncthreads();
-    for (int it = 0; it < iters; ++it) {
-      const int i = it * nth + tid;
-      const uint32_t u = i < N ? keys[i] : 0u;
-      topk_hist_add(sh.hist, (u >> shift) & 255u, i < N && (u & pmask) == prefix);
-    }
-    __syncthreads();
-    if (tid < 32) {
-      const int lane = tid;
-      int c[8], tot = 0;
-#pragma unroll
-      for (int q = 0; q < 8; ++q) {
-        c[q] = sh.hist[255 - 8 * lane - q];
-        tot += c[q];
-      }
-      int incl = tot;
-#pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        const int y = __shfl_up_sync(0xffffffffu, incl, o);
-        if (lane >= o) incl += y;
-      }
-      const int excl = incl - tot;
-      if (excl < rem && rem <= incl) {
-        int cum = excl;
-#pragma unroll
-        for (int q = 0; q < 8; ++q) {
-          if (cum + c[q] >= rem) {
-            sh.prefix = prefix | ((uint32_t)(255 - 8 * lane - q) << shift);
-            sh.rem = rem - cum;
-            break;
-          }
-          cum += c[q];
-        }
-      }
-    }
-    __syncthreads();
-    prefix = sh.prefix;
-    rem = sh.rem;
-    pmask |= 255u << shift;
-    __syncthreads();
-  }
-  const uint32_t T = prefix;
-  const int need_eq = rem;
-  const int ipt = (N + nth - 1) / nth;
-  const int beg = min(N, tid * ipt), end = min(N, beg + ipt);
-  uint32_t gt = 0, eq = 0;
-  for (int i = beg; i < end; ++i) {
-    const uint32_t u = keys[i];
-    gt += u > T;
-    eq += u == T;
-  }
-  const uint32_t base = topk_block_exclusive_scan((gt << 16) | eq, sh.warp_tot);
-  uint32_t gtb = base >> 16, eqb = base & 0xffffu;
+  for (int o = 16; o > 0; o >>= 1) before += __shfl_xor_sync(0xffffffffu, before, o);
+  const uint32_t slot = before + incl - cnt;
+  uint32_t gtb = slot >> 16, eqb = slot & 0xffffu;
   for (int i = beg; i < end; ++i) {
     const uint32_t u = keys[i];
     if (u > T) {
@@ -132,23 +225,113 @@ __device__ __forceinline__ void topk_block_select(const uint32_t* keys, int N, i
   }
 }
 
+// The select of topk_block_select on keys held in registers: thread t owns the
+// KPT keys of indices [t * KPT, t * KPT + KPT) (valid below N), so every
+// per-key loop is unrolled and its loads and atomics are in flight together;
+// every warp ranks the final candidates itself (no barrier after the rank).
+// sh.hist[0] must be cleared and visible; lo/hi are the keys' min and max.
+template <int KPT>
+__device__ __forceinline__ void topk_block_select_reg(const uint32_t (&key)[KPT], int N, int k,
+                                                      uint32_t lo, uint32_t hi, int* out,
+                                                      TopkShared& sh) {
+  const int tid = threadIdx.x, nth = blockDim.x, lane = tid & 31, warp = tid >> 5;
+  const int i0 = tid * KPT;
+  int rem = k;
+  int buf = 0;
+  uint32_t T = lo;
+  int need_eq = rem;
+  for (int pass = 0; pass < 4; ++pass) {
+    if (lo == hi) {
+      T = lo;
+      need_eq = rem;
+      break;
+    }
+    const int hb = 31 - __clz(lo ^ hi);
+    const int shift = hb > 10 ? hb - 10 : 0;
+    const uint32_t base = lo >> shift;
+    int* hist = sh.hist[buf];
+    for (int q = tid; q < kSelectBins; q += nth) sh.hist[buf ^ 1][q] = 0;
+#pragma unroll
+    for (int c = 0; c < KPT; ++c)
+      if (i0 + c < N && key[c] >= lo && key[c] <= hi) atomicAdd(&hist[(key[c] >> shift) - base], 1);
+    if (tid == 0) sh.ncand = 0;
+    __syncthreads();
+    topk_block_find_bin(hist, rem, sh);
+    const uint32_t b0 = (base + (uint32_t)sh.sel) << shift;
+    const int cnt = sh.cnt;
+    rem -= sh.above;
+    lo = max(lo, b0);
+    hi = min(hi, b0 + ((1u << shift) - 1u));
+    buf ^= 1;
+    if (lo != hi && cnt <= kSmallCand) {
+#pragma unroll
+      for (int c = 0; c < KPT; ++c)
+        if (i0 + c < N && key[c] >= lo && key[c] <= hi) {
+          const int p = atomicAdd(&sh.ncand, 1);
+          if (p < kSmallCand) {
+            sh.ckey[p] = key[c];
+            sh.cidx[p] = i0 + c;
+          }
+        }
+      __syncthreads();
+      topk_warp_rank(sh, min(sh.ncand, kSmallCand), rem, T, need_eq);
+      break;
+    }
+  }
+  uint32_t cnt = 0;  // greater << 16 | equal
+#pragma unroll
+  for (int c = 0; c < KPT; ++c)
+    if (i0 + c < N) cnt += (key[c] > T ? 0x10000u : 0u) + (key[c] == T ? 1u : 0u);
+  uint32_t incl = cnt;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint32_t y = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += y;
+  }
+  if (lane == 31) sh.wcnt[warp] = incl;
+  __syncthreads();
+  uint32_t before = lane < warp ? sh.wcnt[lane] : 0u;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) before += __shfl_xor_sync(0xffffffffu, before, o);
+  const uint32_t slot = before + incl - cnt;
+  uint32_t gtb = slot >> 16, eqb = slot & 0xffffu;
+#pragma unroll
+  for (int c = 0; c < KPT; ++c) {
+    if (i0 + c >= N) continue;
+    if (key[c] > T) {
+      out[gtb + min(eqb, (uint32_t)need_eq)] = i0 + c;
+      ++gtb;
+    } else if (key[c] == T) {
+      if (eqb < (uint32_t)need_eq) out[gtb + eqb] = i0 + c;
+      ++eqb;
+    }
+  }
+}
+
 // v_i = (sum over u of partial[row(u)][i], in order) / div: the head-score
 // reduction shared by every path, so all of them give identical bits. Without
 // a head subset, row(u) = u for u < n_part; with one (sel, n_sel positions in a
 // head list of H_sel, in shared memory), row(u) = (u / n_sel) * H_sel +
 // sel[u % n_sel] for u < (n_part / H_sel) * n_sel: the same rows, in the same
 // order, as a head list made of the subset alone.
-// Loads keys[i] and optionally writes the scores. cg: read through L2 only
-// (the partials were written by other CTAs of a still-running grid).
-template <bool CG>
+// Writes keys[i] (and optionally the scores) and returns the thread's min and
+// max key. Every load of a group of columns is issued before the first sum.
 __device__ __forceinline__ void topk_load_partials(const float* P0, int n_part, int N, float div,
                                                    bool zero, float* scores_out, uint32_t* keys,
+                                                   uint32_t& mn, uint32_t& mx,
                                                    const int* sel = nullptr, int n_sel = 0,
                                                    int H_sel = 1) {
   const int tid = threadIdx.x, nth = blockDim.x;
   const int n_sum = sel ? (n_part / H_sel) * n_sel : n_part;
   auto row = [&](int u) -> int { return sel ? (u / n_sel) * H_sel + sel[u % n_sel] : u; };
-  auto ld = [&](size_t off) -> float { return CG ? __ldcg(P0 + off) : __ldg(P0 + off); };
+  auto finish = [&](int i, float s) {
+    const float v = zero ? 0.f : s / div;
+    if (scores_out) scores_out[i] = v;
+    const uint32_t key = float_key(v);
+    keys[i] = key;
+    mn = min(mn, key);
+    mx = max(mx, key);
+  };
   if (n_sum <= 8) {
     // up to 8 partial rows: 4 columns per thread, every load issued first
     int ro[8];
@@ -161,7 +344,7 @@ __device__ __forceinline__ void topk_load_partials(const float* P0, int n_part, 
         const int i = i0 + c * nth + tid;
 #pragma unroll
         for (int u = 0; u < 8; ++u)
-          if (u < n_sum && i < N) t[c][u] = ld((size_t)ro[u] + i);
+          if (u < n_sum && i < N) t[c][u] = __ldg(P0 + (size_t)ro[u] + i);
       }
 #pragma unroll
       for (int c = 0; c < 4; ++c) {
@@ -171,9 +354,7 @@ __device__ __forceinline__ void topk_load_partials(const float* P0, int n_part, 
 #pragma unroll
         for (int u = 0; u < 8; ++u)
           if (u < n_sum) s += t[c][u];
-        const float v = zero ? 0.f : s / div;
-        if (scores_out) scores_out[i] = v;
-        keys[i] = float_key(v);
+        finish(i, s);
       }
     }
   } else {
@@ -190,7 +371,8 @@ __device__ __forceinline__ void topk_load_partials(const float* P0, int n_part, 
         for (int c = 0; c < 4; ++c) {
           const int i = i0 + c * nth + tid;
 #pragma unroll
-          for (int u = 0; u < 8; ++u) t[c][u] = (u0 + u < n_sum && i < N) ? ld((size_t)ro[u] + i) : 0.f;
+          for (int u = 0; u < 8; ++u)
+            t[c][u] = (u0 + u < n_sum && i < N) ? __ldg(P0 + (size_t)ro[u] + i) : 0.f;
         }
 #pragma unroll
         for (int c = 0; c < 4; ++c)
@@ -201,10 +383,34 @@ __device__ __forceinline__ void topk_load_partials(const float* P0, int n_part, 
 #pragma unroll
       for (int c = 0; c < 4; ++c) {
         const int i = i0 + c * nth + tid;
-        if (i >= N) continue;
-        const float v = zero ? 0.f : s[c] / div;
-        if (scores_out) scores_out[i] = v;
-        keys[i] = float_key(v);
+        if (i < N) finish(i, s[c]);
+      }
+    }
+  }
+}
+
+// keys[i] = float_key(scores[i]) (and optionally a copy of the scores), eight
+// loads per thread issued before their keys are written; returns the thread's
+// min and max key
+__device__ __forceinline__ void topk_load_scores(const float* src, int N, float* scores_out,
+                                                 uint32_t* keys, uint32_t& mn, uint32_t& mx) {
+  const int tid = threadIdx.x, nth = blockDim.x;
+  for (int i0 = 0; i0 < N; i0 += 8 * nth) {
+    float v[8];
+#pragma unroll
+    for (int c = 0; c < 8; ++c) {
+      const int i = i0 + c * nth + tid;
+      v[c] = i < N ? __ldg(src + i) : 0.f;
+    }
+#pragma unroll
+    for (int c = 0; c < 8; ++c) {
+      const int i = i0 + c * nth + tid;
+      if (i < N) {
+        if (scores_out) scores_out[i] = v[c];
+        const uint32_t key = float_key(v[c]);
+        keys[i] = key;
+        mn = min(mn, key);
+        mx = max(mx, key);
       }
     }
   }

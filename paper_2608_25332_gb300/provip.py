@@ -28,6 +28,7 @@ F32, BF16 = 0, 1
 ALGO_AUTO, ALGO_SIMT, ALGO_TCGEN05, ALGO_TCGEN05_TWOPASS = 0, 1, 2, 3
 ALGO_TCGEN05_STREAM, ALGO_TCGEN05_CLUSTER = 4, 5
 PRUNE_OVERLAP_PREVIOUS = 1
+PRUNE_CONCURRENT = 2
 
 _P = ctypes.c_void_p
 _I = ctypes.c_int
@@ -48,7 +49,8 @@ _SIGS = {
     "provip_merge_workspace_size": (_Z, [_I, _I, _I, _I]),
     "provip_merge": (_I, [_P, _I, _I, _I, _P, _I, _I, _P, _P, _P, _Z, _P]),
     "provip_similarity_reduce_workspace_size": (_Z, [_I, _I, _I, _I, _I]),
-    "provip_similarity_reduce": (_I, [_P, _I, _I, _I, _P, _P, _I, _P, _I, _I, _P, _P, _P, _P, _P, _Z, _P]),
+    "provip_similarity_reduce": (_I, [_P, _I, _I, _I, _P, _P, _I, _P, _I, _I, _P, _P, _P, _P, _P, _P, _Z,
+                                      _P]),
     "provip_head_scores_workspace_size": (_Z, [_I, _I, _I, _I, _I, _I, _I]),
     "provip_head_scores": (_I, [_P, _P, _I, _I, _I, _I, _I, _P, _I, _P, _P, _P, _I, _I, _I, _P, _I, _I,
                                 _P, _P, _Z, _P]),
@@ -225,29 +227,33 @@ def provip_merge(emb_v, keep_idx, want_merged=True):
 
 
 def provip_similarity_reduce(emb_v, emb_t, text_len, keep_pre, crit_mask=None, want_merged=True,
-                             ws=None, out=None):
-    """Sec. 4.2-4.3 end to end. Returns dict(idx, merged, p, mask); out: the same
-    dict of pre-allocated outputs to write instead."""
+                             ws=None, out=None, want_assign=False):
+    """Sec. 4.2-4.3 end to end. Returns dict(idx, merged, p, mask, assign); out:
+    the same dict of pre-allocated outputs to write instead (assign optional:
+    the merge's nearest-centroid positions [B, N_v], with want_assign or given
+    in out)."""
     B, Nv, D = emb_v.shape
     Ntm = emb_t.shape[1]
     dev = emb_v.device
     if out is not None:
         idx, merged, p, mask = out["idx"], out.get("merged"), out["p"], out["mask"]
+        assign = out.get("assign")
     else:
         idx = torch.empty((B, keep_pre), dtype=torch.int32, device=dev)
         merged = torch.empty((B, keep_pre, D), dtype=emb_v.dtype, device=dev) if want_merged else None
         p = torch.empty((B, Nv), dtype=torch.float32, device=dev)
         mask = torch.empty((B, Ntm), dtype=torch.uint8, device=dev)
+        assign = torch.empty((B, Nv), dtype=torch.int32, device=dev) if (want_assign and want_merged) else None
     L = lib()
     need = L.provip_similarity_reduce_workspace_size(B, Nv, D, Ntm, keep_pre)
     if ws is None or ws.numel() < need:
         ws = workspace(need, dev)
     rc = L.provip_similarity_reduce(_ptr(emb_v), B, Nv, D, _ptr(emb_t), _i32(text_len), Ntm,
                                     _u8(crit_mask), keep_pre, _dtype_code(emb_v), _ptr(idx),
-                                    _ptr(merged), _ptr(p), _ptr(mask), _ptr(ws), ws.numel(),
-                                    _stream(dev))
+                                    _ptr(merged), _i32(assign), _ptr(p), _ptr(mask), _ptr(ws),
+                                    ws.numel(), _stream(dev))
     _check(rc, "provip_similarity_reduce")
-    return dict(idx=idx, merged=merged, p=p, mask=mask)
+    return dict(idx=idx, merged=merged, p=p, mask=mask, assign=assign)
 
 
 # ---------------------------------------------------------------------------

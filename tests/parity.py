@@ -71,3 +71,81 @@ def check_mask_band(mask_gpu, r_ref, rtol, what):
         assert m[above].all() and not m[below].any(), f"{what}: T mask differs outside the band"
     else:
         assert m.all() or not m[below].any(), f"{what}: degenerate T mask"
+
+
+def merge_tol(dtype):
+    """cosine tie band of the nearest-centroid choice: 1e-4 for bf16 inputs
+    (fp32 accumulation of the Gram), 1e-6 for fp32 inputs"""
+    return 1e-6 if dtype == "f32" else 1e-4
+
+
+def out_ulp(x, dtype):
+    """one unit in the last place of the output dtype at |x| (bf16: 8 bits of
+    significand; fp32: numpy's spacing)"""
+    x = np.abs(np.asarray(x, np.float64))
+    if dtype == "f32":
+        return np.spacing(x.astype(np.float32)).astype(np.float64)
+    return 2.0 ** (np.floor(np.log2(np.maximum(x, 1e-30))) - 7)
+
+
+def _unit_rows(X):
+    n = np.linalg.norm(X, axis=1, keepdims=True)
+    return np.where(n > 0, X / np.where(n > 0, n, 1.0), 0.0)
+
+
+def check_merge(Ev, keep, a_gpu, mg_gpu, dtype, what, a_ref, rows, mg_ref=None, centroids=None):
+    """Validity of a nearest-centroid merge (the Sec. 4.3 merge reading) against
+    the oracle's decisions.
+
+    Ev: the sample's visual rows (fp64, as given to the GPU); keep: ascending
+    kept indices; a_gpu [N_v]: the GPU's centroid position of every row; mg_gpu
+    [n1, d]: its merged rows (fp64 view of the output dtype). a_ref: the
+    oracle's centroid positions, valid at least on `rows` (the pruned rows that
+    are checked). mg_ref: the oracle's merged rows when it assigned every row
+    (then every centroid is checked); otherwise `centroids` lists the centroids
+    to check, and each of their GPU members must be in `rows`.
+
+    Rules: kept rows are their own centroid; a checked row whose centroid
+    differs from the oracle's must sit in the tie band (its cosine to the GPU's
+    choice within merge_tol of its cosine to the oracle's, the best); a merged
+    row whose member set equals the oracle's is within one output ulp of the
+    oracle's mean; any other checked merged row is within one output ulp of the
+    fp64 mean over the GPU's own members (a valid choice inside the band)."""
+    n1 = len(keep)
+    nv = Ev.shape[0]
+    a_gpu = np.asarray(a_gpu)
+    assert a_gpu.shape == (nv,), f"{what}: assignment shape {a_gpu.shape}"
+    assert a_gpu.min() >= 0 and a_gpu.max() < n1, f"{what}: centroid position out of range"
+    assert np.array_equal(a_gpu[keep], np.arange(n1)), f"{what}: a kept row is not its own centroid"
+    rows = np.asarray(rows)
+    moved = rows[a_gpu[rows] != a_ref[rows]]
+    if moved.size:
+        U = _unit_rows(Ev[moved])
+        Kg = _unit_rows(Ev[keep[a_gpu[moved]]])
+        Kr = _unit_rows(Ev[keep[a_ref[moved]]])
+        c_gpu = np.sum(U * Kg, axis=1)
+        c_ref = np.sum(U * Kr, axis=1)
+        bad = c_gpu < c_ref - merge_tol(dtype)
+        assert not bad.any(), (f"{what}: {bad.sum()} rows merged into a centroid clearly worse than the "
+                               f"oracle's (rows {moved[bad][:8].tolist()})")
+    if mg_ref is not None:
+        check = np.arange(n1)
+    else:
+        check = np.asarray(centroids)
+    members = {}
+    order = np.argsort(a_gpu, kind="stable")
+    bounds = np.searchsorted(a_gpu[order], np.arange(n1 + 1))
+    for a in check:
+        members[a] = order[bounds[a]:bounds[a + 1]]
+    checked = set(rows.tolist()) | set(np.asarray(keep).tolist())
+    for a in check:
+        mem = members[a]
+        if mg_ref is None:
+            assert set(mem.tolist()) <= checked, f"{what}: centroid {a} has members that were not checked"
+        same = mg_ref is not None and np.array_equal(mem, np.flatnonzero(a_ref == a))
+        expect = mg_ref[a] if same else Ev[mem].mean(axis=0)
+        err = np.abs(np.asarray(mg_gpu[a], np.float64) - expect)
+        lim = out_ulp(expect, dtype) * 1.0001 + 1e-37
+        assert np.all(err <= lim), (f"{what}: merged row {a} ({'oracle member set' if same else 'own members'}"
+                                    f", {len(mem)} rows) beyond one ulp: worst "
+                                    f"{np.max(err / lim):.2f} ulp at column {int(np.argmax(err / lim))}")

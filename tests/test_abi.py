@@ -124,7 +124,7 @@ def test_similarity_validation(L):
     assert L.provip_crit_text(FAKE, 1, 16, 12, FAKE, 1, FAKE, None, None, 0, None) == -2  # D % 8
     assert L.provip_merge(FAKE, 1, 10, 64, FAKE, 11, 1, FAKE, None, None, 0, None) == -1  # keep > N_v
     assert L.provip_merge(FAKE, 1, 10, 16384, FAKE, 5, 1, FAKE, FAKE, None, 0, None) == -2  # D > 8192
-    assert L.provip_similarity_reduce(FAKE, 1, 10, 64, FAKE, FAKE, 8, None, 0, 1, FAKE, None, None,
+    assert L.provip_similarity_reduce(FAKE, 1, 10, 64, FAKE, FAKE, 8, None, 0, 1, FAKE, None, None, None,
                                       None, None, 0, None) == -1  # keep_pre = 0
     assert L.provip_relevance(FAKE, 1, 10, 64, FAKE, FAKE, 8, FAKE, 1, FAKE, None, 0, None) == -3
 

@@ -3,13 +3,14 @@
 The GPU tests are only as strong as tests/parity.py: these CPU cases hand the
 rules outputs with a planted error (a value past the tolerance, a clear winner
 dropped from a keep set, an unsorted or out-of-range index, a T mask that
-disagrees outside the tie band) and check that each is rejected, while correct
-outputs and either choice inside a tie band are accepted.
+disagrees outside the tie band, a merged row off by more than an ulp, a row
+merged into a clearly worse centroid) and check that each is rejected, while
+correct outputs and either choice inside a tie band are accepted.
 """
 import numpy as np
 import pytest
 
-from parity import assert_close_rel, check_mask_band, check_topk_band, rtol_for
+from parity import assert_close_rel, check_mask_band, check_merge, check_topk_band, out_ulp, rtol_for
 
 
 def test_tolerances():
@@ -87,3 +88,71 @@ def test_mask_band():
     # every r equal: the fallback (all rows) is valid
     flat = np.full(5, 0.2)
     check_mask_band(np.ones(5), flat, 1e-3, "fallback")
+
+
+def _merge_case(seed=0, dtype="bf16"):
+    """pruned rows 0..5 near kept rows 6..8; row 5 sits exactly between kept
+    rows 7 and 8 (a cosine tie), so either centroid is valid for it"""
+    rng = np.random.default_rng(seed)
+    d = 16
+    C = rng.standard_normal((3, d))
+    C /= np.linalg.norm(C, axis=1, keepdims=True)
+    Ev = np.zeros((9, d))
+    Ev[6:9] = C * 3.0
+    for j, c in enumerate([0, 0, 1, 1, 2]):
+        Ev[j] = C[c] + 0.05 * rng.standard_normal(d)
+    Ev[5] = C[1] + C[2]  # equidistant from kept rows 7 and 8
+    keep = np.array([6, 7, 8])
+    a_ref = np.array([0, 0, 1, 1, 2, 1, 0, 1, 2])  # the tie goes to the lower position
+    mg = np.stack([Ev[a_ref == a].mean(axis=0) for a in range(3)])
+    rnd = (lambda x: x.astype(np.float32).astype(np.float64)) if dtype == "f32" else \
+        (lambda x: np.round(x * 2.0 ** 20) / 2.0 ** 20)  # well inside one bf16 ulp
+    return Ev, keep, a_ref, mg, rnd
+
+
+def test_merge_rule_accepts_the_oracle_and_a_tie_band_choice():
+    Ev, keep, a_ref, mg, rnd = _merge_case()
+    rows = np.arange(6)
+    check_merge(Ev, keep, a_ref.copy(), rnd(mg), "bf16", "exact", a_ref, rows, mg_ref=mg)
+    # row 5 moved to the other tied centroid: both merged rows become the means over the GPU members
+    a = a_ref.copy()
+    a[5] = 2
+    mg2 = np.stack([Ev[a == k].mean(axis=0) for k in range(3)])
+    check_merge(Ev, keep, a, rnd(mg2), "bf16", "tie move", a_ref, rows, mg_ref=mg)
+    # the sampled form: only centroid 2 and its members are checked
+    check_merge(Ev, keep, a, rnd(mg2), "bf16", "sampled", a_ref, np.array([4, 5]), centroids=[2])
+
+
+def test_merge_rule_rejects_planted_errors():
+    Ev, keep, a_ref, mg, rnd = _merge_case()
+    rows = np.arange(6)
+    # a merged value two ulps off with the oracle's member set
+    bad = mg.copy()
+    bad[1, 3] += 2 * out_ulp(mg[1, 3], "bf16")
+    with pytest.raises(AssertionError, match="beyond one ulp"):
+        check_merge(Ev, keep, a_ref.copy(), bad, "bf16", "value", a_ref, rows, mg_ref=mg)
+    # a row merged into a clearly worse centroid (its value consistent with that choice)
+    a = a_ref.copy()
+    a[0] = 2
+    mg2 = np.stack([Ev[a == k].mean(axis=0) for k in range(3)])
+    with pytest.raises(AssertionError, match="clearly worse"):
+        check_merge(Ev, keep, a, mg2, "bf16", "wrong centroid", a_ref, rows, mg_ref=mg)
+    # a tie-band move whose merged row still holds the oracle's mean (inconsistent)
+    a = a_ref.copy()
+    a[5] = 2
+    with pytest.raises(AssertionError, match="beyond one ulp"):
+        check_merge(Ev, keep, a, mg, "bf16", "stale mean", a_ref, rows, mg_ref=mg)
+    # a kept row that is not its own centroid
+    a = a_ref.copy()
+    a[6] = 1
+    with pytest.raises(AssertionError, match="own centroid"):
+        check_merge(Ev, keep, a, mg, "bf16", "kept row", a_ref, rows, mg_ref=mg)
+    # the sampled form refuses a centroid with unchecked members
+    with pytest.raises(AssertionError, match="not checked"):
+        check_merge(Ev, keep, a_ref.copy(), mg, "bf16", "unchecked", a_ref, np.array([0]), centroids=[0])
+    # fp32 tolerance: one fp32 ulp, not one bf16 ulp
+    Ev, keep, a_ref, mg, rnd = _merge_case(dtype="f32")
+    bad = rnd(mg)
+    bad[2, 0] += 4 * out_ulp(mg[2, 0], "f32")
+    with pytest.raises(AssertionError, match="beyond one ulp"):
+        check_merge(Ev, keep, a_ref.copy(), bad, "f32", "fp32 value", a_ref, rows, mg_ref=mg)
