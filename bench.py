@@ -73,6 +73,13 @@ def parse_args(argv=None):
     ap.add_argument("--streams", type=int, default=None,
                     help="streams of independent batches run concurrently (default: 25 for "
                          "single-sample batches, else 2)")
+    ap.add_argument("--target-s", type=float, default=1.0,
+                    help="seconds of the timed region: the K-step graph is replayed that long, the "
+                         "median repeat reported")
+    ap.add_argument("--no-workloads", action="store_true",
+                    help="skip the video workload block")
+    ap.add_argument("--quick", action="store_true",
+                    help="the headline steps only (no other legs): for profiler captures")
     return ap.parse_args(argv)
 
 
@@ -536,6 +543,121 @@ def run_reference(args, dist):
 # ---------------------------------------------------------------------------
 # the GB300 arm
 # ---------------------------------------------------------------------------
+class Lanes:
+    """S streams of independent batches of one workload (S = 1: a single
+    stream). Lane s has its own inputs (n_copies device copies rotating, so
+    that the data come from HBM), outputs and workspace; step i runs on lane
+    i % S with copy (i // S) % n_copies. Consecutive steps of a lane overlap:
+    each step's head scores may start under that lane's previous compaction
+    (PROVIP_PRUNE_OVERLAP_PREVIOUS); with S > 1 the calls also declare
+    PROVIP_PRUNE_CONCURRENT."""
+
+    def __init__(self, P, synth, w, dev, S, algo, n_copies, seed):
+        import torch
+        self.P, self.torch, self.dev, self.S = P, torch, dev, S
+        flags = P.PRUNE_OVERLAP_PREVIOUS | (P.PRUNE_CONCURRENT if S > 1 else 0)
+        self.lanes = []
+        for s_ in range(S):
+            cpu = synth.in_llm_inputs(w, seed=seed + 7 * s_)
+            cs = [{k: (v.to(dev) if isinstance(v, torch.Tensor) else v) for k, v in cpu.items()}
+                  for _ in range(max(1, n_copies))]
+            st = P.PruneStep(cs[0]["Q"], cs[0]["K"], cs[0]["V"], cs[0]["hidden"], cs[0]["pos"], cpu["head_list"],
+                             w.n_t[1], cpu["N_v"], cpu["keep"], algo=algo, want_scores=False, flags=flags)
+            self.lanes.append((cs, st))
+            if s_ == 0:
+                self.cpu0 = cpu
+        self.vis = self.cpu0["vis_start"]
+        self.streams = [torch.cuda.Stream(device=dev) for _ in range(S)] if S > 1 else None
+
+    def step(self, i):
+        cs, st = self.lanes[i % self.S]
+        c = cs[(i // self.S) % len(cs)]
+        st(c["Q"], c["K"], c["V"], c["hidden"], c["pos"], c["text_start"], c["text_len"], c["seq_len"], self.vis,
+           stream=self.streams[i % self.S] if self.S > 1 else None)
+
+    def run(self, n):
+        """n consecutive steps; with S > 1, forked onto the lane streams and joined"""
+        torch = self.torch
+        if self.S == 1:
+            for i in range(n):
+                self.step(i)
+            return
+        main = torch.cuda.current_stream(self.dev)
+        ev = torch.cuda.Event()
+        ev.record(main)
+        for ls in self.streams:
+            ls.wait_event(ev)
+        for i in range(n):
+            self.step(i)
+        for ls in self.streams:
+            e2 = torch.cuda.Event()
+            e2.record(ls)
+            main.wait_event(e2)
+
+    def graphs(self, K, stream):
+        """CUDA graphs covering exactly K steps (each at most GRAPH_CHUNK steps
+        per lane), each replayed once untimed (a freshly captured graph's first
+        launch runs slower)"""
+        torch = self.torch
+        chunk = GRAPH_CHUNK * self.S
+        sizes, left = [], K
+        while left > 0:
+            sizes.append(min(chunk, left))
+            left -= sizes[-1]
+        made = {}
+        for n in sorted(set(sizes)):
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=stream):
+                self.run(n)
+            made[n] = g
+        torch.cuda.synchronize()
+        for g in made.values():
+            g.replay()
+        torch.cuda.synchronize()
+        return [made[n] for n in sizes]
+
+
+def timed_repeats(torch, graphs, dist, target_s, sampler=None):
+    """Replays the K-step graphs R times back to back between CUDA events (one
+    event per repeat), R sized so that the timed region lasts about target_s;
+    barrier and device synchronisation on both sides. Returns the per-repeat
+    seconds (max over ranks, repeat by repeat) and the clock record."""
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for g in graphs:
+        g.replay()
+    b.record()
+    torch.cuda.synchronize()
+    t1 = max(a.elapsed_time(b) / 1e3, 1e-6)
+    R = int(dist.max(float(max(3, min(20000, math.ceil(target_s / t1))))))
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(R + 1)]
+    if sampler is not None:
+        sampler.start()
+    dist.barrier()
+    torch.cuda.synchronize()
+    w0 = time.time()
+    ev[0].record()
+    for r in range(R):
+        for g in graphs:
+            g.replay()
+        ev[r + 1].record()
+    torch.cuda.synchronize()
+    w1 = time.time()
+    dist.barrier()
+    clocks = sampler.stop(w0, w1) if sampler is not None else None
+    times = [dist.max(ev[r].elapsed_time(ev[r + 1]) / 1e3) for r in range(R)]
+    return times, clocks
+
+
+def summarize(times, units, K, path_bytes, peak):
+    """samples/s from the median repeat, with the spread of the repeats"""
+    med = statistics.median(times)
+    gbs = path_bytes * K / med / 1e9
+    return {"value": units / med, "ms_per_step": 1e3 * med / K, "frac": gbs / peak, "achieved_gbs": gbs,
+            "repeats": {"n": len(times), "min_value": units / max(times), "max_value": units / min(times),
+                        "spread": (max(times) - min(times)) / med}}
+
+
 def run_gb300(args, dist):
     import numpy as np
     import torch
@@ -547,155 +669,75 @@ def run_gb300(args, dist):
     dev = torch.device("cuda", dist.local_rank)
     __graft_entry__.build()
     w = synth.BY_NAME[args.workload]
-    # each rank prunes its own shard of samples (seeded by rank)
-    cpu = synth.in_llm_inputs(w, seed=w.seed + 1000 * dist.rank)
-    vis, nv, keep = cpu["vis_start"], cpu["N_v"], cpu["keep"]
     S = args.streams if args.streams is not None else (25 if w.B == 1 else 2)
     # concurrent streams: the streaming head-score form takes less SM time per
     # sample than the cluster form (at a higher latency), which leaves more of
     # the GPU to the other streams' compactions
     algo_name = "stream" if (args.algo == "auto" and S > 1 and w.dtype == "bf16") else args.algo
-    algo = {"auto": P.ALGO_AUTO, "simt": P.ALGO_SIMT, "tcgen05": P.ALGO_TCGEN05,
-            "stream": P.ALGO_TCGEN05_STREAM, "cluster": P.ALGO_TCGEN05_CLUSTER}[algo_name]
-    copies = []
+    algo_of = {"auto": P.ALGO_AUTO, "simt": P.ALGO_SIMT, "tcgen05": P.ALGO_TCGEN05,
+               "stream": P.ALGO_TCGEN05_STREAM, "cluster": P.ALGO_TCGEN05_CLUSTER}
+    algo = algo_of[algo_name]
     n_copies = max(1, args.copies)
-    for _ in range(n_copies):
-        copies.append({k: (v.to(dev) if isinstance(v, torch.Tensor) else v) for k, v in cpu.items()})
-    g0 = copies[0]
-    # consecutive batches are independent: a step's head scores may start while
-    # the previous step's compaction is still streaming
-    step = P.PruneStep(g0["Q"], g0["K"], g0["V"], g0["hidden"], g0["pos"], g0["head_list"], w.n_t[1], nv, keep,
-                       algo=algo, want_scores=False, flags=P.PRUNE_OVERLAP_PREVIOUS)
-    step_serial = P.PruneStep(g0["Q"], g0["K"], g0["V"], g0["hidden"], g0["pos"], g0["head_list"], w.n_t[1], nv,
-                              keep, algo=algo, want_scores=False, flags=0, ws=step.ws)
-
-    # Concurrent streams of independent batches (single-sample batches cannot
-    # fill the GPU with one dependent chain): stream s takes steps s, s + S, ...
-    # on its own input copies and its own outputs and workspace; lane 0 is the
-    # step and copies above.
-    if S < 1 or args.steps % S:
+    K = args.steps
+    if S < 1 or K % S:
         raise SystemExit(f"--streams {S} must divide --steps")
-    # graphs of GRAPH_CHUNK steps per stream: with many short single-sample
-    # chains, a small graph would spend a visible part of its time filling and
-    # draining the streams
-    chunk = GRAPH_CHUNK * S
-    lanes = [(copies, step)]
-    for s_ in range(1, S):
-        cpu_s = synth.in_llm_inputs(w, seed=w.seed + 1000 * dist.rank + 7 * s_)
-        cs = [{k: (v.to(dev) if isinstance(v, torch.Tensor) else v) for k, v in cpu_s.items()}
-              for _ in range(n_copies)]
-        st_s = P.PruneStep(cs[0]["Q"], cs[0]["K"], cs[0]["V"], cs[0]["hidden"], cs[0]["pos"], cs[0]["head_list"],
-                           w.n_t[1], nv, keep, algo=algo, want_scores=False, flags=P.PRUNE_OVERLAP_PREVIOUS)
-        lanes.append((cs, st_s))
-    lane_streams = [torch.cuda.Stream(device=dev) for _ in range(S)] if S > 1 else None
+    peak, peak_src = hbm_peak()
+    stream = torch.cuda.Stream(device=dev)
+    seed = w.seed + 1000 * dist.rank  # each rank prunes its own shard of samples
 
-    def do_step(i):
-        cs, st = lanes[i % S]
-        c = cs[(i // S) % len(cs)]
-        st(c["Q"], c["K"], c["V"], c["hidden"], c["pos"], c["text_start"], c["text_len"], c["seq_len"], vis,
-           stream=lane_streams[i % S] if S > 1 else None)
-
-    # one stream: with --algo auto, the head-score form the library picks for a
-    # single stream (the streaming form above is chosen for concurrent ones)
-    single_algo = P.ALGO_AUTO if args.algo == "auto" else algo
-    step_one = step if single_algo == algo else P.PruneStep(
-        g0["Q"], g0["K"], g0["V"], g0["hidden"], g0["pos"], g0["head_list"], w.n_t[1], nv, keep,
-        algo=single_algo, want_scores=False, flags=P.PRUNE_OVERLAP_PREVIOUS)
-
-    def do_step_single(i):
-        c = copies[i % len(copies)]
-        step_one(c["Q"], c["K"], c["V"], c["hidden"], c["pos"], c["text_start"], c["text_len"], c["seq_len"],
-                 vis)
-
-    def run_steps(n):
-        # n consecutive steps; with S > 1, fork onto the lane streams and join
-        if S == 1:
-            for i in range(n):
-                do_step(i)
-            return
-        main = torch.cuda.current_stream(dev)
-        ev = torch.cuda.Event()
-        ev.record(main)
-        for ls in lane_streams:
-            ls.wait_event(ev)
-        for i in range(n):
-            do_step(i)
-        for ls in lane_streams:
-            e2 = torch.cuda.Event()
-            e2.record(ls)
-            main.wait_event(e2)
-
-    # warm-up
-    run_steps(max(args.warmup, 1) * S)
+    # ---- the headline: S concurrent streams of independent batches ----
+    lanes = Lanes(P, synth, w, dev, S, algo, n_copies, seed)
+    cpu = lanes.cpu0
+    vis, nv, keep = cpu["vis_start"], cpu["N_v"], cpu["keep"]
+    lanes.run(max(args.warmup, 1) * S)
     torch.cuda.synchronize()
     rc, bits = P.provip_device_status(clear=True)
     if rc != 0:
         raise RuntimeError(f"device status {rc} {bits} after warm-up")
-
-    # graphs of up to `chunk` steps (the step index picks the input copy)
-    K = args.steps
-    sizes = []
-    left = K
-    while left > 0:
-        n = min(chunk, left)
-        sizes.append(n)
-        left -= n
-    graphs = {}
-    stream = torch.cuda.Stream(device=dev)
-    for n in sorted(set(sizes)):
-        g = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(g, stream=stream):
-            run_steps(n)
-        graphs[n] = g
-    torch.cuda.synchronize()
-    # one untimed replay of each graph: the first launch of a freshly captured
-    # graph (upload, cold instruction and address-translation caches) runs
-    # slower than the ones after it
-    for g in graphs.values():
-        g.replay()
-    torch.cuda.synchronize()
-
-    sampler = ClockSampler(visible_device_index(dist.local_rank) if dist.rank == 0 else None)
-    if dist.rank == 0:
-        sampler.start()
-    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    dist.barrier()
-    torch.cuda.synchronize()
-    t_wall0 = time.time()
-    ev0.record()
-    for n in sizes:
-        graphs[n].replay()
-    ev1.record()
-    torch.cuda.synchronize()
-    t_wall1 = time.time()
-    dist.barrier()
-    sec = ev0.elapsed_time(ev1) / 1e3
-    clocks = sampler.stop(t_wall0, t_wall1) if dist.rank == 0 else None
-    max_sec = dist.max(sec)
-    total_samples = dist.sum(float(w.B * K))
-    value = aggregate(total_samples, max_sec)
+    ab = algorithmic_bytes(w, cpu)
+    graphs = lanes.graphs(K, stream)
+    sampler = ClockSampler(visible_device_index(dist.local_rank)) if dist.rank == 0 else None
+    times, clocks = timed_repeats(torch, graphs, dist, args.target_s, sampler)
+    units = dist.sum(float(w.B * K))
+    head = summarize(times, units, K, ab["path"], peak)
+    max_sec = statistics.median(times)
+    value = head["value"]
     rc, bits = P.provip_device_status(clear=True)
     if rc != 0:
         raise RuntimeError(f"device status {rc} {bits} after the timed region")
+    del graphs
+    if args.quick:
+        if dist.rank == 0:
+            print(json.dumps({"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": dist.world, "steps": K,
+                              "warmup": args.warmup, "ms_per_step": 1e3 * max_sec / K, "quick": True,
+                              "config": workload_config(w, algo_name, n_copies), "repeats": head["repeats"]}))
+        return 0
 
-    # per-kernel durations (same launch configuration, graphs of GRAPH_CHUNK launches)
-    ab = algorithmic_bytes(w, cpu)
-    out = step(g0["Q"], g0["K"], g0["V"], g0["hidden"], g0["pos"], g0["text_start"], g0["text_len"],
-               g0["seq_len"], vis)
+    # ---- the same workload on one stream: the configuration as stated ----
+    single_algo = P.ALGO_AUTO if args.algo == "auto" else algo
+    if S > 1:
+        one = Lanes(P, synth, w, dev, 1, single_algo, n_copies, seed)
+        one.run(3)
+        g1 = one.graphs(K, stream)
+        t1s, _ = timed_repeats(torch, g1, dist, args.target_s / 2)
+        single = dict(summarize(t1s, units, K, ab["path"], peak), streams=1,
+                      algo="auto" if single_algo == P.ALGO_AUTO else algo_name)
+        del g1
+    else:
+        single = dict(head, streams=1, algo=algo_name)
+
+    # per-kernel durations of the headline's launch configuration (graphs of
+    # GRAPH_CHUNK launches): the compaction (dominant), head scores + top-k, the
+    # step with no cross-step overlap
+    g0 = lanes.lanes[0][0][0]
+    step0 = lanes.lanes[0][1]
+    copies = lanes.lanes[0][0]
+    out = step0(g0["Q"], g0["K"], g0["V"], g0["hidden"], g0["pos"], g0["text_start"], g0["text_len"], g0["seq_len"],
+                vis)
     idx = out["idx"].clone()
-    outs = (step.hidden_out, step.K_out, step.V_out, step.pos_out)
-    ws_ht = P.workspace(step.ws.numel(), dev)
-
-    def compact_i(i):
-        c = copies[i % len(copies)]
-        P.provip_compact(idx, c["hidden"], c["K"], c["V"], c["pos"], c["seq_len"], vis, nv, out=outs)
-
+    outs = (step0.hidden_out, step0.K_out, step0.V_out, step0.pos_out)
+    ws_ht = P.workspace(step0.ws.numel(), dev)
     heads_host = cpu["head_list"].tolist()
-
-    def head_topk_i(i):
-        c = copies[i % len(copies)]
-        P.provip_head_topk(c["Q"], c["K"], heads_host, c["text_start"], c["text_len"], c["seq_len"], vis, nv,
-                           keep, algo=algo, N_t_max=w.n_t[1], ws=ws_ht, want_scores=False)
 
     def time_graph(fn, reps):
         for i in range(3):
@@ -715,155 +757,210 @@ def run_gb300(args, dist):
         torch.cuda.synchronize()
         return a.elapsed_time(b) / 1e3 / (reps * GRAPH_CHUNK)
 
-    # kernels per step: one-pass head scores (tcgen05, L_max <= 8192), top-k,
-    # compaction; the two-pass and CUDA-core forms launch two head kernels
-    launches_per_step = 3 if (algo_name in ("auto", "tcgen05", "stream", "cluster") and w.dtype == "bf16"
-                              and w.L_max <= 8192) else 4
-    reps = max(1, min(20, K // GRAPH_CHUNK))
-    t_compact = time_graph(compact_i, reps)
-    # context for the fraction: torch's copy_ (the operation the HBM peak was
-    # measured with, there over 2 GiB) on the same bytes (half read, half
-    # written), its source rotating over three buffers as the inputs do, timed
-    # the same way
-    n_el = ab["compact"] // 4  # bf16 elements read (= written)
-    copy_src = [torch.empty(n_el, dtype=torch.bfloat16, device=dev).fill_(1.0) for _ in range(3)]
-    copy_dst = torch.empty(n_el, dtype=torch.bfloat16, device=dev)
-    t_copy = time_graph(lambda i: copy_dst.copy_(copy_src[i % 3]), reps)
-    del copy_src, copy_dst
-    t_head = time_graph(head_topk_i, reps)
+    def compact_i(i):
+        c = copies[i % len(copies)]
+        P.provip_compact(idx, c["hidden"], c["K"], c["V"], c["pos"], c["seq_len"], vis, nv, out=outs)
+
+    def head_topk_i(i):
+        c = copies[i % len(copies)]
+        P.provip_head_topk(c["Q"], c["K"], heads_host, c["text_start"], c["text_len"], c["seq_len"], vis, nv,
+                           keep, algo=algo, N_t_max=w.n_t[1], ws=ws_ht, want_scores=False)
+
+    step_serial = P.PruneStep(g0["Q"], g0["K"], g0["V"], g0["hidden"], g0["pos"], cpu["head_list"], w.n_t[1], nv,
+                              keep, algo=algo, want_scores=False, flags=0, ws=step0.ws)
 
     def serial_i(i):
         c = copies[i % len(copies)]
         step_serial(c["Q"], c["K"], c["V"], c["hidden"], c["pos"], c["text_start"], c["text_len"], c["seq_len"], vis)
 
+    # kernels per step: one-pass head scores (tcgen05, L_max <= 8192), top-k,
+    # compaction; the two-pass and CUDA-core forms launch two head kernels
+    launches_per_step = 3 if (algo_name in ("auto", "tcgen05", "stream", "cluster") and w.dtype == "bf16"
+                              and w.L_max <= 8192) else 4
+    reps = 20
+    t_compact = time_graph(compact_i, reps)
+    t_head = time_graph(head_topk_i, reps)
     t_serial = time_graph(serial_i, reps)
-    # the same step on one stream (each step's head scores overlap the previous
-    # step's compaction, nothing else runs beside it)
-    t_single = time_graph(do_step_single, reps) if S > 1 else None
-    peak, peak_src = hbm_peak()
-
-    # the next rows on the same batches: shallow-layer pruning with the N_VIS
-    # most confident heads of each sample (confidence over every head), and
-    # the middle-layer variant over every head
-    ab_all = algorithmic_bytes(w, cpu, all_heads=True)
-    vh = P.VisualHeadsPruneStep(g0["Q"], g0["K"], g0["V"], g0["hidden"], g0["pos"], w.n_t[1], nv, keep,
-                                min(N_VIS, w.H_q), algo=algo, want_scores=False, want_conf=False,
-                                flags=P.PRUNE_OVERLAP_PREVIOUS)
-    ah = P.PruneStep(g0["Q"], g0["K"], g0["V"], g0["hidden"], g0["pos"], None, w.n_t[1], nv, keep,
-                     algo=algo, want_scores=False, flags=P.PRUNE_OVERLAP_PREVIOUS)
-
-    def vh_i(i):
-        c = copies[i % len(copies)]
-        vh(c["Q"], c["K"], c["V"], c["hidden"], c["pos"], c["text_start"], c["text_len"], c["seq_len"], vis)
-
-    def ah_i(i):
-        c = copies[i % len(copies)]
-        ah(c["Q"], c["K"], c["V"], c["hidden"], c["pos"], c["text_start"], c["text_len"], c["seq_len"], vis)
-
-    def time_lanes(make, reps):
-        # the same steps on the S concurrent streams of the headline: one step
-        # object per lane (own outputs and workspace) over that lane's inputs,
-        # graphs of GRAPH_CHUNK steps per stream; seconds per step (one batch)
-        objs = [make(cs[0]) for cs, _ in lanes]
-
-        def run(n):
-            main = torch.cuda.current_stream(dev)
-            ev = torch.cuda.Event()
-            ev.record(main)
-            for ls in lane_streams:
-                ls.wait_event(ev)
-            for i in range(n):
-                cs = lanes[i % S][0]
-                c = cs[(i // S) % len(cs)]
-                objs[i % S](c["Q"], c["K"], c["V"], c["hidden"], c["pos"], c["text_start"], c["text_len"],
-                            c["seq_len"], vis, stream=lane_streams[i % S])
-            for ls in lane_streams:
-                e2 = torch.cuda.Event()
-                e2.record(ls)
-                main.wait_event(e2)
-
-        run(3 * S)
-        torch.cuda.synchronize()
-        g = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(g, stream=stream):
-            run(GRAPH_CHUNK * S)
-        torch.cuda.synchronize()
-        g.replay()  # untimed first launch
-        torch.cuda.synchronize()
-        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        a.record()
-        for _ in range(reps):
-            g.replay()
-        b.record()
-        torch.cuda.synchronize()
-        return a.elapsed_time(b) / 1e3 / (reps * GRAPH_CHUNK * S)
-
-    def make_vh(c):
-        return P.VisualHeadsPruneStep(c["Q"], c["K"], c["V"], c["hidden"], c["pos"], w.n_t[1], nv, keep,
-                                      min(N_VIS, w.H_q), algo=algo, want_scores=False, want_conf=False,
-                                      flags=P.PRUNE_OVERLAP_PREVIOUS)
-
-    def make_ah(c):
-        return P.PruneStep(c["Q"], c["K"], c["V"], c["hidden"], c["pos"], None, w.n_t[1], nv, keep,
-                           algo=algo, want_scores=False, flags=P.PRUNE_OVERLAP_PREVIOUS)
-
-    next_rows = {}
-    for name, fn, make, extra in (
-            ("visual_heads", vh_i, make_vh, {"n_vis": min(N_VIS, w.H_q), "heads_scored": w.H_q}),
-            ("all_heads", ah_i, make_ah, {"heads_scored": w.H_q})):
-        t = time_graph(fn, reps)
-        gbs = ab_all["path"] / t / 1e9
-        next_rows[name] = dict(extra, us_per_step=t * 1e6, samples_per_s=w.B / t,
-                               algorithmic_bytes=ab_all["path"], achieved_gbs=gbs, frac=gbs / peak)
-        if S > 1:
-            tc = time_lanes(make, reps)
-            gc = ab_all["path"] / tc / 1e9
-            next_rows[name]["streams"] = dict(streams=S, us_per_step=tc * 1e6, samples_per_s=w.B / tc,
-                                              achieved_gbs=gc, frac=gc / peak)
-    rc, bits = P.provip_device_status(clear=True)
-    if rc != 0:
-        raise RuntimeError(f"device status {rc} {bits} after the next-row legs")
     ach = ab["compact"] / t_compact / 1e9
     traffic = None
     if COMPACT_TRAFFIC["bytes"] and COMPACT_TRAFFIC["sha1"] == kernel_sha1("compact.cu") and \
             args.workload == DEFAULT_WORKLOAD:
         traffic = COMPACT_TRAFFIC["bytes"]
-    path_gbs = ab["path"] * K / max_sec / 1e9  # per GPU
 
-    # e2e: host buffers through the C ABI. Every step copies its inputs from
-    # pinned host memory and its outputs back to pinned host memory inside the
-    # timed region; two device buffer sets (each with its own outputs) alternate
-    # so that the copies of one step overlap the pruning of the other (a stream
-    # per copy direction and one for the kernels, ordered by events).
+    # ---- the next rows on the same batches ----
+    ab_all = algorithmic_bytes(w, cpu, all_heads=True)
+    next_rows = {}
+    for name, make in (
+            ("visual_heads", lambda c, fl: P.VisualHeadsPruneStep(
+                c["Q"], c["K"], c["V"], c["hidden"], c["pos"], w.n_t[1], nv, keep, min(N_VIS, w.H_q), algo=algo,
+                want_scores=False, want_conf=False, flags=fl)),
+            ("all_heads", lambda c, fl: P.PruneStep(
+                c["Q"], c["K"], c["V"], c["hidden"], c["pos"], None, w.n_t[1], nv, keep, algo=algo,
+                want_scores=False, flags=fl))):
+        obj = make(g0, P.PRUNE_OVERLAP_PREVIOUS)
+
+        def fn(i, obj=obj):
+            c = copies[i % len(copies)]
+            obj(c["Q"], c["K"], c["V"], c["hidden"], c["pos"], c["text_start"], c["text_len"], c["seq_len"], vis)
+
+        t = time_graph(fn, reps)
+        gbs = ab_all["path"] / t / 1e9
+        next_rows[name] = {"us_per_step": t * 1e6, "samples_per_s": w.B / t, "frac": gbs / peak}
+    next_rows["heads_scored"] = w.H_q
+    next_rows["algorithmic_bytes"] = ab_all["path"]
+    rc, bits = P.provip_device_status(clear=True)
+    if rc != 0:
+        raise RuntimeError(f"device status {rc} {bits} after the per-kernel legs")
+
+    # ---- e2e through the C ABI with host buffers ----
+    e2e = e2e_measure(P, torch, dist, w, cpu, step0, algo, dev, max(1, args.e2e_steps))
+    del lanes
+
+    # ---- the video GQA workload (one sample per batch): as stated, and as
+    # concurrent single-sample batches (an effective batch of S_v) ----
+    workloads = {}
+    if not args.no_workloads and w.name != VIDEO_WORKLOAD:
+        workloads[VIDEO_WORKLOAD] = video_measure(P, synth, torch, dist, dev, stream, args, peak)
+
+    prellm = prellm_measure(w, dev) if dist.rank == 0 else None
+    schedule = schedule_measure(w, dev) if dist.rank == 0 else None
+    ablation = ablation_measure(dev) if dist.rank == 0 else None
+    cpu_base = None
+    if dist.rank == 0 and dist.world == 1 and not args.no_cpu_baseline:
+        cpu_base = cpu_baseline(cpu, w, vis, nv, keep)
+
+    if dist.rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": dist.world, "steps": K,
+            "warmup": args.warmup, "ms_per_step": 1e3 * max_sec / K, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
+            "config": dict(workload_config(w, algo_name, n_copies, e2e["h2d_bytes_per_step"] / 1e6), streams=S,
+                           **({"concurrency": f"{S} streams of independent batches run concurrently (each with its "
+                                              f"own inputs, outputs and workspace); value counts the samples of all "
+                                              f"streams; single_stream is one stream"} if S > 1 else {})),
+            "single_stream": single,
+            "repeats": head["repeats"],
+            "roofline": {"bound": "hbm", "kernel": "compact_kernel", "achieved": ach, "peak": peak,
+                         "peak_source": peak_src, "unit": "GB/s", "frac": ach / peak, "traffic": traffic,
+                         "algorithmic_bytes": ab["compact"], "duration_us": t_compact * 1e6},
+            "path": {"algorithmic_bytes": ab["path"], "achieved_gbs": head["achieved_gbs"], "frac": head["frac"],
+                     "head_topk_us": t_head * 1e6, "compact_us": t_compact * 1e6,
+                     "step_us_without_overlap": t_serial * 1e6},
+            "workloads": workloads,
+            "e2e": e2e,
+            "cpu_baseline": cpu_base,
+            "gpu_launches": launches_per_step * K * head["repeats"]["n"],
+            "prellm": prellm,
+            "next_rows": dict(next_rows, schedule=schedule, ablation=ablation),
+            "clocks": clocks,
+        }
+        print(json.dumps(line))
+    return 0
+
+
+VIDEO_WORKLOAD = "video_gqa_bf16_b1"
+
+
+def video_measure(P, synth, torch, dist, dev, stream, args, peak):
+    """The video GQA workload (B = 1): one stream with the library's automatic
+    head-score form (the configuration as stated), then S_v concurrent streams
+    of independent single-sample batches with the streaming form (an effective
+    batch of S_v), each timed as repeats of 100-step graphs per stream; the
+    compaction alone on one stream for the roofline."""
+    w = synth.BY_NAME[VIDEO_WORKLOAD]
+    seed = w.seed + 1000 * dist.rank
+    n_copies = max(1, args.copies)
+    out = {}
+    for label, S, algo_name in (("single_stream", 1, "auto"), ("streams", 25, "stream")):
+        lanes = Lanes(P, synth, w, dev, S, P.ALGO_AUTO if algo_name == "auto" else P.ALGO_TCGEN05_STREAM,
+                      n_copies, seed)
+        lanes.run(3 * S)
+        K = GRAPH_CHUNK * S
+        graphs = lanes.graphs(K, stream)
+        times, _ = timed_repeats(torch, graphs, dist, args.target_s / 2)
+        ab = algorithmic_bytes(w, lanes.cpu0)
+        r = summarize(times, dist.sum(float(w.B * K)), K, ab["path"], peak)
+        r.update(streams=S, algo=algo_name, us_per_sample=1e6 / r["value"] * dist.world)
+        if S > 1:
+            r["effective_batch"] = S
+        out[label] = r
+        if S == 1:
+            cs, st = lanes.lanes[0]
+            c0 = cs[0]
+            res = st(c0["Q"], c0["K"], c0["V"], c0["hidden"], c0["pos"], c0["text_start"], c0["text_len"],
+                     c0["seq_len"], lanes.vis)
+            idx = res["idx"].clone()
+            outs = (st.hidden_out, st.K_out, st.V_out, st.pos_out)
+
+            def compact_i(i):
+                c = cs[i % len(cs)]
+                P.provip_compact(idx, c["hidden"], c["K"], c["V"], c["pos"], c["seq_len"], lanes.vis,
+                                 lanes.cpu0["N_v"], out=outs)
+
+            for i in range(3):
+                compact_i(i)
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=stream):
+                for i in range(GRAPH_CHUNK):
+                    compact_i(i)
+            g.replay()
+            torch.cuda.synchronize()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record()
+            for _ in range(20):
+                g.replay()
+            b.record()
+            torch.cuda.synchronize()
+            tc = a.elapsed_time(b) / 1e3 / (20 * GRAPH_CHUNK)
+            ach = ab["compact"] / tc / 1e9
+            out["roofline"] = {"bound": "hbm", "kernel": "compact_kernel", "achieved": ach, "peak": peak,
+                               "unit": "GB/s", "frac": ach / peak, "algorithmic_bytes": ab["compact"],
+                               "duration_us": tc * 1e6}
+            out["path_bytes"] = ab["path"]
+        del lanes
+        torch.cuda.synchronize()
+    rc, bits = P.provip_device_status(clear=True)
+    if rc != 0:
+        raise RuntimeError(f"device status {rc} {bits} after the video legs")
+    return out
+
+
+def e2e_measure(P, torch, dist, w, cpu, step0, algo, dev, E):
+    """e2e through the C ABI with host buffers. Every step copies its inputs
+    from pinned host memory and its outputs back to pinned host memory inside
+    the timed region; two device buffer sets (each with its own outputs)
+    alternate so that the copies of one step overlap the pruning of the other
+    (a stream per copy direction and one for the kernels, ordered by events).
+    Three timed runs of E steps, the median reported with the three beside it
+    (the host copies share the machine's memory system with other jobs)."""
+    nv, keep, vis = cpu["N_v"], cpu["keep"], cpu["vis_start"]
     pin = {k: v.pin_memory() for k, v in cpu.items() if isinstance(v, torch.Tensor)}
     out_keys = ("hidden", "K", "V", "pos", "idx", "seq_len")
-    e2e_sets = []
+    sets = []
     for j in range(2):
         db = {k: torch.empty_like(v, device=dev) for k, v in pin.items()}
-        st_j = step if j == 0 else P.PruneStep(db["Q"], db["K"], db["V"], db["hidden"], db["pos"], cpu["head_list"],
-                                              w.n_t[1], nv, keep, algo=algo, want_scores=False,
-                                              flags=P.PRUNE_OVERLAP_PREVIOUS)
+        st_j = P.PruneStep(db["Q"], db["K"], db["V"], db["hidden"], db["pos"], cpu["head_list"], w.n_t[1], nv, keep,
+                           algo=algo, want_scores=False, flags=P.PRUNE_OVERLAP_PREVIOUS)
         outs_j = {"hidden": st_j.hidden_out, "K": st_j.K_out, "V": st_j.V_out, "pos": st_j.pos_out,
                   "idx": st_j.idx, "seq_len": st_j.seq_len_out}
         ho = {k: torch.empty(outs_j[k].shape, dtype=outs_j[k].dtype, pin_memory=True) for k in out_keys}
         ev = {n: torch.cuda.Event() for n in ("comp", "d2h")}
-        e2e_sets.append((db, st_j, ho, ev))
+        sets.append((db, st_j, ho, ev))
     h2d = sum(v.numel() * v.element_size() for v in pin.values())
-    d2h = sum(v.numel() * v.element_size() for v in e2e_sets[0][2].values())
+    d2h = sum(v.numel() * v.element_size() for v in sets[0][2].values())
     s_comp, s_d2h = (torch.cuda.Stream(device=dev) for _ in range(2))
-    # the input copies are spread over N_H2D streams (copy engines) by size
-    N_H2D = 2
-    s_h2ds = [torch.cuda.Stream(device=dev) for _ in range(N_H2D)]
+    n_h2d = 2  # the input copies are spread over two streams (copy engines) by size
+    s_h2ds = [torch.cuda.Stream(device=dev) for _ in range(n_h2d)]
     by_size = sorted(pin, key=lambda k: -pin[k].numel() * pin[k].element_size())
-    h2d_parts = [by_size[i::N_H2D] for i in range(N_H2D)]
+    parts = [by_size[i::n_h2d] for i in range(n_h2d)]
     for j in range(2):
-        e2e_sets[j][3]["h2d_parts"] = [torch.cuda.Event() for _ in range(N_H2D)]
+        sets[j][3]["h2d_parts"] = [torch.cuda.Event() for _ in range(n_h2d)]
     fresh = [True, True]
 
-    def e2e_step(n):
+    def one(n):
         j = n % 2
-        db, st_j, ho, ev = e2e_sets[j]
-        for s_h2d, keys, e_part in zip(s_h2ds, h2d_parts, ev["h2d_parts"]):
+        db, st_j, ho, ev = sets[j]
+        for s_h2d, keys, e_part in zip(s_h2ds, parts, ev["h2d_parts"]):
             with torch.cuda.stream(s_h2d):
                 if not fresh[j]:
                     s_h2d.wait_event(ev["comp"])  # the set's inputs were consumed by step n - 2
@@ -885,85 +982,33 @@ def run_gb300(args, dist):
             ev["d2h"].record(s_d2h)
         fresh[j] = False
 
-    def e2e_run(first, n_steps):
+    def run(first, n_steps):
         main = torch.cuda.current_stream(dev)
         start = torch.cuda.Event()
         start.record(main)
         for st_ in (*s_h2ds, s_comp, s_d2h):
             st_.wait_event(start)
         for n in range(first, first + n_steps):
-            e2e_step(n)
+            one(n)
         for st_ in (*s_h2ds, s_comp, s_d2h):
             done = torch.cuda.Event()
             done.record(st_)
             main.wait_event(done)
 
-    e2e_run(0, 4)
+    run(0, 4)
     torch.cuda.synchronize()
-    E = max(1, args.e2e_steps)
-    # three timed runs of E steps each, the median reported: the host copies
-    # share the machine's memory system with other jobs, so a single run can be
-    # an outlier
-    e2e_runs = []
-    first = 4
+    runs, first = [], 4
     for _ in range(3):
         a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         dist.barrier()
         a.record()
-        e2e_run(first, E)
+        run(first, E)
         b.record()
         torch.cuda.synchronize()
         first += E
-        e2e_sec = dist.max(a.elapsed_time(b) / 1e3)
-        e2e_runs.append(aggregate(dist.sum(float(w.B * E)), e2e_sec))
-    e2e_value = sorted(e2e_runs)[1]
-
-    prellm = prellm_measure(w, dev) if dist.rank == 0 else None
-    schedule = schedule_measure(w, dev) if dist.rank == 0 else None
-    ablation = ablation_measure(dev) if dist.rank == 0 else None
-
-    cpu_base = None
-    if dist.rank == 0 and dist.world == 1 and not args.no_cpu_baseline:
-        cpu_base = cpu_baseline(cpu, w, vis, nv, keep)
-
-    if dist.rank == 0:
-        line = {
-            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": dist.world, "steps": K,
-            "warmup": args.warmup, "ms_per_step": 1e3 * max_sec / K, "higher_is_better": True,
-            "scaling": "weak", "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
-            "config": dict(workload_config(w, algo_name, len(copies),
-                                           sum(v.numel() * v.element_size() for v in pin.values()) / 1e6),
-                           streams=S,
-                           **({"concurrency": f"{S} streams of independent batches run concurrently, each "
-                                              f"with its own inputs, outputs and workspace; value counts the "
-                                              f"samples of all streams"} if S > 1 else {})),
-            "roofline": {"bound": "hbm", "kernel": "compact_kernel", "achieved": ach, "peak": peak,
-                         "peak_source": peak_src, "unit": "GB/s", "frac": ach / peak,
-                         "traffic": traffic, "algorithmic_bytes": ab["compact"],
-                         "duration_us": t_compact * 1e6,
-                         "copy_same_bytes": {"duration_us": t_copy * 1e6,
-                                             "frac": ab["compact"] / t_copy / 1e9 / peak,
-                                             "note": "torch copy_ (the operation the peak was measured "
-                                                     "with, over 2 GiB) on the same bytes, timed the "
-                                                     "same way"}},
-            "path": {"algorithmic_bytes": ab["path"], "achieved_gbs": path_gbs, "frac": path_gbs / peak,
-                     "head_topk_us": t_head * 1e6, "head_topk_bytes": ab["head_topk"],
-                     "compact_us": t_compact * 1e6,
-                     "step_us_without_overlap": t_serial * 1e6,
-                     **({"single_stream": {"algo": "auto" if single_algo == P.ALGO_AUTO else algo_name,
-                                           "value": w.B / t_single, "ms_per_step": t_single * 1e3,
-                                           "frac": ab["path"] / t_single / 1e9 / peak}}
-                        if t_single else {})},
-            "cpu_baseline": cpu_base,
-            "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
-                    "runs": e2e_runs, "note": f"median of 3 timed runs of {E} steps"},
-            "gpu_launches": launches_per_step * K,
-            "prellm": prellm,
-            "next_rows": dict(next_rows, schedule=schedule, ablation=ablation),
-            "clocks": clocks,
-        }
-        print(json.dumps(line))
-    return 0
+        runs.append(aggregate(dist.sum(float(w.B * E)), dist.max(a.elapsed_time(b) / 1e3)))
+    return {"value": sorted(runs)[1], "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+            "runs": runs, "note": f"median of 3 timed runs of {E} steps"}
 
 
 def run_prellm_only(args):

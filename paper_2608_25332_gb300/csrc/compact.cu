@@ -66,6 +66,18 @@ constexpr int kSmallPieces = 4;
 // bytes of rows per CTA below which a compaction that runs alone uses fewer
 // CTAs than two per SM
 constexpr long long kMinCtaBytesAlone = 16 * 1024;
+// kept rows of a CTA whose indices the producer stages in shared memory, and
+// how many of those loads it keeps in flight at once
+constexpr int kIdxStage = 256;
+constexpr int kStageBatch = 16;
+// rows whose (sample, output row, source row) the helper threads work out
+// together before copying them
+constexpr int kMetaRows = 96;
+
+// barrier of the helper threads (warps 1..3; the producer warp does not take part)
+__device__ __forceinline__ void helpers_sync() {
+  asm volatile("bar.sync 1, %0;" ::"n"(kCompactThreads - 32) : "memory");
+}
 
 __device__ __forceinline__ int src_row(const CompactArgs& a, int b, int r, bool& ok) {
   if (r < a.vis_start) return r;
@@ -110,6 +122,8 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(const CompactA
   __shared__ __align__(8) uint64_t bars[kSlots];
   __shared__ char* ring_dst[kSlots];
   __shared__ uint32_t ring_bytes[kSlots];
+  __shared__ int idx_s[kIdxStage];  // the producer's staged kept indices
+  __shared__ int4 meta_s[kMetaRows];  // the helpers' rows: (sample, output row, source row)
   // items per output row: the pieces of the bulk-copied tensors (at least one,
   // so that rows are spread over CTAs even when every tensor is small)
   const int NB = np0 + np1 + np2;
@@ -138,9 +152,41 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(const CompactA
 
   if (threadIdx.x == 0 && NB > 0) {
     const uint64_t pol = policy_evict_first();
+    // The items of a phase are walked in order with running counters (piece
+    // q of row w of sample b), so no item needs a division. The kept visual
+    // indices of the CTA's phase-1 rows are loaded once, kStageBatch at a time
+    // with every load of a batch in flight, right after the wait for the kernel
+    // that writes them; longer ranges read the rest from global memory.
     int phase = 0;
     long long next = beg[0];
-    bool waited = false;
+    int b = 0, w = 0, q = 0, per = 1;
+    int ord = 0;  // rows of the phase started so far (the staged index of a phase-1 row)
+    int sl = 0;
+    auto start_phase = [&](int ph) {
+      if (beg[ph] >= fin[ph]) return;  // nothing of this phase here (per may be 0)
+      per = ph == 0 ? a.L_out - a.keep : a.keep;
+      const long long row = beg[ph] / NP;
+      q = (int)(beg[ph] - row * NP);
+      ord = 0;
+      b = (int)(row / per);
+      w = (int)(row - (long long)b * per);
+      sl = a.seq_len[b];
+      if (ph == 1) {
+        pdl_wait();  // idx is written by the previous kernel
+        const long long r1 = (fin[1] + NP - 1) / NP;
+        const int n = (int)min((long long)kIdxStage, r1 - beg[1] / NP);
+        const int* src = a.idx + beg[1] / NP;
+        for (int j0 = 0; j0 < n; j0 += kStageBatch) {
+          int v[kStageBatch];
+#pragma unroll
+          for (int j = 0; j < kStageBatch; ++j) v[j] = j0 + j < n ? src[j0 + j] : 0;
+#pragma unroll
+          for (int j = 0; j < kStageBatch; ++j)
+            if (j0 + j < n) idx_s[j0 + j] = v[j];
+        }
+      }
+    };
+    start_phase(0);
     // next valid item; false when both phases are exhausted
     auto fetch = [&](Item& it) -> bool {
       for (;;) {
@@ -148,43 +194,51 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(const CompactA
           if (phase == 1) return false;
           phase = 1;
           next = beg[1];
+          start_phase(1);
           continue;
         }
-        if (phase == 1 && !waited) {
-          pdl_wait();  // idx is written by the previous kernel
-          waited = true;
+        ++next;
+        const int cq = q, cw = w, cb = b, csl = sl, cord = ord;
+        if (++q == NP) {  // advance the counters to item i + 1
+          q = 0;
+          ++ord;
+          if (++w == per) {
+            w = 0;
+            ++b;
+            if (next < fin[phase]) sl = a.seq_len[b];
+          }
         }
-        const long long i = next++;
-        const long long row = i / NP;
-        int q = (int)(i - row * NP);
-        int b, r;
-        phase_row(a, phase, row, b, r);
-        const int sl = a.seq_len[b];
-        if (sl > a.L_max || sl < a.vis_start + a.N_v) {
+        if (csl > a.L_max || csl < a.vis_start + a.N_v) {
           set_error(a.err, kErrBadDeviceArg);
           continue;
         }
-        if (r >= sl - a.N_v + a.keep) continue;
-        int t = 0;
-        if (q >= np0) {
-          q -= np0;
+        const int r = phase == 0 ? (cw < a.vis_start ? cw : cw + a.keep) : a.vis_start + cw;
+        if (r >= csl - a.N_v + a.keep) continue;
+        int sr = r;
+        if (phase == 1) {
+          const int v = cord < kIdxStage ? idx_s[cord] : a.idx[(size_t)cb * a.keep + cw];
+          if (v < 0 || v >= a.N_v) {
+            set_error(a.err, kErrBadDeviceArg);
+            continue;
+          }
+          sr = a.vis_start + v;
+        } else if (r >= a.vis_start) {
+          sr = r - a.keep + a.N_v;
+        }
+        int t = 0, pq = cq;
+        if (pq >= np0) {
+          pq -= np0;
           t = 1;
-          if (q >= np1) {
-            q -= np1;
+          if (pq >= np1) {
+            pq -= np1;
             t = 2;
           }
         }
-        bool ok = true;
-        const int sr = src_row(a, b, r, ok);
-        if (!ok) {
-          set_error(a.err, kErrBadDeviceArg);
-          continue;
-        }
         const long long rb = a.row_bytes[t];
-        const long long off = (long long)q * kSlotBytes;
+        const long long off = (long long)pq * kSlotBytes;
         it.bytes = (uint32_t)min((long long)kSlotBytes, rb - off);
-        it.src = a.src[t] + ((long long)b * a.L_max + sr) * rb + off;
-        it.dst = a.dst[t] + ((long long)b * a.L_out + r) * rb + off;
+        it.src = a.src[t] + ((long long)cb * a.L_max + sr) * rb + off;
+        it.dst = a.dst[t] + ((long long)cb * a.L_out + r) * rb + off;
         return true;
       }
     };
@@ -224,62 +278,76 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(const CompactA
     // rows whose first item lies in this CTA's ranges: their position ids, and
     // the rows of the small tensors (16-byte vector copies, a warp per row)
     // a thread per row for the position ids alone, a warp per row with small tensors
+    // Rows are taken kMetaRows at a time: first every helper thread works out
+    // the (sample, output row, source row) of its own rows - their dependent
+    // loads of lengths and kept indices all in flight at once - into shared
+    // memory, then (after a barrier of the helper threads) the copies run.
+    const int ht = (int)threadIdx.x - 32, n_ht = kCompactThreads - 32;
     const int lane = small ? (int)(threadIdx.x & 31) : 0;
-    const int worker = small ? (int)(threadIdx.x >> 5) - 1 : (int)threadIdx.x - 32;
-    const int n_workers = small ? kCompactThreads / 32 - 1 : kCompactThreads - 32;
+    const int worker = small ? (int)(threadIdx.x >> 5) - 1 : ht;
+    const int n_workers = small ? kCompactThreads / 32 - 1 : n_ht;
     for (int ph = 0; ph < 2; ++ph) {
       if (ph == 1) pdl_wait();
       const long long r0 = (beg[ph] + NP - 1) / NP, r1 = (fin[ph] + NP - 1) / NP;
-      for (long long row = r0 + worker; row < r1; row += n_workers) {
-        int b, r;
-        phase_row(a, ph, row, b, r);
-        const int sl = a.seq_len[b];
-        if (sl > a.L_max || sl < a.vis_start + a.N_v || r >= sl - a.N_v + a.keep) continue;
-        bool ok = true;
-        const int sr = src_row(a, b, r, ok);
-        if (!ok) continue;
-        if (a.pos != nullptr)
-          for (int p = lane; p < a.P; p += 32)
-            a.pos_out[((size_t)p * a.B + b) * a.L_out + r] = a.pos[((size_t)p * a.B + b) * a.L_max + sr];
-        // the row's pieces of every small tensor, as one list of 16-byte
-        // pieces: all of a lane's loads are issued before its stores (one
-        // memory round trip per row, not one per tensor)
-        const uint4 *s0 = nullptr, *s1 = nullptr, *s2 = nullptr;
-        uint4 *d0 = nullptr, *d1 = nullptr, *d2 = nullptr;
-        int n0 = 0, n1 = 0, n2 = 0;
-        if (small & 1) {
-          const long long rb = a.row_bytes[0];
-          s0 = reinterpret_cast<const uint4*>(a.src[0] + ((long long)b * a.L_max + sr) * rb);
-          d0 = reinterpret_cast<uint4*>(a.dst[0] + ((long long)b * a.L_out + r) * rb);
-          n0 = (int)(rb / 16);
+      for (long long c0 = r0; c0 < r1; c0 += kMetaRows) {
+        const int nrow = (int)min((long long)kMetaRows, r1 - c0);
+        for (int k = ht; k < nrow; k += n_ht) {
+          int b, r;
+          phase_row(a, ph, c0 + k, b, r);
+          const int sl = a.seq_len[b];
+          bool ok = !(sl > a.L_max || sl < a.vis_start + a.N_v || r >= sl - a.N_v + a.keep);
+          const int sr = ok ? src_row(a, b, r, ok) : 0;
+          meta_s[k] = ok ? make_int4(b, r, sr, 0) : make_int4(-1, 0, 0, 0);
         }
-        if (small & 2) {
-          const long long rb = a.row_bytes[1];
-          s1 = reinterpret_cast<const uint4*>(a.src[1] + ((long long)b * a.L_max + sr) * rb);
-          d1 = reinterpret_cast<uint4*>(a.dst[1] + ((long long)b * a.L_out + r) * rb);
-          n1 = (int)(rb / 16);
-        }
-        if (small & 4) {
-          const long long rb = a.row_bytes[2];
-          s2 = reinterpret_cast<const uint4*>(a.src[2] + ((long long)b * a.L_max + sr) * rb);
-          d2 = reinterpret_cast<uint4*>(a.dst[2] + ((long long)b * a.L_out + r) * rb);
-          n2 = (int)(rb / 16);
-        }
-        const int tot = n0 + n1 + n2;
-        for (int q0 = 0; q0 < tot; q0 += 32 * kSmallPieces) {
-          uint4 v[kSmallPieces];
-#pragma unroll
-          for (int j = 0; j < kSmallPieces; ++j) {
-            const int q = q0 + lane + 32 * j;
-            if (q < tot)
-              v[j] = __ldcs(q < n0 ? s0 + q : (q < n0 + n1 ? s1 + (q - n0) : s2 + (q - n0 - n1)));
+        helpers_sync();
+        for (int k = worker; k < nrow; k += n_workers) {
+          const int4 mt = meta_s[k];
+          if (mt.x < 0) continue;
+          const int b = mt.x, r = mt.y, sr = mt.z;
+          if (a.pos != nullptr)
+            for (int p = lane; p < a.P; p += 32)
+              a.pos_out[((size_t)p * a.B + b) * a.L_out + r] = a.pos[((size_t)p * a.B + b) * a.L_max + sr];
+          // the row's pieces of every small tensor, as one list of 16-byte
+          // pieces: all of a lane's loads are issued before its stores (one
+          // memory round trip per row, not one per tensor)
+          const uint4 *s0 = nullptr, *s1 = nullptr, *s2 = nullptr;
+          uint4 *d0 = nullptr, *d1 = nullptr, *d2 = nullptr;
+          int n0 = 0, n1 = 0, n2 = 0;
+          if (small & 1) {
+            const long long rb = a.row_bytes[0];
+            s0 = reinterpret_cast<const uint4*>(a.src[0] + ((long long)b * a.L_max + sr) * rb);
+            d0 = reinterpret_cast<uint4*>(a.dst[0] + ((long long)b * a.L_out + r) * rb);
+            n0 = (int)(rb / 16);
           }
+          if (small & 2) {
+            const long long rb = a.row_bytes[1];
+            s1 = reinterpret_cast<const uint4*>(a.src[1] + ((long long)b * a.L_max + sr) * rb);
+            d1 = reinterpret_cast<uint4*>(a.dst[1] + ((long long)b * a.L_out + r) * rb);
+            n1 = (int)(rb / 16);
+          }
+          if (small & 4) {
+            const long long rb = a.row_bytes[2];
+            s2 = reinterpret_cast<const uint4*>(a.src[2] + ((long long)b * a.L_max + sr) * rb);
+            d2 = reinterpret_cast<uint4*>(a.dst[2] + ((long long)b * a.L_out + r) * rb);
+            n2 = (int)(rb / 16);
+          }
+          const int tot = n0 + n1 + n2;
+          for (int q0 = 0; q0 < tot; q0 += 32 * kSmallPieces) {
+            uint4 v[kSmallPieces];
 #pragma unroll
-          for (int j = 0; j < kSmallPieces; ++j) {
-            const int q = q0 + lane + 32 * j;
-            if (q < tot) __stcs(q < n0 ? d0 + q : (q < n0 + n1 ? d1 + (q - n0) : d2 + (q - n0 - n1)), v[j]);
+            for (int j = 0; j < kSmallPieces; ++j) {
+              const int q = q0 + lane + 32 * j;
+              if (q < tot)
+                v[j] = __ldcs(q < n0 ? s0 + q : (q < n0 + n1 ? s1 + (q - n0) : s2 + (q - n0 - n1)));
+            }
+#pragma unroll
+            for (int j = 0; j < kSmallPieces; ++j) {
+              const int q = q0 + lane + 32 * j;
+              if (q < tot) __stcs(q < n0 ? d0 + q : (q < n0 + n1 ? d1 + (q - n0) : d2 + (q - n0 - n1)), v[j]);
+            }
           }
         }
+        helpers_sync();  // meta_s is rewritten by the next chunk
       }
     }
   }

@@ -52,3 +52,16 @@ def test_weak_scaling_bookkeeping_gloo():
 def test_aggregate_single_rank():
     import bench
     assert bench.aggregate(80.0, 2.0) == 40.0
+
+
+def test_summarize_takes_the_median_repeat_and_its_spread():
+    import bench
+    times = [0.010, 0.012, 0.011, 0.030, 0.011]  # seconds per repeat of K = 10 steps; one outlier
+    r = bench.summarize(times, units=80.0, K=10, path_bytes=1e6, peak=1000.0)
+    assert r["value"] == pytest.approx(80.0 / 0.011)
+    assert r["ms_per_step"] == pytest.approx(1.1)
+    assert r["achieved_gbs"] == pytest.approx(1e6 * 10 / 0.011 / 1e9)
+    assert r["frac"] == pytest.approx(r["achieved_gbs"] / 1000.0)
+    assert r["repeats"]["n"] == 5
+    assert r["repeats"]["min_value"] == pytest.approx(80.0 / 0.030)
+    assert r["repeats"]["spread"] == pytest.approx((0.030 - 0.010) / 0.011)
