@@ -689,6 +689,7 @@ def run_gb300(args, dist):
     lanes = Lanes(P, synth, w, dev, S, algo, n_copies, seed)
     cpu = lanes.cpu0
     vis, nv, keep = cpu["vis_start"], cpu["N_v"], cpu["keep"]
+    input_mb = sum(v.numel() * v.element_size() for v in cpu.values() if isinstance(v, torch.Tensor)) / 1e6
     lanes.run(max(args.warmup, 1) * S)
     torch.cuda.synchronize()
     rc, bits = P.provip_device_status(clear=True)
@@ -834,7 +835,7 @@ def run_gb300(args, dist):
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": dist.world, "steps": K,
             "warmup": args.warmup, "ms_per_step": 1e3 * max_sec / K, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
-            "config": dict(workload_config(w, algo_name, n_copies, e2e["h2d_bytes_per_step"] / 1e6), streams=S,
+            "config": dict(workload_config(w, algo_name, n_copies, input_mb), streams=S,
                            **({"concurrency": f"{S} streams of independent batches run concurrently (each with its "
                                               f"own inputs, outputs and workspace); value counts the samples of all "
                                               f"streams; single_stream is one stream"} if S > 1 else {})),
@@ -926,59 +927,66 @@ def video_measure(P, synth, torch, dist, dev, stream, args, peak):
 
 
 def e2e_measure(P, torch, dist, w, cpu, step0, algo, dev, E):
-    """e2e through the C ABI with host buffers. Every step copies its inputs
-    from pinned host memory and its outputs back to pinned host memory inside
-    the timed region; two device buffer sets (each with its own outputs)
-    alternate so that the copies of one step overlap the pruning of the other
-    (a stream per copy direction and one for the kernels, ordered by events).
-    Three timed runs of E steps, the median reported with the three beside it
-    (the host copies share the machine's memory system with other jobs)."""
+    """e2e through the C ABI with the batch in pinned host memory. Every step
+    copies to the device what the tensor-core head scores read (each sample's
+    text rows of Q, all of K) and the lengths; the pruning call then reads
+    hidden, V and the position ids where they are, in host memory, and writes
+    the compacted hidden, K, V and position ids straight into pinned host
+    outputs (PROVIP_PRUNE_HOST_ROWS: only the kept rows cross the host link);
+    the kept indices and output lengths are copied back. The bytes declared are
+    the copies plus the kept rows the kernel reads from host memory (in) and
+    the rows it writes there (out). Two device buffer sets alternate so that
+    one step's copies overlap the other's pruning (a stream per copy direction
+    and one for the kernels, ordered by events). Three timed runs of E steps,
+    the median reported with the three beside it (the host link is shared with
+    other jobs)."""
+    import numpy as np
     nv, keep, vis = cpu["N_v"], cpu["keep"], cpu["vis_start"]
     pin = {k: v.pin_memory() for k, v in cpu.items() if isinstance(v, torch.Tensor)}
-    out_keys = ("hidden", "K", "V", "pos", "idx", "seq_len")
+    ts, tl = cpu["text_start"].numpy(), cpu["text_len"].numpy()
+    seq = cpu["seq_len"].numpy().astype(np.int64)
     sets = []
     for j in range(2):
-        db = {k: torch.empty_like(v, device=dev) for k, v in pin.items()}
-        st_j = P.PruneStep(db["Q"], db["K"], db["V"], db["hidden"], db["pos"], cpu["head_list"], w.n_t[1], nv, keep,
-                           algo=algo, want_scores=False, flags=P.PRUNE_OVERLAP_PREVIOUS)
-        outs_j = {"hidden": st_j.hidden_out, "K": st_j.K_out, "V": st_j.V_out, "pos": st_j.pos_out,
-                  "idx": st_j.idx, "seq_len": st_j.seq_len_out}
-        ho = {k: torch.empty(outs_j[k].shape, dtype=outs_j[k].dtype, pin_memory=True) for k in out_keys}
-        ev = {n: torch.cuda.Event() for n in ("comp", "d2h")}
+        db = {k: torch.empty_like(pin[k], device=dev) for k in ("Q", "K", "text_start", "text_len", "seq_len")}
+        st_j = P.PruneStep(db["Q"], db["K"], pin["V"], pin["hidden"], pin["pos"], cpu["head_list"], w.n_t[1], nv,
+                           keep, algo=algo, want_scores=False, flags=P.PRUNE_OVERLAP_PREVIOUS, host_rows=True)
+        ho = {"idx": torch.empty(st_j.idx.shape, dtype=torch.int32, pin_memory=True),
+              "seq_len": torch.empty(st_j.seq_len_out.shape, dtype=torch.int32, pin_memory=True)}
+        ev = {n: torch.cuda.Event() for n in ("h2d", "comp", "d2h")}
         sets.append((db, st_j, ho, ev))
-    h2d = sum(v.numel() * v.element_size() for v in pin.values())
-    d2h = sum(v.numel() * v.element_size() for v in sets[0][2].values())
-    s_comp, s_d2h = (torch.cuda.Stream(device=dev) for _ in range(2))
-    n_h2d = 2  # the input copies are spread over two streams (copy engines) by size
-    s_h2ds = [torch.cuda.Stream(device=dev) for _ in range(n_h2d)]
-    by_size = sorted(pin, key=lambda k: -pin[k].numel() * pin[k].element_size())
-    parts = [by_size[i::n_h2d] for i in range(n_h2d)]
-    for j in range(2):
-        sets[j][3]["h2d_parts"] = [torch.cuda.Event() for _ in range(n_h2d)]
+    es = pin["Q"].element_size()
+    q_rows = int(tl.sum()) * w.H_q * 128 * es
+    small = sum(pin[k].numel() * 4 for k in ("text_start", "text_len", "seq_len"))
+    out_rows = seq - nv + keep
+    row_in = (w.D + w.H_kv * 128) * es + w.P * 4  # hidden + V rows and position ids read in place
+    row_out = (w.D + 2 * w.H_kv * 128) * es + w.P * 4  # hidden, K, V rows and position ids written
+    h2d = q_rows + pin["K"].numel() * es + small + int((out_rows * row_in).sum())
+    d2h = int((out_rows * row_out).sum()) + sets[0][2]["idx"].numel() * 4 + sets[0][2]["seq_len"].numel() * 4
+    s_comp, s_d2h, s_h2d = (torch.cuda.Stream(device=dev) for _ in range(3))
     fresh = [True, True]
 
     def one(n):
         j = n % 2
         db, st_j, ho, ev = sets[j]
-        for s_h2d, keys, e_part in zip(s_h2ds, parts, ev["h2d_parts"]):
-            with torch.cuda.stream(s_h2d):
-                if not fresh[j]:
-                    s_h2d.wait_event(ev["comp"])  # the set's inputs were consumed by step n - 2
-                for k in keys:
-                    db[k].copy_(pin[k], non_blocking=True)
-                e_part.record(s_h2d)
-        with torch.cuda.stream(s_comp):
-            for e_part in ev["h2d_parts"]:
-                s_comp.wait_event(e_part)
+        with torch.cuda.stream(s_h2d):
             if not fresh[j]:
-                s_comp.wait_event(ev["d2h"])  # step n - 2's outputs have left this set
-            r = st_j(db["Q"], db["K"], db["V"], db["hidden"], db["pos"], db["text_start"], db["text_len"],
+                s_h2d.wait_event(ev["comp"])  # the set's device inputs were consumed by step n - 2
+            for b in range(w.B):
+                db["Q"][b, ts[b]:ts[b] + tl[b]].copy_(pin["Q"][b, ts[b]:ts[b] + tl[b]], non_blocking=True)
+            for k in ("K", "text_start", "text_len", "seq_len"):
+                db[k].copy_(pin[k], non_blocking=True)
+            ev["h2d"].record(s_h2d)
+        with torch.cuda.stream(s_comp):
+            s_comp.wait_event(ev["h2d"])
+            if not fresh[j]:
+                s_comp.wait_event(ev["d2h"])  # step n - 2's indices have left this set
+            r = st_j(db["Q"], db["K"], pin["V"], pin["hidden"], pin["pos"], db["text_start"], db["text_len"],
                      db["seq_len"], vis, stream=s_comp)
             ev["comp"].record(s_comp)
         with torch.cuda.stream(s_d2h):
             s_d2h.wait_event(ev["comp"])
-            for k in out_keys:
-                ho[k].copy_(r[k], non_blocking=True)
+            ho["idx"].copy_(r["idx"], non_blocking=True)
+            ho["seq_len"].copy_(r["seq_len"], non_blocking=True)
             ev["d2h"].record(s_d2h)
         fresh[j] = False
 
@@ -986,11 +994,11 @@ def e2e_measure(P, torch, dist, w, cpu, step0, algo, dev, E):
         main = torch.cuda.current_stream(dev)
         start = torch.cuda.Event()
         start.record(main)
-        for st_ in (*s_h2ds, s_comp, s_d2h):
+        for st_ in (s_h2d, s_comp, s_d2h):
             st_.wait_event(start)
         for n in range(first, first + n_steps):
             one(n)
-        for st_ in (*s_h2ds, s_comp, s_d2h):
+        for st_ in (s_h2d, s_comp, s_d2h):
             done = torch.cuda.Event()
             done.record(st_)
             main.wait_event(done)
@@ -1008,7 +1016,9 @@ def e2e_measure(P, torch, dist, w, cpu, step0, algo, dev, E):
         first += E
         runs.append(aggregate(dist.sum(float(w.B * E)), dist.max(a.elapsed_time(b) / 1e3)))
     return {"value": sorted(runs)[1], "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
-            "runs": runs, "note": f"median of 3 timed runs of {E} steps"}
+            "runs": runs, "note": f"median of 3 timed runs of {E} steps; the batch stays in pinned host memory: "
+                                  f"Q text rows and K copied in, kept rows read and compacted rows written in "
+                                  f"place by the kernels (PROVIP_PRUNE_HOST_ROWS)"}
 
 
 def run_prellm_only(args):

@@ -281,7 +281,7 @@ int provip_head_topk(const void *Q, const void *K, int B, int L_max, int H_q, in
  * dependents (the compaction copies the rows that do not depend on the kept
  * indices while the selection finishes).
  *
- * flags: 0, or a combination of the two below.
+ * flags: 0, or a combination of the three below.
  * PROVIP_PRUNE_OVERLAP_PREVIOUS - the call's head-score kernel may start while
  * the kernel before it on the stream (typically the previous call's
  * compaction) is still running; it waits for that kernel only before it
@@ -299,6 +299,16 @@ int provip_head_topk(const void *Q, const void *K, int B, int L_max, int H_q, in
  * without the flag it spreads over every SM, which finishes a call that runs
  * alone soonest. Results are the same either way. */
 #define PROVIP_PRUNE_CONCURRENT 2u
+/* PROVIP_PRUNE_HOST_ROWS - hidden, V and pos, and the outputs hidden_out,
+ * K_out, V_out and pos_out, may be host memory that is pinned and mapped into
+ * the device's address space (cudaHostAlloc; any pointer the GPU can
+ * dereference). The compaction then copies every kept row with 16-byte loads
+ * and stores from the GPU's threads instead of bulk copies, which works for
+ * device and mapped host memory alike, so a caller whose sequences live in
+ * host memory moves only the surviving rows across the host link. Q and K must
+ * still be device memory (the head scores read them through tensor maps), and
+ * so must idx_out, seq_len_out and the scores. Results are the same. */
+#define PROVIP_PRUNE_HOST_ROWS 4u
 size_t provip_prune_workspace_size(int B, int L_max, int H_sel, int N_t_max, int N_v, int algo,
                                    int dtype);
 int provip_prune(const void *Q, const void *K, const void *V, const void *hidden, int B,

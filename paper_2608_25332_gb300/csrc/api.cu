@@ -828,7 +828,7 @@ extern "C" int provip_prune(const void* Q, const void* K, const void* V, const v
                             size_t ws_bytes, unsigned flags, void* stream) {
   NvtxRange nvtx_range("provip_prune");
   // validate both halves before enqueueing anything
-  if (flags & ~(unsigned)(PROVIP_PRUNE_OVERLAP_PREVIOUS | PROVIP_PRUNE_CONCURRENT))
+  if (flags & ~(unsigned)(PROVIP_PRUNE_OVERLAP_PREVIOUS | PROVIP_PRUNE_CONCURRENT | PROVIP_PRUNE_HOST_ROWS))
     return fail(PROVIP_ERR_INVALID_ARG, "prune: unknown flags 0x%x", flags);
   int rc = hs_validate(Q, K, B, L_max, H_q, H_kv, d_h, head_list, H_sel, text_start, text_len,
                        N_t_max, vis_start, N_v, seq_len, dtype, resolve_algo(algo, dtype));
@@ -854,7 +854,8 @@ extern "C" int provip_prune(const void* Q, const void* K, const void* V, const v
   const int form = tc_form(resolve_algo(algo, dtype), B, H_sel, hs_shape(L_max, N_t_max, N_v, algo).n_rb,
                            d->sms);
   cudaError_t e = compact_launch(ca, d->sms, static_cast<cudaStream_t>(stream), true,
-                                 form == PROVIP_ALGO_TCGEN05_STREAM, (flags & PROVIP_PRUNE_CONCURRENT) != 0);
+                                 form == PROVIP_ALGO_TCGEN05_STREAM, (flags & PROVIP_PRUNE_CONCURRENT) != 0,
+                                 (flags & PROVIP_PRUNE_HOST_ROWS) != 0);
   return e == cudaSuccess ? PROVIP_OK : cuda_fail(e, "prune compact");
 }
 
@@ -967,7 +968,7 @@ extern "C" int provip_prune_visual_heads(
     int* vis_heads_out_or_null, float* conf_out_or_null, void* ws, size_t ws_bytes,
     unsigned flags, void* stream) {
   NvtxRange nvtx_range("provip_prune_visual_heads");
-  if (flags & ~(unsigned)(PROVIP_PRUNE_OVERLAP_PREVIOUS | PROVIP_PRUNE_CONCURRENT))
+  if (flags & ~(unsigned)(PROVIP_PRUNE_OVERLAP_PREVIOUS | PROVIP_PRUNE_CONCURRENT | PROVIP_PRUNE_HOST_ROWS))
     return fail(PROVIP_ERR_INVALID_ARG, "prune_visual_heads: unknown flags 0x%x", flags);
   if (keep < 1) return fail(PROVIP_ERR_INVALID_ARG, "prune_visual_heads: keep %d < 1", keep);
   int rc = compact_validate(idx_out ? idx_out : reinterpret_cast<int*>(16), B, N_v, keep, hidden, D,
@@ -989,7 +990,8 @@ extern "C" int provip_prune_visual_heads(
   const int form = tc_form(resolve_algo(algo, dtype), B, H_q, hs_shape(L_max, N_t_max, N_v, algo).n_rb,
                            d->sms);
   cudaError_t e = compact_launch(ca, d->sms, static_cast<cudaStream_t>(stream), true,
-                                 form == PROVIP_ALGO_TCGEN05_STREAM, (flags & PROVIP_PRUNE_CONCURRENT) != 0);
+                                 form == PROVIP_ALGO_TCGEN05_STREAM, (flags & PROVIP_PRUNE_CONCURRENT) != 0,
+                                 (flags & PROVIP_PRUNE_HOST_ROWS) != 0);
   return e == cudaSuccess ? PROVIP_OK : cuda_fail(e, "prune_visual_heads compact");
 }
 

@@ -353,10 +353,97 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(const CompactA
   }
 }
 
+// The compaction for rows in mapped host memory (or any mix of host and device
+// memory): every row is copied by one warp with 16-byte loads and stores, all
+// of a lane's loads of a round (kVecPieces pieces, 4 KiB per warp) issued
+// before its stores, with no bulk (TMA) copies. Rows are dealt to the warps of
+// the grid in turn, phase 0 (the rows that do not depend on idx) first; a
+// warp's lanes resolve a row's (sample, output row, source row) together (the
+// same loads, one transaction).
+constexpr int kVecThreads = 128;
+constexpr int kVecPieces = 8;
+__global__ void __launch_bounds__(kVecThreads) compact_vec_kernel(const CompactArgs a) {
+  const int lane = threadIdx.x & 31;
+  const long long warp = (long long)blockIdx.x * (kVecThreads / 32) + (threadIdx.x >> 5);
+  const long long n_warps = (long long)gridDim.x * (kVecThreads / 32);
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  if (blockIdx.x == 0 && a.seq_len_out != nullptr)
+    for (int b = threadIdx.x; b < a.B; b += blockDim.x) a.seq_len_out[b] = a.seq_len[b] - a.N_v + a.keep;
+  const int n16[3] = {a.n_tensors > 0 ? (int)(a.row_bytes[0] / 16) : 0,
+                      a.n_tensors > 1 ? (int)(a.row_bytes[1] / 16) : 0,
+                      a.n_tensors > 2 ? (int)(a.row_bytes[2] / 16) : 0};
+  const int tot = n16[0] + n16[1] + n16[2];
+  for (int ph = 0; ph < 2; ++ph) {
+    if (ph == 1) pdl_wait();  // idx is written by the previous kernel
+    const long long nrows = ph == 0 ? (long long)a.B * (a.L_out - a.keep) : (long long)a.B * a.keep;
+    for (long long row = warp; row < nrows; row += n_warps) {
+      int b, r;
+      phase_row(a, ph, row, b, r);
+      const int sl = a.seq_len[b];
+      if (sl > a.L_max || sl < a.vis_start + a.N_v) {
+        if (lane == 0) set_error(a.err, kErrBadDeviceArg);
+        continue;
+      }
+      if (r >= sl - a.N_v + a.keep) continue;
+      int sr = r;
+      if (ph == 1) {
+        const int v = a.idx[row];  // row = b * keep + position
+        if (v < 0 || v >= a.N_v) {
+          if (lane == 0) set_error(a.err, kErrBadDeviceArg);
+          continue;
+        }
+        sr = a.vis_start + v;
+      } else if (r >= a.vis_start) {
+        sr = r - a.keep + a.N_v;
+      }
+      if (a.pos != nullptr)
+        for (int p = lane; p < a.P; p += 32)
+          a.pos_out[((size_t)p * a.B + b) * a.L_out + r] = a.pos[((size_t)p * a.B + b) * a.L_max + sr];
+      const uint4* s0 = n16[0] ? reinterpret_cast<const uint4*>(a.src[0] + ((long long)b * a.L_max + sr) * a.row_bytes[0]) : nullptr;
+      const uint4* s1 = n16[1] ? reinterpret_cast<const uint4*>(a.src[1] + ((long long)b * a.L_max + sr) * a.row_bytes[1]) : nullptr;
+      const uint4* s2 = n16[2] ? reinterpret_cast<const uint4*>(a.src[2] + ((long long)b * a.L_max + sr) * a.row_bytes[2]) : nullptr;
+      uint4* d0 = n16[0] ? reinterpret_cast<uint4*>(a.dst[0] + ((long long)b * a.L_out + r) * a.row_bytes[0]) : nullptr;
+      uint4* d1 = n16[1] ? reinterpret_cast<uint4*>(a.dst[1] + ((long long)b * a.L_out + r) * a.row_bytes[1]) : nullptr;
+      uint4* d2 = n16[2] ? reinterpret_cast<uint4*>(a.dst[2] + ((long long)b * a.L_out + r) * a.row_bytes[2]) : nullptr;
+      const int n0 = n16[0], n1 = n16[1];
+      for (int q0 = 0; q0 < tot; q0 += 32 * kVecPieces) {
+        uint4 v[kVecPieces];
+#pragma unroll
+        for (int j = 0; j < kVecPieces; ++j) {
+          const int q = q0 + lane + 32 * j;
+          if (q < tot) v[j] = __ldcs(q < n0 ? s0 + q : (q < n0 + n1 ? s1 + (q - n0) : s2 + (q - n0 - n1)));
+        }
+#pragma unroll
+        for (int j = 0; j < kVecPieces; ++j) {
+          const int q = q0 + lane + 32 * j;
+          if (q < tot) __stcs(q < n0 ? d0 + q : (q < n0 + n1 ? d1 + (q - n0) : d2 + (q - n0 - n1)), v[j]);
+        }
+      }
+    }
+  }
+}
+
 }  // namespace
 
 cudaError_t compact_launch(const CompactArgs& a, int num_sms, cudaStream_t s, bool pdl, bool allow_deep,
-                           bool concurrent) {
+                           bool concurrent, bool host_rows) {
+  if (host_rows) {
+    // rows in mapped host memory: plain vector copies over the whole GPU
+    const long long rows = (long long)a.B * a.L_out;
+    long long grid = (long long)kCtasPerSm * num_sms;
+    const long long need = (rows + kVecThreads / 32 - 1) / (kVecThreads / 32);
+    if (grid > need) grid = need > 0 ? need : 1;
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr[1];
+    cfg.gridDim = dim3((unsigned)grid);
+    cfg.blockDim = dim3(kVecThreads);
+    cfg.stream = s;
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = pdl ? 1 : 0;
+    return cudaLaunchKernelEx(&cfg, compact_vec_kernel, a);
+  }
   static std::atomic<bool> configured[64];  // per device, zero-initialised
   int dev = 0;
   cudaGetDevice(&dev);

@@ -150,8 +150,10 @@ struct CompactArgs {
 // head-score CTA per SM, not for the cluster form's larger one). concurrent:
 // other calls run beside this one on other streams, so a small problem takes
 // only the CTAs its bytes fill (otherwise it spreads over every SM).
+// host_rows: sources or destinations may be mapped host memory, so every row is
+// copied with 16-byte loads and stores (no bulk copies).
 cudaError_t compact_launch(const CompactArgs& a, int num_sms, cudaStream_t s, bool pdl = false,
-                           bool allow_deep = true, bool concurrent = false);
+                           bool allow_deep = true, bool concurrent = false, bool host_rows = false);
 
 // ---------------------------------------------------------------------------
 // pre-LLM similarity pass (Sec. 4.2-4.3)

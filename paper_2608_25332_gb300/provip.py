@@ -29,6 +29,7 @@ ALGO_AUTO, ALGO_SIMT, ALGO_TCGEN05, ALGO_TCGEN05_TWOPASS = 0, 1, 2, 3
 ALGO_TCGEN05_STREAM, ALGO_TCGEN05_CLUSTER = 4, 5
 PRUNE_OVERLAP_PREVIOUS = 1
 PRUNE_CONCURRENT = 2
+PRUNE_HOST_ROWS = 4
 
 _P = ctypes.c_void_p
 _I = ctypes.c_int
@@ -126,6 +127,18 @@ def _ptr(t):
     return ctypes.c_void_p(t.data_ptr())
 
 
+def _ptr_host_ok(t):
+    """a device tensor, or a pinned host tensor (mapped into the device's
+    address space) for the arguments PROVIP_PRUNE_HOST_ROWS allows there"""
+    if t is not None and not t.is_cuda:
+        if not t.is_pinned():
+            raise ProvipError(ERR_INVALID_ARG, "a host tensor must be pinned (pin_memory())")
+        if not t.is_contiguous():
+            raise ProvipError(ERR_INVALID_ARG, "tensor must be contiguous")
+        return ctypes.c_void_p(t.data_ptr())
+    return _ptr(t)
+
+
 def _stream(device):
     return ctypes.c_void_p(torch.cuda.current_stream(device).cuda_stream)
 
@@ -136,6 +149,14 @@ def _i32(t):
     if t.dtype != torch.int32:
         raise ProvipError(ERR_INVALID_ARG, "index/length tensors must be int32")
     return _ptr(t)
+
+
+def _i32_host_ok(t):
+    if t is None:
+        return None
+    if t.dtype != torch.int32:
+        raise ProvipError(ERR_INVALID_ARG, "index/length tensors must be int32")
+    return _ptr_host_ok(t)
 
 
 def _u8(t):
@@ -334,18 +355,24 @@ class PruneStep:
     """Pre-allocated outputs + workspace for repeated provip_prune calls (one shape)."""
 
     def __init__(self, Q, K, V, hidden, pos, head_list, N_t_max, N_v, keep, algo=ALGO_AUTO,
-                 want_scores=True, flags=0, ws=None, device=None):
+                 want_scores=True, flags=0, ws=None, device=None, host_rows=False):
         """Q, K, V, hidden, pos give the shapes and dtypes (meta tensors are fine
-        with device=...)."""
+        with device=...). host_rows: the compacted outputs are pinned host
+        tensors, and hidden, V and pos may be pinned host tensors too
+        (PROVIP_PRUNE_HOST_ROWS)."""
         B, Lm, Hq, dh = Q.shape
         self.shape = (B, Lm, Hq, K.shape[2], dh, hidden.shape[2])
         self.heads, self.H_sel = _heads_arg(head_list, Q.shape[2])
         self.N_t_max, self.N_v, self.keep, self.algo = int(N_t_max), int(N_v), int(keep), algo
-        self.flags = int(flags)
+        self.flags = int(flags) | (PRUNE_HOST_ROWS if host_rows else 0)
         dev = Q.device if device is None else torch.device(device)
         self.dtype = _dtype_code(Q)
         L_out = Lm - N_v + keep
         self.hidden_out, self.K_out, self.V_out, self.pos_out = _outs(hidden, K, V, pos, B, L_out, dev)
+        if host_rows:
+            self.hidden_out, self.K_out, self.V_out, self.pos_out = (
+                None if t is None else torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
+                for t in (self.hidden_out, self.K_out, self.V_out, self.pos_out))
         self.idx = torch.empty((B, keep), dtype=torch.int32, device=dev)
         self.seq_len_out = torch.empty(B, dtype=torch.int32, device=dev)
         self.scores = torch.empty((B, N_v), dtype=torch.float32, device=dev) if want_scores else None
@@ -357,11 +384,14 @@ class PruneStep:
         B, Lm, Hq, Hkv, dh, D = self.shape
         P = pos.shape[0] if pos is not None else 0
         st = ctypes.c_void_p(stream.cuda_stream) if stream is not None else _stream(Q.device)
-        rc = lib().provip_prune(_ptr(Q), _ptr(K), _ptr(V), _ptr(hidden), B, Lm, Hq, Hkv, dh, D,
+        hp = _ptr_host_ok if self.flags & PRUNE_HOST_ROWS else _ptr
+        rc = lib().provip_prune(_ptr(Q), _ptr(K), hp(V), hp(hidden), B, Lm, Hq, Hkv, dh, D,
                                 self.heads, self.H_sel, _i32(text_start), _i32(text_len),
                                 _u8(row_mask), self.N_t_max, vis_start, self.N_v, _i32(seq_len),
-                                _i32(pos), P, self.keep, self.dtype, self.algo, _ptr(self.hidden_out),
-                                _ptr(self.K_out), _ptr(self.V_out), _i32(self.pos_out),
+                                _i32_host_ok(pos) if hp is _ptr_host_ok else _i32(pos), P, self.keep,
+                                self.dtype, self.algo, hp(self.hidden_out), hp(self.K_out),
+                                hp(self.V_out),
+                                _i32_host_ok(self.pos_out) if hp is _ptr_host_ok else _i32(self.pos_out),
                                 _ptr(self.idx), _i32(self.seq_len_out), _ptr(self.scores),
                                 _ptr(self.ws), self.ws.numel(), self.flags, st)
         _check(rc, "provip_prune")

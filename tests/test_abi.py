@@ -98,7 +98,7 @@ def test_visual_heads_validation(L):
         1, 0, FAKE, FAKE, FAKE, None, FAKE, None, None, None, None, None, 0, flags, None)
     assert prune(0) == -1                     # keep < 1
     assert prune(51) == -1                    # keep > N_v
-    assert prune(5, flags=4) == -1            # unknown flag
+    assert prune(5, flags=8) == -1            # unknown flag
     assert prune(5) == -3                     # workspace too small
 
 
