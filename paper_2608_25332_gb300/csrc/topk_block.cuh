@@ -19,6 +19,7 @@
 #pragma once
 
 #include "common.cuh"
+#include "kernels.h"
 
 namespace provip {
 
@@ -412,6 +413,119 @@ __device__ __forceinline__ void topk_load_scores(const float* src, int N, float*
         mn = min(mn, key);
         mx = max(mx, key);
       }
+    }
+  }
+}
+
+// Row count of sample b for the score division: the valid text rows, counted
+// by the whole block (a block barrier inside).
+__device__ __forceinline__ int block_count_rows(const TopkArgs& a, int b) {
+  __shared__ int cnt;
+  if (threadIdx.x == 0) cnt = 0;
+  __syncthreads();
+  const int tl = a.text_len[b];
+  int mine = 0;
+  for (int j = threadIdx.x; j < a.N_t_max; j += blockDim.x)
+    mine += (j < tl) && (a.row_mask == nullptr || a.row_mask[(size_t)b * a.N_t_max + j] != 0);
+  if (mine) atomicAdd(&cnt, mine);
+  __syncthreads();
+  return cnt;
+}
+
+// Thread t's KPT keys (indices t * KPT + c, c < KPT; 0 past N) from the scores
+// or the head partials (the same sums, in the same order, as
+// load_sample_keys), with the thread's min and max key. Every load of a group
+// of partial rows is issued before the first sum.
+template <int KPT>
+__device__ __forceinline__ void load_keys_reg(const TopkArgs& a, int b, uint32_t (&key)[KPT],
+                                              uint32_t& mn, uint32_t& mx) {
+  const int N = a.N, i0 = threadIdx.x * KPT;
+  float v[KPT];
+  if (a.partial != nullptr) {
+    __shared__ int sel[kMaxHeads];
+    int nrows;
+    if (a.row_mask == nullptr && a.sel == nullptr) {
+      nrows = min(max(a.text_len[b], 0), a.N_t_max);
+    } else {
+      if (a.sel != nullptr)
+        for (int q = threadIdx.x; q < a.n_sel; q += blockDim.x) sel[q] = a.sel[(size_t)b * a.n_sel + q];
+      nrows = block_count_rows(a, b);  // synchronises the block (sel is visible after it)
+    }
+    const int n_sum = a.sel != nullptr ? (a.n_part / a.H_sel) * a.n_sel : a.n_part;
+    const float div = (float)(a.sel != nullptr ? a.n_sel : a.H_sel) * (float)nrows;
+    const float* P0 = a.partial + (size_t)b * a.n_part * N;
+    // N % 4 == 0 and an aligned base: every row and every thread's columns start
+    // on 16 bytes, and a group of 4 columns lies wholly below N or wholly past it
+    const bool vec = (N & 3) == 0 && (reinterpret_cast<uintptr_t>(P0) & 15u) == 0;
+    constexpr int G = KPT >= 16 ? 2 : 32 / KPT;  // rows per group: 32 to 64 loads in flight
+    float s[KPT];
+#pragma unroll
+    for (int c = 0; c < KPT; ++c) s[c] = 0.f;
+    for (int u0 = 0; u0 < n_sum; u0 += G) {
+      int ro[G];
+#pragma unroll
+      for (int u = 0; u < G; ++u) {
+        const int uu = u0 + u;
+        ro[u] = uu < n_sum ? (a.sel != nullptr ? (uu / a.n_sel) * a.H_sel + sel[uu % a.n_sel] : uu) * N : 0;
+      }
+      float t[KPT][G];
+      if (vec) {
+        // 16-byte loads of the thread's KPT consecutive columns
+#pragma unroll
+        for (int u = 0; u < G; ++u)
+#pragma unroll
+          for (int c4 = 0; c4 < KPT / 4; ++c4) {
+            float4 f = make_float4(0.f, 0.f, 0.f, 0.f);
+            if (u0 + u < n_sum && i0 + 4 * c4 < N)
+              f = __ldg(reinterpret_cast<const float4*>(P0 + (size_t)ro[u] + i0) + c4);
+            t[4 * c4 + 0][u] = f.x;
+            t[4 * c4 + 1][u] = f.y;
+            t[4 * c4 + 2][u] = f.z;
+            t[4 * c4 + 3][u] = f.w;
+          }
+      } else {
+#pragma unroll
+        for (int c = 0; c < KPT; ++c)
+#pragma unroll
+          for (int u = 0; u < G; ++u)
+            t[c][u] = (u0 + u < n_sum && i0 + c < N) ? __ldg(P0 + (size_t)ro[u] + i0 + c) : 0.f;
+      }
+#pragma unroll
+      for (int c = 0; c < KPT; ++c)
+#pragma unroll
+        for (int u = 0; u < G; ++u)
+          if (u0 + u < n_sum) s[c] += t[c][u];
+    }
+#pragma unroll
+    for (int c = 0; c < KPT; ++c) v[c] = nrows <= 0 ? 0.f : s[c] / div;
+  } else {
+    const float* src = a.scores + (size_t)b * N;
+    if ((N & 3) == 0 && (reinterpret_cast<uintptr_t>(src) & 15u) == 0) {
+#pragma unroll
+      for (int c4 = 0; c4 < KPT / 4; ++c4) {
+        float4 f = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (i0 + 4 * c4 < N) f = __ldg(reinterpret_cast<const float4*>(src + i0) + c4);
+        v[4 * c4 + 0] = f.x;
+        v[4 * c4 + 1] = f.y;
+        v[4 * c4 + 2] = f.z;
+        v[4 * c4 + 3] = f.w;
+      }
+    } else {
+#pragma unroll
+      for (int c = 0; c < KPT; ++c) v[c] = i0 + c < N ? __ldg(src + i0 + c) : 0.f;
+    }
+  }
+  float* so = a.scores_out ? a.scores_out + (size_t)b * N : nullptr;
+  mn = 0xffffffffu;
+  mx = 0u;
+#pragma unroll
+  for (int c = 0; c < KPT; ++c) {
+    key[c] = 0u;
+    if (i0 + c < N) {
+      if (so) so[i0 + c] = v[c];
+      key[c] = float_key(v[c]);
+      mn = min(mn, key[c]);
+      mx = max(mx, key[c]);
     }
   }
 }
