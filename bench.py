@@ -774,10 +774,7 @@ def run_gb300(args, dist):
         c = copies[i % len(copies)]
         step_serial(c["Q"], c["K"], c["V"], c["hidden"], c["pos"], c["text_start"], c["text_len"], c["seq_len"], vis)
 
-    # kernels per step: one-pass head scores (tcgen05, L_max <= 8192), top-k,
-    # compaction; the two-pass and CUDA-core forms launch two head kernels
-    launches_per_step = 3 if (algo_name in ("auto", "tcgen05", "stream", "cluster") and w.dtype == "bf16"
-                              and w.L_max <= 8192) else 4
+    launches_per_step = kernels_per_step(w, algo_name)
     reps = 20
     t_compact = time_graph(compact_i, reps)
     t_head = time_graph(head_topk_i, reps)
@@ -924,6 +921,15 @@ def video_measure(P, synth, torch, dist, dev, stream, args, peak):
     if rc != 0:
         raise RuntimeError(f"device status {rc} {bits} after the video legs")
     return out
+
+
+def kernels_per_step(w, algo_name):
+    """Kernels one pruning step launches: the one-pass tensor-core head scores
+    (L_max <= 8192; the streaming or the cluster form), the top-k and the
+    compaction; the two-pass and CUDA-core forms launch two head kernels."""
+    if w.dtype != "bf16" or w.L_max > 8192 or algo_name not in ("auto", "tcgen05", "stream", "cluster"):
+        return 4
+    return 3
 
 
 def e2e_measure(P, torch, dist, w, cpu, step0, algo, dev, E):
