@@ -9,7 +9,10 @@
 // indices (prefix and text rows), then the kept visual rows - and every CTA
 // owns a contiguous range of each phase. Launched as a programmatic dependent
 // of the kernel that writes idx, the first phase overlaps that kernel; the
-// threads that read idx wait for it (griddepcontrol.wait, a no-op otherwise). One thread per CTA
+// threads that read idx wait for it (griddepcontrol.wait). A call on its own
+// (no programmatic dependency) splits the two phases as one list over four
+// CTAs per SM, and each CTA loads its kept indices at once, alongside the
+// sequence lengths: its few rows are then one short chain of round trips. One thread per CTA
 // streams its range through a ring of shared-memory slots: a cp.async.bulk load
 // (global -> shared, completion on the slot's mbarrier) and, once it lands, a
 // cp.async.bulk store (shared -> global, bulk group). A slot is refilled as soon
@@ -115,9 +118,15 @@ __device__ __forceinline__ void phase_row(const CompactArgs& a, int phase, long 
   }
 }
 
+// alone: launched with no programmatic dependency (nothing to overlap, idx is
+// ready at the start): the two phases' items are split over the CTAs as one
+// list, the producer stages its kept indices before its first load, and the
+// helpers resolve and copy all their rows in one pass. Otherwise each phase is
+// split over every CTA, and idx is read only after the wait.
 template <int kSlots>
 __global__ void __launch_bounds__(kCompactThreads) compact_kernel(const CompactArgs a, int np0,
-                                                                   int np1, int np2, int small) {
+                                                                   int np1, int np2, int small,
+                                                                   int alone) {
   extern __shared__ __align__(128) uint8_t slots[];
   __shared__ __align__(8) uint64_t bars[kSlots];
   __shared__ char* ring_dst[kSlots];
@@ -128,13 +137,21 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(const CompactA
   // so that rows are spread over CTAs even when every tensor is small)
   const int NB = np0 + np1 + np2;
   const int NP = NB > 0 ? NB : 1;
-  long long rows[2] = {(long long)a.B * (a.L_out - a.keep), (long long)a.B * a.keep};
+  const long long items[2] = {(long long)a.B * (a.L_out - a.keep) * NP, (long long)a.B * a.keep * NP};
   long long beg[2], fin[2];
-  for (int ph = 0; ph < 2; ++ph) {
-    const long long total = rows[ph] * NP;
-    const long long per = (total + gridDim.x - 1) / gridDim.x;
-    beg[ph] = min(total, (long long)blockIdx.x * per);
-    fin[ph] = min(total, beg[ph] + per);
+  if (alone) {
+    // [phase 0 | phase 1] as one list, in equal shares (they differ by at most one)
+    const long long T = items[0] + items[1];
+    const long long lo = T * blockIdx.x / gridDim.x, hi = T * (blockIdx.x + 1) / gridDim.x;
+    beg[0] = min(lo, items[0]);
+    fin[0] = min(hi, items[0]);
+    beg[1] = max(lo, items[0]) - items[0];
+    fin[1] = max(hi, items[0]) - items[0];
+  } else {
+    for (int ph = 0; ph < 2; ++ph) {
+      beg[ph] = items[ph] * blockIdx.x / gridDim.x;
+      fin[ph] = items[ph] * (blockIdx.x + 1) / gridDim.x;
+    }
   }
 
   // a kernel launched as this grid's programmatic dependent may start now (it
@@ -162,6 +179,21 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(const CompactA
     int b = 0, w = 0, q = 0, per = 1;
     int ord = 0;  // rows of the phase started so far (the staged index of a phase-1 row)
     int sl = 0;
+    // the kept indices of this CTA's phase-1 rows into idx_s
+    auto stage_idx = [&]() {
+      if (beg[1] >= fin[1]) return;
+      const long long r1 = (fin[1] + NP - 1) / NP;
+      const int n = (int)min((long long)kIdxStage, r1 - beg[1] / NP);
+      const int* src = a.idx + beg[1] / NP;
+      for (int j0 = 0; j0 < n; j0 += kStageBatch) {
+        int v[kStageBatch];
+#pragma unroll
+        for (int j = 0; j < kStageBatch; ++j) v[j] = j0 + j < n ? src[j0 + j] : 0;
+#pragma unroll
+        for (int j = 0; j < kStageBatch; ++j)
+          if (j0 + j < n) idx_s[j0 + j] = v[j];
+      }
+    };
     auto start_phase = [&](int ph) {
       if (beg[ph] >= fin[ph]) return;  // nothing of this phase here (per may be 0)
       per = ph == 0 ? a.L_out - a.keep : a.keep;
@@ -171,21 +203,12 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(const CompactA
       b = (int)(row / per);
       w = (int)(row - (long long)b * per);
       sl = a.seq_len[b];
-      if (ph == 1) {
+      if (ph == 1 && !alone) {
         pdl_wait();  // idx is written by the previous kernel
-        const long long r1 = (fin[1] + NP - 1) / NP;
-        const int n = (int)min((long long)kIdxStage, r1 - beg[1] / NP);
-        const int* src = a.idx + beg[1] / NP;
-        for (int j0 = 0; j0 < n; j0 += kStageBatch) {
-          int v[kStageBatch];
-#pragma unroll
-          for (int j = 0; j < kStageBatch; ++j) v[j] = j0 + j < n ? src[j0 + j] : 0;
-#pragma unroll
-          for (int j = 0; j < kStageBatch; ++j)
-            if (j0 + j < n) idx_s[j0 + j] = v[j];
-        }
+        stage_idx();
       }
     };
+    if (alone) stage_idx();  // in flight with the lengths start_phase loads
     start_phase(0);
     // next valid item; false when both phases are exhausted
     auto fetch = [&](Item& it) -> bool {
@@ -286,68 +309,83 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(const CompactA
     const int lane = small ? (int)(threadIdx.x & 31) : 0;
     const int worker = small ? (int)(threadIdx.x >> 5) - 1 : ht;
     const int n_workers = small ? kCompactThreads / 32 - 1 : n_ht;
-    for (int ph = 0; ph < 2; ++ph) {
-      if (ph == 1) pdl_wait();
-      const long long r0 = (beg[ph] + NP - 1) / NP, r1 = (fin[ph] + NP - 1) / NP;
-      for (long long c0 = r0; c0 < r1; c0 += kMetaRows) {
-        const int nrow = (int)min((long long)kMetaRows, r1 - c0);
-        for (int k = ht; k < nrow; k += n_ht) {
-          int b, r;
-          phase_row(a, ph, c0 + k, b, r);
-          const int sl = a.seq_len[b];
-          bool ok = !(sl > a.L_max || sl < a.vis_start + a.N_v || r >= sl - a.N_v + a.keep);
-          const int sr = ok ? src_row(a, b, r, ok) : 0;
-          meta_s[k] = ok ? make_int4(b, r, sr, 0) : make_int4(-1, 0, 0, 0);
+    // (sample, output row, source row) of row `row` of phase ph into meta_s[k]
+    auto meta_row = [&](int ph, long long row, int k) {
+      int b, r;
+      phase_row(a, ph, row, b, r);
+      const int sl = a.seq_len[b];
+      bool ok = !(sl > a.L_max || sl < a.vis_start + a.N_v || r >= sl - a.N_v + a.keep);
+      const int sr = ok ? src_row(a, b, r, ok) : 0;
+      meta_s[k] = ok ? make_int4(b, r, sr, 0) : make_int4(-1, 0, 0, 0);
+    };
+    // the copies of the rows in meta_s[0..nrow)
+    auto copy_rows = [&](int nrow) {
+      for (int k = worker; k < nrow; k += n_workers) {
+        const int4 mt = meta_s[k];
+        if (mt.x < 0) continue;
+        const int b = mt.x, r = mt.y, sr = mt.z;
+        if (a.pos != nullptr)
+          for (int p = lane; p < a.P; p += 32)
+            a.pos_out[((size_t)p * a.B + b) * a.L_out + r] = a.pos[((size_t)p * a.B + b) * a.L_max + sr];
+        // the row's pieces of every small tensor, as one list of 16-byte
+        // pieces: all of a lane's loads are issued before its stores (one
+        // memory round trip per row, not one per tensor)
+        const uint4 *s0 = nullptr, *s1 = nullptr, *s2 = nullptr;
+        uint4 *d0 = nullptr, *d1 = nullptr, *d2 = nullptr;
+        int n0 = 0, n1 = 0, n2 = 0;
+        if (small & 1) {
+          const long long rb = a.row_bytes[0];
+          s0 = reinterpret_cast<const uint4*>(a.src[0] + ((long long)b * a.L_max + sr) * rb);
+          d0 = reinterpret_cast<uint4*>(a.dst[0] + ((long long)b * a.L_out + r) * rb);
+          n0 = (int)(rb / 16);
         }
-        helpers_sync();
-        for (int k = worker; k < nrow; k += n_workers) {
-          const int4 mt = meta_s[k];
-          if (mt.x < 0) continue;
-          const int b = mt.x, r = mt.y, sr = mt.z;
-          if (a.pos != nullptr)
-            for (int p = lane; p < a.P; p += 32)
-              a.pos_out[((size_t)p * a.B + b) * a.L_out + r] = a.pos[((size_t)p * a.B + b) * a.L_max + sr];
-          // the row's pieces of every small tensor, as one list of 16-byte
-          // pieces: all of a lane's loads are issued before its stores (one
-          // memory round trip per row, not one per tensor)
-          const uint4 *s0 = nullptr, *s1 = nullptr, *s2 = nullptr;
-          uint4 *d0 = nullptr, *d1 = nullptr, *d2 = nullptr;
-          int n0 = 0, n1 = 0, n2 = 0;
-          if (small & 1) {
-            const long long rb = a.row_bytes[0];
-            s0 = reinterpret_cast<const uint4*>(a.src[0] + ((long long)b * a.L_max + sr) * rb);
-            d0 = reinterpret_cast<uint4*>(a.dst[0] + ((long long)b * a.L_out + r) * rb);
-            n0 = (int)(rb / 16);
-          }
-          if (small & 2) {
-            const long long rb = a.row_bytes[1];
-            s1 = reinterpret_cast<const uint4*>(a.src[1] + ((long long)b * a.L_max + sr) * rb);
-            d1 = reinterpret_cast<uint4*>(a.dst[1] + ((long long)b * a.L_out + r) * rb);
-            n1 = (int)(rb / 16);
-          }
-          if (small & 4) {
-            const long long rb = a.row_bytes[2];
-            s2 = reinterpret_cast<const uint4*>(a.src[2] + ((long long)b * a.L_max + sr) * rb);
-            d2 = reinterpret_cast<uint4*>(a.dst[2] + ((long long)b * a.L_out + r) * rb);
-            n2 = (int)(rb / 16);
-          }
-          const int tot = n0 + n1 + n2;
-          for (int q0 = 0; q0 < tot; q0 += 32 * kSmallPieces) {
-            uint4 v[kSmallPieces];
+        if (small & 2) {
+          const long long rb = a.row_bytes[1];
+          s1 = reinterpret_cast<const uint4*>(a.src[1] + ((long long)b * a.L_max + sr) * rb);
+          d1 = reinterpret_cast<uint4*>(a.dst[1] + ((long long)b * a.L_out + r) * rb);
+          n1 = (int)(rb / 16);
+        }
+        if (small & 4) {
+          const long long rb = a.row_bytes[2];
+          s2 = reinterpret_cast<const uint4*>(a.src[2] + ((long long)b * a.L_max + sr) * rb);
+          d2 = reinterpret_cast<uint4*>(a.dst[2] + ((long long)b * a.L_out + r) * rb);
+          n2 = (int)(rb / 16);
+        }
+        const int tot = n0 + n1 + n2;
+        for (int q0 = 0; q0 < tot; q0 += 32 * kSmallPieces) {
+          uint4 v[kSmallPieces];
 #pragma unroll
-            for (int j = 0; j < kSmallPieces; ++j) {
-              const int q = q0 + lane + 32 * j;
-              if (q < tot)
-                v[j] = __ldcs(q < n0 ? s0 + q : (q < n0 + n1 ? s1 + (q - n0) : s2 + (q - n0 - n1)));
-            }
+          for (int j = 0; j < kSmallPieces; ++j) {
+            const int q = q0 + lane + 32 * j;
+            if (q < tot)
+              v[j] = __ldcs(q < n0 ? s0 + q : (q < n0 + n1 ? s1 + (q - n0) : s2 + (q - n0 - n1)));
+          }
 #pragma unroll
-            for (int j = 0; j < kSmallPieces; ++j) {
-              const int q = q0 + lane + 32 * j;
-              if (q < tot) __stcs(q < n0 ? d0 + q : (q < n0 + n1 ? d1 + (q - n0) : d2 + (q - n0 - n1)), v[j]);
-            }
+          for (int j = 0; j < kSmallPieces; ++j) {
+            const int q = q0 + lane + 32 * j;
+            if (q < tot) __stcs(q < n0 ? d0 + q : (q < n0 + n1 ? d1 + (q - n0) : d2 + (q - n0 - n1)), v[j]);
           }
         }
-        helpers_sync();  // meta_s is rewritten by the next chunk
+      }
+    };
+    const long long r0[2] = {(beg[0] + NP - 1) / NP, (beg[1] + NP - 1) / NP};
+    const long long r1[2] = {(fin[0] + NP - 1) / NP, (fin[1] + NP - 1) / NP};
+    const int n0 = (int)(r1[0] - r0[0]), n1 = (int)(r1[1] - r0[1]);
+    if (alone && n0 + n1 <= kMetaRows) {
+      // every row of both phases resolved, then copied, in one pass
+      for (int k = ht; k < n0 + n1; k += n_ht) meta_row(k < n0 ? 0 : 1, k < n0 ? r0[0] + k : r0[1] + (k - n0), k);
+      helpers_sync();
+      copy_rows(n0 + n1);
+    } else {
+      for (int ph = 0; ph < 2; ++ph) {
+        if (ph == 1) pdl_wait();
+        for (long long c0 = r0[ph]; c0 < r1[ph]; c0 += kMetaRows) {
+          const int nrow = (int)min((long long)kMetaRows, r1[ph] - c0);
+          for (int k = ht; k < nrow; k += n_ht) meta_row(ph, c0 + k, k);
+          helpers_sync();
+          copy_rows(nrow);
+          helpers_sync();  // meta_s is rewritten by the next chunk
+        }
       }
     }
   }
@@ -467,7 +505,9 @@ cudaError_t compact_launch(const CompactArgs& a, int num_sms, cudaStream_t s, bo
   }
   const int nb = np[0] + np[1] + np[2];
   const long long total = (long long)a.B * a.L_out * (nb > 0 ? nb : 1);
-  long long grid = (long long)kCtasPerSm * num_sms;
+  // Two CTAs per SM when the call follows a kernel it overlaps (room is left
+  // for the next step's head-score CTAs), four when it runs on its own.
+  long long grid = (long long)(pdl ? kCtasPerSm : 2 * kCtasPerSm) * num_sms;
   // Alone, the compaction spreads over every SM (a small problem is bound by
   // the latency of each CTA's few copies, so more CTAs finish it sooner). With
   // concurrent calls on other streams, a small problem takes at least
@@ -490,8 +530,9 @@ cudaError_t compact_launch(const CompactArgs& a, int num_sms, cudaStream_t s, bo
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = pdl ? 1 : 0;
-  return deep ? cudaLaunchKernelEx(&cfg, compact_kernel<kSlotsDeep>, a, np[0], np[1], np[2], small)
-              : cudaLaunchKernelEx(&cfg, compact_kernel<kSlotsShort>, a, np[0], np[1], np[2], small);
+  const int alone = pdl ? 0 : 1;
+  return deep ? cudaLaunchKernelEx(&cfg, compact_kernel<kSlotsDeep>, a, np[0], np[1], np[2], small, alone)
+              : cudaLaunchKernelEx(&cfg, compact_kernel<kSlotsShort>, a, np[0], np[1], np[2], small, alone);
 }
 
 }  // namespace provip
