@@ -51,7 +51,10 @@ constexpr int kSlotBytes = PROVIP_COMPACT_SLOT_BYTES;
 constexpr int kSlotsShort = PROVIP_COMPACT_SLOTS;
 constexpr int kSlotsDeep = PROVIP_COMPACT_DEEP_SLOTS;
 constexpr int kCtasPerSm = PROVIP_COMPACT_CTAS_PER_SM;
+// a producer warp and three helper warps; a fourth helper warp when the helpers
+// copy rows of small tensors (one round of copies for four rows per CTA)
 constexpr int kCompactThreads = 128;
+constexpr int kCompactThreadsSmall = 160;
 #ifndef PROVIP_COMPACT_MIN_CTA_KIB
 #define PROVIP_COMPACT_MIN_CTA_KIB 160
 #endif
@@ -77,9 +80,9 @@ constexpr int kStageBatch = 16;
 // together before copying them
 constexpr int kMetaRows = 96;
 
-// barrier of the helper threads (warps 1..3; the producer warp does not take part)
+// barrier of the helper threads (warps 1..; the producer warp does not take part)
 __device__ __forceinline__ void helpers_sync() {
-  asm volatile("bar.sync 1, %0;" ::"n"(kCompactThreads - 32) : "memory");
+  asm volatile("bar.sync 1, %0;" ::"r"(blockDim.x - 32) : "memory");
 }
 
 __device__ __forceinline__ int src_row(const CompactArgs& a, int b, int r, bool& ok) {
@@ -124,7 +127,7 @@ __device__ __forceinline__ void phase_row(const CompactArgs& a, int phase, long 
 // helpers resolve and copy all their rows in one pass. Otherwise each phase is
 // split over every CTA, and idx is read only after the wait.
 template <int kSlots>
-__global__ void __launch_bounds__(kCompactThreads) compact_kernel(const CompactArgs a, int np0,
+__global__ void __launch_bounds__(kCompactThreadsSmall) compact_kernel(const CompactArgs a, int np0,
                                                                    int np1, int np2, int small,
                                                                    int alone) {
   extern __shared__ __align__(128) uint8_t slots[];
@@ -149,8 +152,9 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(const CompactA
     fin[1] = max(hi, items[0]) - items[0];
   } else {
     for (int ph = 0; ph < 2; ++ph) {
-      beg[ph] = items[ph] * blockIdx.x / gridDim.x;
-      fin[ph] = items[ph] * (blockIdx.x + 1) / gridDim.x;
+      const long long per = (items[ph] + gridDim.x - 1) / gridDim.x;
+      beg[ph] = min(items[ph], (long long)blockIdx.x * per);
+      fin[ph] = min(items[ph], beg[ph] + per);
     }
   }
 
@@ -305,10 +309,10 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(const CompactA
     // the (sample, output row, source row) of its own rows - their dependent
     // loads of lengths and kept indices all in flight at once - into shared
     // memory, then (after a barrier of the helper threads) the copies run.
-    const int ht = (int)threadIdx.x - 32, n_ht = kCompactThreads - 32;
+    const int ht = (int)threadIdx.x - 32, n_ht = (int)blockDim.x - 32;
     const int lane = small ? (int)(threadIdx.x & 31) : 0;
     const int worker = small ? (int)(threadIdx.x >> 5) - 1 : ht;
-    const int n_workers = small ? kCompactThreads / 32 - 1 : n_ht;
+    const int n_workers = small ? (int)blockDim.x / 32 - 1 : n_ht;
     // (sample, output row, source row) of row `row` of phase ph into meta_s[k]
     auto meta_row = [&](int ph, long long row, int k) {
       int b, r;
@@ -523,7 +527,7 @@ cudaError_t compact_launch(const CompactArgs& a, int num_sms, cudaStream_t s, bo
   cudaLaunchConfig_t cfg = {};
   cudaLaunchAttribute attr[1];
   cfg.gridDim = dim3((unsigned)grid);
-  cfg.blockDim = dim3(kCompactThreads);
+  cfg.blockDim = dim3(small ? kCompactThreadsSmall : kCompactThreads);
   cfg.dynamicSmemBytes = (size_t)(deep ? kSlotsDeep : kSlotsShort) * kSlotBytes;
   cfg.stream = s;
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
