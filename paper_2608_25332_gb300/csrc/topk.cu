@@ -50,12 +50,12 @@ __device__ __forceinline__ void load_sample_keys(const TopkArgs& a, int b, uint3
 __global__ void __launch_bounds__(kTopkMaxThreads) topk_kernel(const TopkArgs a) {
   extern __shared__ uint32_t keys[];
   __shared__ TopkShared sh;
+  for (int q = threadIdx.x; q < kSelectBins; q += blockDim.x) sh.hist[0][q] = 0;
   // launched as a programmatic dependent: wait until the kernel that writes the
   // scores has completed (which, for overlapped calls, implies the previous
   // compaction has completed too)
   asm volatile("griddepcontrol.wait;" ::: "memory");
   const int b = blockIdx.x;
-  for (int q = threadIdx.x; q < kSelectBins; q += blockDim.x) sh.hist[0][q] = 0;
   uint32_t mn, mx, lo, hi;
   load_sample_keys(a, b, keys, a.scores_out ? a.scores_out + (size_t)b * a.N : nullptr, mn, mx);
   topk_block_range(mn, mx, sh, lo, hi);  // its barrier also publishes the keys and the cleared histogram
@@ -73,10 +73,11 @@ constexpr int kRegMaxThreads = 512;
 template <int KPT>
 __global__ void __launch_bounds__(kRegMaxThreads) topk_reg_kernel(const TopkArgs a) {
   __shared__ TopkShared sh;
-  // a programmatic dependent: wait for the kernel that writes the scores
+  // the histogram is cleared while the kernel that writes the scores finishes
+  for (int q = threadIdx.x; q < kSelectBins; q += blockDim.x) sh.hist[0][q] = 0;
+  // a programmatic dependent: wait for that kernel
   asm volatile("griddepcontrol.wait;" ::: "memory");
   const int b = blockIdx.x;
-  for (int q = threadIdx.x; q < kSelectBins; q += blockDim.x) sh.hist[0][q] = 0;
   uint32_t key[KPT], mn, mx, lo, hi;
   load_keys_reg<KPT>(a, b, key, mn, mx);
   topk_block_range(mn, mx, sh, lo, hi);  // its barrier also publishes the cleared histogram
