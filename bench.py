@@ -45,12 +45,13 @@ DEFAULT_WORKLOAD = "llava_next_7b_bf16_b8"
 FALLBACK_HBM_GBS = 6800.0
 GRAPH_CHUNK = 100
 N_COPIES = 3
+L2_BYTES = 129e6  # GB300's L2; the rotating inputs of a timed loop span at least 3x this
 N_VIS = 6  # visual heads per pruning layer (the paper's setting, Sec. 5.1)
 
 # DRAM traffic of one compaction launch on the default workload, from the ncu
 # capture summarised in profiles/ (null when the kernel source has changed
 # since: the sha1 of the kernel file is checked at run time).
-COMPACT_TRAFFIC = {"sha1": "5d122551ff6fe2cfedc2e5435c94ad4bcc9ee65a", "bytes": 115629056,
+COMPACT_TRAFFIC = {"sha1": "4d447a409e84a515a32c928dcba8278a535f9f57", "bytes": 115457280,
                    "profile": "profiles/prune_llava_next_b8_kernels.md"}
 
 
@@ -67,6 +68,9 @@ def parse_args(argv=None):
     ap.add_argument("--e2e-steps", type=int, default=20)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--copies", type=int, default=N_COPIES, help="rotating device copies of the inputs")
+    ap.add_argument("--compact-only", action="store_true",
+                    help="time the compaction alone (provip_compact, no programmatic dependency) on --workload "
+                         "and print one JSON line (the command the compaction profiles use)")
     ap.add_argument("--prellm-only", action="store_true",
                     help="time only the pre-LLM pass (provip_similarity_reduce) and print its JSON")
     ap.add_argument("--prellm-reps", type=int, default=20)
@@ -553,12 +557,19 @@ class Lanes:
     PROVIP_PRUNE_CONCURRENT."""
 
     def __init__(self, P, synth, w, dev, S, algo, n_copies, seed):
+        import math
         import torch
         self.P, self.torch, self.dev, self.S = P, torch, dev, S
         flags = P.PRUNE_OVERLAP_PREVIOUS | (P.PRUNE_CONCURRENT if S > 1 else 0)
         self.lanes = []
         for s_ in range(S):
             cpu = synth.in_llm_inputs(w, seed=seed + 7 * s_)
+            if s_ == 0:
+                # at least n_copies per lane, and enough that all lanes' inputs span 3x the L2
+                self.copy_bytes = sum(v.numel() * v.element_size() for v in cpu.values()
+                                      if isinstance(v, torch.Tensor))
+                n_copies = max(1, n_copies, math.ceil(3 * L2_BYTES / (S * self.copy_bytes)))
+                self.n_copies = n_copies
             cs = [{k: (v.to(dev) if isinstance(v, torch.Tensor) else v) for k, v in cpu.items()}
                   for _ in range(max(1, n_copies))]
             st = P.PruneStep(cs[0]["Q"], cs[0]["K"], cs[0]["V"], cs[0]["hidden"], cs[0]["pos"], cpu["head_list"],
@@ -711,7 +722,8 @@ def run_gb300(args, dist):
         if dist.rank == 0:
             print(json.dumps({"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": dist.world, "steps": K,
                               "warmup": args.warmup, "ms_per_step": 1e3 * max_sec / K, "quick": True,
-                              "config": workload_config(w, algo_name, n_copies), "repeats": head["repeats"]}))
+                              "config": workload_config(w, algo_name, lanes.n_copies, input_mb),
+                              "repeats": head["repeats"]}))
         return 0
 
     # ---- the same workload on one stream: the configuration as stated ----
@@ -722,7 +734,9 @@ def run_gb300(args, dist):
         g1 = one.graphs(K, stream)
         t1s, _ = timed_repeats(torch, g1, dist, args.target_s / 2)
         single = dict(summarize(t1s, units, K, ab["path"], peak), streams=1,
-                      algo="auto" if single_algo == P.ALGO_AUTO else algo_name)
+                      algo="auto" if single_algo == P.ALGO_AUTO else algo_name,
+                      l2=f"inputs larger than L2: {one.n_copies} rotating device copies of "
+                         f"{one.copy_bytes / 1e6:.0f} MB")
         del g1
     else:
         single = dict(head, streams=1, algo=algo_name)
@@ -832,7 +846,7 @@ def run_gb300(args, dist):
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": dist.world, "steps": K,
             "warmup": args.warmup, "ms_per_step": 1e3 * max_sec / K, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
-            "config": dict(workload_config(w, algo_name, n_copies, input_mb), streams=S,
+            "config": dict(workload_config(w, algo_name, lanes.n_copies, input_mb), streams=S,
                            **({"concurrency": f"{S} streams of independent batches run concurrently (each with its "
                                               f"own inputs, outputs and workspace); value counts the samples of all "
                                               f"streams; single_stream is one stream"} if S > 1 else {})),
@@ -878,7 +892,9 @@ def video_measure(P, synth, torch, dist, dev, stream, args, peak):
         times, _ = timed_repeats(torch, graphs, dist, args.target_s / 2)
         ab = algorithmic_bytes(w, lanes.cpu0)
         r = summarize(times, dist.sum(float(w.B * K)), K, ab["path"], peak)
-        r.update(streams=S, algo=algo_name, us_per_sample=1e6 / r["value"] * dist.world)
+        r.update(streams=S, algo=algo_name, us_per_sample=1e6 / r["value"] * dist.world,
+                 l2=f"inputs larger than L2: {S} x {lanes.n_copies} rotating device copies of "
+                    f"{lanes.copy_bytes / 1e6:.0f} MB")
         if S > 1:
             r["effective_batch"] = S
         out[label] = r
@@ -1037,10 +1053,68 @@ def run_prellm_only(args):
     return 0
 
 
+def run_compact_only(args):
+    """The compaction on its own: one pruning step gives idx, then --steps calls
+    of provip_compact on rotating input copies (a CUDA graph of them, replayed
+    after one untimed launch), timed with events."""
+    import torch
+    import __graft_entry__
+    from paper_2608_25332_gb300 import provip as P
+    from paper_2608_25332_gb300 import synth
+    __graft_entry__.build()
+    dev = torch.device("cuda", 0)
+    w = synth.BY_NAME[args.workload]
+    cpu = synth.in_llm_inputs(w)
+    copy_bytes = sum(v.numel() * v.element_size() for v in cpu.values() if isinstance(v, torch.Tensor))
+    n_copies = max(1, args.copies, -(-int(3 * L2_BYTES) // copy_bytes))  # rotating inputs span 3x the L2
+    copies = [{k: (v.to(dev) if isinstance(v, torch.Tensor) else v) for k, v in cpu.items()}
+              for _ in range(n_copies)]
+    c0 = copies[0]
+    vis, nv, keep = cpu["vis_start"], cpu["N_v"], cpu["keep"]
+    st = P.PruneStep(c0["Q"], c0["K"], c0["V"], c0["hidden"], c0["pos"], cpu["head_list"], w.n_t[1], nv, keep,
+                     want_scores=False)
+    idx = st(c0["Q"], c0["K"], c0["V"], c0["hidden"], c0["pos"], c0["text_start"], c0["text_len"],
+             c0["seq_len"], vis)["idx"].clone()
+    outs = (st.hidden_out, st.K_out, st.V_out, st.pos_out)
+    n = max(1, min(args.steps, 500))
+
+    def call(i):
+        c = copies[i % len(copies)]
+        P.provip_compact(idx, c["hidden"], c["K"], c["V"], c["pos"], c["seq_len"], vis, nv, out=outs)
+
+    for i in range(max(args.warmup, 1)):
+        call(i)
+    stream = torch.cuda.Stream(device=dev)
+    stream.wait_stream(torch.cuda.current_stream())
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        for i in range(n):
+            call(i)
+    g.replay()
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    g.replay()
+    b.record()
+    torch.cuda.synchronize()
+    rc, bits = P.provip_device_status(clear=True)
+    if rc != 0 or bits != 0:
+        raise RuntimeError(f"device status {rc} {bits}")
+    us = a.elapsed_time(b) * 1e3 / n
+    ab = algorithmic_bytes(w, cpu)["compact"]
+    peak, src = hbm_peak()
+    print(json.dumps({"compact_only": {"workload": w.name, "calls": n, "us_per_call": us, "copies": n_copies,
+                                       "algorithmic_bytes": ab, "achieved_gbs": ab / us / 1e3,
+                                       "frac": ab / us / 1e3 / peak, "peak_source": src}}))
+    return 0
+
+
 def main(argv=None):
     args = parse_args(argv)
     if args.prellm_only:
         return run_prellm_only(args)
+    if args.compact_only:
+        return run_compact_only(args)
     dist = Dist()
     if args.impl == "reference":
         dist.init("gloo")
