@@ -54,6 +54,35 @@ struct DevInfo {
 DevInfo g_dev[64];
 std::mutex g_dev_mu;  // serialises the first lookup of each device
 
+// A second stream per host thread and device for the part of a call that can
+// run beside the rest (forked from the caller's stream and joined back with
+// the two events), so that calls from different threads never share one. They
+// live until the process ends: destroying them at thread exit could run after
+// the CUDA runtime has shut down.
+struct SideStream {
+  cudaStream_t s = nullptr;
+  cudaEvent_t fork = nullptr, join = nullptr;
+};
+thread_local SideStream tl_side[64];
+int side_stream(SideStream** out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+  if (dev < 0 || dev >= 64) return fail(PROVIP_ERR_UNSUPPORTED, "device ordinal %d >= 64", dev);
+  SideStream& x = tl_side[dev];
+  if (x.s == nullptr) {
+    e = cudaStreamCreateWithFlags(&x.s, cudaStreamNonBlocking);
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&x.fork, cudaEventDisableTiming);
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&x.join, cudaEventDisableTiming);
+    if (e != cudaSuccess) {
+      x = SideStream();
+      return cuda_fail(e, "side stream");
+    }
+  }
+  *out = &x;
+  return PROVIP_OK;
+}
+
 // per-device facts, looked up once with that device current (safe from several
 // host threads: the first caller fills them under the lock, later ones read them
 // after an acquire of `init`)
@@ -646,15 +675,27 @@ extern "C" int provip_similarity_reduce(const void* emb_v, int B, int N_v, int D
   const uint8_t* mask = crit_mask_or_null;
   uint8_t* mask_dst = mask_out_or_null ? mask_out_or_null : w.mask;
   cudaError_t e = cudaSuccess;
+  cudaEvent_t mask_ready = nullptr;
   if (!mask) {
-    e = crit_text_launch(a, mask_dst, nullptr, w.G, s);
+    // the critical text rows (their Gram and threshold) run on a side stream
+    // beside the relevance Gram, which reads no mask; the stream waits for
+    // them before the kernel that takes the max over the critical rows
+    SideStream* side;
+    if ((rc = side_stream(&side))) return rc;
+    e = cudaEventRecord(side->fork, s);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(side->s, side->fork, 0);
+    if (e == cudaSuccess) e = crit_text_launch(a, mask_dst, nullptr, w.G, side->s);
+    if (e == cudaSuccess) e = cudaEventRecord(side->join, side->s);
+    if (e == cudaSuccess) mask_ready = side->join;
     mask = mask_dst;
   } else if (mask_out_or_null) {
     e = cudaMemcpyAsync(mask_out_or_null, mask, (size_t)B * N_t_max, cudaMemcpyDeviceToDevice, s);
   }
   float* p = p_out_or_null ? p_out_or_null : w.p;
-  if (e == cudaSuccess)
-    e = relevance_launch(a, mask, w.inv_v, p, w.sum, w.mu, w.invt, rel_splits(B, N_v), d->sms, s);
+  if (e == cudaSuccess) {
+    e = relevance_launch(a, mask, w.inv_v, p, w.sum, w.mu, w.invt, rel_splits(B, N_v), d->sms, s, mask_ready);
+    if (e != cudaSuccess && mask_ready != nullptr) cudaStreamWaitEvent(s, mask_ready, 0);  // join even so
+  }
   if (e == cudaSuccess) {
     TopkArgs t;
     memset(&t, 0, sizeof(t));

@@ -175,10 +175,14 @@ cudaError_t vis_inv_norm_launch(const SimArgs& a, float* inv_v, cudaStream_t s);
 // Sec. 4.3: p[b][j] = max_{i in T} cos(t_i, v_j) - mu_i; also writes inv_v (the
 // inverse norms of the visual rows, used again by the merge). ws_sum holds
 // n_split partial sums over row chunks and their total.
-// ws_sum holds max((n_split + 1) * B * D, relevance_fused_floats(B, N_v, N_t_max)) floats
+// ws_sum holds max((n_split + 1) * B * D, relevance_fused_floats(B, N_v, N_t_max)) floats.
+// mask_ready (optional): an event recorded where the mask is written (another
+// stream); s waits for it before the first kernel that reads the mask, so that
+// the kernels before that one run beside the mask's producer.
 cudaError_t relevance_launch(const SimArgs& a, const uint8_t* mask, float* inv_v,
                              float* p, float* ws_sum, float* ws_mu, float* ws_invt,
-                             int n_split, int num_sms, cudaStream_t s);
+                             int n_split, int num_sms, cudaStream_t s,
+                             cudaEvent_t mask_ready = nullptr);
 // Sec. 4.3 merge: assign[b][j] and merged[b][a][:]
 // n_split: the SIMT split (sized by the caller); ws_pruned: [B][N_v] ints and
 // ws_perm: [B][N_v][D] bf16 for the tcgen05 path (null: CUDA-core path);
@@ -200,7 +204,8 @@ size_t relevance_fused_floats(int B, int N_v, int N_t_max);
 // reads the text rows' inverse norms inv_t [B][N_t_max]; writes inv_v and p;
 // ws holds relevance_fused_floats(...) floats
 cudaError_t relevance_tc_launch(const SimArgs& a, const uint8_t* mask, const float* inv_t, float* inv_v,
-                                float* p, float* ws, int num_sms, cudaStream_t s);
+                                float* p, float* ws, int num_sms, cudaStream_t s,
+                                cudaEvent_t mask_ready = nullptr);
 bool merge_tc_supported(const SimArgs& a, int keep, int n_split);
 // pruned: the rows not kept, ascending ([B][N_v - keep], from merge_index_kernel)
 cudaError_t merge_argmax_tc_launch(const SimArgs& a, const int* keep_idx, int keep,

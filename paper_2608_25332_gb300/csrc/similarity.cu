@@ -873,14 +873,14 @@ cudaError_t vis_inv_norm_launch(const SimArgs& a, float* inv_v, cudaStream_t s) 
 
 cudaError_t relevance_launch(const SimArgs& a, const uint8_t* mask, float* inv_v, float* p,
                              float* ws_sum, float* ws_mu, float* ws_invt, int n_split,
-                             int num_sms, cudaStream_t s) {
+                             int num_sms, cudaStream_t s, cudaEvent_t mask_ready) {
   // bf16 with at most 128 text rows: the text rows' inverse norms, one
   // tensor-core read of the visual rows (norms, cosines and de-meaning sums)
   // and a small max kernel
   if (relevance_tc_supported(a)) {
     const size_t rows = (size_t)a.B * a.N_t_max;
     inv_norm_kernel<__nv_bfloat16><<<(unsigned)((rows + 7) / 8), 256, 0, s>>>(a.emb_t, rows, a.D, ws_invt);
-    return relevance_tc_launch(a, mask, ws_invt, inv_v, p, ws_sum, num_sms, s);
+    return relevance_tc_launch(a, mask, ws_invt, inv_v, p, ws_sum, num_sms, s, mask_ready);
   }
   const int chunk = (a.N_v + n_split - 1) / n_split;
   dim3 g1((a.D + 255) / 256, a.B, n_split);
@@ -920,11 +920,19 @@ cudaError_t relevance_launch(const SimArgs& a, const uint8_t* mask, float* inv_v
     if (!fused) vis_sum_kernel<float><<<g1, 256, 0, s>>>(a, inv_v, ws_sum, chunk);
     vis_sum_reduce_kernel<<<g4, 256, 0, s>>>(a, ws_sum, n_split, total);
     text_mu_kernel<float><<<g2, 256, 0, s>>>(a, total, ws_mu, ws_invt);
+    if (mask_ready != nullptr) {
+      const cudaError_t e = cudaStreamWaitEvent(s, mask_ready, 0);  // the first kernel that reads the mask
+      if (e != cudaSuccess) return e;
+    }
     relevance_kernel<float><<<g3, 256, 0, s>>>(a, mask, inv_v, ws_mu, ws_invt, p);
   } else {
     if (!fused) vis_sum_kernel<__nv_bfloat16><<<g1, 256, 0, s>>>(a, inv_v, ws_sum, chunk);
     vis_sum_reduce_kernel<<<g4, 256, 0, s>>>(a, ws_sum, n_split, total);
     text_mu_kernel<__nv_bfloat16><<<g2, 256, 0, s>>>(a, total, ws_mu, ws_invt);
+    if (mask_ready != nullptr) {
+      const cudaError_t e = cudaStreamWaitEvent(s, mask_ready, 0);
+      if (e != cudaSuccess) return e;
+    }
     relevance_kernel<__nv_bfloat16><<<g3, 256, 0, s>>>(a, mask, inv_v, ws_mu, ws_invt, p);
   }
   return cudaGetLastError();

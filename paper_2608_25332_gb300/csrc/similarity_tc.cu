@@ -623,7 +623,7 @@ size_t relevance_fused_floats(int B, int N_v, int N_t_max) {
 }
 
 cudaError_t relevance_tc_launch(const SimArgs& a, const uint8_t* mask, const float* inv_t, float* inv_v,
-                                float* p, float* ws, int num_sms, cudaStream_t s) {
+                                float* p, float* ws, int num_sms, cudaStream_t s, cudaEvent_t mask_ready) {
   static std::atomic<bool> smem_set[64];  // per device, zero-initialised
   int dev = 0;
   cudaGetDevice(&dev);
@@ -654,6 +654,10 @@ cudaError_t relevance_tc_launch(const SimArgs& a, const uint8_t* mask, const flo
                         (uint32_t)r.NT))
     return cudaErrorInvalidValue;
   relevance_fused_tc<<<dim3(r.n_vt, a.B), kThreads, smem, s>>>(r, mapV, mapT);
+  if (mask_ready != nullptr) {
+    e = cudaStreamWaitEvent(s, mask_ready, 0);  // the first kernel that reads the mask
+    if (e != cudaSuccess) return e;
+  }
   relevance_finish_kernel<<<dim3((a.N_v + 255) / 256, a.B), 256, 0, s>>>(r, a.text_len, mask, p);
   return cudaGetLastError();
 }
