@@ -266,9 +266,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (threadIdx.x < 32) tmem_dealloc(pipe.tmem, kMergeTmemCols);
 }
 
-// relevance_fused_tc: one read of the visual rows gives, per 128-row tile of
-// sample b (A = the 128 visual rows, B = [the same 128 visual rows ; the text
-// rows], both already adjacent in the stage, so one MMA of N = 128 + NT),
+// relevance_fused_tc: one read of the visual rows gives, per tile of R visual
+// rows of sample b (R = 128, 96 or 64, chosen so that the tiles spread evenly
+// over the SMs; A = the tile's rows, B = [the same R visual rows ; the text
+// rows], both already adjacent in the stage, so one MMA of N = R + NT; the
+// MMA's 128 A rows run past the R visual rows and their results are unused),
 //   * |v_j|^2 from the diagonal of the visual x visual block (thread = TMEM
 //     lane = visual row j reads its own column),
 //   * the cosines Y[b][j][i] = <v_j, t_i> |t_i|^-1 |v_j|^-1 (|t_i|^-1 from a
@@ -280,7 +282,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 struct RelFusedArgs {
   int B, N_v, D, N_t_max;
   int NT;        // text rows in the MMA (N_t_max rounded up to 16)
-  int n_vt;      // 128-row visual tiles per sample
+  int R;         // visual rows per tile (128, 96 or 64)
+  int n_vt;      // visual tiles per sample
   int n_stages;  // shared-memory ring depth
   const float* inv_t;  // [B][N_t_max]
   float* inv_v;  // [B][N_v]
@@ -308,10 +311,11 @@ __global__ void __launch_bounds__(kThreads, 2)
   __shared__ float s_invt[kBM];
   __shared__ float red[4][kBM];
   const int b = blockIdx.y, tile = blockIdx.x;
-  const int n0 = tile * kBM;
+  const int R = a.R;
+  const int n0 = tile * R;
   const int n_k = (a.D + kBK - 1) / kBK;
   const int NS = a.n_stages;
-  const uint32_t st_bytes = (uint32_t)kABytes + (uint32_t)a.NT * 128u;
+  const uint32_t st_bytes = (uint32_t)(R + a.NT) * 128u;
   const uint32_t sbase = smem_u32(smem_raw);
   uint8_t* stages = smem_raw + (((sbase + 1023u) & ~1023u) - sbase);
   if (threadIdx.x == 0) {
@@ -347,12 +351,12 @@ __global__ void __launch_bounds__(kThreads, 2)
         // rows past the sample's last visual row belong to the next sample (or
         // lie past the tensor and read as zeros): computed, never stored
         tma_load_2d(sa, &mapV, kb * kBK, b * a.N_v + n0, &pipe.full[s]);
-        tma_load_2d(sa + kABytes, &mapT, kb * kBK, b * a.N_t_max, &pipe.full[s]);
+        tma_load_2d(sa + R * 128, &mapT, kb * kBK, b * a.N_t_max, &pipe.full[s]);
       }
     }
   } else if (warp == 1) {
     if (lane == 0) {
-      const uint32_t idesc = idesc_bf16_f32(kBM, kBM + a.NT);
+      const uint32_t idesc = idesc_bf16_f32(kBM, R + a.NT);
       for (int kb = 0; kb < n_k; ++kb) {
         const int s = kb % NS;
         const uint32_t ph = (uint32_t)(kb / NS) & 1u;
@@ -374,7 +378,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     const int quad = warp & 3;
     const int r = quad * 32 + lane;
     const int j = n0 + r;
-    const bool rv = j < a.N_v;
+    const bool rv = r < R && j < a.N_v;
     s_invt[r] = r < a.N_t_max ? a.inv_t[(size_t)b * a.N_t_max + r] : 0.f;
     asm volatile("bar.sync 1, 128;" ::: "memory");  // s_invt complete (epilogue warps)
     const bool ok = warp_mbar_wait(&pipe.acc_full, 0, a.err) && !pipe.fail;
@@ -392,7 +396,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     float* yrow = a.Y + ((size_t)b * a.N_v + (rv ? j : 0)) * a.NT;
 #pragma unroll 1
     for (int cb = 0; cb * 32 < a.NT; ++cb) {
-      tmem_ld32(taddr + (uint32_t)(kBM + cb * 32), v);
+      tmem_ld32(taddr + (uint32_t)(R + cb * 32), v);
       tc_wait_ld();
 #pragma unroll
       for (int i = 0; i < 32; ++i) v[i] = v[i] * s_invt[cb * 32 + i] * iv;
@@ -618,8 +622,25 @@ bool relevance_tc_supported(const SimArgs& a) { return a.dtype == 1 && a.N_t_max
 static int rel_nt(int N_t_max) { return (N_t_max + 15) / 16 * 16; }
 
 size_t relevance_fused_floats(int B, int N_v, int N_t_max) {
-  const int NT = rel_nt(N_t_max), n_vt = (N_v + kBM - 1) / kBM;
+  const int NT = rel_nt(N_t_max), n_vt = (N_v + 63) / 64;  // tiles of the smallest R
   return (size_t)B * N_v * NT + (size_t)B * n_vt * NT;
+}
+
+// Visual rows per relevance tile: the R of 128, 96 and 64 whose tiles give the
+// busiest SM the fewest rows to take in (its tiles' visual and text rows,
+// ceil(tiles / SMs) tiles), the larger R on a tie.
+static int rel_tile_rows(int B, int N_v, int NT, int num_sms) {
+  int best = kBM;
+  long long best_cost = -1;
+  for (int R = kBM; R >= 64; R -= 32) {
+    const long long tiles = (long long)B * ((N_v + R - 1) / R);
+    const long long cost = ((tiles + num_sms - 1) / num_sms) * (R + NT);
+    if (best_cost < 0 || cost < best_cost) {
+      best_cost = cost;
+      best = R;
+    }
+  }
+  return best;
 }
 
 cudaError_t relevance_tc_launch(const SimArgs& a, const uint8_t* mask, const float* inv_t, float* inv_v,
@@ -636,20 +657,24 @@ cudaError_t relevance_tc_launch(const SimArgs& a, const uint8_t* mask, const flo
   r.D = a.D;
   r.N_t_max = a.N_t_max;
   r.NT = rel_nt(a.N_t_max);
-  r.n_vt = (a.N_v + kBM - 1) / kBM;
+  r.R = rel_tile_rows(a.B, a.N_v, r.NT, num_sms);
+  r.n_vt = (a.N_v + r.R - 1) / r.R;
   r.inv_t = inv_t;
   r.inv_v = inv_v;
   r.Y = ws;
   r.part = ws + (size_t)a.B * a.N_v * r.NT;
   r.err = a.err;
   // one CTA per SM when the tiles do not fill the GPU (deeper ring), else two
-  const size_t st_bytes = (size_t)kABytes + (size_t)r.NT * 128;
-  const size_t budget = (long long)a.B * r.n_vt <= num_sms ? kSmemMax - 1024 : 110 * 1024 - 1024;
+  // the MMA reads 128 A rows (16 KiB) from the start of a stage: the last
+  // stage keeps that much room even when R + NT rows are fewer
+  const size_t st_bytes = (size_t)(r.R + r.NT) * 128;
+  const size_t tail = st_bytes > (size_t)kABytes ? 0 : (size_t)kABytes - st_bytes;
+  const size_t budget = ((long long)a.B * r.n_vt <= num_sms ? kSmemMax - 1024 : 110 * 1024 - 1024) - tail;
   int ns = (int)(budget / st_bytes);
   r.n_stages = ns > kRelMaxStages ? kRelMaxStages : (ns < 2 ? 2 : ns);
-  const size_t smem = (size_t)r.n_stages * st_bytes + 1024;
+  const size_t smem = (size_t)r.n_stages * st_bytes + tail + 1024;
   CUtensorMap mapV, mapT;
-  if (make_tmap_bf16_2d(&mapV, a.emb_v, (uint64_t)a.B * a.N_v, (uint64_t)a.D, (uint64_t)a.D * 2, kBM) ||
+  if (make_tmap_bf16_2d(&mapV, a.emb_v, (uint64_t)a.B * a.N_v, (uint64_t)a.D, (uint64_t)a.D * 2, (uint32_t)r.R) ||
       make_tmap_bf16_2d(&mapT, a.emb_t, (uint64_t)a.B * a.N_t_max, (uint64_t)a.D, (uint64_t)a.D * 2,
                         (uint32_t)r.NT))
     return cudaErrorInvalidValue;
