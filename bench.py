@@ -826,6 +826,7 @@ def run_gb300(args, dist):
 
     # ---- e2e through the C ABI with host buffers ----
     e2e = e2e_measure(P, torch, dist, w, cpu, step0, algo, dev, max(1, args.e2e_steps))
+    head_copies = lanes.n_copies
     del lanes
 
     # ---- the video GQA workload (one sample per batch): as stated, and as
@@ -846,7 +847,7 @@ def run_gb300(args, dist):
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": dist.world, "steps": K,
             "warmup": args.warmup, "ms_per_step": 1e3 * max_sec / K, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
-            "config": dict(workload_config(w, algo_name, lanes.n_copies, input_mb), streams=S,
+            "config": dict(workload_config(w, algo_name, head_copies, input_mb), streams=S,
                            **({"concurrency": f"{S} streams of independent batches run concurrently (each with its "
                                               f"own inputs, outputs and workspace); value counts the samples of all "
                                               f"streams; single_stream is one stream"} if S > 1 else {})),
@@ -950,65 +951,103 @@ def kernels_per_step(w, algo_name):
 
 def e2e_measure(P, torch, dist, w, cpu, step0, algo, dev, E):
     """e2e through the C ABI with the batch in pinned host memory. Every step
-    copies to the device what the tensor-core head scores read (each sample's
-    text rows of Q, all of K) and the lengths; the pruning call then reads
-    hidden, V and the position ids where they are, in host memory, and writes
-    the compacted hidden, K, V and position ids straight into pinned host
-    outputs (PROVIP_PRUNE_HOST_ROWS: only the kept rows cross the host link);
-    the kept indices and output lengths are copied back. The bytes declared are
-    the copies plus the kept rows the kernel reads from host memory (in) and
-    the rows it writes there (out). Two device buffer sets alternate so that
-    one step's copies overlap the other's pruning (a stream per copy direction
-    and one for the kernels, ordered by events). Three timed runs of E steps,
-    the median reported with the three beside it (the host link is shared with
-    other jobs)."""
+    copies to the device what the tensor-core head scores read through tensor
+    maps: each sample's text rows of Q and, with one 2-D copy per key/value head
+    the selected query heads use, that head's key columns of every row; and the
+    lengths. provip_head_topk selects on the device, then provip_compact reads
+    the kept rows of hidden, K, V and the position ids where they are, in host
+    memory (the library detects it: only the surviving rows cross the host
+    link), and writes the compacted rows into device buffers, the input of the
+    layers after the pruning; the kept indices and output lengths are copied
+    back. The bytes declared are the copies plus the rows the compaction reads
+    from host memory (in) and the indices and lengths (out). Two buffer sets
+    alternate so that one step's copies overlap the other's kernels (a stream
+    per copy direction and one for the kernels, ordered by events). Three timed
+    runs of E steps, the median reported with the three beside it (the host link
+    is shared with other jobs)."""
+    import ctypes
     import numpy as np
+    cudart = ctypes.CDLL("libcudart.so.13")
+    memcpy2d = cudart.cudaMemcpy2DAsync
+    memcpy2d.argtypes = [ctypes.c_void_p, ctypes.c_size_t, ctypes.c_void_p, ctypes.c_size_t, ctypes.c_size_t,
+                         ctypes.c_size_t, ctypes.c_int, ctypes.c_void_p]
+    memcpy2d.restype = ctypes.c_int
+    H2D = 1  # cudaMemcpyHostToDevice
+    L = P.lib()
     nv, keep, vis = cpu["N_v"], cpu["keep"], cpu["vis_start"]
+    B, Lm, Hq, dh = cpu["Q"].shape
+    Hkv, D, Pn = cpu["K"].shape[2], cpu["hidden"].shape[2], cpu["pos"].shape[0]
+    heads, hs = P._heads_arg(cpu["head_list"], Hq)
+    kv_used = sorted({int(h) // (Hq // Hkv) for h in cpu["head_list"].tolist()})
     pin = {k: v.pin_memory() for k, v in cpu.items() if isinstance(v, torch.Tensor)}
     ts, tl = cpu["text_start"].numpy(), cpu["text_len"].numpy()
     seq = cpu["seq_len"].numpy().astype(np.int64)
+    L_out = Lm - nv + keep
+    es = pin["Q"].element_size()
+    dt = P._dtype_code(pin["Q"])
+    ws_bytes = L.provip_head_scores_workspace_size(B, Lm, hs, w.n_t[1], nv, algo, dt)
     sets = []
     for j in range(2):
-        db = {k: torch.empty_like(pin[k], device=dev) for k in ("Q", "K", "text_start", "text_len", "seq_len")}
-        st_j = P.PruneStep(db["Q"], db["K"], pin["V"], pin["hidden"], pin["pos"], cpu["head_list"], w.n_t[1], nv,
-                           keep, algo=algo, want_scores=False, flags=P.PRUNE_OVERLAP_PREVIOUS, host_rows=True)
-        ho = {"idx": torch.empty(st_j.idx.shape, dtype=torch.int32, pin_memory=True),
-              "seq_len": torch.empty(st_j.seq_len_out.shape, dtype=torch.int32, pin_memory=True)}
+        db = {k: torch.zeros_like(pin[k], device=dev) for k in ("Q", "K", "text_start", "text_len", "seq_len")}
+        outs = {"idx": torch.empty((B, keep), dtype=torch.int32, device=dev),
+                "hidden": torch.empty((B, L_out, D), dtype=pin["hidden"].dtype, device=dev),
+                "K": torch.empty((B, L_out, Hkv, dh), dtype=pin["K"].dtype, device=dev),
+                "V": torch.empty((B, L_out, Hkv, dh), dtype=pin["V"].dtype, device=dev),
+                "pos": torch.empty((Pn, B, L_out), dtype=torch.int32, device=dev),
+                "seq_len": torch.empty(B, dtype=torch.int32, device=dev)}
+        ws = P.workspace(ws_bytes, dev)
+        ho = {"idx": torch.empty((B, keep), dtype=torch.int32, pin_memory=True),
+              "seq_len": torch.empty(B, dtype=torch.int32, pin_memory=True)}
         ev = {n: torch.cuda.Event() for n in ("h2d", "comp", "d2h")}
-        sets.append((db, st_j, ho, ev))
-    es = pin["Q"].element_size()
-    q_rows = int(tl.sum()) * w.H_q * 128 * es
+        sets.append((db, outs, ws, ho, ev))
+    q_rows = int(tl.sum()) * Hq * dh * es
+    k_cols = len(kv_used) * B * Lm * dh * es
     small = sum(pin[k].numel() * 4 for k in ("text_start", "text_len", "seq_len"))
     out_rows = seq - nv + keep
-    row_in = (w.D + w.H_kv * 128) * es + w.P * 4  # hidden + V rows and position ids read in place
-    row_out = (w.D + 2 * w.H_kv * 128) * es + w.P * 4  # hidden, K, V rows and position ids written
-    h2d = q_rows + pin["K"].numel() * es + small + int((out_rows * row_in).sum())
-    d2h = int((out_rows * row_out).sum()) + sets[0][2]["idx"].numel() * 4 + sets[0][2]["seq_len"].numel() * 4
+    row_in = (D + 2 * Hkv * dh) * es + Pn * 4  # hidden, K and V rows and position ids read in place
+    h2d = q_rows + k_cols + small + int((out_rows * row_in).sum())
+    d2h = sets[0][3]["idx"].numel() * 4 + sets[0][3]["seq_len"].numel() * 4
     s_comp, s_d2h, s_h2d = (torch.cuda.Stream(device=dev) for _ in range(3))
     fresh = [True, True]
+    kp, kpitch, kw = pin["K"].data_ptr(), Hkv * dh * es, dh * es
 
     def one(n):
         j = n % 2
-        db, st_j, ho, ev = sets[j]
+        db, outs, ws, ho, ev = sets[j]
         with torch.cuda.stream(s_h2d):
             if not fresh[j]:
                 s_h2d.wait_event(ev["comp"])  # the set's device inputs were consumed by step n - 2
-            for b in range(w.B):
+            for b in range(B):
                 db["Q"][b, ts[b]:ts[b] + tl[b]].copy_(pin["Q"][b, ts[b]:ts[b] + tl[b]], non_blocking=True)
-            for k in ("K", "text_start", "text_len", "seq_len"):
+            for g in kv_used:
+                rc = memcpy2d(db["K"].data_ptr() + g * kw, kpitch, kp + g * kw, kpitch, kw, B * Lm, H2D,
+                              s_h2d.cuda_stream)
+                if rc != 0:
+                    raise RuntimeError(f"cudaMemcpy2DAsync returned {rc}")
+            for k in ("text_start", "text_len", "seq_len"):
                 db[k].copy_(pin[k], non_blocking=True)
             ev["h2d"].record(s_h2d)
         with torch.cuda.stream(s_comp):
             s_comp.wait_event(ev["h2d"])
             if not fresh[j]:
                 s_comp.wait_event(ev["d2h"])  # step n - 2's indices have left this set
-            r = st_j(db["Q"], db["K"], pin["V"], pin["hidden"], pin["pos"], db["text_start"], db["text_len"],
-                     db["seq_len"], vis, stream=s_comp)
+            st = ctypes.c_void_p(s_comp.cuda_stream)
+            rc = L.provip_head_topk(P._ptr(db["Q"]), P._ptr(db["K"]), B, Lm, Hq, Hkv, dh, heads, hs,
+                                    P._i32(db["text_start"]), P._i32(db["text_len"]), None, w.n_t[1], vis, nv,
+                                    P._i32(db["seq_len"]), keep, dt, algo, P._ptr(outs["idx"]), None,
+                                    P._ptr(ws), ws.numel(), st)
+            P._check(rc, "provip_head_topk")
+            rc = L.provip_compact(P._ptr(outs["idx"]), B, nv, keep, P._ptr_host_ok(pin["hidden"]), D,
+                                  P._ptr_host_ok(pin["K"]), P._ptr_host_ok(pin["V"]), Hkv, dh,
+                                  P._i32_host_ok(pin["pos"]), Pn, P._i32(db["seq_len"]), Lm, vis, dt,
+                                  P._ptr(outs["hidden"]), P._ptr(outs["K"]), P._ptr(outs["V"]),
+                                  P._i32(outs["pos"]), P._i32(outs["seq_len"]), st)
+            P._check(rc, "provip_compact")
             ev["comp"].record(s_comp)
         with torch.cuda.stream(s_d2h):
             s_d2h.wait_event(ev["comp"])
-            ho["idx"].copy_(r["idx"], non_blocking=True)
-            ho["seq_len"].copy_(r["seq_len"], non_blocking=True)
+            ho["idx"].copy_(outs["idx"], non_blocking=True)
+            ho["seq_len"].copy_(outs["seq_len"], non_blocking=True)
             ev["d2h"].record(s_d2h)
         fresh[j] = False
 
@@ -1027,6 +1066,18 @@ def e2e_measure(P, torch, dist, w, cpu, step0, algo, dev, E):
 
     run(0, 4)
     torch.cuda.synchronize()
+    # the e2e path's kept indices and rows are those of the device-resident step
+    ref = step0(*(lambda c: (c["Q"], c["K"], c["V"], c["hidden"], c["pos"], c["text_start"], c["text_len"],
+                             c["seq_len"], vis))({k: (v.to(dev) if isinstance(v, torch.Tensor) else v)
+                                                  for k, v in cpu.items()}))
+    torch.cuda.synchronize()
+    slo = ref["seq_len"].cpu()
+    same = torch.equal(sets[1][3]["idx"], ref["idx"].cpu()) and torch.equal(sets[1][3]["seq_len"], slo)
+    for k in ("hidden", "K", "V"):
+        for b_ in range(B):
+            same = same and torch.equal(sets[1][1][k][b_, :int(slo[b_])], ref[k][b_, :int(slo[b_])])
+    if not same:
+        raise RuntimeError("e2e path disagrees with the device-resident step")
     runs, first = [], 4
     for _ in range(3):
         a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -1039,8 +1090,9 @@ def e2e_measure(P, torch, dist, w, cpu, step0, algo, dev, E):
         runs.append(aggregate(dist.sum(float(w.B * E)), dist.max(a.elapsed_time(b) / 1e3)))
     return {"value": sorted(runs)[1], "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
             "runs": runs, "note": f"median of 3 timed runs of {E} steps; the batch stays in pinned host memory: "
-                                  f"Q text rows and K copied in, kept rows read and compacted rows written in "
-                                  f"place by the kernels (PROVIP_PRUNE_HOST_ROWS)"}
+                                  f"Q text rows and the used key heads copied in, kept rows read in place by the "
+                                  f"compaction, compacted rows left on the device, kept indices and lengths read "
+                                  f"back"}
 
 
 def run_prellm_only(args):

@@ -245,6 +245,12 @@ int provip_head_scores_noalloc(const void *Q, const void *K, int B, int L_max, i
  * carried, not renumbered. seq_len_out [B] (may be NULL) = seq_len - N_v + keep.
  * Output rows >= seq_len_out[b] are left untouched.
  *   idx [B, keep] int32 ascending in [0, N_v) (device).
+ * hidden, K, V, pos and the four outputs may each be device memory or host
+ * memory the device can dereference (pinned and mapped, cudaHostAlloc):
+ * host memory is detected (cudaPointerGetAttributes) and every row is then
+ * copied with 16-byte loads and stores from the GPU's threads instead of bulk
+ * copies, so that only the surviving rows cross the host link. Results are
+ * the same.
  * Row sizes (D and H_kv*d_h elements) must be multiples of 16 bytes and every
  * tensor pointer 16-byte aligned. */
 int provip_compact(const int *idx, int B, int N_v, int keep, const void *hidden, int D,

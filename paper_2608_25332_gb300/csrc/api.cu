@@ -7,6 +7,7 @@
 #include <string.h>
 
 #include <atomic>
+#include <initializer_list>
 #include <mutex>
 
 #include <nvtx3/nvToolsExt.h>
@@ -758,6 +759,23 @@ extern "C" int provip_head_scores(const void* Q, const void* K, int B, int L_max
   return e == cudaSuccess ? PROVIP_OK : cuda_fail(e, "head_scores reduce");
 }
 
+// true if any pointer is host memory (pinned and mapped, or memory the device
+// reaches through the system's address translation): the rows are then copied
+// with vector loads and stores, which work on any memory the device can
+// dereference, instead of bulk copies
+static bool any_host_memory(std::initializer_list<const void*> ptrs) {
+  for (const void* p : ptrs) {
+    if (p == nullptr) continue;
+    cudaPointerAttributes at;
+    if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+      cudaGetLastError();  // not known to the runtime: not device memory
+      return true;
+    }
+    if (at.type != cudaMemoryTypeDevice && at.type != cudaMemoryTypeManaged) return true;
+  }
+  return false;
+}
+
 extern "C" int provip_compact(const int* idx, int B, int N_v, int keep, const void* hidden, int D,
                               const void* K, const void* V, int H_kv, int d_h, const int* pos,
                               int P, const int* seq_len, int L_max, int vis_start, int dtype,
@@ -772,7 +790,8 @@ extern "C" int provip_compact(const int* idx, int B, int N_v, int keep, const vo
   CompactArgs a = compact_args(idx, B, N_v, keep, hidden, D, K, V, H_kv, d_h, pos, P, seq_len,
                                L_max, vis_start, dtype, hidden_out, K_out, V_out, pos_out,
                                seq_len_out, d->status);
-  cudaError_t e = compact_launch(a, d->sms, static_cast<cudaStream_t>(stream));
+  const bool host_rows = any_host_memory({hidden, K, V, pos, hidden_out, K_out, V_out, pos_out});
+  cudaError_t e = compact_launch(a, d->sms, static_cast<cudaStream_t>(stream), false, true, false, host_rows);
   return e == cudaSuccess ? PROVIP_OK : cuda_fail(e, "compact launch");
 }
 

@@ -321,16 +321,19 @@ def _outs(hidden, K, V, pos, B, L_out, device=None):
 
 
 def provip_compact(idx, hidden, K, V, pos, seq_len, vis_start, N_v, out=None):
+    """hidden, K, V, pos and the outputs may be device tensors or pinned host
+    tensors (the library detects host memory); idx and seq_len live on the
+    device, and the outputs default to device tensors."""
     B, Lm, D = hidden.shape
     keep = idx.shape[1]
     Hkv, dh = (K.shape[2], K.shape[3]) if K is not None else (0, 0)
     P = pos.shape[0] if pos is not None else 0
-    ho, ko, vo, po = out if out is not None else _outs(hidden, K, V, pos, B, Lm - N_v + keep)
-    slo = torch.empty(B, dtype=torch.int32, device=hidden.device)
-    rc = lib().provip_compact(_i32(idx), B, N_v, keep, _ptr(hidden), D, _ptr(K), _ptr(V), Hkv, dh,
-                              _i32(pos), P, _i32(seq_len), Lm, vis_start, _dtype_code(hidden),
-                              _ptr(ho), _ptr(ko), _ptr(vo), _i32(po), _i32(slo),
-                              _stream(hidden.device))
+    ho, ko, vo, po = out if out is not None else _outs(hidden, K, V, pos, B, Lm - N_v + keep, idx.device)
+    slo = torch.empty(B, dtype=torch.int32, device=idx.device)
+    rc = lib().provip_compact(_i32(idx), B, N_v, keep, _ptr_host_ok(hidden), D, _ptr_host_ok(K), _ptr_host_ok(V),
+                              Hkv, dh, _i32_host_ok(pos), P, _i32(seq_len), Lm, vis_start, _dtype_code(hidden),
+                              _ptr_host_ok(ho), _ptr_host_ok(ko), _ptr_host_ok(vo), _i32_host_ok(po), _i32(slo),
+                              _stream(idx.device))
     _check(rc, "provip_compact")
     return dict(hidden=ho, K=ko, V=vo, pos=po, seq_len=slo)
 

@@ -57,3 +57,37 @@ def test_host_rows_match_device_rows(name, batch, flags):
     for b in range(slo.shape[0]):
         n = int(slo[b])
         assert torch.equal(got["pos"][:, b, :n], ref["pos"][:, b, :n].cpu())
+
+
+@pytest.mark.parametrize("name,batch", [("llava_next_7b_bf16_b8", 2), ("video_gqa_bf16_b1", None),
+                                        ("llava15_7b_bf16_b16", 5)])
+@pytest.mark.parametrize("outputs", ["device", "host"])
+def test_compact_detects_host_memory(name, batch, outputs):
+    """provip_compact with hidden, K, V and the position ids in pinned host
+    memory (detected by the library), writing device or host outputs, gives the
+    bytes of the all-device call."""
+    w = synth.BY_NAME[name]
+    cpu = synth.in_llm_inputs(w, batch=batch)
+    g = {k: (v.to(DEV) if isinstance(v, torch.Tensor) else v) for k, v in cpu.items()}
+    st = P.PruneStep(g["Q"], g["K"], g["V"], g["hidden"], g["pos"], cpu["head_list"], w.n_t[1], g["N_v"],
+                     g["keep"], want_scores=False)
+    idx = st(g["Q"], g["K"], g["V"], g["hidden"], g["pos"], g["text_start"], g["text_len"], g["seq_len"],
+             g["vis_start"])["idx"].clone()
+    ref = P.provip_compact(idx, g["hidden"], g["K"], g["V"], g["pos"], g["seq_len"], g["vis_start"], g["N_v"])
+    hst = {k: cpu[k].pin_memory() for k in ("hidden", "K", "V", "pos")}
+    out = None
+    if outputs == "host":
+        out = tuple(torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
+                    for t in (ref["hidden"], ref["K"], ref["V"], ref["pos"]))
+    got = P.provip_compact(idx, hst["hidden"], hst["K"], hst["V"], hst["pos"], g["seq_len"], g["vis_start"],
+                           g["N_v"], out=out)
+    torch.cuda.synchronize()
+    assert torch.equal(got["seq_len"], ref["seq_len"])
+    slo = ref["seq_len"].cpu()
+    for k in ("hidden", "K", "V"):
+        for b in range(slo.shape[0]):
+            n = int(slo[b])
+            assert torch.equal(got[k][b, :n].cpu().view(torch.int16), ref[k][b, :n].cpu().view(torch.int16)), (k, b)
+    for b in range(slo.shape[0]):
+        n = int(slo[b])
+        assert torch.equal(got["pos"][:, b, :n].cpu(), ref["pos"][:, b, :n].cpu())
