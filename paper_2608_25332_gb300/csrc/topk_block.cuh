@@ -10,8 +10,8 @@
 // builds a shared histogram of the digits, and one warp finds the bin that
 // holds the k-th largest key; the range becomes that bin's keys. A range of
 // one key value ends the search, and so does a bin of at most kSmallCand keys:
-// they are gathered and one warp ranks them exactly by (key, lower index
-// first). Spread-out keys take one pass; a 32-bit range needs at most three.
+// they are gathered and ranked exactly by (key, lower index first), a warp per
+// 32 of them. Spread-out keys take one pass; a 32-bit range needs at most three.
 // The threshold key T and how many keys equal to T are taken (need_eq) then
 // give every selected element its output slot, #(greater before i) +
 // min(#(equal before i), need_eq), from counts of (greater, equal) in index
@@ -24,7 +24,7 @@
 namespace provip {
 
 constexpr int kSelectBins = 2048;  // one 11-bit digit
-constexpr int kSmallCand = 32;
+constexpr int kSmallCand = 128;  // at most a warp per 32 candidates: blocks of >= 128 threads
 
 struct TopkShared {
   __align__(16) int hist[2][kSelectBins];  // double-buffered: the next pass's is cleared during this one
@@ -32,6 +32,8 @@ struct TopkShared {
   uint32_t wcnt[32];         // packed (greater << 16 | equal) counts per warp
   int sel, above, cnt;       // chosen bin, keys above it in the range, keys in it
   int ncand;
+  uint32_t rkey;             // the candidates' threshold key and the equal keys taken
+  int rneed;
   __align__(16) uint32_t ckey[kSmallCand];
   __align__(16) int cidx[kSmallCand];
 };
@@ -118,28 +120,45 @@ __device__ __forceinline__ void topk_block_find_bin(const int* hist, int rem, To
 
 // Exact rank of the rem-th largest of the nc <= kSmallCand candidates (key,
 // index) in shared memory: the threshold key T and how many keys equal to T
-// are taken. Lane l ranks candidate l against all of them, read with 16-byte
-// broadcast loads; every warp that calls it gets the same answer.
-__device__ __forceinline__ void topk_warp_rank(const TopkShared& sh, int nc, int rem, uint32_t& T,
-                                               int& need_eq) {
-  const int lane = threadIdx.x & 31;
-  const uint32_t ku = lane < nc ? sh.ckey[lane] : 0u;
-  const int ki = lane < nc ? sh.cidx[lane] : 0x7fffffff;
-  int rank = 0;
+// are taken. Warp w ranks candidates 32w..32w+31 against all of them (16-byte
+// broadcast loads); the warp holding the candidate of rank rem - 1 (exactly one
+// has it, 1 <= rem <= nc) counts the candidates above its key and publishes
+// both. Called by every thread of a block of at least kSmallCand threads; one
+// barrier.
+__device__ __forceinline__ void topk_block_rank(TopkShared& sh, int nc, int rem, uint32_t& T,
+                                                int& need_eq) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  if (warp * 32 < nc) {  // warp-uniform
+    const int c = warp * 32 + lane;
+    const uint32_t ku = c < nc ? sh.ckey[c] : 0u;
+    const int ki = c < nc ? sh.cidx[c] : 0x7fffffff;
+    int rank = 0;
+    const int nq = (nc + 3) >> 2;
+    for (int q = 0; q < nq; ++q) {
+      const uint4 kv = reinterpret_cast<const uint4*>(sh.ckey)[q];
+      const int4 iv = reinterpret_cast<const int4*>(sh.cidx)[q];
+      // branch-free: (j < nc) & (key_j > key or (key_j == key and idx_j < idx))
+      rank += (int)((4 * q + 0 < nc) & ((kv.x > ku) | ((kv.x == ku) & (iv.x < ki))));
+      rank += (int)((4 * q + 1 < nc) & ((kv.y > ku) | ((kv.y == ku) & (iv.y < ki))));
+      rank += (int)((4 * q + 2 < nc) & ((kv.z > ku) | ((kv.z == ku) & (iv.z < ki))));
+      rank += (int)((4 * q + 3 < nc) & ((kv.w > ku) | ((kv.w == ku) & (iv.w < ki))));
+    }
+    const unsigned hit = __ballot_sync(0xffffffffu, c < nc && rank == rem - 1);
+    if (hit) {
+      const uint32_t t = __shfl_sync(0xffffffffu, ku, __ffs(hit) - 1);
+      int gt = 0;
+      for (int j = lane; j < nc; j += 32) gt += sh.ckey[j] > t ? 1 : 0;
 #pragma unroll
-  for (int q = 0; q < kSmallCand / 4; ++q) {
-    const uint4 kv = reinterpret_cast<const uint4*>(sh.ckey)[q];
-    const int4 iv = reinterpret_cast<const int4*>(sh.cidx)[q];
-    // branch-free: (j < nc) & (key_j > key or (key_j == key and idx_j < idx))
-    rank += (int)((4 * q + 0 < nc) & ((kv.x > ku) | ((kv.x == ku) & (iv.x < ki))));
-    rank += (int)((4 * q + 1 < nc) & ((kv.y > ku) | ((kv.y == ku) & (iv.y < ki))));
-    rank += (int)((4 * q + 2 < nc) & ((kv.z > ku) | ((kv.z == ku) & (iv.z < ki))));
-    rank += (int)((4 * q + 3 < nc) & ((kv.w > ku) | ((kv.w == ku) & (iv.w < ki))));
+      for (int o = 16; o > 0; o >>= 1) gt += __shfl_xor_sync(0xffffffffu, gt, o);
+      if (lane == 0) {
+        sh.rkey = t;
+        sh.rneed = rem - gt;
+      }
+    }
   }
-  const unsigned hit = __ballot_sync(0xffffffffu, lane < nc && rank == rem - 1);
-  T = __shfl_sync(0xffffffffu, ku, hit ? __ffs(hit) - 1 : 0);
-  const unsigned gt = __ballot_sync(0xffffffffu, lane < nc && ku > T);
-  need_eq = rem - __popc(gt);
+  __syncthreads();
+  T = sh.rkey;
+  need_eq = sh.rneed;
 }
 
 // Selects the k largest of keys[0..N) (shared memory) into out[0..k), given the
@@ -189,7 +208,7 @@ __device__ __forceinline__ void topk_block_select(const uint32_t* keys, int N, i
         }
       }
       __syncthreads();
-      topk_warp_rank(sh, min(sh.ncand, kSmallCand), rem, T, need_eq);
+      topk_block_rank(sh, min(sh.ncand, kSmallCand), rem, T, need_eq);
       break;
     }
   }
@@ -228,8 +247,7 @@ __device__ __forceinline__ void topk_block_select(const uint32_t* keys, int N, i
 
 // The select of topk_block_select on keys held in registers: thread t owns the
 // KPT keys of indices [t * KPT, t * KPT + KPT) (valid below N), so every
-// per-key loop is unrolled and its loads and atomics are in flight together;
-// every warp ranks the final candidates itself (no barrier after the rank).
+// per-key loop is unrolled and its loads and atomics are in flight together.
 // sh.hist[0] must be cleared and visible; lo/hi are the keys' min and max.
 template <int KPT>
 __device__ __forceinline__ void topk_block_select_reg(const uint32_t (&key)[KPT], int N, int k,
@@ -275,7 +293,7 @@ __device__ __forceinline__ void topk_block_select_reg(const uint32_t (&key)[KPT]
           }
         }
       __syncthreads();
-      topk_warp_rank(sh, min(sh.ncand, kSmallCand), rem, T, need_eq);
+      topk_block_rank(sh, min(sh.ncand, kSmallCand), rem, T, need_eq);
       break;
     }
   }
