@@ -96,6 +96,16 @@ const char *provip_last_error(void);
 /* Library version as 10000*major + 100*minor + patch. */
 int provip_version(void);
 
+/* Process-wide switches of the library's kernel choice (tests and measurement
+ * use them to reach every form); they apply to calls enqueued after the switch.
+ *   PROVIP_OPT_MERGE_PAIRS: 1 (default) lets the bf16 nearest-centroid Gram of
+ *   the merge (Sec. 4.3) run on pairs of SMs (tcgen05 cta_group::2, one M = 256
+ *   MMA over two CTAs) where two-CTA clusters fit; 0 keeps it on single SMs.
+ * Returns PROVIP_OK, or PROVIP_ERR_INVALID_ARG for an unknown option or a value
+ * outside {0, 1}. */
+#define PROVIP_OPT_MERGE_PAIRS 1
+int provip_set_option(int option, int value);
+
 /* Synchronises the current device, then returns the device status word of the
  * current device (PROVIP_DEVSTAT_* bits) in *bits and clears it when `clear`
  * is non-zero. Returns PROVIP_ERR_TIMEOUT if the TIMEOUT bit is set,

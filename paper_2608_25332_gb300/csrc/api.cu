@@ -440,6 +440,15 @@ extern "C" const char* provip_last_error(void) { return g_last_error; }
 
 extern "C" int provip_version(void) { return 10000; }
 
+extern "C" int provip_set_option(int option, int value) {
+  if (value != 0 && value != 1) return fail(PROVIP_ERR_INVALID_ARG, "set_option: value %d", value);
+  if (option == PROVIP_OPT_MERGE_PAIRS) {
+    merge_pair_enable(value);
+    return PROVIP_OK;
+  }
+  return fail(PROVIP_ERR_INVALID_ARG, "set_option: unknown option %d", option);
+}
+
 extern "C" int provip_device_status(unsigned* bits, int clear) {
   DevInfo* d;
   int rc = dev_info(&d);

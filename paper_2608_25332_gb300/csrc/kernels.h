@@ -208,12 +208,40 @@ cudaError_t relevance_tc_launch(const SimArgs& a, const uint8_t* mask, const flo
                                 cudaEvent_t mask_ready = nullptr);
 bool merge_tc_supported(const SimArgs& a, int keep, int n_split);
 // pruned: the rows not kept, ascending ([B][N_v - keep], from merge_index_kernel)
+// Writes the permuted copy perm, then runs the Gram on pairs of SMs when they
+// are usable (*n_split_out = its column ranges), else on single SMs with n_split
+// column splits (*n_split_out = n_split).
 cudaError_t merge_argmax_tc_launch(const SimArgs& a, const int* keep_idx, int keep,
                                    const float* inv_v, const int* pruned, void* perm,
-                                   int n_split, float* ws_best, int* ws_bidx, cudaStream_t s);
+                                   int n_split, float* ws_best, int* ws_bidx, int num_sms,
+                                   int* n_split_out, cudaStream_t s);
 // N split of the tcgen05 merge Gram (fewest waves x tiles per CTA) and its upper bound
 int merge_tc_split(int B, int N_v, int keep, int num_sms);
 constexpr int kMergeMaxSplit = 16;
+
+// the merge Gram on pairs of SMs (tcgen05 cta_group::2, merge_pair_tc.cu)
+constexpr int kMergePairHeights = 4;
+// A tile is (512-row group of one sample's pruned rows, range of its kept
+// columns); groups x_hi .. Q-1 split the columns into n_lo ranges, groups
+// 0 .. x_hi-1 into n_lo + 1.
+struct MergePairPlan {
+  int n_quads;  // 512-row groups of pruned rows per sample
+  int Q;        // groups of the batch: B * n_quads
+  int n_lo;     // column ranges of groups x_hi .. Q-1
+  int x_hi;     // groups with n_lo + 1 ranges
+  int T;        // tiles
+  int P;        // clusters of two CTAs (pairs of SMs), at most T
+  int n_slots;  // partial slots per row: n_lo + (x_hi > 0), <= kMergeMaxSplit
+  int n_heights;                     // distinct B rows per CTA (N / 2) of the tiles
+  int heights[kMergePairHeights];
+};
+bool merge_pair_plan(int B, int n_pruned, int keep, int D, int num_sms, MergePairPlan* p);
+// bf16, the pair form enabled, and a two-CTA cluster of it fits on this device
+bool merge_pair_usable(const SimArgs& a);
+void merge_pair_enable(int on);
+cudaError_t merge_argmax_pair_launch(const SimArgs& a, const int* keep_idx, int keep, const float* inv_v,
+                                     const int* pruned, const void* perm, const MergePairPlan& plan,
+                                     float* ws_best, int* ws_bidx, cudaStream_t s);
 
 // host helper: encode a 2-D bf16 row table [rows, cols] (row stride in bytes)
 // as a tensor map with 64 x box_rows boxes and 128-byte swizzle.

@@ -951,9 +951,8 @@ cudaError_t merge_launch(const SimArgs& a, const int* keep_idx, int keep, const 
   merge_index_kernel<<<a.B, 1024, 0, s>>>(keep_idx, keep, a.N_v, kpos, tc ? ws_pruned : nullptr, a.err);
   if (tc) {
     cudaError_t e = merge_argmax_tc_launch(a, keep_idx, keep, inv_v, ws_pruned, ws_perm, tc_split, ws_best,
-                                           ws_bidx, s);
+                                           ws_bidx, num_sms, &n_split, s);
     if (e != cudaSuccess) return e;
-    n_split = tc_split;
   } else {
     dim3 g((a.N_v + kSimtBM - 1) / kSimtBM, a.B, n_split);
     if (a.dtype == 0)

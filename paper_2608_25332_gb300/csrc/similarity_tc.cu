@@ -584,18 +584,29 @@ bool merge_tc_supported(const SimArgs& a, int keep, int n_split) {
 
 cudaError_t merge_argmax_tc_launch(const SimArgs& a, const int* keep_idx, int keep, const float* inv_v,
                                    const int* pruned, void* perm, int n_split,
-                                   float* ws_best, int* ws_bidx, cudaStream_t s) {
-  static std::atomic<bool> smem_set[64];  // per device, zero-initialised
-  int dev = 0;
-  cudaGetDevice(&dev);
-  const size_t smem = merge_tc_smem();
-  cudaError_t e = set_smem(merge_argmax_tc, smem, &smem_set[dev < 64 ? dev : 0]);
-  if (e != cudaSuccess) return e;
+                                   float* ws_best, int* ws_bidx, int num_sms, int* n_split_out,
+                                   cudaStream_t s) {
   const int n_pruned = a.N_v - keep;  // pruned: the rows not kept, ascending (merge_index_kernel)
+  MergePairPlan plan;
+  const bool pairs = merge_pair_usable(a) && merge_pair_plan(a.B, n_pruned, keep, a.D, num_sms, &plan);
+  cudaError_t e = cudaSuccess;
+  if (!pairs) {
+    static std::atomic<bool> smem_set[64];  // per device, zero-initialised
+    int dev = 0;
+    cudaGetDevice(&dev);
+    e = set_smem(merge_argmax_tc, merge_tc_smem(), &smem_set[dev < 64 ? dev : 0]);
+    if (e != cudaSuccess) return e;
+  }
   dim3 gg((a.N_v + 7) / 8, a.B);
   gather_perm_kernel<<<gg, 256, 0, s>>>(static_cast<const __nv_bfloat16*>(a.emb_v), pruned, keep_idx,
                                         n_pruned, keep, a.N_v, a.D, static_cast<__nv_bfloat16*>(perm),
                                         a.err);
+  if (pairs) {
+    *n_split_out = plan.n_slots;
+    return merge_argmax_pair_launch(a, keep_idx, keep, inv_v, pruned, perm, plan, ws_best, ws_bidx, s);
+  }
+  *n_split_out = n_split;
+  const size_t smem = merge_tc_smem();
   CUtensorMap mapE;
   if (make_tmap_bf16_2d(&mapE, perm, (uint64_t)a.B * a.N_v, (uint64_t)a.D, (uint64_t)a.D * 2, 128))
     return cudaErrorInvalidValue;

@@ -40,6 +40,7 @@ _SIGS = {
     "provip_status_string": (ctypes.c_char_p, [_I]),
     "provip_last_error": (ctypes.c_char_p, []),
     "provip_version": (_I, []),
+    "provip_set_option": (_I, [_I, _I]),
     "provip_device_status": (_I, [_P, _I]),
     "provip_selftest_wait_timeout": (_I, [_P]),
     "provip_crit_text_workspace_size": (_Z, [_I, _I, _I]),
@@ -190,6 +191,14 @@ def provip_selftest_wait_timeout(device="cuda:0"):
 
 def provip_version() -> int:
     return lib().provip_version()
+
+
+OPT_MERGE_PAIRS = 1
+
+
+def provip_set_option(option: int, value: int) -> None:
+    """Process-wide kernel-choice switch (PROVIP_OPT_*), for calls enqueued after it."""
+    _check(lib().provip_set_option(int(option), int(value)), "provip_set_option")
 
 
 # ---------------------------------------------------------------------------

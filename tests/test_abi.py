@@ -55,6 +55,13 @@ def test_status_strings_and_version(L):
     assert L.provip_version() >= 10000
 
 
+def test_set_option_validation(L):
+    assert L.provip_set_option(1, 0) == 0  # PROVIP_OPT_MERGE_PAIRS off ...
+    assert L.provip_set_option(1, 1) == 0  # ... and back to the default
+    assert L.provip_set_option(1, 2) == -1
+    assert L.provip_set_option(99, 1) == -1
+
+
 def _heads(*h):
     return (ctypes.c_int * len(h))(*h)
 

@@ -74,6 +74,35 @@ def test_similarity_reduce_random_shapes(seed):
     _check_reduce(ev, et, tl, keep_pre, dtype, f"seed {seed} {dtype} B={B} N_v={N_v} D={D} tl={tls} keep={keep_pre}")
 
 
+@pytest.mark.parametrize("pairs", [1, 0])
+@pytest.mark.parametrize("B,N_v,D,keep", [
+    (6, 1000, 256, 237),   # two 512-row groups, the second ending inside its first half
+    (2, 700, 136, 640),    # 60 pruned rows; ten 64-column ranges, a partial last K slice
+    (5, 513, 128, 1),      # one kept row; 512 pruned rows fill one group exactly
+    (3, 800, 64, 130),     # the second group's second half holds 32 rows
+    (40, 800, 64, 500),    # 120 tiles: two per pair of SMs, the accumulators reused
+])
+def test_merge_ragged_groups(B, N_v, D, keep, pairs):
+    """provip_merge (bf16) with random keep sets over ragged row groups and
+    column ranges, every sample against the oracle's merge, with the Gram on
+    pairs of SMs (pairs=1) and on single SMs (pairs=0)."""
+    rng = np.random.default_rng(7000 + N_v + keep)
+    ev, _, _ = _pre_case(7100 + N_v, B, N_v, D, (1,), "bf16")
+    keeps = np.stack([np.sort(rng.choice(N_v, keep, replace=False)) for _ in range(B)]).astype(np.int32)
+    P.provip_set_option(P.OPT_MERGE_PAIRS, pairs)
+    try:
+        assign, merged = P.provip_merge(ev.to(DEV), torch.from_numpy(keeps).to(DEV))
+        torch.cuda.synchronize()
+    finally:
+        P.provip_set_option(P.OPT_MERGE_PAIRS, 1)
+    Evn = ev.float().numpy().astype(np.float64)
+    for b in range(B):
+        a_ref, mg_ref = oracle.merge(Evn[b], keeps[b])
+        check_merge(Evn[b], keeps[b], assign[b].cpu().numpy(), merged[b].float().cpu().numpy().astype(np.float64),
+                    "bf16", f"merge B={B} N_v={N_v} D={D} keep={keep} pairs={pairs} [{b}]", a_ref,
+                    np.setdiff1d(np.arange(N_v), keeps[b]), mg_ref=mg_ref)
+
+
 def _check_reduce(ev, et, tl, keep_pre, dtype, what):
     B, N_v = ev.shape[0], ev.shape[1]
     rt = rtol_for(dtype)

@@ -159,16 +159,26 @@ def test_similarity_pass_matches_oracle(name):
     _pmap(lambda b: merge_check(b, False), parted)
 
 
-@pytest.mark.parametrize("name", [w.name for w in synth.WORKLOADS])
-def test_merge_matches_oracle(name):
+# bf16 merges run their Gram on pairs of SMs by default; pairs=0 holds the
+# single-SM form to the oracle as well
+MERGE_CASES = [(w.name, 1) for w in synth.WORKLOADS] + \
+    [(w.name, 0) for w in synth.WORKLOADS if w.dtype == "bf16"]
+
+
+@pytest.mark.parametrize("name,pairs", MERGE_CASES)
+def test_merge_matches_oracle(name, pairs):
     """provip_merge on the whole batch in one call, each sample with the
     oracle's own keep set (so every sample reaches the merge): the stand-alone
     merge path, with its own inverse norms."""
     w, cpu, g = inputs(name)
     fronts = _pmap(lambda b: _oracle_front(w, cpu, b), range(w.B))
     keeps = np.stack([f["keep"] for f in fronts])
-    assign, merged = P.provip_merge(g["emb_v"], torch.from_numpy(keeps).to(DEV))
-    torch.cuda.synchronize()
+    P.provip_set_option(P.OPT_MERGE_PAIRS, pairs)
+    try:
+        assign, merged = P.provip_merge(g["emb_v"], torch.from_numpy(keeps).to(DEV))
+        torch.cuda.synchronize()
+    finally:
+        P.provip_set_option(P.OPT_MERGE_PAIRS, 1)
     a_h = assign.cpu().numpy()
     mg_h = merged.float().cpu().numpy().astype(np.float64)
     exact = w.N_v <= EXACT_MERGE_MAX_NV
