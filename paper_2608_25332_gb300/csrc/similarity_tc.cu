@@ -15,6 +15,7 @@
 // crit_gram_tc: the text Gram E_t E_t^T, split over K.
 #include "common.cuh"
 #include "kernels.h"
+#include "merge_epi.cuh"
 #include "tc_gemm.cuh"
 
 namespace provip {
@@ -71,6 +72,8 @@ constexpr int kMergeStages = 3;
 constexpr int kMergeBBytes = kMergeBN * kBK * 2;                 // 32 KiB
 constexpr int kMergeStageBytes = 2 * kABytes + kMergeBBytes;     // A0 | A1 | B: 64 KiB
 constexpr uint32_t kMergeTmemCols = 2 * kMergeBN;                // one accumulator per M tile
+constexpr int kMergeEpiWarps = 8;  // two per TMEM lane quadrant, splitting each tile's columns
+constexpr int kMergeThreads = 64 + 32 * kMergeEpiWarps;
 
 struct MergePipe {
   uint64_t full[kMergeStages];
@@ -89,11 +92,13 @@ struct MergePipe {
 // between that tile's last MMA and the next tile's first (the producer keeps
 // loading meanwhile). The last N tile's MMA is only as wide as its kept rows
 // (rounded up to 16).
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(kMergeThreads, 1)
     merge_argmax_tc(const MergeTcArgs a, const __grid_constant__ CUtensorMap mapE) {
   extern __shared__ uint8_t smem_raw[];
   __shared__ MergePipe pipe;
   __shared__ int sidx_a[2 * kBM];
+  __shared__ float xbest[2][kBM];  // the upper column halves' (max, position) per row
+  __shared__ int xidx[2][kBM];
   const int b = blockIdx.z, split = blockIdx.y;
   const int m0 = blockIdx.x * 2 * kBM;
   const bool has1 = m0 + kBM < a.n_pruned;  // the second M tile holds pruned rows
@@ -116,7 +121,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&pipe.empty[s], 1);
     }
     mbar_init(&pipe.acc_full, 1);
-    mbar_init(&pipe.acc_empty, 4);  // one arrival per epilogue warp
+    mbar_init(&pipe.acc_empty, kMergeEpiWarps);  // one arrival per epilogue warp
     pipe.fail = 0;
     fence_mbar_init();
   }
@@ -195,8 +200,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int* pr = a.pruned + (size_t)b * a.n_pruned;
       const int* kp = a.keep_idx + (size_t)b * a.keep;
       const int et = threadIdx.x - 64;
-      for (int r = et; r < 2 * kBM; r += 128) sidx_a[r] = m0 + r < a.n_pruned ? pr[m0 + r] : 0;
-      for (int q = et; q < n_keep; q += 128) {
+      constexpr int kEpi = 32 * kMergeEpiWarps;
+      for (int r = et; r < 2 * kBM; r += kEpi) sidx_a[r] = m0 + r < a.n_pruned ? pr[m0 + r] : 0;
+      for (int q = et; q < n_keep; q += kEpi) {
         int j = kp[a0 + q];
         if (j < 0 || j >= a.N_v) {
           set_error(a.err, kErrBadDeviceArg);
@@ -204,51 +210,76 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         skinv[q] = a.inv_v[(size_t)b * a.N_v + j];
       }
-      asm volatile("bar.sync 1, 128;" ::: "memory");  // tables complete (epilogue warps)
-      // epilogue: row r of each M tile, running (max, first index) over the range
+      asm volatile("bar.sync 1, %0;" ::"n"(kEpi) : "memory");  // tables complete (epilogue warps)
+      // epilogue: row r of each M tile; the two warps of a lane quadrant take
+      // the lower and the upper half of each tile's 32-column pieces (their
+      // tensor-memory loads double-buffered), each keeping a running (max,
+      // first position) over the range, merged at the end
       const int quad = warp & 3;
+      const int half = (warp - 2) / 4;
       const int r = quad * 32 + lane;
-      float best0 = -INFINITY, best1 = -INFINITY;
-      int bidx0 = 0x7fffffff, bidx1 = 0x7fffffff;
+      RowBest r0, r1;
+      r0.init();
+      r1.init();
       bool ok = true;
       for (int t = 0; t < n_tiles; ++t) {
         ok = warp_mbar_wait(&pipe.acc_full, (uint32_t)t & 1u, a.err) && !pipe.fail;
         if (!ok) break;
         tc_fence_after();
         const uint32_t taddr = pipe.tmem + ((uint32_t)(quad * 32) << 16);
-        const int ncb = (tile_cols(t) + 31) / 32;
+        const int ncb = (tile_cols(t) + 31) / 32, mid = (ncb + 1) / 2;
+        const int cb0 = half ? mid : 0, cb1 = half ? ncb : mid;
+        const int sh = has1 ? 1 : 0;
+        const int npc = (cb1 - cb0) << sh;
+        auto piece = [&](int j, float* v) {
+          tmem_ld32(taddr + (uint32_t)((j & sh) * kMergeBN + (cb0 + (j >> sh)) * 32), v);
+        };
+        auto reduce = [&](int j, const float* v) {
+          const int q0 = t * kMergeBN + (cb0 + (j >> sh)) * 32;  // position within the range
+          if (j & sh)
+            r1.add32(v, skinv + q0, q0, n_keep, a0);
+          else
+            r0.add32(v, skinv + q0, q0, n_keep, a0);
+        };
+        float va[32], vb[32];
+        if (npc > 0) piece(0, va);
 #pragma unroll 1
-        for (int cb = 0; cb < ncb; ++cb) {
-          float v0[32], v1[32];
-          tmem_ld32(taddr + cb * 32, v0);
-          if (has1) tmem_ld32(taddr + kMergeBN + cb * 32, v1);
-          tc_wait_ld();
-          const int q0 = t * kMergeBN + cb * 32;  // position within the range
-#pragma unroll
-          for (int i = 0; i < 32; ++i) {
-            const int q = q0 + i;
-            if (q < n_keep) {
-              const float sk = skinv[q];
-              const float x0 = v0[i] * sk;
-              if (x0 > best0) {
-                best0 = x0;
-                bidx0 = a0 + q;
-              }
-              if (has1) {
-                const float x1 = v1[i] * sk;
-                if (x1 > best1) {
-                  best1 = x1;
-                  bidx1 = a0 + q;
-                }
-              }
-            }
+        for (int j = 0; j < npc; j += 2) {
+          tc_wait_ld_into(va);
+          if (j + 1 < npc) piece(j + 1, vb);
+          reduce(j, va);
+          if (j + 1 < npc) {
+            tc_wait_ld_into(vb);
+            if (j + 2 < npc) piece(j + 2, va);
+            reduce(j + 1, vb);
           }
         }
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&pipe.acc_empty);
       }
-      if (ok && !pipe.fail) {
+      float best0, best1;
+      int bidx0, bidx1;
+      r0.result(best0, bidx0);
+      r1.result(best1, bidx1);
+      if (half) {
+        xbest[0][r] = best0;
+        xidx[0][r] = bidx0;
+        xbest[1][r] = best1;
+        xidx[1][r] = bidx1;
+      }
+      asm volatile("bar.sync 1, %0;" ::"n"(kEpi) : "memory");  // the upper halves' results
+      if (!half) {
+        if (merge_better(xbest[0][r], xidx[0][r], best0, bidx0)) {
+          best0 = xbest[0][r];
+          bidx0 = xidx[0][r];
+        }
+        if (merge_better(xbest[1][r], xidx[1][r], best1, bidx1)) {
+          best1 = xbest[1][r];
+          bidx1 = xidx[1][r];
+        }
+      }
+      if (!half && ok && !pipe.fail) {
         const size_t o = ((size_t)split * a.B + b) * a.N_v;
         if (m0 + r < a.n_pruned) {
           a.ws_best[o + sidx_a[r]] = best0;
@@ -624,7 +655,7 @@ cudaError_t merge_argmax_tc_launch(const SimArgs& a, const int* keep_idx, int ke
   m.ws_bidx = ws_bidx;
   m.err = a.err;
   dim3 grid((n_pruned + 2 * kBM - 1) / (2 * kBM), n_split, a.B);
-  merge_argmax_tc<<<grid, kThreads, smem, s>>>(m, mapE);
+  merge_argmax_tc<<<grid, kMergeThreads, smem, s>>>(m, mapE);
   return cudaGetLastError();
 }
 
