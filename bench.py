@@ -227,8 +227,9 @@ def prellm_measure(w, dev, reps=20):
                    "note": "the whole pass (text Gram, relevance, top-k, gather, merge Gram, "
                            "assignment, means) against the sustained tensor peak"},
             "assign_us": us_assign, "assign_gram_flops": flops,
-            "tensor_roofline": {"bound": "tensor", "kernel": "merge_argmax_tc (timed with its gather, "
-                                "norm and assignment kernels)", "achieved": ach, "peak": peak,
+            "tensor_roofline": {"bound": "tensor", "kernel": "merge_argmax_pair_tc (bf16 merge Gram on "
+                                "pairs of SMs; timed with its gather, norm and assignment kernels)",
+                                "achieved": ach, "peak": peak,
                                 "peak_source": src, "unit": "TFLOP/s", "frac": ach / peak}}
 
 
