@@ -42,6 +42,7 @@
 
 #include <math.h>
 
+#include <mutex>
 #include <vector>
 
 namespace provip {
@@ -484,7 +485,7 @@ void merge_pair_enable(int on) { g_pair_enabled.store(on ? 1 : 0); }
 // ring's pace: a stage's loads take about 2700 clocks from issue to landing,
 // and four stages fit in shared memory), plus 9000 clocks of epilogue and
 // refill per tile.
-bool merge_pair_plan(int B, int n_pruned, int keep, int D, int num_sms, MergePairPlan* p) {
+static bool merge_pair_search(int B, int n_pruned, int keep, int D, int num_sms, MergePairPlan* p) {
   if (B < 1 || n_pruned < 1 || keep < 1 || D < 1 || num_sms < 2) return false;
   const int n_quads = (n_pruned + kPairQuadRows - 1) / kPairQuadRows;
   const long long Q = (long long)B * n_quads;
@@ -541,6 +542,43 @@ bool merge_pair_plan(int B, int n_pruned, int keep, int D, int num_sms, MergePai
     }
   }
   return best >= 0;
+}
+
+// The search simulates every candidate's deal (tens to hundreds of
+// microseconds of host time): its results are kept per shape, the last
+// kPlanCache shapes, for the calls that follow.
+namespace {
+constexpr int kPlanCache = 16;
+struct PlanEntry {
+  int B, n_pruned, keep, D, num_sms;
+  bool ok;
+  MergePairPlan plan;
+};
+std::mutex g_plan_mu;
+PlanEntry g_plans[kPlanCache];
+int g_plan_n = 0, g_plan_next = 0;
+}  // namespace
+
+bool merge_pair_plan(int B, int n_pruned, int keep, int D, int num_sms, MergePairPlan* p) {
+  {
+    std::lock_guard<std::mutex> lock(g_plan_mu);
+    for (int i = 0; i < g_plan_n; ++i) {
+      const PlanEntry& e = g_plans[i];
+      if (e.B == B && e.n_pruned == n_pruned && e.keep == keep && e.D == D && e.num_sms == num_sms) {
+        if (e.ok) *p = e.plan;
+        return e.ok;
+      }
+    }
+  }
+  MergePairPlan plan;
+  const bool ok = merge_pair_search(B, n_pruned, keep, D, num_sms, &plan);
+  std::lock_guard<std::mutex> lock(g_plan_mu);
+  PlanEntry& e = g_plans[g_plan_next];
+  e = PlanEntry{B, n_pruned, keep, D, num_sms, ok, plan};
+  g_plan_next = (g_plan_next + 1) % kPlanCache;
+  if (g_plan_n < kPlanCache) ++g_plan_n;
+  if (ok) *p = plan;
+  return ok;
 }
 
 bool merge_pair_usable(const SimArgs& a) {
