@@ -81,6 +81,7 @@ def test_similarity_reduce_random_shapes(seed):
     (5, 513, 128, 1),      # one kept row; 512 pruned rows fill one group exactly
     (3, 800, 64, 130),     # the second group's second half holds 32 rows
     (40, 800, 64, 500),    # 120 tiles: two per pair of SMs, the accumulators reused
+    (1, 4500, 64, 4200),   # more kept rows than 16 ranges of 256: the single-SM form either way
 ])
 def test_merge_ragged_groups(B, N_v, D, keep, pairs):
     """provip_merge (bf16) with random keep sets over ragged row groups and
