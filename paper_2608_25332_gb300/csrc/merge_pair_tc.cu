@@ -589,8 +589,9 @@ bool merge_pair_usable(const SimArgs& a) {
   if (st == 0) {
     st = 2;
     const size_t smem = pair_smem();
-    if (cudaFuncSetAttribute(merge_argmax_pair_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) ==
-        cudaSuccess) {
+    cudaError_t e = cudaFuncSetAttribute(merge_argmax_pair_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)smem);
+    if (e == cudaSuccess) {
       cudaLaunchConfig_t cfg = {};
       cudaLaunchAttribute attr[1];
       attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -603,9 +604,12 @@ bool merge_pair_usable(const SimArgs& a) {
       cfg.attrs = attr;
       cfg.numAttrs = 1;
       int n = 0;
-      if (cudaOccupancyMaxActiveClusters(&n, merge_argmax_pair_tc, &cfg) == cudaSuccess && n > 0) st = 1;
+      e = cudaOccupancyMaxActiveClusters(&n, merge_argmax_pair_tc, &cfg);
+      if (e == cudaSuccess && n > 0) st = 1;
     }
-    cudaGetLastError();  // a refused attribute or query leaves no sticky error
+    // a refused attribute or query falls back to the single-SM form: clear the
+    // error it left (only then, so that no earlier error of the caller is lost)
+    if (e != cudaSuccess) cudaGetLastError();
     g_pair_ok[dev].store(st, std::memory_order_release);
   }
   return st == 1;
