@@ -715,13 +715,18 @@ extern "C" int provip_similarity_reduce(const void* emb_v, int B, int N_v, int D
     t.k = keep_pre;
     t.idx_out = idx_out;
     t.err = d->status;
+    if (merged_out_or_null && topk_writes_index(N_v)) {
+      // the selection also writes the merge's kept-position map and pruned list
+      t.kpos_out = assign_out_or_null ? assign_out_or_null : w.assign;
+      t.pruned_out = w.pruned;
+    }
     e = topk_launch(t, s);
   }
   if (e == cudaSuccess && merged_out_or_null)
     e = merge_launch(a, idx_out, keep_pre, w.inv_v, assign_out_or_null ? assign_out_or_null : w.assign,
                      merged_out_or_null, w.best, w.bidx,
                      merge_splits(B, N_v, keep_pre), w.pruned,
-                     dtype == PROVIP_BF16 ? w.perm : nullptr, d->sms, s);
+                     dtype == PROVIP_BF16 ? w.perm : nullptr, d->sms, s, topk_writes_index(N_v));
   return e == cudaSuccess ? PROVIP_OK : cuda_fail(e, "similarity_reduce launch");
 }
 

@@ -119,12 +119,20 @@ struct TopkArgs {
   float* scores_out;         // optional [B][N]
   int B, N, k;
   int* idx_out;              // [B][k]
+  // optional (N above the rank kernel's range, see topk_writes_index): the
+  // merge's index, kpos_out [B][N] (the output slot of a selected element,
+  // else -1) and pruned_out [B][N - k] (the others, ascending)
+  int* kpos_out;
+  int* pruned_out;
   unsigned* err;
 };
 constexpr int kTopkMaxN = 49152;
 // pdl: launched as a programmatic dependent of the previous kernel on the
 // stream (the kernel waits for it before reading its inputs)
 cudaError_t topk_launch(const TopkArgs& a, cudaStream_t s, bool pdl = false);
+// whether topk_launch fills kpos_out / pruned_out for N keys (the block
+// selects do; the cluster rank kernel for small N does not)
+bool topk_writes_index(int N);
 
 // ---------------------------------------------------------------------------
 // compaction: rows [0, vis_start) ++ vis_start + idx ++ [vis_start + N_v, seq_len)
@@ -187,9 +195,12 @@ cudaError_t relevance_launch(const SimArgs& a, const uint8_t* mask, float* inv_v
 // n_split: the SIMT split (sized by the caller); ws_pruned: [B][N_v] ints and
 // ws_perm: [B][N_v][D] bf16 for the tcgen05 path (null: CUDA-core path);
 // num_sms for its split choice
+// index_ready: the kept-position map (in assign) and the pruned list (in
+// ws_pruned) were written by the top-k that chose keep_idx (topk_writes_index)
 cudaError_t merge_launch(const SimArgs& a, const int* keep_idx, int keep, const float* inv_v,
                          int* assign, void* merged, float* ws_best, int* ws_bidx,
-                         int n_split, int* ws_pruned, void* ws_perm, int num_sms, cudaStream_t s);
+                         int n_split, int* ws_pruned, void* ws_perm, int num_sms, cudaStream_t s,
+                         bool index_ready = false);
 
 // tcgen05 forms of the pre-LLM Grams (bf16), used by the launchers above
 bool crit_gram_tc_supported(const SimArgs& a);

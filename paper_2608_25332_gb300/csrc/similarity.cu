@@ -940,7 +940,7 @@ cudaError_t relevance_launch(const SimArgs& a, const uint8_t* mask, float* inv_v
 
 cudaError_t merge_launch(const SimArgs& a, const int* keep_idx, int keep, const float* inv_v,
                          int* assign, void* merged, float* ws_best, int* ws_bidx, int n_split,
-                         int* ws_pruned, void* ws_perm, int num_sms, cudaStream_t s) {
+                         int* ws_pruned, void* ws_perm, int num_sms, cudaStream_t s, bool index_ready) {
   // kpos lives in `assign` until the final assignment overwrites it: it is
   // read by merge_argmax_kernel and merge_assign_kernel (same index only).
   int* kpos = assign;
@@ -948,7 +948,8 @@ cudaError_t merge_launch(const SimArgs& a, const int* keep_idx, int keep, const 
   const int tc_split = merge_tc_split(a.B, a.N_v, keep, num_sms);
   const bool tc = ws_pruned != nullptr && ws_perm != nullptr && merge_tc_supported(a, keep, tc_split);
   // the kept-position map, and the pruned rows for the tensor-core Gram
-  merge_index_kernel<<<a.B, 1024, 0, s>>>(keep_idx, keep, a.N_v, kpos, tc ? ws_pruned : nullptr, a.err);
+  if (!index_ready)
+    merge_index_kernel<<<a.B, 1024, 0, s>>>(keep_idx, keep, a.N_v, kpos, tc ? ws_pruned : nullptr, a.err);
   if (tc) {
     cudaError_t e = merge_argmax_tc_launch(a, keep_idx, keep, inv_v, ws_pruned, ws_perm, tc_split, ws_best,
                                            ws_bidx, num_sms, &n_split, s);

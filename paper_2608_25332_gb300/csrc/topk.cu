@@ -63,7 +63,9 @@ __global__ void __launch_bounds__(kTopkMaxThreads) topk_kernel(const TopkArgs a)
   // through it the next call's head scores, which rewrite the partials) may
   // start. idx is only read by the compaction after this grid completes.
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-  topk_block_select(keys, a.N, a.k, lo, hi, a.idx_out + (size_t)b * a.k, sh);
+  topk_block_select(keys, a.N, a.k, lo, hi, a.idx_out + (size_t)b * a.k, sh,
+                    a.kpos_out ? a.kpos_out + (size_t)b * a.N : nullptr,
+                    a.kpos_out ? a.pruned_out + (size_t)b * (a.N - a.k) : nullptr);
 }
 
 // Up to 16384 keys: they stay in registers, 4 to 32 per thread (at most 512
@@ -84,7 +86,9 @@ __global__ void __launch_bounds__(kRegMaxThreads) topk_reg_kernel(const TopkArgs
   // the scores are consumed: the next kernel may start (it waits for this
   // grid's completion before reading idx)
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-  topk_block_select_reg<KPT>(key, a.N, a.k, lo, hi, a.idx_out + (size_t)b * a.k, sh);
+  topk_block_select_reg<KPT>(key, a.N, a.k, lo, hi, a.idx_out + (size_t)b * a.k, sh,
+                             a.kpos_out ? a.kpos_out + (size_t)b * a.N : nullptr,
+                             a.kpos_out ? a.pruned_out + (size_t)b * (a.N - a.k) : nullptr);
 }
 
 // Small N (<= kRankUseMaxN): selection by exact ranks, for latency. A cluster of
@@ -172,6 +176,8 @@ __global__ void __launch_bounds__(kRankThreads) topk_rank_kernel(const TopkArgs 
   cluster_sync_all();  // no CTA leaves while a peer may still read its count
 }
 }  // namespace
+
+bool topk_writes_index(int N) { return !(N <= kRankUseMaxN && N <= kRankMaxN); }
 
 cudaError_t topk_launch(const TopkArgs& a, cudaStream_t s, bool pdl) {
   static std::atomic<bool> configured[64];  // per device, zero-initialised

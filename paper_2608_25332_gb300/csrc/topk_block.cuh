@@ -15,7 +15,9 @@
 // The threshold key T and how many keys equal to T are taken (need_eq) then
 // give every selected element its output slot, #(greater before i) +
 // min(#(equal before i), need_eq), from counts of (greater, equal) in index
-// order scanned within warps and then across them.
+// order scanned within warps and then across them. The same count gives, when
+// asked for, the merge's index (Sec. 4.3): kpos[i] = the slot of a selected i,
+// else -1, and the unselected elements in ascending order, pruned[i - slot].
 #pragma once
 
 #include "common.cuh"
@@ -165,7 +167,8 @@ __device__ __forceinline__ void topk_block_rank(TopkShared& sh, int nc, int rem,
 // keys' min lo and max hi. Must be called by every thread of the block; keys
 // and sh.hist[0] (cleared) must be visible (synced).
 __device__ __forceinline__ void topk_block_select(const uint32_t* keys, int N, int k, uint32_t lo,
-                                                  uint32_t hi, int* out, TopkShared& sh) {
+                                                  uint32_t hi, int* out, TopkShared& sh, int* kpos = nullptr,
+                                                  int* pruned = nullptr) {
   const int tid = threadIdx.x, nth = blockDim.x, lane = tid & 31, warp = tid >> 5;
   int rem = k;  // keys still to take from [lo, hi]
   int buf = 0;
@@ -235,12 +238,19 @@ __device__ __forceinline__ void topk_block_select(const uint32_t* keys, int N, i
   uint32_t gtb = slot >> 16, eqb = slot & 0xffffu;
   for (int i = beg; i < end; ++i) {
     const uint32_t u = keys[i];
+    const uint32_t before_i = gtb + min(eqb, (uint32_t)need_eq);  // elements kept before i
+    bool kept = false;
     if (u > T) {
-      out[gtb + min(eqb, (uint32_t)need_eq)] = i;
+      kept = true;
       ++gtb;
     } else if (u == T) {
-      if (eqb < (uint32_t)need_eq) out[gtb + eqb] = i;
+      kept = eqb < (uint32_t)need_eq;
       ++eqb;
+    }
+    if (kept) out[before_i] = i;
+    if (kpos != nullptr) {
+      kpos[i] = kept ? (int)before_i : -1;
+      if (!kept) pruned[i - (int)before_i] = i;
     }
   }
 }
@@ -252,7 +262,8 @@ __device__ __forceinline__ void topk_block_select(const uint32_t* keys, int N, i
 template <int KPT>
 __device__ __forceinline__ void topk_block_select_reg(const uint32_t (&key)[KPT], int N, int k,
                                                       uint32_t lo, uint32_t hi, int* out,
-                                                      TopkShared& sh) {
+                                                      TopkShared& sh, int* kpos = nullptr,
+                                                      int* pruned = nullptr) {
   const int tid = threadIdx.x, nth = blockDim.x, lane = tid & 31, warp = tid >> 5;
   const int i0 = tid * KPT;
   int rem = k;
@@ -317,12 +328,19 @@ __device__ __forceinline__ void topk_block_select_reg(const uint32_t (&key)[KPT]
 #pragma unroll
   for (int c = 0; c < KPT; ++c) {
     if (i0 + c >= N) continue;
+    const uint32_t before_i = gtb + min(eqb, (uint32_t)need_eq);  // elements kept before i0 + c
+    bool kept = false;
     if (key[c] > T) {
-      out[gtb + min(eqb, (uint32_t)need_eq)] = i0 + c;
+      kept = true;
       ++gtb;
     } else if (key[c] == T) {
-      if (eqb < (uint32_t)need_eq) out[gtb + eqb] = i0 + c;
+      kept = eqb < (uint32_t)need_eq;
       ++eqb;
+    }
+    if (kept) out[before_i] = i0 + c;
+    if (kpos != nullptr) {
+      kpos[i0 + c] = kept ? (int)before_i : -1;
+      if (!kept) pruned[i0 + c - (int)before_i] = i0 + c;
     }
   }
 }
