@@ -324,6 +324,7 @@ struct RelFusedArgs {
 };
 
 constexpr int kRelMaxStages = 8;
+constexpr int kRelFinishRows = 8;  // rows per warp of relevance_finish_kernel
 constexpr uint32_t kRelTmemCols = 256;  // 128 visual + <= 128 text columns
 
 struct RelPipe {
@@ -464,8 +465,8 @@ __global__ void __launch_bounds__(kThreads, 2)
   if (threadIdx.x < 32) tmem_dealloc(pipe.tmem, kRelTmemCols);
 }
 
-// mu_i from the tile sums (tile order), then p_j = max over the critical rows
-// of Y[b][j][i] - mu_i; an empty T gives -inf. Loads go out 32 at a time.
+// mu_i from the tile sums (tile order; every CTA forms all of mu), then p_j =
+// max over the critical rows of Y[b][j][i] - mu_i; an empty T gives -inf.
 __global__ void __launch_bounds__(256) relevance_finish_kernel(const RelFusedArgs a, const int* text_len,
                                                                const uint8_t* mask, float* p) {
   __shared__ float mu[kBM];
@@ -490,26 +491,32 @@ __global__ void __launch_bounds__(256) relevance_finish_kernel(const RelFusedArg
     valid[c] = v;
   }
   __syncthreads();
-  const int j = blockIdx.x * blockDim.x + threadIdx.x;
-  if (j >= a.N_v) return;
-  const float4* y = reinterpret_cast<const float4*>(a.Y + ((size_t)b * a.N_v + j) * a.NT);
-  float best = -INFINITY;
-  for (int q0 = 0; q0 < a.NT / 4; q0 += 32) {  // NT <= 128: one batch
-    float4 f[32];
+  // a warp per kRelFinishRows rows: lane q reads the 16-byte piece q of each row
+  // (NT <= 128: at most 32 pieces), every row's load in flight, then a warp max
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int nq = a.NT / 4;
+  const int j0 = (blockIdx.x * (blockDim.x >> 5) + warp) * kRelFinishRows;
+  const bool has = lane < nq;
+  const int c = lane * 4;
+  const float m0 = has ? mu[c] : 0.f, m1 = has ? mu[c + 1] : 0.f, m2 = has ? mu[c + 2] : 0.f,
+              m3 = has ? mu[c + 3] : 0.f;
+  const bool v0 = has && valid[c], v1 = has && valid[c + 1], v2 = has && valid[c + 2], v3 = has && valid[c + 3];
+  const float4* y = reinterpret_cast<const float4*>(a.Y + (size_t)b * a.N_v * a.NT);
+  float4 f[kRelFinishRows];
 #pragma unroll
-    for (int u = 0; u < 32; ++u)
-      if (q0 + u < a.NT / 4) f[u] = y[q0 + u];
+  for (int r = 0; r < kRelFinishRows; ++r)
+    f[r] = (has && j0 + r < a.N_v) ? y[(size_t)(j0 + r) * nq + lane] : make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
-    for (int u = 0; u < 32; ++u) {
-      if (q0 + u >= a.NT / 4) break;
-      const int c = (q0 + u) * 4;
-      if (valid[c]) best = fmaxf(best, f[u].x - mu[c]);
-      if (valid[c + 1]) best = fmaxf(best, f[u].y - mu[c + 1]);
-      if (valid[c + 2]) best = fmaxf(best, f[u].z - mu[c + 2]);
-      if (valid[c + 3]) best = fmaxf(best, f[u].w - mu[c + 3]);
-    }
+  for (int r = 0; r < kRelFinishRows; ++r) {
+    float best = -INFINITY;
+    if (v0) best = fmaxf(best, f[r].x - m0);
+    if (v1) best = fmaxf(best, f[r].y - m1);
+    if (v2) best = fmaxf(best, f[r].z - m2);
+    if (v3) best = fmaxf(best, f[r].w - m3);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) best = fmaxf(best, __shfl_xor_sync(0xffffffffu, best, o));
+    if (lane == 0 && j0 + r < a.N_v) p[(size_t)b * a.N_v + j0 + r] = best;
   }
-  p[(size_t)b * a.N_v + j] = best;
 }
 
 // G = E_t E_t^T for one sample (<= 128 text rows), split over K: CTA x of
@@ -725,7 +732,8 @@ cudaError_t relevance_tc_launch(const SimArgs& a, const uint8_t* mask, const flo
     e = cudaStreamWaitEvent(s, mask_ready, 0);  // the first kernel that reads the mask
     if (e != cudaSuccess) return e;
   }
-  relevance_finish_kernel<<<dim3((a.N_v + 255) / 256, a.B), 256, 0, s>>>(r, a.text_len, mask, p);
+  relevance_finish_kernel<<<dim3((a.N_v + 8 * kRelFinishRows - 1) / (8 * kRelFinishRows), a.B), 256, 0, s>>>(
+      r, a.text_len, mask, p);
   return cudaGetLastError();
 }
 
