@@ -630,6 +630,7 @@ using MeanSmall = MeanCfg<128, 4, 3, 256, 8>;       // row bytes <= 128 * 4 * 16
 using MeanBf16 = MeanCfg<256, 4, 4, 1024, 4>;       // bf16 rows <= 8192 elements
 using MeanF32 = MeanCfg<256, 8, 4, 1024, 2>;        // fp32 rows <= 8192 elements
 constexpr int kMeanSmallRowBytes = 128 * 4 * 16;
+constexpr int kSortSmemKeep = 6144;  // centroids whose counters the sort keeps in shared memory (48 KiB)
 template <typename C> size_t merge_mean_smem(int row_bytes) { return (size_t)C::kSlots * row_bytes; }
 
 // Counting sort of one sample's rows by centroid (one CTA of 1024 threads):
@@ -637,15 +638,20 @@ template <typename C> size_t merge_mean_smem(int row_bytes) { return (size_t)C::
 // members[b][offset[a] ..] the rows of a in no particular order (the means
 // rank them). The block-wide barriers order the phases (global memory of this
 // block only).
+template <bool kSmem>
 __global__ void __launch_bounds__(1024) merge_sort_kernel(const int* assign, int N_v, int keep, int* count,
                                                           int* offset, int* cursor, int* members) {
+  extern __shared__ int sort_sm[];  // kSmem: counts [keep], then offsets / cursors [keep]
   __shared__ uint32_t warp_tot[32];
   __shared__ uint32_t carry;
   const int b = blockIdx.x;
   const int* as = assign + (size_t)b * N_v;
-  int* cnt = count + (size_t)b * keep;
-  int* off = offset + (size_t)b * keep;
-  int* cur = cursor + (size_t)b * keep;
+  int* cnt_g = count + (size_t)b * keep;
+  int* off_g = offset + (size_t)b * keep;
+  // the counters: shared memory for at most kSortSmemKeep centroids, else the
+  // global scratch (cursor)
+  int* cnt = kSmem ? sort_sm : cnt_g;
+  int* cur = kSmem ? sort_sm + keep : cursor + (size_t)b * keep;
   for (int q = threadIdx.x; q < keep; q += blockDim.x) {
     cnt[q] = 0;
     cur[q] = 0;
@@ -680,14 +686,24 @@ __global__ void __launch_bounds__(1024) merge_sort_kernel(const int* assign, int
       warp_tot[lane] = ti - t;
     }
     __syncthreads();
-    if (ap < keep) off[ap] = (int)(carry + warp_tot[warp] + incl - v);
+    if (ap < keep) {
+      const int o = (int)(carry + warp_tot[warp] + incl - v);
+      off_g[ap] = o;
+      if (kSmem) {
+        cnt_g[ap] = (int)v;
+        cur[ap] = o;  // the fill's running position
+      }
+    }
     __syncthreads();
     if (threadIdx.x == 1023) carry += warp_tot[31] + incl;
     __syncthreads();
   }
   for (int j = threadIdx.x; j < N_v; j += blockDim.x) {
     const int ap = as[j];
-    if (ap >= 0 && ap < keep) members[(size_t)b * N_v + off[ap] + atomicAdd(&cur[ap], 1)] = j;
+    if (ap >= 0 && ap < keep) {
+      const int pos = kSmem ? atomicAdd(&cur[ap], 1) : off_g[ap] + atomicAdd(&cur[ap], 1);
+      members[(size_t)b * N_v + pos] = j;
+    }
   }
 }
 
@@ -970,7 +986,11 @@ cudaError_t merge_launch(const SimArgs& a, const int* keep_idx, int keep, const 
     int* off = cnt + (size_t)a.B * keep;
     int* cur = off + (size_t)a.B * keep;
     int* mem = reinterpret_cast<int*>(ws_best);
-    merge_sort_kernel<<<a.B, 1024, 0, s>>>(assign, a.N_v, keep, cnt, off, cur, mem);
+    if (keep <= kSortSmemKeep)
+      merge_sort_kernel<true><<<a.B, 1024, (size_t)2 * keep * sizeof(int), s>>>(assign, a.N_v, keep, cnt, off,
+                                                                                cur, mem);
+    else
+      merge_sort_kernel<false><<<a.B, 1024, 0, s>>>(assign, a.N_v, keep, cnt, off, cur, mem);
     dim3 gm(keep, a.B);
     static std::atomic<bool> configured[64];  // per device, zero-initialised
     int dev = 0;
