@@ -269,6 +269,10 @@ __global__ void __launch_bounds__(kPairThreads, 1)
   tc_fence_before();
   pair_cluster_sync();  // both CTAs' barriers initialised, the pair's tensor memory allocated
   tc_fence_after();
+  // launched as a programmatic dependent of the gather: the set-up above ran
+  // under its tail; the permuted copy and the index tables are read after this
+  pdl_wait_prior();
+  pdl_allow_next();
 
   if (warp == 0) {
     if (lane == 0) {
@@ -639,17 +643,19 @@ cudaError_t merge_argmax_pair_launch(const SimArgs& a, const int* keep_idx, int 
   m.ws_bidx = ws_bidx;
   m.err = a.err;
   cudaLaunchConfig_t cfg = {};
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = 2;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.gridDim = dim3((unsigned)(2 * plan.P), 1, 1);
   cfg.blockDim = dim3(kPairThreads, 1, 1);
   cfg.dynamicSmemBytes = pair_smem();
   cfg.stream = s;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 2;
   return cudaLaunchKernelEx(&cfg, merge_argmax_pair_tc, m, maps);
 }
 

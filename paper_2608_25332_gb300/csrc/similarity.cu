@@ -588,6 +588,8 @@ __global__ void __launch_bounds__(256) merge_argmax_kernel(const SimArgs a, cons
 // assign[b][j]: own position for kept rows, best over splits for the others
 __global__ void merge_assign_kernel(const SimArgs a, const int* kpos, int n_split,
                                     const float* ws_best, const int* ws_bidx, int* assign) {
+  pdl_wait_prior();  // the partials come from the Gram before
+  pdl_allow_next();
   const size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= (size_t)a.B * a.N_v) return;
   const int kp = kpos[i];
@@ -644,6 +646,8 @@ __global__ void __launch_bounds__(1024) merge_sort_kernel(const int* assign, int
   extern __shared__ int sort_sm[];  // kSmem: counts [keep], then offsets / cursors [keep]
   __shared__ uint32_t warp_tot[32];
   __shared__ uint32_t carry;
+  pdl_wait_prior();  // the assignment comes from the kernel before
+  pdl_allow_next();
   const int b = blockIdx.x;
   const int* as = assign + (size_t)b * N_v;
   int* cnt_g = count + (size_t)b * keep;
@@ -750,6 +754,7 @@ __global__ void __launch_bounds__(C::kThreads, C::kMinBlocks)
   constexpr int kPieces = C::kPieces;
   const int ap = blockIdx.x, b = blockIdx.y;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  pdl_wait_prior();  // the member lists come from the sort before
   const T* E = static_cast<const T*>(a.emb_v) + (size_t)b * a.N_v * a.D;
   T* out = static_cast<T*>(merged) + ((size_t)b * keep + ap) * a.D;
   const uint32_t row_bytes = (uint32_t)a.D * (uint32_t)sizeof(T);
@@ -978,7 +983,9 @@ cudaError_t merge_launch(const SimArgs& a, const int* keep_idx, int keep, const 
       merge_argmax_kernel<__nv_bfloat16><<<g, 256, 0, s>>>(a, keep_idx, keep, inv_v, kpos, n_split, ws_best,
                                                            ws_bidx);
   }
-  merge_assign_kernel<<<(unsigned)((nb + 255) / 256), 256, 0, s>>>(a, kpos, n_split, ws_best, ws_bidx, assign);
+  cudaError_t el = launch_pdl(merge_assign_kernel, dim3((unsigned)((nb + 255) / 256)), dim3(256), 0, s, a,
+                              (const int*)kpos, n_split, (const float*)ws_best, (const int*)ws_bidx, assign);
+  if (el != cudaSuccess) return el;
   if (merged != nullptr) {
     // counting sort of the rows by centroid; the scratch reuses ws_best/ws_bidx
     // (the argmax partials are consumed by merge_assign_kernel above)
@@ -986,11 +993,13 @@ cudaError_t merge_launch(const SimArgs& a, const int* keep_idx, int keep, const 
     int* off = cnt + (size_t)a.B * keep;
     int* cur = off + (size_t)a.B * keep;
     int* mem = reinterpret_cast<int*>(ws_best);
-    if (keep <= kSortSmemKeep)
-      merge_sort_kernel<true><<<a.B, 1024, (size_t)2 * keep * sizeof(int), s>>>(assign, a.N_v, keep, cnt, off,
-                                                                                cur, mem);
-    else
-      merge_sort_kernel<false><<<a.B, 1024, 0, s>>>(assign, a.N_v, keep, cnt, off, cur, mem);
+    cudaError_t es = keep <= kSortSmemKeep
+                         ? launch_pdl(merge_sort_kernel<true>, dim3(a.B), dim3(1024),
+                                      (size_t)2 * keep * sizeof(int), s, (const int*)assign, a.N_v, keep, cnt,
+                                      off, cur, mem)
+                         : launch_pdl(merge_sort_kernel<false>, dim3(a.B), dim3(1024), 0, s, (const int*)assign,
+                                      a.N_v, keep, cnt, off, cur, mem);
+    if (es != cudaSuccess) return es;
     dim3 gm(keep, a.B);
     static std::atomic<bool> configured[64];  // per device, zero-initialised
     int dev = 0;
@@ -1007,22 +1016,25 @@ cudaError_t merge_launch(const SimArgs& a, const int* keep_idx, int keep, const 
       configured[dev] = true;
     }
     const int row_bytes = a.D * (a.dtype == 0 ? 4 : 2);
+    cudaError_t em;
     if (row_bytes <= kMeanSmallRowBytes) {
       const size_t smem = merge_mean_smem<MeanSmall>(row_bytes);
       if (a.dtype == 0)
-        merge_mean_kernel<float, double, MeanSmall><<<gm, MeanSmall::kThreads, smem, s>>>(a, assign, cnt, off, mem,
-                                                                                        keep, merged);
+        em = launch_pdl(merge_mean_kernel<float, double, MeanSmall>, gm, dim3(MeanSmall::kThreads), smem, s, a,
+                        (const int*)assign, (const int*)cnt, (const int*)off, (const int*)mem, keep, merged);
       else
-        merge_mean_kernel<__nv_bfloat16, float, MeanSmall><<<gm, MeanSmall::kThreads, smem, s>>>(
-            a, assign, cnt, off, mem, keep, merged);
+        em = launch_pdl(merge_mean_kernel<__nv_bfloat16, float, MeanSmall>, gm, dim3(MeanSmall::kThreads), smem,
+                        s, a, (const int*)assign, (const int*)cnt, (const int*)off, (const int*)mem, keep, merged);
     } else if (a.dtype == 0) {
-      merge_mean_kernel<float, double, MeanF32><<<gm, MeanF32::kThreads, merge_mean_smem<MeanF32>(row_bytes), s>>>(
-          a, assign, cnt, off, mem, keep, merged);
+      em = launch_pdl(merge_mean_kernel<float, double, MeanF32>, gm, dim3(MeanF32::kThreads),
+                      merge_mean_smem<MeanF32>(row_bytes), s, a, (const int*)assign, (const int*)cnt,
+                      (const int*)off, (const int*)mem, keep, merged);
     } else {
-      merge_mean_kernel<__nv_bfloat16, float, MeanBf16>
-          <<<gm, MeanBf16::kThreads, merge_mean_smem<MeanBf16>(row_bytes), s>>>(a, assign, cnt, off, mem, keep,
-                                                                              merged);
+      em = launch_pdl(merge_mean_kernel<__nv_bfloat16, float, MeanBf16>, gm, dim3(MeanBf16::kThreads),
+                      merge_mean_smem<MeanBf16>(row_bytes), s, a, (const int*)assign, (const int*)cnt,
+                      (const int*)off, (const int*)mem, keep, merged);
     }
+    if (em != cudaSuccess) return em;
   }
   return cudaGetLastError();
 }

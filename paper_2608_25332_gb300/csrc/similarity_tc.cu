@@ -30,6 +30,8 @@ __global__ void __launch_bounds__(256) gather_perm_kernel(const __nv_bfloat16* E
                                                           const int* keep_idx, int n_pruned, int keep,
                                                           int N_v, int D, __nv_bfloat16* perm,
                                                           unsigned* err) {
+  pdl_wait_prior();  // pruned and keep_idx come from the kernels before
+  pdl_allow_next();  // the Gram may set itself up meanwhile
   const int b = blockIdx.y;
   const int r = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
   if (r >= N_v) return;
@@ -636,9 +638,9 @@ cudaError_t merge_argmax_tc_launch(const SimArgs& a, const int* keep_idx, int ke
     if (e != cudaSuccess) return e;
   }
   dim3 gg((a.N_v + 7) / 8, a.B);
-  gather_perm_kernel<<<gg, 256, 0, s>>>(static_cast<const __nv_bfloat16*>(a.emb_v), pruned, keep_idx,
-                                        n_pruned, keep, a.N_v, a.D, static_cast<__nv_bfloat16*>(perm),
-                                        a.err);
+  e = launch_pdl(gather_perm_kernel, gg, dim3(256), 0, s, static_cast<const __nv_bfloat16*>(a.emb_v), pruned,
+                 keep_idx, n_pruned, keep, a.N_v, a.D, static_cast<__nv_bfloat16*>(perm), a.err);
+  if (e != cudaSuccess) return e;
   if (pairs) {
     *n_split_out = plan.n_slots;
     return merge_argmax_pair_launch(a, keep_idx, keep, inv_v, pruned, perm, plan, ws_best, ws_bidx, s);
