@@ -720,7 +720,7 @@ extern "C" int provip_similarity_reduce(const void* emb_v, int B, int N_v, int D
       t.kpos_out = assign_out_or_null ? assign_out_or_null : w.assign;
       t.pruned_out = w.pruned;
     }
-    e = topk_launch(t, s);
+    e = topk_launch(t, s, true);  // a programmatic dependent of the relevance's last kernel
   }
   if (e == cudaSuccess && merged_out_or_null)
     e = merge_launch(a, idx_out, keep_pre, w.inv_v, assign_out_or_null ? assign_out_or_null : w.assign,

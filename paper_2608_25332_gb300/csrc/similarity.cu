@@ -185,6 +185,7 @@ __global__ void __launch_bounds__(kFinishThreads) crit_finish_kernel(const SimAr
 template <typename T>
 __global__ void __launch_bounds__(256) inv_norm_kernel(const void* X, size_t rows, int D,
                                                        float* inv) {
+  pdl_allow_next();  // a dependent reads inv only after this grid completes
   const size_t row = (size_t)blockIdx.x * 8 + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (row >= rows) return;

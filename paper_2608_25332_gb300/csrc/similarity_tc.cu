@@ -413,6 +413,9 @@ __global__ void __launch_bounds__(kThreads, 2)
     const int r = quad * 32 + lane;
     const int j = n0 + r;
     const bool rv = r < R && j < a.N_v;
+    // launched as a programmatic dependent of the text-row norms: the loads and
+    // MMAs ran under that kernel; its output (and every write below) waits here
+    pdl_wait_prior();
     s_invt[r] = r < a.N_t_max ? a.inv_t[(size_t)b * a.N_t_max + r] : 0.f;
     asm volatile("bar.sync 1, 128;" ::: "memory");  // s_invt complete (epilogue warps)
     const bool ok = warp_mbar_wait(&pipe.acc_full, 0, a.err) && !pipe.fail;
@@ -471,6 +474,7 @@ __global__ void __launch_bounds__(kThreads, 2)
 // max over the critical rows of Y[b][j][i] - mu_i; an empty T gives -inf.
 __global__ void __launch_bounds__(256) relevance_finish_kernel(const RelFusedArgs a, const int* text_len,
                                                                const uint8_t* mask, float* p) {
+  pdl_allow_next();  // the top-k reads p only after this grid completes
   __shared__ float mu[kBM];
   __shared__ int valid[kBM];
   const int b = blockIdx.y;
@@ -729,7 +733,8 @@ cudaError_t relevance_tc_launch(const SimArgs& a, const uint8_t* mask, const flo
       make_tmap_bf16_2d(&mapT, a.emb_t, (uint64_t)a.B * a.N_t_max, (uint64_t)a.D, (uint64_t)a.D * 2,
                         (uint32_t)r.NT))
     return cudaErrorInvalidValue;
-  relevance_fused_tc<<<dim3(r.n_vt, a.B), kThreads, smem, s>>>(r, mapV, mapT);
+  e = launch_pdl(relevance_fused_tc, dim3(r.n_vt, a.B), dim3(kThreads), smem, s, r, mapV, mapT);
+  if (e != cudaSuccess) return e;
   if (mask_ready != nullptr) {
     e = cudaStreamWaitEvent(s, mask_ready, 0);  // the first kernel that reads the mask
     if (e != cudaSuccess) return e;
