@@ -622,7 +622,9 @@ extern "C" int provip_merge(const void* emb_v, int B, int N_v, int D, const int*
   merge_ws(c, B, N_v, D, keep, w);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   SimArgs a = sim_args(emb_v, nullptr, nullptr, B, N_v, D, 1, dtype, d->status);
-  cudaError_t e = vis_inv_norm_launch(a, w.inv_v, s);
+  // the cosine's kept-row factor 1/|e_k| is all the nearest-centroid argmax
+  // needs (the pruned row's own norm is the same for every kept k)
+  cudaError_t e = kept_inv_norm_launch(a, keep_idx, keep, w.inv_v, s);
   if (e == cudaSuccess)
     e = merge_launch(a, keep_idx, keep, w.inv_v, assign_out, merged_out, w.best, w.bidx,
                      merge_splits(B, N_v, keep), w.pruned, dtype == PROVIP_BF16 ? w.perm : nullptr,

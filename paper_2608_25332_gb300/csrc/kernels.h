@@ -180,6 +180,10 @@ cudaError_t crit_text_launch(const SimArgs& a, uint8_t* mask, float* r_out, floa
                              cudaStream_t s);
 // inverse L2 norms of every visual row (0 for a zero row): inv_v [B][N_v]
 cudaError_t vis_inv_norm_launch(const SimArgs& a, float* inv_v, cudaStream_t s);
+// the same for the kept rows keep_idx [B][keep] only (inv_v[b][keep_idx[b][q]]),
+// which is all the merge reads
+cudaError_t kept_inv_norm_launch(const SimArgs& a, const int* keep_idx, int keep, float* inv_v,
+                                 cudaStream_t s);
 // Sec. 4.3: p[b][j] = max_{i in T} cos(t_i, v_j) - mu_i; also writes inv_v (the
 // inverse norms of the visual rows, used again by the merge). ws_sum holds
 // n_split partial sums over row chunks and their total.

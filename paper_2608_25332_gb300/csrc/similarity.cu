@@ -883,6 +883,46 @@ cudaError_t crit_text_launch(const SimArgs& a, uint8_t* mask, float* r_out, floa
   return cudaGetLastError();
 }
 
+// 1/|e_j| (0 for a zero row) of the kept rows j = keep_idx[b][q] only, into
+// inv_v[b][j] (the merge reads no other): a warp per row; an index out of range
+// is reported and skipped.
+template <typename T>
+__global__ void __launch_bounds__(256) kept_inv_norm_kernel(const void* X, const int* keep_idx, int keep,
+                                                            int N_v, int D, size_t rows, float* inv_v,
+                                                            unsigned* err) {
+  const size_t row = (size_t)blockIdx.x * 8 + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (row >= rows) return;
+  const size_t b = row / (size_t)keep;
+  const int j = keep_idx[row];
+  if (j < 0 || j >= N_v) {
+    if (lane == 0) set_error(err, kErrBadDeviceArg);
+    return;
+  }
+  const T* p = static_cast<const T*>(X) + (b * (size_t)N_v + (size_t)j) * (size_t)D;
+  float s = 0.f;
+  for (int e = lane * 8; e < D; e += 256) {
+    float v[8];
+    load8(p + e, v);
+#pragma unroll
+    for (int q = 0; q < 8; ++q) s = fmaf(v[q], v[q], s);
+  }
+  s = warp_sum(s);
+  if (lane == 0) inv_v[b * (size_t)N_v + (size_t)j] = s > 0.f ? 1.f / sqrtf(s) : 0.f;
+}
+
+cudaError_t kept_inv_norm_launch(const SimArgs& a, const int* keep_idx, int keep, float* inv_v,
+                                 cudaStream_t s) {
+  const size_t rows = (size_t)a.B * keep;
+  const unsigned grid = (unsigned)((rows + 7) / 8);
+  if (a.dtype == 0)
+    kept_inv_norm_kernel<float><<<grid, 256, 0, s>>>(a.emb_v, keep_idx, keep, a.N_v, a.D, rows, inv_v, a.err);
+  else
+    kept_inv_norm_kernel<__nv_bfloat16><<<grid, 256, 0, s>>>(a.emb_v, keep_idx, keep, a.N_v, a.D, rows, inv_v,
+                                                            a.err);
+  return cudaGetLastError();
+}
+
 cudaError_t vis_inv_norm_launch(const SimArgs& a, float* inv_v, cudaStream_t s) {
   const size_t rows = (size_t)a.B * a.N_v;
   const unsigned grid = (unsigned)((rows + 7) / 8);
