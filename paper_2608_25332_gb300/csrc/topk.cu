@@ -72,7 +72,9 @@ __global__ void __launch_bounds__(kTopkMaxThreads) topk_kernel(const TopkArgs a)
 // threads, so a thread may hold 128 registers), thread t owning the contiguous
 // indices [t * KPT, t * KPT + KPT).
 constexpr int kRegMaxThreads = 512;
-template <int KPT>
+// kIndex: also write the merge's index (kpos_out, pruned_out), a separate
+// instantiation so that the plain selection carries none of that code
+template <int KPT, bool kIndex>
 __global__ void __launch_bounds__(kRegMaxThreads) topk_reg_kernel(const TopkArgs a) {
   __shared__ TopkShared sh;
   // the histogram is cleared while the kernel that writes the scores finishes
@@ -86,9 +88,9 @@ __global__ void __launch_bounds__(kRegMaxThreads) topk_reg_kernel(const TopkArgs
   // the scores are consumed: the next kernel may start (it waits for this
   // grid's completion before reading idx)
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-  topk_block_select_reg<KPT>(key, a.N, a.k, lo, hi, a.idx_out + (size_t)b * a.k, sh,
-                             a.kpos_out ? a.kpos_out + (size_t)b * a.N : nullptr,
-                             a.kpos_out ? a.pruned_out + (size_t)b * (a.N - a.k) : nullptr);
+  topk_block_select_reg<KPT, kIndex>(key, a.N, a.k, lo, hi, a.idx_out + (size_t)b * a.k, sh,
+                                     kIndex ? a.kpos_out + (size_t)b * a.N : nullptr,
+                                     kIndex ? a.pruned_out + (size_t)b * (a.N - a.k) : nullptr);
 }
 
 // Small N (<= kRankUseMaxN): selection by exact ranks, for latency. A cluster of
@@ -224,10 +226,16 @@ cudaError_t topk_launch(const TopkArgs& a, cudaStream_t s, bool pdl) {
     int nt = ((a.N + kpt - 1) / kpt + 31) / 32 * 32;
     cfg.blockDim = dim3((unsigned)(nt < 128 ? 128 : nt));
     cfg.dynamicSmemBytes = 0;
-    if (kpt == 4) return cudaLaunchKernelEx(&cfg, topk_reg_kernel<4>, a);
-    if (kpt == 8) return cudaLaunchKernelEx(&cfg, topk_reg_kernel<8>, a);
-    if (kpt == 16) return cudaLaunchKernelEx(&cfg, topk_reg_kernel<16>, a);
-    return cudaLaunchKernelEx(&cfg, topk_reg_kernel<32>, a);
+    if (a.kpos_out != nullptr) {
+      if (kpt == 4) return cudaLaunchKernelEx(&cfg, topk_reg_kernel<4, true>, a);
+      if (kpt == 8) return cudaLaunchKernelEx(&cfg, topk_reg_kernel<8, true>, a);
+      if (kpt == 16) return cudaLaunchKernelEx(&cfg, topk_reg_kernel<16, true>, a);
+      return cudaLaunchKernelEx(&cfg, topk_reg_kernel<32, true>, a);
+    }
+    if (kpt == 4) return cudaLaunchKernelEx(&cfg, topk_reg_kernel<4, false>, a);
+    if (kpt == 8) return cudaLaunchKernelEx(&cfg, topk_reg_kernel<8, false>, a);
+    if (kpt == 16) return cudaLaunchKernelEx(&cfg, topk_reg_kernel<16, false>, a);
+    return cudaLaunchKernelEx(&cfg, topk_reg_kernel<32, false>, a);
   }
   return cudaLaunchKernelEx(&cfg, topk_kernel, a);
 }

@@ -259,7 +259,7 @@ __device__ __forceinline__ void topk_block_select(const uint32_t* keys, int N, i
 // KPT keys of indices [t * KPT, t * KPT + KPT) (valid below N), so every
 // per-key loop is unrolled and its loads and atomics are in flight together.
 // sh.hist[0] must be cleared and visible; lo/hi are the keys' min and max.
-template <int KPT>
+template <int KPT, bool kIndex = false>
 __device__ __forceinline__ void topk_block_select_reg(const uint32_t (&key)[KPT], int N, int k,
                                                       uint32_t lo, uint32_t hi, int* out,
                                                       TopkShared& sh, int* kpos = nullptr,
@@ -325,22 +325,34 @@ __device__ __forceinline__ void topk_block_select_reg(const uint32_t (&key)[KPT]
   for (int o = 16; o > 0; o >>= 1) before += __shfl_xor_sync(0xffffffffu, before, o);
   const uint32_t slot = before + incl - cnt;
   uint32_t gtb = slot >> 16, eqb = slot & 0xffffu;
+  if constexpr (kIndex) {
 #pragma unroll
-  for (int c = 0; c < KPT; ++c) {
-    if (i0 + c >= N) continue;
-    const uint32_t before_i = gtb + min(eqb, (uint32_t)need_eq);  // elements kept before i0 + c
-    bool kept = false;
-    if (key[c] > T) {
-      kept = true;
-      ++gtb;
-    } else if (key[c] == T) {
-      kept = eqb < (uint32_t)need_eq;
-      ++eqb;
-    }
-    if (kept) out[before_i] = i0 + c;
-    if (kpos != nullptr) {
+    for (int c = 0; c < KPT; ++c) {
+      if (i0 + c >= N) continue;
+      const uint32_t before_i = gtb + min(eqb, (uint32_t)need_eq);  // elements kept before i0 + c
+      bool kept = false;
+      if (key[c] > T) {
+        kept = true;
+        ++gtb;
+      } else if (key[c] == T) {
+        kept = eqb < (uint32_t)need_eq;
+        ++eqb;
+      }
+      if (kept) out[before_i] = i0 + c;
       kpos[i0 + c] = kept ? (int)before_i : -1;
       if (!kept) pruned[i0 + c - (int)before_i] = i0 + c;
+    }
+  } else {
+#pragma unroll
+    for (int c = 0; c < KPT; ++c) {
+      if (i0 + c >= N) continue;
+      if (key[c] > T) {
+        out[gtb + min(eqb, (uint32_t)need_eq)] = i0 + c;
+        ++gtb;
+      } else if (key[c] == T) {
+        if (eqb < (uint32_t)need_eq) out[gtb + eqb] = i0 + c;
+        ++eqb;
+      }
     }
   }
 }
