@@ -18,7 +18,7 @@
 //
 // A group splits its kept columns into n_lo or n_lo + 1 ranges (see
 // pair_tile); the tiles are dealt to the clusters in snake order (see
-// pair_round_tile), so that the busiest pair of SMs gets as little work as the
+// pair_deal_tile), so that the busiest pair of SMs gets as little work as the
 // ranges allow, and the tiles of one group run side by side on different pairs
 // and share its A rows through L2. Each CTA loads only the N/2 kept rows its
 // half of the MMA reads (one tensor map per distinct N/2 of the plan).
@@ -224,11 +224,11 @@ __host__ __device__ __forceinline__ PairTile pair_tile(const MergePairPlan& p, i
   g.N = (g.nv + 31) / 32 * 32;         // MMA width: N / 2 rows of B per CTA, a multiple of 16
   return g;
 }
-// Tile of pair p in round r (snake order: pairs 0 .. P-1 take tiles r*P ..
-// in rounds 0, 2, ..., and in reverse order in rounds 1, 3, ..., so that a
+// Tile of pair p in deal r (snake order: pairs 0 .. P-1 take tiles r*P ..
+// in deals 0, 2, ..., and in reverse order in deals 1, 3, ..., so that a
 // pair given one of the first, wider tiles gets one of the last, narrower ones);
 // -1 past the last tile.
-__host__ __device__ __forceinline__ int pair_round_tile(const MergePairPlan& p, int pair, int r) {
+__host__ __device__ __forceinline__ int pair_deal_tile(const MergePairPlan& p, int pair, int r) {
   const int k = (r & 1) ? (r + 1) * p.P - 1 - pair : r * p.P + pair;
   return k < p.T ? k : -1;
 }
@@ -279,7 +279,7 @@ __global__ void __launch_bounds__(kPairThreads, 1)
       // both CTAs load their rows of every stage; completion counts on the
       // even CTA's full barrier, which expects the bytes of both
       int it = 0;
-      for (int rd = 0, k; (k = pair_round_tile(pl, pair, rd)) >= 0 && !pipe.fail; ++rd) {
+      for (int rd = 0, k; (k = pair_deal_tile(pl, pair, rd)) >= 0 && !pipe.fail; ++rd) {
         const PairTile g = pair_tile(pl, a.n_pruned, a.keep, k);
         const int row_a = g.b * a.N_v + g.m0 + (int)rank * kBM;
         const int row_b = g.b * a.N_v + a.n_pruned + g.c0 + (int)rank * (g.N / 2);
@@ -315,7 +315,7 @@ __global__ void __launch_bounds__(kPairThreads, 1)
   } else if (warp == 1) {
     if (rank == 0 && lane == 0) {
       int it = 0, ti = 0;
-      for (int rd = 0, k; (k = pair_round_tile(pl, pair, rd)) >= 0; ++rd, ++ti) {
+      for (int rd = 0, k; (k = pair_deal_tile(pl, pair, rd)) >= 0; ++rd, ++ti) {
         const PairTile g = pair_tile(pl, a.n_pruned, a.keep, k);
         // both epilogues have read the previous tile's accumulators
         if (!pipe.fail && !mbar_wait_cluster(&pipe.acc_empty, ((uint32_t)ti & 1u) ^ 1u, a.err)) pipe.fail = 1;
@@ -356,7 +356,7 @@ __global__ void __launch_bounds__(kPairThreads, 1)
     const int r = quad * 32 + lane;
     const uint32_t acc_empty = cluster_addr(&pipe.acc_empty, 0);
     int ti = 0;
-    for (int rd = 0, k; (k = pair_round_tile(pl, pair, rd)) >= 0; ++rd, ++ti) {
+    for (int rd = 0, k; (k = pair_deal_tile(pl, pair, rd)) >= 0; ++rd, ++ti) {
       const PairTile g = pair_tile(pl, a.n_pruned, a.keep, k);
       const int* pr = a.pruned + (size_t)g.b * a.n_pruned;
       const int* kp = a.keep_idx + (size_t)g.b * a.keep;
@@ -526,7 +526,7 @@ static bool merge_pair_search(int B, int n_pruned, int keep, int D, int num_sms,
       }
     load.assign(c.P, 0.0);
     for (int pr = 0; pr < c.P; ++pr) {
-      for (int r = 0, k; (k = pair_round_tile(c, pr, r)) >= 0; ++r) {
+      for (int r = 0, k; (k = pair_deal_tile(c, pr, r)) >= 0; ++r) {
         const PairTile g = pair_tile(c, n_pruned, keep, k);
         load[pr] += (double)n_k * fmax((g.has1 ? 4.0 : 2.0) * g.N, 960.0) + 9000.0;
       }
