@@ -1,6 +1,7 @@
 // Pre-LLM pass (Sec. 4.3) on 5th-generation tensor cores (bf16).
 //
-// merge_argmax_tc: the pruned x kept cosine Gram fused with the row argmax.
+// merge_argmax_tc: the pruned x kept cosine Gram fused with the row argmax, on
+//   single SMs (the form on pairs of SMs is merge_pair_tc.cu, the default).
 //   A = the pruned visual rows of two 128-row M tiles, B = the kept rows of a
 //   range of 256-row N tiles shared by both, read as contiguous tiles of a
 //   per-sample copy of E_v permuted to [pruned | kept] by one bandwidth-bound
@@ -92,8 +93,10 @@ struct MergePipe {
 // 8.4 MFLOP instead of 48 KiB for 4.2 MFLOP with a single M tile. The two
 // accumulators fill the 512 TMEM columns: the epilogue of an N tile runs
 // between that tile's last MMA and the next tile's first (the producer keeps
-// loading meanwhile). The last N tile's MMA is only as wide as its kept rows
-// (rounded up to 16).
+// loading meanwhile), so it is kept short: eight warps, two per TMEM lane
+// quadrant, each taking half of a tile's 32-column pieces with its loads
+// double-buffered and four interleaved running maxima per row (RowBest). The
+// last N tile's MMA is only as wide as its kept rows (rounded up to 16).
 __global__ void __launch_bounds__(kMergeThreads, 1)
     merge_argmax_tc(const MergeTcArgs a, const __grid_constant__ CUtensorMap mapE) {
   extern __shared__ uint8_t smem_raw[];
