@@ -3,8 +3,9 @@
 // every pruned row of every sample must get each partial slot written exactly
 // once (by its range's tile, or as the spare slot of a group with fewer
 // ranges), every range must be 1..256 columns wide, its box height one of the
-// plan's, and each pair's tiles distinct. Prints "ok" per shape or the first
-// violation. Built and run by tests/test_merge_plan.py (host code only: no
+// plan's, and each pair's tiles distinct, and a second request for the same
+// shape (from the plan cache) must give the same plan. Prints "ok" per shape or
+// the first violation. Built and run by tests/test_merge_plan.py (host code only: no
 // GPU is touched).
 #include "../paper_2608_25332_gb300/csrc/merge_pair_tc.cu"
 
@@ -27,6 +28,15 @@ static int check(int B, int N_v, int keep, int D, int sms) {
     // the single-SM form
     printf("noplan B=%d N_v=%d keep=%d\n", B, N_v, keep);
     return 0;
+  }
+  // a second request (answered from the plan cache once the shape is known)
+  // gives the same plan
+  MergePairPlan q;
+  if (!merge_pair_plan(B, n_pruned, keep, D, sms, &q) || q.n_quads != p.n_quads || q.Q != p.Q ||
+      q.n_lo != p.n_lo || q.x_hi != p.x_hi || q.T != p.T || q.P != p.P || q.n_slots != p.n_slots ||
+      q.n_heights != p.n_heights) {
+    printf("B=%d N_v=%d keep=%d: a second request gave another plan\n", B, N_v, keep);
+    return 1;
   }
   if (p.P < 1 || p.P > sms / 2 || p.n_slots < 1 || p.n_slots > kMergeMaxSplit || p.n_heights < 1 ||
       p.n_heights > kMergePairHeights) {
